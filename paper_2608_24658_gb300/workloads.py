@@ -1,0 +1,394 @@
+"""Seeded synthetic fork-tree decode workloads.
+
+This module only draws inputs: tree shapes, node lengths, page tables and
+q/K/V values.  It holds none of the attention arithmetic, imports neither the
+CUDA binding nor the oracle, and is the one piece of code both sides share.
+
+A workload is one decode step of every live branch of a parallel-reasoning
+fork tree.  The paper's runtime dispatches each <Subtask>/<Trial> entry of a
+<Parallel> region as an independent worker (Sec. 3.4); threads may nest further
+<Parallel> regions (Fig. 4, rule W -> <Thread> B </Thread>), so the tree can
+be deeper than one level, as in the 24-puzzle example of Fig. 3 (three subtasks
+with four, one and three trials).
+
+Tree encoding (what ``parason_attn_plan`` takes):
+  parent[i]        parent node of node i, -1 for a root; parent[i] < i
+  node_len[i]      tokens held by node i (a leaf's count includes the token
+                   decoded this step)
+  node_page_ptr    CSR offsets [num_nodes + 1] into page_ids
+  page_ids         physical page of each node's j-th logical page; node i owns
+                   exactly ceil(node_len[i] / page_size) pages and no page is
+                   shared between nodes
+  leaf_node[b]     node holding branch b's private suffix; branch b's query is
+                   row b of q
+
+Value recipe: q, K, V ~ N(0, 1) rounded to the KV dtype (q scaled by 1/sqrt(d)
+in the 16-branch Llama-3-8B-shape workload); fp8 KV is the bf16 draw divided
+by a per-kv-head scale amax/448 and rounded to e4m3.  Draw order per seed:
+node lengths in node order, the page permutation, q, K, V.
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field, replace
+from typing import Optional, Sequence
+
+import numpy as np
+import torch
+
+PAGE_SIZE = 16
+E4M3_MAX = 448.0
+
+
+@dataclass
+class ForkTree:
+    name: str
+    num_q_heads: int
+    num_kv_heads: int
+    head_dim: int
+    mode: str                      # "bf16" | "fp32" | "fp8"
+    parent: np.ndarray
+    node_len: np.ndarray
+    node_page_ptr: np.ndarray
+    page_ids: np.ndarray
+    leaf_node: np.ndarray
+    num_physical_pages: int
+    q: torch.Tensor                # [L, H_q, d]
+    k_pages: torch.Tensor          # [P, H_kv, page_size, d]
+    v_pages: torch.Tensor
+    k_scale: Optional[torch.Tensor] = None   # [H_kv] fp32, fp8 mode
+    v_scale: Optional[torch.Tensor] = None
+    sm_scale: float = 0.0          # 0 => 1/sqrt(head_dim)
+    page_size: int = PAGE_SIZE
+    meta: dict = field(default_factory=dict)
+
+    @property
+    def num_nodes(self) -> int:
+        return len(self.parent)
+
+    @property
+    def num_leaves(self) -> int:
+        return len(self.leaf_node)
+
+    @property
+    def group(self) -> int:
+        return self.num_q_heads // self.num_kv_heads
+
+    def path(self, b: int) -> list:
+        """Nodes on the path root -> leaf of branch b, root first."""
+        out, n = [], int(self.leaf_node[b])
+        while n >= 0:
+            out.append(n)
+            n = int(self.parent[n])
+        return out[::-1]
+
+    def leaves_under(self) -> np.ndarray:
+        """Number of branches whose path contains each node."""
+        cnt = np.zeros(self.num_nodes, dtype=np.int64)
+        for b in range(self.num_leaves):
+            for n in self.path(b):
+                cnt[n] += 1
+        return cnt
+
+    def unique_tokens(self) -> int:
+        """Tokens of every node on some branch's path, each node counted once."""
+        cnt = self.leaves_under()
+        return int(self.node_len[cnt > 0].sum())
+
+    def path_tokens(self) -> int:
+        """Tokens summed over branches with no sharing (every branch's full path)."""
+        return int(sum(int(self.node_len[self.path(b)].sum()) for b in range(self.num_leaves)))
+
+    def kv_elem_bytes(self) -> int:
+        return {"bf16": 2, "fp32": 4, "fp8": 1}[self.mode]
+
+    def q_elem_bytes(self) -> int:
+        return 4 if self.mode == "fp32" else 2
+
+    def to(self, device) -> "ForkTree":
+        mv = lambda t: None if t is None else t.to(device)
+        return replace(self, q=mv(self.q), k_pages=mv(self.k_pages),
+                       v_pages=mv(self.v_pages), k_scale=mv(self.k_scale),
+                       v_scale=mv(self.v_scale))
+
+
+# ----------------------------------------------------------------------------
+# page tables
+# ----------------------------------------------------------------------------
+
+def assign_pages(node_len: Sequence[int], rng: Optional[np.random.Generator] = None,
+                 permute: bool = False, page_size: int = PAGE_SIZE,
+                 extra_pages: int = 0):
+    """Give every node ceil(len/page_size) fresh pages, node-major.
+
+    With ``permute`` the logical->physical map is a random permutation drawn
+    from ``rng`` (this is the draw that follows the node lengths).  Returns
+    (node_page_ptr, page_ids, num_physical_pages).
+    """
+    counts = np.array([(int(n) + page_size - 1) // page_size for n in node_len], dtype=np.int64)
+    ptr = np.zeros(len(counts) + 1, dtype=np.int64)
+    np.cumsum(counts, out=ptr[1:])
+    total = int(ptr[-1])
+    num_phys = total + int(extra_pages)
+    if permute:
+        assert rng is not None
+        perm = rng.permutation(num_phys)[:total]
+    else:
+        perm = np.arange(total)
+    return ptr.astype(np.int32), perm.astype(np.int32), num_phys
+
+
+# ----------------------------------------------------------------------------
+# value draws
+# ----------------------------------------------------------------------------
+
+def _randn(shape, gen, device, dtype, chunk_rows: int = 1 << 14):
+    """N(0,1) draw of ``shape`` in float32, rounded to ``dtype``.
+
+    Drawn in slices along dim 0 so that multi-GB KV pools never need an fp32
+    copy of the whole pool; the slice size is fixed, so the values depend only
+    on the seed.
+    """
+    out = torch.empty(shape, dtype=dtype, device=device)
+    for s in range(0, shape[0], chunk_rows):
+        e = min(shape[0], s + chunk_rows)
+        out[s:e] = torch.randn((e - s,) + tuple(shape[1:]), generator=gen,
+                               device=device, dtype=torch.float32).to(dtype)
+    return out
+
+
+def _quantize_e4m3(pages_bf16: torch.Tensor, chunk_rows: int = 1 << 14):
+    """Per-kv-head scale amax/448 and the e4m3 rounding of pages/scale."""
+    hkv = pages_bf16.shape[1]
+    amax = torch.zeros(hkv, dtype=torch.float32, device=pages_bf16.device)
+    for s in range(0, pages_bf16.shape[0], chunk_rows):
+        blk = pages_bf16[s:s + chunk_rows].float().abs()
+        amax = torch.maximum(amax, blk.amax(dim=(0, 2, 3)))
+    scale = torch.where(amax > 0, amax / E4M3_MAX, torch.ones_like(amax))
+    out = torch.empty(pages_bf16.shape, dtype=torch.float8_e4m3fn, device=pages_bf16.device)
+    for s in range(0, pages_bf16.shape[0], chunk_rows):
+        blk = pages_bf16[s:s + chunk_rows].float() / scale.view(1, -1, 1, 1)
+        out[s:s + chunk_rows] = blk.to(torch.float8_e4m3fn)
+    return out, scale
+
+
+def _fill_tail_slots(tree: ForkTree, value: float):
+    """Write ``value`` into the unused slots of every node's last page."""
+    ps = tree.page_size
+    for n in range(tree.num_nodes):
+        ln = int(tree.node_len[n])
+        if ln % ps == 0:
+            continue
+        page = int(tree.page_ids[int(tree.node_page_ptr[n + 1]) - 1])
+        for pages in (tree.k_pages, tree.v_pages):
+            if pages.dtype == torch.float8_e4m3fn:
+                pages.view(torch.uint8)[page, :, ln % ps:, :] = 0x7F if math.isnan(value) else 0
+            else:
+                pages[page, :, ln % ps:, :] = value
+
+
+def build_tree(name: str, parent, node_len, leaf_node, *, num_q_heads: int,
+               num_kv_heads: int, head_dim: int, mode: str = "bf16", seed: int = 0,
+               rng: Optional[np.random.Generator] = None, permute_pages: bool = False,
+               extra_pages: int = 0, q_std: float = 1.0, device="cpu",
+               tail_value: Optional[float] = None, sm_scale: float = 0.0,
+               meta: Optional[dict] = None) -> ForkTree:
+    """Assemble a workload from a tree shape; draws pages, then q, K, V."""
+    if rng is None:
+        rng = np.random.default_rng(seed)
+    parent = np.asarray(parent, dtype=np.int32)
+    node_len = np.asarray(node_len, dtype=np.int32)
+    leaf_node = np.asarray(leaf_node, dtype=np.int32)
+    ptr, pages, nphys = assign_pages(node_len, rng, permute_pages, PAGE_SIZE, extra_pages)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(rng.integers(0, 2**62)))
+    L = len(leaf_node)
+    q_dtype = torch.float32 if mode == "fp32" else torch.bfloat16
+    kv_draw_dtype = torch.float32 if mode == "fp32" else torch.bfloat16
+    q = torch.randn((L, num_q_heads, head_dim), generator=gen, device=device,
+                    dtype=torch.float32)
+    if q_std != 1.0:
+        q = q * q_std
+    q = q.to(q_dtype)
+    shape = (max(nphys, 1), num_kv_heads, PAGE_SIZE, head_dim)
+    k = _randn(shape, gen, device, kv_draw_dtype)
+    v = _randn(shape, gen, device, kv_draw_dtype)
+    k_scale = v_scale = None
+    if mode == "fp8":
+        k, k_scale = _quantize_e4m3(k)
+        v, v_scale = _quantize_e4m3(v)
+    tree = ForkTree(name=name, num_q_heads=num_q_heads, num_kv_heads=num_kv_heads,
+                    head_dim=head_dim, mode=mode, parent=parent, node_len=node_len,
+                    node_page_ptr=ptr, page_ids=pages, leaf_node=leaf_node,
+                    num_physical_pages=nphys, q=q, k_pages=k, v_pages=v,
+                    k_scale=k_scale, v_scale=v_scale, sm_scale=sm_scale,
+                    meta=dict(meta or {}))
+    if tail_value is not None:
+        _fill_tail_slots(tree, tail_value)
+    return tree
+
+
+# ----------------------------------------------------------------------------
+# the five workloads
+# ----------------------------------------------------------------------------
+
+def _uniform(rng, lo, hi):
+    return int(rng.integers(lo, hi + 1))      # inclusive bounds
+
+
+def tiny_fork(mode="bf16", device="cpu", **kw) -> ForkTree:
+    """1 request, 4 branches, 8 q / 2 kv heads, d 64, prefix 256, suffixes 32/40/48/64."""
+    rng = np.random.default_rng(0)
+    parent = [-1, 0, 0, 0, 0]
+    node_len = [256, 32, 40, 48, 64]
+    return build_tree("tiny_fork_h8_2_d64", parent, node_len, [1, 2, 3, 4], num_q_heads=8,
+                      num_kv_heads=2, head_dim=64, mode=mode, rng=rng, device=device, **kw)
+
+
+def llama3_trials(mode="bf16", device="cpu", **kw) -> ForkTree:
+    """Llama-3-8B attention shape (32 q / 8 kv, d 128), prefix 2048, 16 trials U[512,4096]."""
+    rng = np.random.default_rng(1)
+    lens = [2048] + [_uniform(rng, 512, 4096) for _ in range(16)]
+    parent = [-1] + [0] * 16
+    return build_tree("llama3_8b_prefix2048_16trials", parent, lens, list(range(1, 17)),
+                      num_q_heads=32, num_kv_heads=8, head_dim=128, mode=mode, rng=rng,
+                      q_std=1.0 / math.sqrt(128.0), device=device, **kw)
+
+
+def subtask_trial_tree(mode="bf16", device="cpu", **kw) -> ForkTree:
+    """Two-level tree: root 4096, 8 subtasks x 1024, 8 trials each U[256,2048]; 64/8/128."""
+    rng = np.random.default_rng(2)
+    parent, lens, leaves = [-1], [4096], []
+    for s in range(8):
+        parent.append(0)
+        lens.append(1024)
+    for s in range(8):
+        for t in range(8):
+            parent.append(1 + s)
+            lens.append(_uniform(rng, 256, 2048))
+            leaves.append(len(parent) - 1)
+    return build_tree("two_level_root4096_8x1024_64trials", parent, lens, leaves,
+                      num_q_heads=64, num_kv_heads=8, head_dim=128, mode=mode, rng=rng,
+                      device=device, **kw)
+
+
+def lognormal_prefix(rng, median=2048, sigma=0.5, lo=1024, hi=8192) -> int:
+    x = math.exp(math.log(median) + sigma * float(rng.standard_normal()))
+    return int(min(hi, max(lo, int(round(x)))))
+
+
+def batched_serving(mode="bf16", device="cpu", requests=32, branches=32, **kw) -> ForkTree:
+    """32 requests x 32 trials (1024 branches), lognormal prefixes, U[256,8192], permuted pages."""
+    rng = np.random.default_rng(3)
+    parent, lens, leaves = [], [], []
+    for r in range(requests):
+        root = len(parent)
+        parent.append(-1)
+        lens.append(lognormal_prefix(rng))
+        for b in range(branches):
+            parent.append(root)
+            lens.append(_uniform(rng, 256, 8192))
+            leaves.append(len(parent) - 1)
+    return build_tree(f"batched_{requests}req_x{branches}_permuted", parent, lens, leaves,
+                      num_q_heads=32, num_kv_heads=8, head_dim=128, mode=mode, rng=rng,
+                      permute_pages=True, device=device, **kw)
+
+
+def long_reasoning(mode="bf16", device="cpu", branches=128, **kw) -> ForkTree:
+    """Prefix 32768, 128 branches U[4096,16384], 64/8/128; bf16 or fp8 e4m3 KV."""
+    rng = np.random.default_rng(4)
+    lens = [32768] + [_uniform(rng, 4096, 16384) for _ in range(branches)]
+    parent = [-1] + [0] * branches
+    return build_tree(f"long_prefix32768_{branches}x4k_16k", parent, lens,
+                      list(range(1, branches + 1)), num_q_heads=64, num_kv_heads=8,
+                      head_dim=128, mode=mode, rng=rng, device=device, **kw)
+
+
+CONFIGS = {1: tiny_fork, 2: llama3_trials, 3: subtask_trial_tree, 4: batched_serving,
+           5: long_reasoning}
+
+
+def make_config(idx: int, mode: Optional[str] = None, device="cpu", **kw) -> ForkTree:
+    fn = CONFIGS[idx]
+    return fn(mode=mode or "bf16", device=device, **kw)
+
+
+# ----------------------------------------------------------------------------
+# small fixtures
+# ----------------------------------------------------------------------------
+
+def figure3_tree(mode="bf16", device="cpu", seed=11, h_q=8, h_kv=2, d=64,
+                 trunk=40, subtask=(24, 17, 33), trial_len=None, **kw) -> ForkTree:
+    """Shape of the 24-puzzle example: 3 subtask threads with 4, 1 and 3 trials."""
+    rng = np.random.default_rng(seed)
+    parent, lens, leaves = [-1], [trunk], []
+    for s, n_trials in enumerate((4, 1, 3)):
+        parent.append(0)
+        lens.append(subtask[s])
+    for s, n_trials in enumerate((4, 1, 3)):
+        for t in range(n_trials):
+            parent.append(1 + s)
+            lens.append(int(rng.integers(1, 70)) if trial_len is None else trial_len)
+            leaves.append(len(parent) - 1)
+    return build_tree("figure3_3subtasks_4_1_3_trials", parent, lens, leaves, num_q_heads=h_q,
+                      num_kv_heads=h_kv, head_dim=d, mode=mode, rng=rng, device=device, **kw)
+
+
+def random_tree(seed: int, *, num_requests=2, depth=3, fanout=(1, 4), len_range=(0, 80),
+                h_q=8, h_kv=2, d=64, mode="bf16", device="cpu", permute_pages=True,
+                extra_pages=3, leaf_min_len=1, **kw) -> ForkTree:
+    """Random forest of nested parallel regions (depth levels below each root)."""
+    rng = np.random.default_rng(seed)
+    parent, lens, leaves = [], [], []
+
+    def grow(node, level):
+        if level == depth:
+            leaves.append(node)
+            return
+        k = int(rng.integers(fanout[0], fanout[1] + 1))
+        for _ in range(k):
+            parent.append(node)
+            lens.append(0)
+            grow(len(parent) - 1, level + 1)
+
+    for _ in range(num_requests):
+        parent.append(-1)
+        lens.append(0)
+        grow(len(parent) - 1, 0)
+    leafset = set(leaves)
+    for n in range(len(parent)):
+        lo = max(len_range[0], leaf_min_len) if n in leafset else len_range[0]
+        lens[n] = int(rng.integers(lo, len_range[1] + 1))
+    return build_tree(f"random_forest_seed{seed}", parent, lens, leaves, num_q_heads=h_q,
+                      num_kv_heads=h_kv, head_dim=d, mode=mode, rng=rng,
+                      permute_pages=permute_pages, extra_pages=extra_pages, device=device, **kw)
+
+
+def host_subset(tree: ForkTree, sel: Sequence[int]) -> ForkTree:
+    """Host copy of only what branches ``sel`` read, with a compact page table.
+
+    Lets a CPU check of a multi-GB workload copy a few MB: the selected
+    branches keep their order (branch i of the result is sel[i]), their path
+    nodes keep their lengths, and their pages are copied to the host.
+    """
+    nodes = sorted({n for b in sel for n in tree.path(int(b))})
+    remap = {n: i for i, n in enumerate(nodes)}
+    parent = [remap[int(tree.parent[n])] if tree.parent[n] >= 0 else -1 for n in nodes]
+    node_len = [int(tree.node_len[n]) for n in nodes]
+    phys = []
+    ptr = [0]
+    for n in nodes:
+        phys.extend(int(p) for p in tree.page_ids[tree.node_page_ptr[n]:tree.node_page_ptr[n + 1]])
+        ptr.append(len(phys))
+    idx = torch.as_tensor(phys if phys else [0], dtype=torch.long, device=tree.k_pages.device)
+    k = tree.k_pages.index_select(0, idx).cpu()
+    v = tree.v_pages.index_select(0, idx).cpu()
+    sel_t = torch.as_tensor(list(sel), dtype=torch.long, device=tree.q.device)
+    q = tree.q.index_select(0, sel_t).cpu()
+    return replace(tree, name=tree.name + "_subset", parent=np.array(parent, np.int32),
+                   node_len=np.array(node_len, np.int32), node_page_ptr=np.array(ptr, np.int32),
+                   page_ids=np.arange(len(phys), dtype=np.int32),
+                   leaf_node=np.array([remap[int(tree.leaf_node[b])] for b in sel], np.int32),
+                   num_physical_pages=len(phys), q=q, k_pages=k, v_pages=v,
+                   k_scale=None if tree.k_scale is None else tree.k_scale.cpu(),
+                   v_scale=None if tree.v_scale is None else tree.v_scale.cpu())
