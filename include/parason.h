@@ -1,0 +1,261 @@
+/*
+ * parason.h -- C ABI of the GB300 (sm_103a) fork-tree decode-attention library.
+ *
+ * Parallel reasoning forks one request into Subtask branches (all results
+ * needed) and Trial branches (speculative attempts) (paper Sec. 3.1); threads
+ * may nest further parallel regions (Fig. 4, rule W -> <Thread> B </Thread>),
+ * so the live branches form a fork tree.  The runtime decodes every branch
+ * as an independent worker (Sec. 3.4) and concatenates the branch outputs
+ * into the context that follows (Fig. 1 caption), so each decode step needs,
+ * for every branch b, softmax attention of b's query over b's whole context:
+ * the KV of every tree node on the path root -> b, root first.
+ *
+ * This library computes exactly that, reading every shared node's KV from
+ * HBM once for all the branches under it.  Sharing, tiling and splitting are
+ * rearrangements of the same sums; the result is plain attention.
+ *
+ * Conventions for every entry point:
+ *   - "host" pointers are read during the call only; "device" pointers are
+ *     CUDA device memory owned by the caller and must stay valid until the
+ *     work queued on `stream` has finished.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Every
+ *     entry point that takes a stream only enqueues work on it, except
+ *     parason_plan_check, which synchronises it.
+ *   - No entry point throws; every failure is a parason_status.  Nothing is
+ *     allocated by parason_attn_decode or parason_lse_merge.
+ *
+ * Layouts (row-major, innermost last):
+ *   q         [num_leaves, H_q, head_dim]                 (branch b = row b)
+ *   k_pages   [num_physical_pages, H_kv, page_size, head_dim]
+ *   v_pages   same as k_pages
+ *   out       [num_leaves, H_q, head_dim]   same dtype as q
+ *   lse       [num_leaves, H_q] fp32, natural log of sum_t exp(s_t)
+ *   q head h reads kv head h / (H_q / H_kv)  (grouped-query attention)
+ *   s_t = sm_scale * <q, k_t>, sm_scale = 1/sqrt(head_dim) unless given.
+ */
+#ifndef PARASON_H
+#define PARASON_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* cudaStream_t without including the CUDA headers (same type). */
+struct CUstream_st;
+typedef struct CUstream_st *parason_stream_t;
+
+typedef enum {
+    PARASON_OK = 0,
+    PARASON_EINVAL = 1,       /* malformed argument, tree or page table   */
+    PARASON_ENOMEM = 2,       /* host or device allocation failed (plan)  */
+    PARASON_ECUDA = 3,        /* a CUDA runtime call failed               */
+    PARASON_ETIMEOUT = 4,     /* a bounded device wait expired            */
+    PARASON_EUNSUPPORTED = 5  /* valid but not implemented (shape / mode) */
+} parason_status;
+
+typedef enum {
+    PARASON_BF16 = 0,         /* q, K, V, out bf16; fp32 accumulation     */
+    PARASON_FP32 = 1,         /* q, K, V, out fp32; fp32 FMA throughout   */
+    PARASON_FP8_E4M3_KV = 2   /* q, out bf16; K, V OCP e4m3 bytes with one
+                                 fp32 scale per kv head for K and for V   */
+} parason_mode;
+
+typedef struct {
+    int32_t num_q_heads;      /* H_q, multiple of H_kv                    */
+    int32_t num_kv_heads;     /* H_kv                                     */
+    int32_t head_dim;         /* 64 or 128                                */
+    int32_t page_size;        /* tokens per KV page; must be 16           */
+    int32_t mode;             /* a parason_mode                           */
+    float sm_scale;           /* 0 => 1/sqrt(head_dim)                    */
+} parason_attn_config;
+
+typedef struct parason_plan_s *parason_plan;
+
+/*
+ * Build the decode plan of one fork tree (the branch set of Sec. 3.4 at one
+ * decode step) and upload its metadata on `stream`.
+ *
+ * Tree, all host arrays:
+ *   parent[num_nodes]        parent node, -1 for a root; parent[i] < i.
+ *                            Several roots (several requests) are allowed.
+ *   node_len[num_nodes]      tokens held by each node (>= 0); a branch's own
+ *                            node includes the token decoded this step.
+ *   node_page_ptr[num_nodes+1]  CSR offsets into page_ids; node i owns
+ *                            exactly ceil(node_len[i] / page_size) pages.
+ *   page_ids[node_page_ptr[num_nodes]]  physical page of node i's j-th page
+ *                            at page_ids[node_page_ptr[i] + j], in
+ *                            [0, num_physical_pages); no page is owned by two
+ *                            nodes.  Token t of node i sits in slot
+ *                            t % page_size of its page t / page_size.
+ *   leaf_node[num_leaves]    node holding branch b's private suffix; distinct
+ *                            nodes with no children.  Branch b's query is
+ *                            row b of q.
+ *
+ * Returns PARASON_EINVAL for: bad config (H_q % H_kv != 0, head_dim not 64 or
+ * 128, page_size != 16, unknown mode, negative or non-finite sm_scale), a
+ * parent out of range or not smaller than its child, a negative length, a
+ * page count that is not ceil(len/page_size), a page id out of range or owned
+ * twice, a leaf out of range, repeated or with children, or a NULL pointer.
+ * PARASON_ENOMEM / PARASON_ECUDA if the metadata cannot be allocated or
+ * copied.  On success *out owns host and device memory until
+ * parason_plan_destroy.  The plan is immutable and may be used by any number
+ * of decode calls, but calls that share a workspace must not overlap.
+ */
+parason_status parason_attn_plan(const parason_attn_config *cfg, int32_t num_nodes,
+                                 const int32_t *parent, const int32_t *node_len,
+                                 const int32_t *node_page_ptr, const int32_t *page_ids,
+                                 int32_t num_leaves, const int32_t *leaf_node,
+                                 int64_t num_physical_pages, parason_stream_t stream,
+                                 parason_plan *out);
+
+/*
+ * Same validation and work decomposition as parason_attn_plan, but no device
+ * memory and no CUDA call: the plan can be inspected (parason_plan_info,
+ * parason_plan_export) on a machine without a GPU.  parason_attn_decode on
+ * it returns PARASON_EINVAL.  `num_sms` is the SM count the work split
+ * targets (152 on GB300).
+ */
+parason_status parason_attn_plan_host(const parason_attn_config *cfg, int32_t num_nodes,
+                                      const int32_t *parent, const int32_t *node_len,
+                                      const int32_t *node_page_ptr, const int32_t *page_ids,
+                                      int32_t num_leaves, const int32_t *leaf_node,
+                                      int64_t num_physical_pages, int32_t num_sms,
+                                      parason_plan *out);
+
+/* Device workspace (bytes) that parason_attn_decode needs for this plan:
+ * the split partial results (o, m, l) of every work item.  0 for NULL. */
+size_t parason_plan_workspace_bytes(parason_plan plan);
+
+/*
+ * One decode step: out[b, h, :] = softmax(s) V over branch b's root->leaf KV.
+ * Asynchronous on `stream`; allocates nothing; capturable in a CUDA graph.
+ *
+ *   q        device, [num_leaves, H_q, head_dim], bf16 (fp32 in FP32 mode)
+ *   k_pages  device, [num_physical_pages, H_kv, 16, head_dim], bf16 / fp32 /
+ *            e4m3 bytes by mode, 16-byte aligned
+ *   v_pages  device, same layout and dtype as k_pages
+ *   k_scale, v_scale  device fp32 [H_kv] in FP8 mode (k = e4m3 * k_scale),
+ *            ignored otherwise (may be NULL)
+ *   out      device, [num_leaves, H_q, head_dim], dtype of q
+ *   lse      device fp32 [num_leaves, H_q] or NULL.  A branch whose whole
+ *            path holds no token gets out = 0 and lse = -inf.
+ *   workspace  device, at least parason_plan_workspace_bytes(plan) bytes,
+ *            256-byte aligned; no contents are kept between calls.
+ *
+ * Slots of a node's last page past node_len are never read into the result,
+ * whatever they hold (NaN included).  Returns PARASON_EINVAL on a host-only
+ * plan, a NULL or misaligned buffer or a short workspace, PARASON_ECUDA if a
+ * launch fails.  Device-side failures (a bounded wait that expired) are
+ * reported by parason_plan_check.
+ */
+parason_status parason_attn_decode(parason_plan plan, const void *q, const void *k_pages,
+                                   const void *v_pages, const float *k_scale,
+                                   const float *v_scale, void *out, float *lse,
+                                   void *workspace, size_t workspace_bytes,
+                                   parason_stream_t stream);
+
+/*
+ * Combine two attention results over disjoint key sets A and B (for example
+ * two KV ranges of one branch, or a branch's context before and after a join)
+ * into the result over A u B, row by row:
+ *   o = (e^{lse_a} o_a + e^{lse_b} o_b) / (e^{lse_a} + e^{lse_b})
+ *   lse = ln(e^{lse_a} + e^{lse_b})
+ * A side with lse = -inf is empty; both empty gives o = 0, lse = -inf.
+ * o_a, o_b, o_out: device [rows, head_dim], bf16 (PARASON_BF16 and
+ * PARASON_FP8_E4M3_KV) or fp32 (PARASON_FP32); lse_*: device fp32 [rows].
+ * o_out / lse_out may alias the inputs row for row.  Asynchronous on stream.
+ */
+parason_status parason_lse_merge(const void *o_a, const float *lse_a, const void *o_b,
+                                 const float *lse_b, void *o_out, float *lse_out,
+                                 int64_t rows, int32_t head_dim, int32_t mode,
+                                 parason_stream_t stream);
+
+/* Synchronise `stream`, then read and clear the plan's device error word:
+ * PARASON_ETIMEOUT if a kernel gave up a bounded wait since the last check,
+ * PARASON_ECUDA if the stream reports an error, else PARASON_OK. */
+parason_status parason_plan_check(parason_plan plan, parason_stream_t stream);
+
+/* Release the plan's host and device memory.  NULL is a no-op.  Work queued
+ * with the plan must have finished. */
+void parason_plan_destroy(parason_plan plan);
+
+/* Static English name of a status. */
+const char *parason_status_string(parason_status status);
+
+/* ---------------------------------------------------------------------------
+ * Inspection, testing and measurement
+ * ------------------------------------------------------------------------- */
+
+typedef struct {
+    int32_t num_items;          /* work items of the attention kernel       */
+    int32_t num_leaves;
+    int32_t num_merge_entries;  /* partial results folded by the merge      */
+    int32_t chunk_pages;        /* split-K chunk length in pages            */
+    int64_t num_slots;          /* partial (o, m, l) rows in the workspace  */
+    int64_t unique_tokens;      /* tokens of nodes some branch reads, once  */
+    int64_t path_tokens;        /* sum over branches of their path tokens   */
+    int32_t num_sms;            /* SM count the split targeted              */
+    int32_t on_device;          /* 1 if decode can run on this plan         */
+} parason_plan_info;
+
+parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info);
+
+/*
+ * Copy one of the plan's host-side tables into `dst` (host, `bytes` long):
+ *   PARASON_TABLE_ITEMS      int32 [num_items][8]: first page position in
+ *                            page_ids, page count, valid tokens in the last
+ *                            page, first branch (index into the DFS branch
+ *                            order), first node row, row count, kv head,
+ *                            partial slot of node row 0
+ *   PARASON_TABLE_DFS_LEAVES int32 [num_leaves]: branches in DFS order
+ *   PARASON_TABLE_MERGE_PTR  int32 [num_leaves + 1]: CSR into the entries
+ *   PARASON_TABLE_MERGE      int32 [num_merge_entries][2]: (base, stride);
+ *                            q head h = j*g + r of the branch reads the
+ *                            partial slot base + j*stride + r
+ * Returns PARASON_EINVAL if `bytes` is smaller than the table.
+ */
+enum {
+    PARASON_TABLE_ITEMS = 0,
+    PARASON_TABLE_DFS_LEAVES = 1,
+    PARASON_TABLE_MERGE_PTR = 2,
+    PARASON_TABLE_MERGE = 3
+};
+parason_status parason_plan_export(parason_plan plan, int32_t table, void *dst, size_t bytes);
+
+/*
+ * Debug controls.  `wait_limit_ns` bounds every device-side wait of the
+ * plan's kernels (default 2e9 ns; 0 keeps the current value).  Flag
+ * PARASON_DEBUG_SKIP_FIRST_LOAD makes each attention CTA skip issuing its
+ * first KV load, so its consumers' wait can only expire: the kernel records
+ * PARASON_ETIMEOUT, lets its other copies land, and exits; the output is
+ * then undefined.  Used to test the timeout path without faulting the GPU.
+ */
+enum { PARASON_DEBUG_SKIP_FIRST_LOAD = 1u };
+parason_status parason_plan_set_debug(parason_plan plan, uint32_t flags, int64_t wait_limit_ns);
+
+/*
+ * Per-kernel timing for benchmarks.  After parason_plan_enable_timing(plan,
+ * n) every decode records CUDA events on its stream around its attention
+ * kernel and its merge kernel, for up to n calls.  parason_plan_read_timing
+ * synchronises on the last event and writes the durations (ms) of the
+ * recorded calls to attn_ms[] and merge_ms[] (either may be NULL), sets
+ * *count, and starts a new recording.  n = 0 disables timing.
+ */
+parason_status parason_plan_enable_timing(parason_plan plan, int32_t max_calls);
+parason_status parason_plan_read_timing(parason_plan plan, float *attn_ms, float *merge_ms,
+                                        int32_t capacity, int32_t *count);
+
+/* Number of kernel launches one parason_attn_decode call of this plan makes. */
+int32_t parason_plan_launches_per_decode(parason_plan plan);
+
+/* Library version, "major.minor.patch". */
+const char *parason_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PARASON_H */

@@ -1,0 +1,84 @@
+// internal.h -- types shared by the planner and the kernels of libparason.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "parason.h"
+
+namespace parason {
+
+// One unit of attention work: a tile of up to 64 query rows of one tree node
+// and one kv head, against one contiguous chunk of that node's pages.
+//
+// The rows of node n are its branches in DFS order times the g = H_q/H_kv
+// q heads of the kv head: node row r is branch dfs_leaf[leaf_lo + r / g],
+// q head kv_head * g + r % g.  The item writes the partial result (o, m, l)
+// of node row r to partial slot slot_base + r.
+struct WorkItem {
+    int32_t page_pos;    // index in page_ids of the chunk's first page
+    int32_t num_pages;   // pages in the chunk (>= 1)
+    int32_t last_valid;  // valid tokens in the chunk's last page (1..16)
+    int32_t leaf_lo;     // DFS position of the node's first branch
+    int32_t row0;        // first node row of this tile
+    int32_t nrows;       // rows in this tile (1..64)
+    int32_t kv_head;
+    int32_t slot_base;   // partial slot of node row 0 for (node, chunk, kv head)
+};
+static_assert(sizeof(WorkItem) == 32, "WorkItem is a 32-byte device record");
+
+constexpr int kPageSize = 16;
+constexpr int kMaxTileRows = 64;
+constexpr int kErrWords = 4;            // device error record: code, block, site, aux
+
+// Where a bounded wait gave up (error record word 2).
+enum WaitSite : int32_t {
+    kSiteConsumerFull = 1,
+    kSiteProducerEmpty = 2,
+};
+
+struct AttnArgs {
+    const WorkItem *items;
+    const int32_t *page_ids;
+    const int32_t *dfs_leaf;
+    const void *q;
+    float *part_o;          // [num_slots, head_dim]   sum_t 2^(x_t - m) v_t
+    float2 *part_ml;        // [num_slots]             (m, sum_t 2^(x_t - m))
+    const float *k_scale;   // FP8 mode
+    const float *v_scale;
+    int32_t *err;           // kErrWords ints
+    long long wait_limit_ns;
+    uint32_t debug_flags;
+    int32_t num_items;
+    int32_t num_q_heads;
+    int32_t num_kv_heads;
+    int32_t group;
+    float scale_log2;       // sm_scale * log2(e): x_t = scale_log2 * <q, k_t>
+};
+
+struct MergeArgs {
+    const int32_t *merge_ptr;   // [num_leaves + 1]
+    const int2 *merge_ent;      // (base, stride)
+    const float *part_o;
+    const float2 *part_ml;
+    void *out;
+    float *lse;
+    int32_t num_leaves;
+    int32_t num_q_heads;
+    int32_t group;
+};
+
+// Kernel launchers; each returns the launch's cudaError_t.
+cudaError_t launch_attn_bf16(const AttnArgs &a, const CUtensorMap &tmap_k,
+                             const CUtensorMap &tmap_v, int head_dim, cudaStream_t stream);
+cudaError_t launch_attn_fp8(const AttnArgs &a, const CUtensorMap &tmap_k,
+                            const CUtensorMap &tmap_v, int head_dim, cudaStream_t stream);
+cudaError_t launch_attn_fp32(const AttnArgs &a, const float *k_pages, const float *v_pages,
+                             int head_dim, cudaStream_t stream);
+cudaError_t launch_merge(const MergeArgs &a, int head_dim, int mode, cudaStream_t stream);
+cudaError_t launch_lse_merge(const void *o_a, const float *lse_a, const void *o_b,
+                             const float *lse_b, void *o_out, float *lse_out, int64_t rows,
+                             int head_dim, int mode, cudaStream_t stream);
+
+}  // namespace parason

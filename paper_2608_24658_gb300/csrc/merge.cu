@@ -1,0 +1,192 @@
+// merge.cu -- log-sum-exp merge kernels.
+//
+// tree merge: branch b's attention over its root->leaf KV is the softmax over
+// the union of the key sets of every (node, chunk) partial on its path, so
+//   M = max_i m_i,  L = sum_i l_i 2^(m_i - M),  o = sum_i o_i 2^(m_i - M) / L,
+//   lse = (M + log2 L) ln 2
+// with the partials in the log2 domain of the attention kernels.  Every
+// branch's result is needed because branch outputs are concatenated into the
+// context that follows (paper Fig. 1, Sec. 3.1).
+//
+// lse merge: two normalised results over disjoint key sets with natural-log
+// lse combine with weights e^{lse_a}, e^{lse_b}.
+#include <cuda_bf16.h>
+
+#include "internal.h"
+
+namespace parason {
+namespace {
+
+constexpr int kMergeThreads = 128;
+constexpr float kLn2 = 0.69314718055994530942f;
+
+template <int D>
+struct Vec;
+template <>
+struct Vec<128> {
+    static constexpr int N = 4;
+};
+template <>
+struct Vec<64> {
+    static constexpr int N = 2;
+};
+
+template <int N>
+__device__ __forceinline__ void load_f32(const float *p, float (&v)[N]) {
+    if constexpr (N == 4) {
+        const float4 t = *reinterpret_cast<const float4 *>(p);
+        v[0] = t.x, v[1] = t.y, v[2] = t.z, v[3] = t.w;
+    } else {
+        const float2 t = *reinterpret_cast<const float2 *>(p);
+        v[0] = t.x, v[1] = t.y;
+    }
+}
+
+template <int N>
+__device__ __forceinline__ void store_out(void *out, int64_t off, const float (&v)[N], bool bf16) {
+    if (bf16) {
+        __nv_bfloat16 *o = static_cast<__nv_bfloat16 *>(out) + off;
+        if constexpr (N == 4) {
+            __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]);
+            __nv_bfloat162 b = __floats2bfloat162_rn(v[2], v[3]);
+            uint2 u;
+            u.x = *reinterpret_cast<uint32_t *>(&a);
+            u.y = *reinterpret_cast<uint32_t *>(&b);
+            *reinterpret_cast<uint2 *>(o) = u;
+        } else {
+            *reinterpret_cast<__nv_bfloat162 *>(o) = __floats2bfloat162_rn(v[0], v[1]);
+        }
+    } else {
+        float *o = static_cast<float *>(out) + off;
+        if constexpr (N == 4)
+            *reinterpret_cast<float4 *>(o) = make_float4(v[0], v[1], v[2], v[3]);
+        else
+            *reinterpret_cast<float2 *>(o) = make_float2(v[0], v[1]);
+    }
+}
+
+template <int N>
+__device__ __forceinline__ void load_in(const void *in, int64_t off, float (&v)[N], bool bf16) {
+    if (bf16) {
+        const __nv_bfloat16 *p = static_cast<const __nv_bfloat16 *>(in) + off;
+        if constexpr (N == 4) {
+            const uint2 u = *reinterpret_cast<const uint2 *>(p);
+            const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162 *>(&u.x);
+            const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162 *>(&u.y);
+            v[0] = __low2float(a), v[1] = __high2float(a);
+            v[2] = __low2float(b), v[3] = __high2float(b);
+        } else {
+            const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162 *>(p);
+            v[0] = __low2float(a), v[1] = __high2float(a);
+        }
+    } else {
+        load_f32<N>(static_cast<const float *>(in) + off, v);
+    }
+}
+
+// one warp per (branch, q head)
+template <int D>
+__global__ void __launch_bounds__(kMergeThreads)
+    tree_merge_kernel(const MergeArgs a, bool out_bf16) {
+    constexpr int N = Vec<D>::N;
+    const int64_t w = (static_cast<int64_t>(blockIdx.x) * kMergeThreads + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (w >= static_cast<int64_t>(a.num_leaves) * a.num_q_heads) return;
+    const int b = static_cast<int>(w / a.num_q_heads), h = static_cast<int>(w % a.num_q_heads);
+    const int j = h / a.group, r = h % a.group;
+    const int e0 = a.merge_ptr[b], e1 = a.merge_ptr[b + 1];
+
+    float M = -INFINITY;
+    for (int e = e0; e < e1; ++e) {
+        const int2 ent = a.merge_ent[e];
+        const int64_t slot = static_cast<int64_t>(ent.x) + static_cast<int64_t>(j) * ent.y + r;
+        M = fmaxf(M, a.part_ml[slot].x);
+    }
+    float L = 0.f;
+    float acc[N];
+#pragma unroll
+    for (int i = 0; i < N; ++i) acc[i] = 0.f;
+    for (int e = e0; e < e1; ++e) {
+        const int2 ent = a.merge_ent[e];
+        const int64_t slot = static_cast<int64_t>(ent.x) + static_cast<int64_t>(j) * ent.y + r;
+        const float2 ml = a.part_ml[slot];
+        const float sc = exp2f(ml.x - M);
+        L += sc * ml.y;
+        float v[N];
+        load_f32<N>(a.part_o + slot * D + lane * N, v);
+#pragma unroll
+        for (int i = 0; i < N; ++i) acc[i] += sc * v[i];
+    }
+    const bool empty = !(L > 0.f);
+    const float inv = empty ? 0.f : 1.f / L;
+#pragma unroll
+    for (int i = 0; i < N; ++i) acc[i] *= inv;
+    const int64_t row = static_cast<int64_t>(b) * a.num_q_heads + h;
+    store_out<N>(a.out, row * D + lane * N, acc, out_bf16);
+    if (a.lse && lane == 0) a.lse[row] = empty ? -INFINITY : (M + log2f(L)) * kLn2;
+}
+
+template <int D>
+__global__ void __launch_bounds__(kMergeThreads)
+    lse_merge_kernel(const void *o_a, const float *lse_a, const void *o_b, const float *lse_b,
+                     void *o_out, float *lse_out, int64_t rows, bool bf16) {
+    constexpr int N = Vec<D>::N;
+    const int64_t row = (static_cast<int64_t>(blockIdx.x) * kMergeThreads + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (row >= rows) return;
+    const float la = lse_a[row], lb = lse_b[row];
+    float va[N], vb[N], o[N];
+    load_in<N>(o_a, row * D + lane * N, va, bf16);
+    load_in<N>(o_b, row * D + lane * N, vb, bf16);
+    float lse;
+    if (la == -INFINITY && lb == -INFINITY) {
+#pragma unroll
+        for (int i = 0; i < N; ++i) o[i] = 0.f;
+        lse = -INFINITY;
+    } else {
+        const float mx = fmaxf(la, lb);
+        const float wa = expf(la - mx), wb = expf(lb - mx);
+        const float inv = 1.f / (wa + wb);
+#pragma unroll
+        for (int i = 0; i < N; ++i) o[i] = (wa * va[i] + wb * vb[i]) * inv;
+        lse = mx + logf(wa + wb);
+    }
+    __syncwarp();   // every lane has read its inputs before any lane writes (aliasing)
+    store_out<N>(o_out, row * D + lane * N, o, bf16);
+    if (lane == 0) lse_out[row] = lse;
+}
+
+}  // namespace
+
+cudaError_t launch_merge(const MergeArgs &a, int head_dim, int mode, cudaStream_t stream) {
+    const int64_t warps = static_cast<int64_t>(a.num_leaves) * a.num_q_heads;
+    if (warps == 0) return cudaSuccess;
+    const int64_t blocks = (warps * 32 + kMergeThreads - 1) / kMergeThreads;
+    const bool bf16 = mode != PARASON_FP32;
+    if (head_dim == 128)
+        tree_merge_kernel<128><<<static_cast<unsigned>(blocks), kMergeThreads, 0, stream>>>(a, bf16);
+    else if (head_dim == 64)
+        tree_merge_kernel<64><<<static_cast<unsigned>(blocks), kMergeThreads, 0, stream>>>(a, bf16);
+    else
+        return cudaErrorNotSupported;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_lse_merge(const void *o_a, const float *lse_a, const void *o_b,
+                             const float *lse_b, void *o_out, float *lse_out, int64_t rows,
+                             int head_dim, int mode, cudaStream_t stream) {
+    if (rows <= 0) return cudaSuccess;
+    const int64_t blocks = (rows * 32 + kMergeThreads - 1) / kMergeThreads;
+    const bool bf16 = mode != PARASON_FP32;
+    if (head_dim == 128)
+        lse_merge_kernel<128><<<static_cast<unsigned>(blocks), kMergeThreads, 0, stream>>>(
+            o_a, lse_a, o_b, lse_b, o_out, lse_out, rows, bf16);
+    else if (head_dim == 64)
+        lse_merge_kernel<64><<<static_cast<unsigned>(blocks), kMergeThreads, 0, stream>>>(
+            o_a, lse_a, o_b, lse_b, o_out, lse_out, rows, bf16);
+    else
+        return cudaErrorNotSupported;
+    return cudaGetLastError();
+}
+
+}  // namespace parason

@@ -1,0 +1,684 @@
+// plan.cpp -- host planner and C ABI of libparason.
+//
+// The planner turns a fork tree (branches of Subtask/Trial parallel regions
+// decoded as independent workers, paper Sec. 3.4; nested regions per Fig. 4)
+// into work items for the attention kernel and merge lists for the merge
+// kernel:
+//
+//  * every node n that some branch reads is processed once per kv head, with
+//    all R_n = (#branches under n) * g query rows stacked into tiles of up to
+//    64 rows, so the node's KV is read from HBM once for all of them;
+//  * long nodes are cut into chunks of whole pages (split-K) so that the
+//    grid fills the GPU; each (node, chunk, kv head) has R_n partial slots;
+//  * branch b's result is the log-sum-exp merge of the partial slots of every
+//    node on its root->leaf path and every chunk of those nodes.
+#include <algorithm>
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <vector>
+
+#include <cudaTypedefs.h>
+
+#include "internal.h"
+
+using parason::WorkItem;
+
+namespace {
+
+constexpr int kMinChunkPages = 8;
+constexpr int kItemsPerSm = 4;          // ~2 resident CTAs x 2 waves
+constexpr int64_t kDefaultWaitNs = 2000000000LL;
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+int tile_rows_for(int32_t rows, int32_t mode) {
+    if (mode == PARASON_FP32) return 16;
+    if (rows <= 16) return 16;
+    if (rows <= 32) return 32;
+    return 64;
+}
+
+}  // namespace
+
+struct parason_plan_s {
+    parason_attn_config cfg{};
+    int32_t group = 1;
+    int32_t num_nodes = 0;
+    int32_t num_leaves = 0;
+    int64_t num_phys = 0;
+    int32_t num_sms = 152;
+    int32_t chunk_pages = kMinChunkPages;
+    std::vector<WorkItem> items;
+    std::vector<int32_t> page_ids;
+    std::vector<int32_t> dfs_leaf;
+    std::vector<int32_t> merge_ptr;
+    std::vector<int32_t> merge_ent;   // pairs (base, stride)
+    int64_t num_slots = 0;
+    int64_t unique_tokens = 0;
+    int64_t path_tokens = 0;
+
+    // device side
+    bool on_device = false;
+    int device = -1;
+    void *d_blob = nullptr;
+    WorkItem *d_items = nullptr;
+    int32_t *d_page_ids = nullptr;
+    int32_t *d_dfs_leaf = nullptr;
+    int32_t *d_merge_ptr = nullptr;
+    int2 *d_merge_ent = nullptr;
+    int32_t *d_err = nullptr;
+    uint32_t debug_flags = 0;
+    int64_t wait_limit_ns = kDefaultWaitNs;
+
+    // tensor maps of the last KV pools seen
+    std::mutex tm_mutex;
+    const void *tm_k_ptr = nullptr;
+    const void *tm_v_ptr = nullptr;
+    CUtensorMap tm_k{};
+    CUtensorMap tm_v{};
+
+    // timing
+    int32_t timing_cap = 0;
+    int32_t timing_n = 0;
+    std::vector<cudaEvent_t> events;   // 3 per recorded call
+};
+
+namespace {
+
+// ---------------------------------------------------------------------------
+// validation and work decomposition (no CUDA calls)
+// ---------------------------------------------------------------------------
+
+parason_status validate_config(const parason_attn_config *cfg) {
+    if (!cfg) return PARASON_EINVAL;
+    if (cfg->num_q_heads <= 0 || cfg->num_kv_heads <= 0) return PARASON_EINVAL;
+    if (cfg->num_q_heads % cfg->num_kv_heads != 0) return PARASON_EINVAL;
+    if (cfg->head_dim != 64 && cfg->head_dim != 128) return PARASON_EINVAL;
+    if (cfg->page_size != parason::kPageSize) return PARASON_EINVAL;
+    if (cfg->mode != PARASON_BF16 && cfg->mode != PARASON_FP32 &&
+        cfg->mode != PARASON_FP8_E4M3_KV)
+        return PARASON_EINVAL;
+    if (!(cfg->sm_scale >= 0.0f) || !std::isfinite(cfg->sm_scale)) return PARASON_EINVAL;
+    return PARASON_OK;
+}
+
+parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int32_t num_nodes,
+                          const int32_t *parent, const int32_t *node_len,
+                          const int32_t *node_page_ptr, const int32_t *page_ids,
+                          int32_t num_leaves, const int32_t *leaf_node,
+                          int64_t num_phys, int32_t num_sms) {
+    parason_status st = validate_config(cfg);
+    if (st != PARASON_OK) return st;
+    if (num_nodes < 0 || num_leaves < 0 || num_phys < 0) return PARASON_EINVAL;
+    if (num_nodes > 0 && (!parent || !node_len || !node_page_ptr)) return PARASON_EINVAL;
+    if (num_leaves > 0 && !leaf_node) return PARASON_EINVAL;
+    if (num_leaves > 0 && num_nodes == 0) return PARASON_EINVAL;
+
+    const int32_t H_kv = cfg->num_kv_heads;
+    const int32_t g = cfg->num_q_heads / H_kv;
+    p->cfg = *cfg;
+    p->group = g;
+    p->num_nodes = num_nodes;
+    p->num_leaves = num_leaves;
+    p->num_phys = num_phys;
+    p->num_sms = num_sms > 0 ? num_sms : 152;
+
+    // tree and page table
+    if (num_nodes > 0 && node_page_ptr[0] != 0) return PARASON_EINVAL;
+    for (int32_t i = 0; i < num_nodes; ++i) {
+        if (parent[i] < -1 || parent[i] >= i) return PARASON_EINVAL;
+        if (node_len[i] < 0) return PARASON_EINVAL;
+        const int64_t want = (static_cast<int64_t>(node_len[i]) + parason::kPageSize - 1) /
+                             parason::kPageSize;
+        if (static_cast<int64_t>(node_page_ptr[i + 1]) - node_page_ptr[i] != want)
+            return PARASON_EINVAL;
+    }
+    const int64_t total_pages = num_nodes > 0 ? node_page_ptr[num_nodes] : 0;
+    if (total_pages > 0 && !page_ids) return PARASON_EINVAL;
+    // rows addressed by the kernels: (page * H_kv + kv_head) * 16 must fit int32
+    if (num_phys > 0 &&
+        (num_phys * static_cast<int64_t>(H_kv) * parason::kPageSize) > INT32_MAX)
+        return PARASON_EUNSUPPORTED;
+    {
+        std::vector<int32_t> sorted(static_cast<size_t>(total_pages));
+        if (total_pages > 0)
+            std::memcpy(sorted.data(), page_ids, sizeof(int32_t) * static_cast<size_t>(total_pages));
+        std::sort(sorted.begin(), sorted.end());
+        for (int64_t i = 0; i < total_pages; ++i) {
+            if (sorted[i] < 0 || sorted[i] >= num_phys) return PARASON_EINVAL;
+            if (i > 0 && sorted[i] == sorted[i - 1]) return PARASON_EINVAL;
+        }
+    }
+    p->page_ids.resize(static_cast<size_t>(total_pages));
+    if (total_pages > 0)
+        std::memcpy(p->page_ids.data(), page_ids, sizeof(int32_t) * static_cast<size_t>(total_pages));
+
+    // branches: distinct, in range, childless
+    std::vector<int32_t> leaf_of_node(num_nodes, -1);
+    std::vector<int32_t> nchild(num_nodes, 0);
+    for (int32_t i = 0; i < num_nodes; ++i)
+        if (parent[i] >= 0) nchild[parent[i]]++;
+    for (int32_t b = 0; b < num_leaves; ++b) {
+        const int32_t n = leaf_node[b];
+        if (n < 0 || n >= num_nodes) return PARASON_EINVAL;
+        if (leaf_of_node[n] != -1) return PARASON_EINVAL;
+        if (nchild[n] != 0) return PARASON_EINVAL;
+        leaf_of_node[n] = b;
+    }
+
+    // branches under each node, and DFS order: parent[i] < i, so a reverse
+    // sweep accumulates subtree counts and a forward sweep lays the subtrees
+    // out contiguously (children in index order).
+    std::vector<int64_t> cnt(num_nodes, 0), lo(num_nodes, 0), next_child(num_nodes, 0);
+    for (int32_t i = 0; i < num_nodes; ++i) cnt[i] = leaf_of_node[i] >= 0 ? 1 : 0;
+    for (int32_t i = num_nodes - 1; i >= 0; --i)
+        if (parent[i] >= 0) cnt[parent[i]] += cnt[i];
+    int64_t root_cursor = 0;
+    for (int32_t i = 0; i < num_nodes; ++i) {
+        if (parent[i] < 0) {
+            lo[i] = root_cursor;
+            root_cursor += cnt[i];
+        } else {
+            lo[i] = lo[parent[i]] + next_child[parent[i]];
+            next_child[parent[i]] += cnt[i];
+        }
+    }
+    p->dfs_leaf.assign(num_leaves, -1);
+    for (int32_t b = 0; b < num_leaves; ++b) p->dfs_leaf[lo[leaf_node[b]]] = b;
+
+    // work decomposition
+    const int32_t mode = cfg->mode;
+    int64_t units = 0;
+    for (int32_t n = 0; n < num_nodes; ++n) {
+        if (cnt[n] == 0 || node_len[n] == 0) continue;
+        const int64_t R = cnt[n] * g;
+        const int rt = tile_rows_for(static_cast<int32_t>(std::min<int64_t>(R, 1 << 20)), mode);
+        units += static_cast<int64_t>(node_page_ptr[n + 1] - node_page_ptr[n]) * H_kv *
+                 ((R + rt - 1) / rt);
+        p->unique_tokens += node_len[n];
+    }
+    const int64_t target = static_cast<int64_t>(p->num_sms) * kItemsPerSm;
+    int64_t chunk = target > 0 ? (units + target - 1) / target : units;
+    chunk = std::max<int64_t>(chunk, kMinChunkPages);
+    p->chunk_pages = static_cast<int32_t>(std::min<int64_t>(chunk, INT32_MAX));
+
+    std::vector<int64_t> slot_first(num_nodes, -1);
+    std::vector<int32_t> nchunks(num_nodes, 0);
+    int64_t slots = 0;
+    std::vector<std::pair<int64_t, WorkItem>> keyed;
+    for (int32_t n = 0; n < num_nodes; ++n) {
+        if (cnt[n] == 0 || node_len[n] == 0) continue;
+        const int64_t R = cnt[n] * g;
+        if (R > INT32_MAX / 4) return PARASON_EUNSUPPORTED;
+        const int rt = tile_rows_for(static_cast<int32_t>(R), mode);
+        const int32_t P = node_page_ptr[n + 1] - node_page_ptr[n];
+        const int32_t nc = static_cast<int32_t>((P + chunk - 1) / chunk);
+        const int32_t base = P / nc, rem = P % nc;
+        nchunks[n] = nc;
+        slot_first[n] = slots;
+        int32_t pg = 0;
+        for (int32_t c = 0; c < nc; ++c) {
+            const int32_t np = base + (c < rem ? 1 : 0);
+            const bool has_last = (pg + np == P);
+            const int32_t last_valid =
+                has_last ? node_len[n] - (P - 1) * parason::kPageSize : parason::kPageSize;
+            for (int32_t j = 0; j < H_kv; ++j) {
+                const int64_t sb = slots + static_cast<int64_t>(c) * H_kv * R +
+                                   static_cast<int64_t>(j) * R;
+                for (int64_t r0 = 0; r0 < R; r0 += rt) {
+                    WorkItem it;
+                    it.page_pos = node_page_ptr[n] + pg;
+                    it.num_pages = np;
+                    it.last_valid = last_valid;
+                    it.leaf_lo = static_cast<int32_t>(lo[n]);
+                    it.row0 = static_cast<int32_t>(r0);
+                    it.nrows = static_cast<int32_t>(std::min<int64_t>(rt, R - r0));
+                    it.kv_head = j;
+                    if (sb > INT32_MAX) return PARASON_EUNSUPPORTED;
+                    it.slot_base = static_cast<int32_t>(sb);
+                    // cost: pages, weighted by the MMA work of wide tiles
+                    const int64_t rgc = it.nrows <= 16 ? 1 : (it.nrows <= 32 ? 2 : 4);
+                    keyed.emplace_back(static_cast<int64_t>(np) * (3 + rgc), it);
+                }
+            }
+            pg += np;
+        }
+        slots += static_cast<int64_t>(nc) * H_kv * R;
+        if (slots > INT32_MAX) return PARASON_EUNSUPPORTED;
+    }
+    // longest items first, so the tail of the grid is made of short ones
+    std::stable_sort(keyed.begin(), keyed.end(),
+                     [](const auto &a, const auto &b) { return a.first > b.first; });
+    p->items.clear();
+    p->items.reserve(keyed.size());
+    for (auto &kv : keyed) p->items.push_back(kv.second);
+    if (p->items.size() > static_cast<size_t>(INT32_MAX)) return PARASON_EUNSUPPORTED;
+    p->num_slots = slots;
+
+    // merge lists: every chunk of every node on the branch's path
+    p->merge_ptr.assign(num_leaves + 1, 0);
+    p->merge_ent.clear();
+    std::vector<int32_t> path;
+    for (int32_t b = 0; b < num_leaves; ++b) {
+        path.clear();
+        for (int32_t n = leaf_node[b]; n >= 0; n = parent[n]) path.push_back(n);
+        std::reverse(path.begin(), path.end());
+        const int64_t pos = lo[leaf_node[b]];
+        for (int32_t n : path) {
+            p->path_tokens += node_len[n];
+            if (nchunks[n] == 0) continue;
+            const int64_t R = cnt[n] * g;
+            for (int32_t c = 0; c < nchunks[n]; ++c) {
+                const int64_t base =
+                    slot_first[n] + static_cast<int64_t>(c) * H_kv * R + (pos - lo[n]) * g;
+                p->merge_ent.push_back(static_cast<int32_t>(base));
+                p->merge_ent.push_back(static_cast<int32_t>(R));
+            }
+        }
+        p->merge_ptr[b + 1] = static_cast<int32_t>(p->merge_ent.size() / 2);
+    }
+    return PARASON_OK;
+}
+
+// ---------------------------------------------------------------------------
+// device side
+// ---------------------------------------------------------------------------
+
+parason_status upload(parason_plan_s *p, cudaStream_t stream) {
+    if (cudaGetDevice(&p->device) != cudaSuccess) return PARASON_ECUDA;
+    const size_t n_items = p->items.size() * sizeof(WorkItem);
+    const size_t n_pages = p->page_ids.size() * sizeof(int32_t);
+    const size_t n_dfs = p->dfs_leaf.size() * sizeof(int32_t);
+    const size_t n_mptr = p->merge_ptr.size() * sizeof(int32_t);
+    const size_t n_ment = p->merge_ent.size() * sizeof(int32_t);
+    const size_t n_err = parason::kErrWords * sizeof(int32_t);
+    size_t off[6], total = 0;
+    const size_t sizes[6] = {n_items, n_pages, n_dfs, n_mptr, n_ment, n_err};
+    for (int i = 0; i < 6; ++i) {
+        off[i] = total;
+        total = align_up(total + std::max<size_t>(sizes[i], 4), kAlign);
+    }
+    if (cudaMalloc(&p->d_blob, total) != cudaSuccess) {
+        cudaGetLastError();
+        p->d_blob = nullptr;
+        return PARASON_ENOMEM;
+    }
+    char *base = static_cast<char *>(p->d_blob);
+    p->d_items = reinterpret_cast<WorkItem *>(base + off[0]);
+    p->d_page_ids = reinterpret_cast<int32_t *>(base + off[1]);
+    p->d_dfs_leaf = reinterpret_cast<int32_t *>(base + off[2]);
+    p->d_merge_ptr = reinterpret_cast<int32_t *>(base + off[3]);
+    p->d_merge_ent = reinterpret_cast<int2 *>(base + off[4]);
+    p->d_err = reinterpret_cast<int32_t *>(base + off[5]);
+    const void *src[5] = {p->items.data(), p->page_ids.data(), p->dfs_leaf.data(),
+                          p->merge_ptr.data(), p->merge_ent.data()};
+    for (int i = 0; i < 5; ++i) {
+        if (sizes[i] == 0) continue;
+        if (cudaMemcpyAsync(base + off[i], src[i], sizes[i], cudaMemcpyHostToDevice, stream) !=
+            cudaSuccess)
+            return PARASON_ECUDA;
+    }
+    if (cudaMemsetAsync(p->d_err, 0, n_err, stream) != cudaSuccess) return PARASON_ECUDA;
+    // the host vectors are pageable: make sure the copies have consumed them
+    // before the caller can free its own arrays (ours stay alive anyway)
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return PARASON_ECUDA;
+    p->on_device = true;
+    return PARASON_OK;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+    });
+    return fn;
+}
+
+// KV pool [P, H_kv, 16, d] seen as rows of 128-byte segments:
+//   dim0 = 128 bytes of one segment (64 bf16 or 128 e4m3), dim1 = segment in
+//   the token row, dim2 = token row (page * H_kv + kv_head) * 16 + slot.
+// One box {seg, nseg, 16} is one page of one kv head; 128-byte swizzle.
+parason_status encode_kv_map(CUtensorMap *map, const void *pages, int64_t num_phys,
+                             int32_t H_kv, int32_t head_dim, int32_t mode) {
+    auto fn = encode_fn();
+    if (!fn) return PARASON_ECUDA;
+    const int esize = (mode == PARASON_FP8_E4M3_KV) ? 1 : 2;
+    const CUtensorMapDataType dt =
+        (mode == PARASON_FP8_E4M3_KV) ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    const int row_bytes = head_dim * esize;
+    if (row_bytes % 128 != 0) return PARASON_EUNSUPPORTED;
+    const int nseg = row_bytes / 128;
+    const int seg_elems = 128 / esize;
+    const cuuint64_t rows = static_cast<cuuint64_t>(num_phys) * H_kv * parason::kPageSize;
+    cuuint64_t dims[3] = {static_cast<cuuint64_t>(seg_elems), static_cast<cuuint64_t>(nseg), rows};
+    cuuint64_t strides[2] = {128, static_cast<cuuint64_t>(row_bytes)};
+    cuuint32_t box[3] = {static_cast<cuuint32_t>(seg_elems), static_cast<cuuint32_t>(nseg),
+                         static_cast<cuuint32_t>(parason::kPageSize)};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = fn(map, dt, 3, const_cast<void *>(pages), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? PARASON_OK : PARASON_ECUDA;
+}
+
+parason_status record_event(parason_plan_s *p, int which, cudaStream_t stream) {
+    if (p->timing_cap <= 0 || p->timing_n >= p->timing_cap) return PARASON_OK;
+    cudaEvent_t ev = p->events[3 * p->timing_n + which];
+    return cudaEventRecord(ev, stream) == cudaSuccess ? PARASON_OK : PARASON_ECUDA;
+}
+
+void free_events(parason_plan_s *p) {
+    for (auto e : p->events)
+        if (e) cudaEventDestroy(e);
+    p->events.clear();
+    p->timing_cap = p->timing_n = 0;
+}
+
+}  // namespace
+
+extern "C" {
+
+parason_status parason_attn_plan_host(const parason_attn_config *cfg, int32_t num_nodes,
+                                      const int32_t *parent, const int32_t *node_len,
+                                      const int32_t *node_page_ptr, const int32_t *page_ids,
+                                      int32_t num_leaves, const int32_t *leaf_node,
+                                      int64_t num_physical_pages, int32_t num_sms,
+                                      parason_plan *out) {
+    if (!out) return PARASON_EINVAL;
+    *out = nullptr;
+    auto *p = new (std::nothrow) parason_plan_s();
+    if (!p) return PARASON_ENOMEM;
+    parason_status st;
+    try {
+        st = build_host(p, cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves,
+                        leaf_node, num_physical_pages, num_sms);
+    } catch (const std::bad_alloc &) {
+        st = PARASON_ENOMEM;
+    }
+    if (st != PARASON_OK) {
+        delete p;
+        return st;
+    }
+    *out = p;
+    return PARASON_OK;
+}
+
+parason_status parason_attn_plan(const parason_attn_config *cfg, int32_t num_nodes,
+                                 const int32_t *parent, const int32_t *node_len,
+                                 const int32_t *node_page_ptr, const int32_t *page_ids,
+                                 int32_t num_leaves, const int32_t *leaf_node,
+                                 int64_t num_physical_pages, parason_stream_t stream,
+                                 parason_plan *out) {
+    if (!out) return PARASON_EINVAL;
+    *out = nullptr;
+    // validate before touching CUDA, so malformed input is EINVAL everywhere
+    parason_status st = validate_config(cfg);
+    if (st != PARASON_OK) return st;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+        // still report malformed trees as EINVAL on machines without a GPU
+        parason_plan probe = nullptr;
+        st = parason_attn_plan_host(cfg, num_nodes, parent, node_len, node_page_ptr, page_ids,
+                                    num_leaves, leaf_node, num_physical_pages, 152, &probe);
+        parason_plan_destroy(probe);
+        cudaGetLastError();
+        return st != PARASON_OK ? st : PARASON_ECUDA;
+    }
+    parason_plan p = nullptr;
+    st = parason_attn_plan_host(cfg, num_nodes, parent, node_len, node_page_ptr, page_ids,
+                                num_leaves, leaf_node, num_physical_pages, sms, &p);
+    if (st != PARASON_OK) return st;
+    st = upload(p, reinterpret_cast<cudaStream_t>(stream));
+    if (st != PARASON_OK) {
+        parason_plan_destroy(p);
+        return st;
+    }
+    *out = p;
+    return PARASON_OK;
+}
+
+size_t parason_plan_workspace_bytes(parason_plan p) {
+    if (!p) return 0;
+    const size_t o = align_up(static_cast<size_t>(p->num_slots) * p->cfg.head_dim * sizeof(float), kAlign);
+    const size_t ml = align_up(static_cast<size_t>(p->num_slots) * sizeof(float2), kAlign);
+    return o + ml;
+}
+
+parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_pages,
+                                   const void *v_pages, const float *k_scale,
+                                   const float *v_scale, void *out, float *lse,
+                                   void *workspace, size_t workspace_bytes,
+                                   parason_stream_t stream_) {
+    if (!p || !p->on_device) return PARASON_EINVAL;
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    if (p->num_leaves == 0) return PARASON_OK;
+    if (!q || !out) return PARASON_EINVAL;
+    const bool has_items = !p->items.empty();
+    if (has_items) {
+        if (!k_pages || !v_pages || !workspace) return PARASON_EINVAL;
+        if (workspace_bytes < parason_plan_workspace_bytes(p)) return PARASON_EINVAL;
+        if (reinterpret_cast<uintptr_t>(workspace) % kAlign) return PARASON_EINVAL;
+        if (reinterpret_cast<uintptr_t>(k_pages) % 16 || reinterpret_cast<uintptr_t>(v_pages) % 16)
+            return PARASON_EINVAL;
+        if (p->cfg.mode == PARASON_FP8_E4M3_KV && (!k_scale || !v_scale)) return PARASON_EINVAL;
+    }
+    if (reinterpret_cast<uintptr_t>(q) % 16 || reinterpret_cast<uintptr_t>(out) % 16)
+        return PARASON_EINVAL;
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) return PARASON_ECUDA;
+    if (dev != p->device) return PARASON_EINVAL;
+
+    const int d = p->cfg.head_dim;
+    float *part_o = static_cast<float *>(workspace);
+    float2 *part_ml = reinterpret_cast<float2 *>(
+        static_cast<char *>(workspace) +
+        align_up(static_cast<size_t>(p->num_slots) * d * sizeof(float), kAlign));
+    const float sm_scale = p->cfg.sm_scale > 0.0f ? p->cfg.sm_scale : 1.0f / std::sqrt(static_cast<float>(d));
+
+    parason_status st = record_event(p, 0, stream);
+    if (st != PARASON_OK) return st;
+    if (has_items) {
+        parason::AttnArgs a{};
+        a.items = p->d_items;
+        a.page_ids = p->d_page_ids;
+        a.dfs_leaf = p->d_dfs_leaf;
+        a.q = q;
+        a.part_o = part_o;
+        a.part_ml = part_ml;
+        a.k_scale = k_scale;
+        a.v_scale = v_scale;
+        a.err = p->d_err;
+        a.wait_limit_ns = p->wait_limit_ns;
+        a.debug_flags = p->debug_flags;
+        a.num_items = static_cast<int32_t>(p->items.size());
+        a.num_q_heads = p->cfg.num_q_heads;
+        a.num_kv_heads = p->cfg.num_kv_heads;
+        a.group = p->group;
+        a.scale_log2 = sm_scale * 1.4426950408889634f;
+        cudaError_t e;
+        if (p->cfg.mode == PARASON_FP32) {
+            e = parason::launch_attn_fp32(a, static_cast<const float *>(k_pages),
+                                          static_cast<const float *>(v_pages), d, stream);
+        } else {
+            CUtensorMap tk, tv;
+            {
+                std::lock_guard<std::mutex> lock(p->tm_mutex);
+                if (p->tm_k_ptr != k_pages) {
+                    st = encode_kv_map(&p->tm_k, k_pages, p->num_phys, p->cfg.num_kv_heads, d, p->cfg.mode);
+                    if (st != PARASON_OK) return st;
+                    p->tm_k_ptr = k_pages;
+                }
+                if (p->tm_v_ptr != v_pages) {
+                    st = encode_kv_map(&p->tm_v, v_pages, p->num_phys, p->cfg.num_kv_heads, d, p->cfg.mode);
+                    if (st != PARASON_OK) return st;
+                    p->tm_v_ptr = v_pages;
+                }
+                tk = p->tm_k;
+                tv = p->tm_v;
+            }
+            e = (p->cfg.mode == PARASON_BF16) ? parason::launch_attn_bf16(a, tk, tv, d, stream)
+                                              : parason::launch_attn_fp8(a, tk, tv, d, stream);
+        }
+        if (e == cudaErrorNotSupported) return PARASON_EUNSUPPORTED;
+        if (e != cudaSuccess) return PARASON_ECUDA;
+    }
+    st = record_event(p, 1, stream);
+    if (st != PARASON_OK) return st;
+    parason::MergeArgs m{};
+    m.merge_ptr = p->d_merge_ptr;
+    m.merge_ent = p->d_merge_ent;
+    m.part_o = part_o;
+    m.part_ml = part_ml;
+    m.out = out;
+    m.lse = lse;
+    m.num_leaves = p->num_leaves;
+    m.num_q_heads = p->cfg.num_q_heads;
+    m.group = p->group;
+    if (parason::launch_merge(m, d, p->cfg.mode, stream) != cudaSuccess) return PARASON_ECUDA;
+    st = record_event(p, 2, stream);
+    if (st != PARASON_OK) return st;
+    if (p->timing_cap > 0 && p->timing_n < p->timing_cap) p->timing_n++;
+    return PARASON_OK;
+}
+
+parason_status parason_lse_merge(const void *o_a, const float *lse_a, const void *o_b,
+                                 const float *lse_b, void *o_out, float *lse_out, int64_t rows,
+                                 int32_t head_dim, int32_t mode, parason_stream_t stream) {
+    if (rows < 0 || (head_dim != 64 && head_dim != 128)) return PARASON_EINVAL;
+    if (mode != PARASON_BF16 && mode != PARASON_FP32 && mode != PARASON_FP8_E4M3_KV)
+        return PARASON_EINVAL;
+    if (rows == 0) return PARASON_OK;
+    if (!o_a || !lse_a || !o_b || !lse_b || !o_out || !lse_out) return PARASON_EINVAL;
+    const uintptr_t mis = reinterpret_cast<uintptr_t>(o_a) | reinterpret_cast<uintptr_t>(o_b) |
+                          reinterpret_cast<uintptr_t>(o_out);
+    if (mis % 16) return PARASON_EINVAL;
+    cudaError_t e = parason::launch_lse_merge(o_a, lse_a, o_b, lse_b, o_out, lse_out, rows, head_dim,
+                                              mode, reinterpret_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? PARASON_OK : PARASON_ECUDA;
+}
+
+parason_status parason_plan_check(parason_plan p, parason_stream_t stream) {
+    if (!p || !p->on_device) return PARASON_EINVAL;
+    if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return PARASON_ECUDA;
+    int32_t rec[parason::kErrWords] = {0, 0, 0, 0};
+    if (cudaMemcpy(rec, p->d_err, sizeof rec, cudaMemcpyDeviceToHost) != cudaSuccess)
+        return PARASON_ECUDA;
+    if (rec[0] != 0) {
+        if (cudaMemset(p->d_err, 0, sizeof rec) != cudaSuccess) return PARASON_ECUDA;
+        return rec[0] == PARASON_ETIMEOUT ? PARASON_ETIMEOUT : PARASON_ECUDA;
+    }
+    return PARASON_OK;
+}
+
+void parason_plan_destroy(parason_plan p) {
+    if (!p) return;
+    free_events(p);
+    if (p->d_blob) cudaFree(p->d_blob);
+    delete p;
+}
+
+const char *parason_status_string(parason_status s) {
+    switch (s) {
+    case PARASON_OK: return "ok";
+    case PARASON_EINVAL: return "invalid argument";
+    case PARASON_ENOMEM: return "out of memory";
+    case PARASON_ECUDA: return "CUDA error";
+    case PARASON_ETIMEOUT: return "device wait timed out";
+    case PARASON_EUNSUPPORTED: return "unsupported";
+    }
+    return "unknown status";
+}
+
+parason_status parason_plan_get_info(parason_plan p, parason_plan_info *info) {
+    if (!p || !info) return PARASON_EINVAL;
+    info->num_items = static_cast<int32_t>(p->items.size());
+    info->num_leaves = p->num_leaves;
+    info->num_merge_entries = static_cast<int32_t>(p->merge_ent.size() / 2);
+    info->chunk_pages = p->chunk_pages;
+    info->num_slots = p->num_slots;
+    info->unique_tokens = p->unique_tokens;
+    info->path_tokens = p->path_tokens;
+    info->num_sms = p->num_sms;
+    info->on_device = p->on_device ? 1 : 0;
+    return PARASON_OK;
+}
+
+parason_status parason_plan_export(parason_plan p, int32_t table, void *dst, size_t bytes) {
+    if (!p) return PARASON_EINVAL;
+    const void *src = nullptr;
+    size_t n = 0;
+    switch (table) {
+    case PARASON_TABLE_ITEMS: src = p->items.data(); n = p->items.size() * sizeof(WorkItem); break;
+    case PARASON_TABLE_DFS_LEAVES: src = p->dfs_leaf.data(); n = p->dfs_leaf.size() * 4; break;
+    case PARASON_TABLE_MERGE_PTR: src = p->merge_ptr.data(); n = p->merge_ptr.size() * 4; break;
+    case PARASON_TABLE_MERGE: src = p->merge_ent.data(); n = p->merge_ent.size() * 4; break;
+    default: return PARASON_EINVAL;
+    }
+    if (bytes < n || (n > 0 && !dst)) return PARASON_EINVAL;
+    if (n) std::memcpy(dst, src, n);
+    return PARASON_OK;
+}
+
+parason_status parason_plan_set_debug(parason_plan p, uint32_t flags, int64_t wait_limit_ns) {
+    if (!p || wait_limit_ns < 0) return PARASON_EINVAL;
+    p->debug_flags = flags;
+    if (wait_limit_ns > 0) p->wait_limit_ns = wait_limit_ns;
+    return PARASON_OK;
+}
+
+parason_status parason_plan_enable_timing(parason_plan p, int32_t max_calls) {
+    if (!p || max_calls < 0 || !p->on_device) return PARASON_EINVAL;
+    free_events(p);
+    if (max_calls == 0) return PARASON_OK;
+    p->events.assign(static_cast<size_t>(max_calls) * 3, nullptr);
+    for (auto &e : p->events) {
+        if (cudaEventCreate(&e) != cudaSuccess) {
+            e = nullptr;
+            free_events(p);
+            return PARASON_ECUDA;
+        }
+    }
+    p->timing_cap = max_calls;
+    p->timing_n = 0;
+    return PARASON_OK;
+}
+
+parason_status parason_plan_read_timing(parason_plan p, float *attn_ms, float *merge_ms,
+                                        int32_t capacity, int32_t *count) {
+    if (!p || !count || capacity < 0) return PARASON_EINVAL;
+    const int32_t n = std::min(p->timing_n, capacity);
+    if (p->timing_n > 0 && cudaEventSynchronize(p->events[3 * (p->timing_n - 1) + 2]) != cudaSuccess)
+        return PARASON_ECUDA;
+    for (int32_t i = 0; i < n; ++i) {
+        float a = 0.f, m = 0.f;
+        if (cudaEventElapsedTime(&a, p->events[3 * i], p->events[3 * i + 1]) != cudaSuccess ||
+            cudaEventElapsedTime(&m, p->events[3 * i + 1], p->events[3 * i + 2]) != cudaSuccess)
+            return PARASON_ECUDA;
+        if (attn_ms) attn_ms[i] = a;
+        if (merge_ms) merge_ms[i] = m;
+    }
+    *count = n;
+    p->timing_n = 0;
+    return PARASON_OK;
+}
+
+int32_t parason_plan_launches_per_decode(parason_plan p) {
+    if (!p || p->num_leaves == 0) return 0;
+    return (p->items.empty() ? 0 : 1) + 1;
+}
+
+const char *parason_version(void) { return "0.1.0"; }
+
+}  // extern "C"

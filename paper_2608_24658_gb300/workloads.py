@@ -192,14 +192,25 @@ def build_tree(name: str, parent, node_len, leaf_node, *, num_q_heads: int,
                rng: Optional[np.random.Generator] = None, permute_pages: bool = False,
                extra_pages: int = 0, q_std: float = 1.0, device="cpu",
                tail_value: Optional[float] = None, sm_scale: float = 0.0,
-               meta: Optional[dict] = None) -> ForkTree:
-    """Assemble a workload from a tree shape; draws pages, then q, K, V."""
+               meta: Optional[dict] = None, values: bool = True) -> ForkTree:
+    """Assemble a workload from a tree shape; draws pages, then q, K, V.
+
+    ``values=False`` stops after the page table (tensors are left empty): the
+    tree shape of a multi-GB workload without its q/K/V.
+    """
     if rng is None:
         rng = np.random.default_rng(seed)
     parent = np.asarray(parent, dtype=np.int32)
     node_len = np.asarray(node_len, dtype=np.int32)
     leaf_node = np.asarray(leaf_node, dtype=np.int32)
     ptr, pages, nphys = assign_pages(node_len, rng, permute_pages, PAGE_SIZE, extra_pages)
+    if not values:
+        empty = torch.empty(0)
+        return ForkTree(name=name, num_q_heads=num_q_heads, num_kv_heads=num_kv_heads,
+                        head_dim=head_dim, mode=mode, parent=parent, node_len=node_len,
+                        node_page_ptr=ptr, page_ids=pages, leaf_node=leaf_node,
+                        num_physical_pages=nphys, q=empty, k_pages=empty, v_pages=empty,
+                        sm_scale=sm_scale, meta=dict(meta or {}))
     gen = torch.Generator(device=device)
     gen.manual_seed(int(rng.integers(0, 2**62)))
     L = len(leaf_node)

@@ -1,0 +1,161 @@
+"""Planner work lists, checked bit-exactly against the tree (CPU only).
+
+The checks recompute from the tree alone what the work items and merge lists
+must cover, and compare exactly:
+  * every (node, kv head, node row) of every node some branch reads is
+    computed over every page of that node exactly once;
+  * every item row maps to a (branch, q head) whose path contains the node;
+  * partial slots written by items are unique and fill [0, num_slots);
+  * branch b / q head h merges exactly the slots written for its row by the
+    items of the nodes on its path;
+  * last-page token counts match the node lengths.
+"""
+import collections
+
+import numpy as np
+import pytest
+
+from paper_2608_24658_gb300 import _lib, build
+from paper_2608_24658_gb300.api import Plan
+from paper_2608_24658_gb300 import workloads as W
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    build.build()
+
+
+def node_of_page_pos(tree):
+    """node owning each position of page_ids."""
+    owner = np.full(int(tree.node_page_ptr[-1]), -1, dtype=np.int64)
+    for n in range(tree.num_nodes):
+        owner[tree.node_page_ptr[n]:tree.node_page_ptr[n + 1]] = n
+    return owner
+
+
+def verify_plan(tree, plan):
+    g = tree.group
+    H_kv = tree.num_kv_heads
+    info = plan.info()
+    items = plan.export(_lib.TABLE_ITEMS)
+    dfs = plan.export(_lib.TABLE_DFS_LEAVES)
+    mptr = plan.export(_lib.TABLE_MERGE_PTR)
+    ment = plan.export(_lib.TABLE_MERGE)
+    assert sorted(dfs.tolist()) == list(range(tree.num_leaves))
+    owner = node_of_page_pos(tree)
+    paths = [set(tree.path(b)) for b in range(tree.num_leaves)]
+    under = collections.defaultdict(set)
+    for b, p in enumerate(paths):
+        for n in p:
+            under[n].add(b)
+
+    # coverage[(node, kv_head, branch, r)] -> list of page positions covered
+    coverage = collections.defaultdict(list)
+    written = {}                                 # slot -> (node, kvh, branch, r)
+    slots_of = collections.defaultdict(list)     # (branch, h) -> slots written for it
+    for it in items:
+        page_pos, npg, last_valid, leaf_lo, row0, nrows, kvh, slot_base = (int(x) for x in it)
+        assert npg >= 1 and 1 <= nrows <= 64 and 0 <= kvh < H_kv
+        n = int(owner[page_pos])
+        assert n >= 0 and owner[page_pos + npg - 1] == n, "chunk crosses a node boundary"
+        P = tree.node_page_ptr[n + 1] - tree.node_page_ptr[n]
+        ends_node = page_pos + npg == tree.node_page_ptr[n + 1]
+        want_last = int(tree.node_len[n]) - 16 * (P - 1) if ends_node else 16
+        assert last_valid == want_last
+        for row in range(row0, row0 + nrows):
+            b = int(dfs[leaf_lo + row // g])
+            r = row % g
+            assert n in paths[b], "item row belongs to a branch outside the node's subtree"
+            coverage[(n, kvh, b, r)].extend(range(page_pos, page_pos + npg))
+            slot = slot_base + row
+            assert slot not in written, "partial slot written twice"
+            written[slot] = (n, kvh, b, r)
+            slots_of[(b, kvh * g + r)].append(slot)
+    assert sorted(written) == list(range(info["num_slots"]))
+    # every node some branch reads, every kv head, every row: all pages exactly once
+    for n, bs in under.items():
+        if tree.node_len[n] == 0:
+            continue
+        pages = list(range(tree.node_page_ptr[n], tree.node_page_ptr[n + 1]))
+        for kvh in range(H_kv):
+            for b in bs:
+                for r in range(g):
+                    assert sorted(coverage[(n, kvh, b, r)]) == pages
+    # nothing computed for nodes no branch reads
+    assert all(k[0] in under and tree.node_len[k[0]] > 0 for k in coverage)
+    # merge lists: exactly the slots written for (branch, head)
+    assert mptr[0] == 0 and mptr[-1] == len(ment)
+    for b in range(tree.num_leaves):
+        for h in range(tree.num_q_heads):
+            j, r = divmod(h, g)
+            got = sorted(int(base) + j * int(stride) + r for base, stride in ment[mptr[b]:mptr[b + 1]])
+            assert got == sorted(slots_of[(b, h)]), (b, h)
+    assert info["unique_tokens"] == tree.unique_tokens()
+    assert info["path_tokens"] == tree.path_tokens()
+    return info
+
+
+CASES = {
+    "figure3": lambda: W.figure3_tree(values=False),
+    "tiny_fork": lambda: W.make_config(1, values=False),
+    "llama3_trials": lambda: W.make_config(2, values=False),
+    "two_level": lambda: W.make_config(3, values=False),
+    "random_forest_0": lambda: W.random_tree(0, values=False),
+    "random_forest_1": lambda: W.random_tree(1, depth=4, fanout=(0, 3), values=False),
+    "random_forest_g1": lambda: W.random_tree(2, h_q=4, h_kv=4, values=False),
+    "random_forest_g16": lambda: W.random_tree(3, h_q=32, h_kv=2, values=False),
+    "random_forest_g6": lambda: W.random_tree(4, h_q=12, h_kv=2, values=False),
+    "chain_with_empty": lambda: W.build_tree("chain", [-1, 0, 1, 2], [17, 0, 33, 5], [3],
+                                             num_q_heads=6, num_kv_heads=3, head_dim=64,
+                                             values=False),
+    "empty_path": lambda: W.build_tree("empty", [-1, 0, 0], [0, 0, 5], [1, 2], num_q_heads=4,
+                                       num_kv_heads=2, head_dim=64, values=False),
+    "unused_branch_node": lambda: W.build_tree("unused", [-1, 0, 0, 1], [40, 20, 30, 9], [3],
+                                               num_q_heads=4, num_kv_heads=2, head_dim=64,
+                                               values=False),
+    "wide_node": lambda: W.build_tree("wide", [-1] + [0] * 40, [700] + [3] * 40,
+                                      list(range(1, 41)), num_q_heads=16, num_kv_heads=2,
+                                      head_dim=128, values=False),
+}
+
+
+@pytest.mark.parametrize("name", sorted(CASES))
+@pytest.mark.parametrize("mode", ["bf16", "fp32"])
+def test_plan_covers_tree_exactly(name, mode):
+    tree = CASES[name]()
+    tree.mode = mode
+    with Plan.for_tree(tree, host_only=True) as plan:
+        verify_plan(tree, plan)
+
+
+@pytest.mark.parametrize("idx", [4, 5])
+def test_plan_large_configs(idx):
+    tree = W.make_config(idx, values=False)
+    with Plan.for_tree(tree, host_only=True) as plan:
+        info = plan.info()
+        items = plan.export(_lib.TABLE_ITEMS)
+        # partial traffic stays a small fraction of the unique KV bytes
+        kv_bytes = info["unique_tokens"] * 2 * tree.num_kv_heads * tree.head_dim * 2
+        part_bytes = info["num_slots"] * (tree.head_dim * 4 + 8) * 2
+        assert part_bytes < 0.05 * kv_bytes, part_bytes / kv_bytes
+        assert len(items) >= 152
+        # pages of all items of one (kv head, first tile) sum to the unique pages
+        one = items[(items[:, 6] == 0) & (items[:, 4] == 0)]
+        assert one[:, 1].sum() == sum(
+            tree.node_page_ptr[n + 1] - tree.node_page_ptr[n]
+            for n in range(tree.num_nodes) if tree.node_len[n] > 0)
+
+
+def test_plan_deterministic():
+    tree = W.make_config(3, values=False)
+    with Plan.for_tree(tree, host_only=True) as a, Plan.for_tree(tree, host_only=True) as b:
+        for t in range(4):
+            assert np.array_equal(a.export(t), b.export(t))
+
+
+def test_plan_sm_count_changes_split_only():
+    tree = W.make_config(2, values=False)
+    for sms in (1, 16, 152, 1000):
+        with Plan.for_tree(tree, host_only=True, num_sms=sms) as plan:
+            assert plan.info()["num_sms"] == sms
+            verify_plan(tree, plan)
