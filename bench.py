@@ -244,6 +244,7 @@ def run_gpu(args):
     build.build()
     tree = make_workload(args, device=dev)
     plan = Plan.for_tree(tree)
+    plan_info = plan.info()
     ws = plan.workspace(dev)
     out = torch.empty_like(tree.q)
     lse = torch.empty(tree.q.shape[:2], dtype=torch.float32, device=dev)
@@ -366,6 +367,9 @@ def run_gpu(args):
         "roofline": roofline, "cpu_baseline": cpu, "clocks": clocks,
         "wall_s_timed_region": wall,
         "algorithmic": {"bytes_per_step": ab["step"], "flops_per_step": algorithmic_flops(tree)},
+        "plan": {k: v for k, v in plan_info.items()
+                 if k in ("num_items", "num_ctas", "ctas_per_sm", "chunk_pages", "num_slots",
+                          "num_merge_entries")},
     }
     print(json.dumps(line), flush=True)
     plan.close()

@@ -199,6 +199,9 @@ typedef struct {
     int64_t path_tokens;        /* sum over branches of their path tokens   */
     int32_t num_sms;            /* SM count the split targeted              */
     int32_t on_device;          /* 1 if decode can run on this plan         */
+    int32_t num_ctas;           /* CTAs of the persistent attention kernel  */
+    int32_t num_empty_leaves;   /* branches whose whole path is empty       */
+    int32_t ctas_per_sm;        /* resident CTAs per SM the grid assumes    */
 } parason_plan_info;
 
 parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info);
@@ -215,13 +218,22 @@ parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info)
  *   PARASON_TABLE_MERGE      int32 [num_merge_entries][2]: (base, stride);
  *                            q head h = j*g + r of the branch reads the
  *                            partial slot base + j*stride + r
+ *   PARASON_TABLE_SCHEDULE_PTR int32 [num_ctas + 1]: CSR of the persistent
+ *                            kernel's per-CTA item lists
+ *   PARASON_TABLE_SCHEDULE   int32 [num_items]: item indices, CTA by CTA
+ *   PARASON_TABLE_TARGETS    int32 [num_leaves][H_kv]: items whose rows
+ *                            include (branch, kv head); the merge of that
+ *                            pair runs when the last of them finishes
  * Returns PARASON_EINVAL if `bytes` is smaller than the table.
  */
 enum {
     PARASON_TABLE_ITEMS = 0,
     PARASON_TABLE_DFS_LEAVES = 1,
     PARASON_TABLE_MERGE_PTR = 2,
-    PARASON_TABLE_MERGE = 3
+    PARASON_TABLE_MERGE = 3,
+    PARASON_TABLE_SCHEDULE_PTR = 4,
+    PARASON_TABLE_SCHEDULE = 5,
+    PARASON_TABLE_TARGETS = 6
 };
 parason_status parason_plan_export(parason_plan plan, int32_t table, void *dst, size_t bytes);
 

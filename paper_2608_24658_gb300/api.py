@@ -124,7 +124,10 @@ class Plan:
         shape = {_lib.TABLE_ITEMS: (inf["num_items"], 8),
                  _lib.TABLE_DFS_LEAVES: (inf["num_leaves"],),
                  _lib.TABLE_MERGE_PTR: (inf["num_leaves"] + 1,),
-                 _lib.TABLE_MERGE: (inf["num_merge_entries"], 2)}[table]
+                 _lib.TABLE_MERGE: (inf["num_merge_entries"], 2),
+                 _lib.TABLE_SCHEDULE_PTR: (inf["num_ctas"] + 1,),
+                 _lib.TABLE_SCHEDULE: (inf["num_items"],),
+                 _lib.TABLE_TARGETS: (inf["num_leaves"], self.num_kv_heads)}[table]
         buf = np.zeros(shape, dtype=np.int32)
         check(_lib.load().parason_plan_export(self.handle, table, _ptr(buf), buf.nbytes),
               "plan_export")

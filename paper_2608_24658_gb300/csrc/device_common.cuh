@@ -67,6 +67,28 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
     }
 }
 
+// Named barrier over the first NTHREADS threads that also ORs a predicate:
+// every participant gets the same answer, so decisions taken on it (leave a
+// loop, skip an epilogue) are uniform and no warp is left at a later barrier.
+template <int NTHREADS>
+__device__ __forceinline__ bool bar_sync_or(int id, bool pred) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.or.pred q, %2, %3, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"(static_cast<uint32_t>(pred)), "r"(id), "n"(NTHREADS)
+        : "memory");
+    return r != 0;
+}
+
+template <int NTHREADS>
+__device__ __forceinline__ void bar_sync(int id) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "n"(NTHREADS) : "memory");
+}
+
 // Record the first device-side failure of a launch: code, block, site.
 __device__ __forceinline__ void record_error(int32_t *err, int32_t code, int32_t site) {
     if (atomicCAS(err, 0, code) == 0) {

@@ -55,6 +55,24 @@ struct AttnArgs {
     int32_t num_kv_heads;
     int32_t group;
     float scale_log2;       // sm_scale * log2(e): x_t = scale_log2 * <q, k_t>
+
+    // persistent schedule: CTA c runs items cta_items[cta_ptr[c] .. cta_ptr[c+1])
+    const int32_t *cta_ptr;
+    const int32_t *cta_items;
+    int32_t num_ctas;
+
+    // fused merge: the CTA whose item brings counters[b * H_kv + j] to
+    // targets[b * H_kv + j] merges branch b, kv head j into out / lse and
+    // sets the counter back to 0
+    int32_t *counters;
+    const int32_t *targets;
+    const int32_t *merge_ptr;
+    const int2 *merge_ent;
+    void *out;
+    float *lse;
+    const int32_t *empty_leaves;    // branches whose whole path is empty
+    int32_t num_empty_leaves;
+    int32_t num_leaves;
 };
 
 struct MergeArgs {
@@ -68,6 +86,9 @@ struct MergeArgs {
     int32_t num_q_heads;
     int32_t group;
 };
+
+// Resident CTAs per SM of the persistent attention kernel (sets its attributes).
+cudaError_t attn_bf16_ctas_per_sm(int head_dim, int *ctas_per_sm);
 
 // Kernel launchers; each returns the launch's cudaError_t.
 cudaError_t launch_attn_bf16(const AttnArgs &a, const CUtensorMap &tmap_k,

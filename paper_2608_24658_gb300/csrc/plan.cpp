@@ -18,6 +18,7 @@
 #include <cstring>
 #include <mutex>
 #include <new>
+#include <queue>
 #include <vector>
 
 #include <cudaTypedefs.h>
@@ -29,11 +30,19 @@ using parason::WorkItem;
 namespace {
 
 constexpr int kMinChunkPages = 8;
-constexpr int kItemsPerSm = 4;          // ~2 resident CTAs x 2 waves
+constexpr int kItemsPerSm = 8;          // 2 persistent CTAs x ~4 items each
+constexpr int kDefaultCtasPerSm = 2;    // persistent attention CTAs per SM (host plans)
 constexpr int64_t kDefaultWaitNs = 2000000000LL;
 constexpr size_t kAlign = 256;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Relative time of an item: its pages, weighted by the MMA work of wide tiles
+// (every consumer warp of a 64-row tile reads every page).
+int64_t item_cost(const WorkItem &it) {
+    const int64_t rgc = it.nrows <= 16 ? 1 : (it.nrows <= 32 ? 2 : 4);
+    return static_cast<int64_t>(it.num_pages) * (3 + rgc);
+}
 
 int tile_rows_for(int32_t rows, int32_t mode) {
     if (mode == PARASON_FP32) return 16;
@@ -51,12 +60,17 @@ struct parason_plan_s {
     int32_t num_leaves = 0;
     int64_t num_phys = 0;
     int32_t num_sms = 152;
+    int32_t ctas_per_sm = kDefaultCtasPerSm;
     int32_t chunk_pages = kMinChunkPages;
     std::vector<WorkItem> items;
     std::vector<int32_t> page_ids;
     std::vector<int32_t> dfs_leaf;
     std::vector<int32_t> merge_ptr;
     std::vector<int32_t> merge_ent;   // pairs (base, stride)
+    std::vector<int32_t> cta_ptr;     // persistent schedule (CSR over CTAs)
+    std::vector<int32_t> cta_items;
+    std::vector<int32_t> targets;     // items per (branch, kv head)
+    std::vector<int32_t> empty_leaves;
     int64_t num_slots = 0;
     int64_t unique_tokens = 0;
     int64_t path_tokens = 0;
@@ -70,6 +84,11 @@ struct parason_plan_s {
     int32_t *d_dfs_leaf = nullptr;
     int32_t *d_merge_ptr = nullptr;
     int2 *d_merge_ent = nullptr;
+    int32_t *d_cta_ptr = nullptr;
+    int32_t *d_cta_items = nullptr;
+    int32_t *d_counters = nullptr;
+    int32_t *d_targets = nullptr;
+    int32_t *d_empty = nullptr;
     int32_t *d_err = nullptr;
     uint32_t debug_flags = 0;
     int64_t wait_limit_ns = kDefaultWaitNs;
@@ -110,7 +129,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                           const int32_t *parent, const int32_t *node_len,
                           const int32_t *node_page_ptr, const int32_t *page_ids,
                           int32_t num_leaves, const int32_t *leaf_node,
-                          int64_t num_phys, int32_t num_sms) {
+                          int64_t num_phys, int32_t num_sms, int32_t ctas_per_sm) {
     parason_status st = validate_config(cfg);
     if (st != PARASON_OK) return st;
     if (num_nodes < 0 || num_leaves < 0 || num_phys < 0) return PARASON_EINVAL;
@@ -126,6 +145,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     p->num_leaves = num_leaves;
     p->num_phys = num_phys;
     p->num_sms = num_sms > 0 ? num_sms : 152;
+    p->ctas_per_sm = ctas_per_sm > 0 ? ctas_per_sm : kDefaultCtasPerSm;
 
     // tree and page table
     if (num_nodes > 0 && node_page_ptr[0] != 0) return PARASON_EINVAL;
@@ -240,9 +260,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                     it.kv_head = j;
                     if (sb > INT32_MAX) return PARASON_EUNSUPPORTED;
                     it.slot_base = static_cast<int32_t>(sb);
-                    // cost: pages, weighted by the MMA work of wide tiles
-                    const int64_t rgc = it.nrows <= 16 ? 1 : (it.nrows <= 32 ? 2 : 4);
-                    keyed.emplace_back(static_cast<int64_t>(np) * (3 + rgc), it);
+                    keyed.emplace_back(item_cost(it), it);
                 }
             }
             pg += np;
@@ -281,6 +299,42 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         }
         p->merge_ptr[b + 1] = static_cast<int32_t>(p->merge_ent.size() / 2);
     }
+
+    // items that feed each (branch, kv head), and branches with no item at all
+    p->targets.assign(static_cast<size_t>(num_leaves) * H_kv, 0);
+    for (const WorkItem &it : p->items) {
+        const int32_t pos_lo = it.row0 / g, pos_hi = (it.row0 + it.nrows - 1) / g;
+        for (int32_t pos = pos_lo; pos <= pos_hi; ++pos) {
+            const int32_t b = p->dfs_leaf[it.leaf_lo + pos];
+            p->targets[static_cast<size_t>(b) * H_kv + it.kv_head]++;
+        }
+    }
+    p->empty_leaves.clear();
+    for (int32_t b = 0; b < num_leaves; ++b)
+        if (p->targets[static_cast<size_t>(b) * H_kv] == 0) p->empty_leaves.push_back(b);
+
+    // persistent schedule: longest item first onto the least loaded CTA
+    const int32_t n_items = static_cast<int32_t>(p->items.size());
+    const int32_t n_ctas =
+        std::max<int32_t>(1, std::min<int32_t>(p->num_sms * p->ctas_per_sm, n_items));
+    std::vector<std::vector<int32_t>> per(n_ctas);
+    {
+        using Load = std::pair<int64_t, int32_t>;
+        std::priority_queue<Load, std::vector<Load>, std::greater<Load>> heap;
+        for (int32_t c = 0; c < n_ctas; ++c) heap.emplace(0, c);
+        for (int32_t i = 0; i < n_items; ++i) {     // items are sorted by cost, longest first
+            Load l = heap.top();
+            heap.pop();
+            per[l.second].push_back(i);
+            heap.emplace(l.first + item_cost(p->items[i]), l.second);
+        }
+    }
+    p->cta_ptr.assign(n_ctas + 1, 0);
+    p->cta_items.clear();
+    for (int32_t c = 0; c < n_ctas; ++c) {
+        p->cta_items.insert(p->cta_items.end(), per[c].begin(), per[c].end());
+        p->cta_ptr[c + 1] = static_cast<int32_t>(p->cta_items.size());
+    }
     return PARASON_OK;
 }
 
@@ -295,10 +349,17 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     const size_t n_dfs = p->dfs_leaf.size() * sizeof(int32_t);
     const size_t n_mptr = p->merge_ptr.size() * sizeof(int32_t);
     const size_t n_ment = p->merge_ent.size() * sizeof(int32_t);
+    const size_t n_cptr = p->cta_ptr.size() * sizeof(int32_t);
+    const size_t n_citems = p->cta_items.size() * sizeof(int32_t);
+    const size_t n_targets = p->targets.size() * sizeof(int32_t);
+    const size_t n_empty = p->empty_leaves.size() * sizeof(int32_t);
     const size_t n_err = parason::kErrWords * sizeof(int32_t);
-    size_t off[6], total = 0;
-    const size_t sizes[6] = {n_items, n_pages, n_dfs, n_mptr, n_ment, n_err};
-    for (int i = 0; i < 6; ++i) {
+    constexpr int kArrays = 11;
+    size_t off[kArrays], total = 0;
+    // the last two (counters, error record) are zero-filled, not copied
+    const size_t sizes[kArrays] = {n_items, n_pages,   n_dfs,    n_mptr,    n_ment, n_cptr,
+                                   n_citems, n_targets, n_empty, n_targets, n_err};
+    for (int i = 0; i < kArrays; ++i) {
         off[i] = total;
         total = align_up(total + std::max<size_t>(sizes[i], 4), kAlign);
     }
@@ -313,10 +374,18 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     p->d_dfs_leaf = reinterpret_cast<int32_t *>(base + off[2]);
     p->d_merge_ptr = reinterpret_cast<int32_t *>(base + off[3]);
     p->d_merge_ent = reinterpret_cast<int2 *>(base + off[4]);
-    p->d_err = reinterpret_cast<int32_t *>(base + off[5]);
-    const void *src[5] = {p->items.data(), p->page_ids.data(), p->dfs_leaf.data(),
-                          p->merge_ptr.data(), p->merge_ent.data()};
-    for (int i = 0; i < 5; ++i) {
+    p->d_cta_ptr = reinterpret_cast<int32_t *>(base + off[5]);
+    p->d_cta_items = reinterpret_cast<int32_t *>(base + off[6]);
+    p->d_targets = reinterpret_cast<int32_t *>(base + off[7]);
+    p->d_empty = reinterpret_cast<int32_t *>(base + off[8]);
+    p->d_counters = reinterpret_cast<int32_t *>(base + off[9]);
+    p->d_err = reinterpret_cast<int32_t *>(base + off[10]);
+    const void *src[9] = {p->items.data(),     p->page_ids.data(),  p->dfs_leaf.data(),
+                          p->merge_ptr.data(), p->merge_ent.data(), p->cta_ptr.data(),
+                          p->cta_items.data(), p->targets.data(),   p->empty_leaves.data()};
+    if (n_targets > 0 && cudaMemsetAsync(p->d_counters, 0, n_targets, stream) != cudaSuccess)
+        return PARASON_ECUDA;
+    for (int i = 0; i < 9; ++i) {
         if (sizes[i] == 0) continue;
         if (cudaMemcpyAsync(base + off[i], src[i], sizes[i], cudaMemcpyHostToDevice, stream) !=
             cudaSuccess)
@@ -401,7 +470,7 @@ parason_status parason_attn_plan_host(const parason_attn_config *cfg, int32_t nu
     parason_status st;
     try {
         st = build_host(p, cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves,
-                        leaf_node, num_physical_pages, num_sms);
+                        leaf_node, num_physical_pages, num_sms, kDefaultCtasPerSm);
     } catch (const std::bad_alloc &) {
         st = PARASON_ENOMEM;
     }
@@ -435,10 +504,24 @@ parason_status parason_attn_plan(const parason_attn_config *cfg, int32_t num_nod
         cudaGetLastError();
         return st != PARASON_OK ? st : PARASON_ECUDA;
     }
-    parason_plan p = nullptr;
-    st = parason_attn_plan_host(cfg, num_nodes, parent, node_len, node_page_ptr, page_ids,
-                                num_leaves, leaf_node, num_physical_pages, sms, &p);
-    if (st != PARASON_OK) return st;
+    int ctas_per_sm = kDefaultCtasPerSm;
+    if (cfg->mode != PARASON_FP32) {
+        if (parason::attn_bf16_ctas_per_sm(cfg->head_dim, &ctas_per_sm) != cudaSuccess)
+            return PARASON_ECUDA;
+        if (ctas_per_sm < 1) return PARASON_EUNSUPPORTED;
+    }
+    auto *p = new (std::nothrow) parason_plan_s();
+    if (!p) return PARASON_ENOMEM;
+    try {
+        st = build_host(p, cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves,
+                        leaf_node, num_physical_pages, sms, ctas_per_sm);
+    } catch (const std::bad_alloc &) {
+        st = PARASON_ENOMEM;
+    }
+    if (st != PARASON_OK) {
+        delete p;
+        return st;
+    }
     st = upload(p, reinterpret_cast<cudaStream_t>(stream));
     if (st != PARASON_OK) {
         parason_plan_destroy(p);
@@ -488,6 +571,7 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
 
     parason_status st = record_event(p, 0, stream);
     if (st != PARASON_OK) return st;
+    const bool fused = has_items && p->cfg.mode != PARASON_FP32;
     if (has_items) {
         parason::AttnArgs a{};
         a.items = p->d_items;
@@ -506,6 +590,18 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
         a.num_kv_heads = p->cfg.num_kv_heads;
         a.group = p->group;
         a.scale_log2 = sm_scale * 1.4426950408889634f;
+        a.cta_ptr = p->d_cta_ptr;
+        a.cta_items = p->d_cta_items;
+        a.num_ctas = static_cast<int32_t>(p->cta_ptr.size()) - 1;
+        a.counters = p->d_counters;
+        a.targets = p->d_targets;
+        a.merge_ptr = p->d_merge_ptr;
+        a.merge_ent = p->d_merge_ent;
+        a.out = out;
+        a.lse = lse;
+        a.empty_leaves = p->d_empty;
+        a.num_empty_leaves = static_cast<int32_t>(p->empty_leaves.size());
+        a.num_leaves = p->num_leaves;
         cudaError_t e;
         if (p->cfg.mode == PARASON_FP32) {
             e = parason::launch_attn_fp32(a, static_cast<const float *>(k_pages),
@@ -545,7 +641,8 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
     m.num_leaves = p->num_leaves;
     m.num_q_heads = p->cfg.num_q_heads;
     m.group = p->group;
-    if (parason::launch_merge(m, d, p->cfg.mode, stream) != cudaSuccess) return PARASON_ECUDA;
+    if (!fused && parason::launch_merge(m, d, p->cfg.mode, stream) != cudaSuccess)
+        return PARASON_ECUDA;
     st = record_event(p, 2, stream);
     if (st != PARASON_OK) return st;
     if (p->timing_cap > 0 && p->timing_n < p->timing_cap) p->timing_n++;
@@ -576,7 +673,11 @@ parason_status parason_plan_check(parason_plan p, parason_stream_t stream) {
     if (cudaMemcpy(rec, p->d_err, sizeof rec, cudaMemcpyDeviceToHost) != cudaSuccess)
         return PARASON_ECUDA;
     if (rec[0] != 0) {
+        // an aborted launch leaves merge counters part-way: start them over
         if (cudaMemset(p->d_err, 0, sizeof rec) != cudaSuccess) return PARASON_ECUDA;
+        if (!p->targets.empty() &&
+            cudaMemset(p->d_counters, 0, p->targets.size() * sizeof(int32_t)) != cudaSuccess)
+            return PARASON_ECUDA;
         return rec[0] == PARASON_ETIMEOUT ? PARASON_ETIMEOUT : PARASON_ECUDA;
     }
     return PARASON_OK;
@@ -612,6 +713,9 @@ parason_status parason_plan_get_info(parason_plan p, parason_plan_info *info) {
     info->path_tokens = p->path_tokens;
     info->num_sms = p->num_sms;
     info->on_device = p->on_device ? 1 : 0;
+    info->num_ctas = p->cta_ptr.empty() ? 0 : static_cast<int32_t>(p->cta_ptr.size()) - 1;
+    info->ctas_per_sm = p->ctas_per_sm;
+    info->num_empty_leaves = static_cast<int32_t>(p->empty_leaves.size());
     return PARASON_OK;
 }
 
@@ -624,6 +728,9 @@ parason_status parason_plan_export(parason_plan p, int32_t table, void *dst, siz
     case PARASON_TABLE_DFS_LEAVES: src = p->dfs_leaf.data(); n = p->dfs_leaf.size() * 4; break;
     case PARASON_TABLE_MERGE_PTR: src = p->merge_ptr.data(); n = p->merge_ptr.size() * 4; break;
     case PARASON_TABLE_MERGE: src = p->merge_ent.data(); n = p->merge_ent.size() * 4; break;
+    case PARASON_TABLE_SCHEDULE_PTR: src = p->cta_ptr.data(); n = p->cta_ptr.size() * 4; break;
+    case PARASON_TABLE_SCHEDULE: src = p->cta_items.data(); n = p->cta_items.size() * 4; break;
+    case PARASON_TABLE_TARGETS: src = p->targets.data(); n = p->targets.size() * 4; break;
     default: return PARASON_EINVAL;
     }
     if (bytes < n || (n > 0 && !dst)) return PARASON_EINVAL;
@@ -676,7 +783,8 @@ parason_status parason_plan_read_timing(parason_plan p, float *attn_ms, float *m
 
 int32_t parason_plan_launches_per_decode(parason_plan p) {
     if (!p || p->num_leaves == 0) return 0;
-    return (p->items.empty() ? 0 : 1) + 1;
+    if (p->items.empty()) return 1;                       // merge kernel only
+    return p->cfg.mode == PARASON_FP32 ? 2 : 1;           // bf16/fp8 merge is fused
 }
 
 const char *parason_version(void) { return "0.1.0"; }

@@ -92,6 +92,21 @@ def verify_plan(tree, plan):
             assert got == sorted(slots_of[(b, h)]), (b, h)
     assert info["unique_tokens"] == tree.unique_tokens()
     assert info["path_tokens"] == tree.path_tokens()
+    # persistent schedule: every item exactly once, no empty CTA
+    sptr = plan.export(_lib.TABLE_SCHEDULE_PTR)
+    sched = plan.export(_lib.TABLE_SCHEDULE)
+    assert sorted(sched.tolist()) == list(range(len(items)))
+    assert sptr[0] == 0 and sptr[-1] == len(items) and np.all(np.diff(sptr) >= 1 if len(items) else True)
+    assert info["num_ctas"] == max(1, min(info["ctas_per_sm"] * info["num_sms"], len(items)))
+    # merge targets: the items whose rows include (branch, kv head)
+    targets = plan.export(_lib.TABLE_TARGETS)
+    want = np.zeros((tree.num_leaves, H_kv), dtype=np.int64)
+    for it in items:
+        _, _, _, leaf_lo, row0, nrows, kvh, _ = (int(x) for x in it)
+        for b in {int(dfs[leaf_lo + row // g]) for row in range(row0, row0 + nrows)}:
+            want[b, kvh] += 1
+    assert np.array_equal(targets, want)
+    assert info["num_empty_leaves"] == int((want[:, 0] == 0).sum()) if tree.num_leaves else True
     return info
 
 
