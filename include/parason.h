@@ -193,15 +193,15 @@ typedef struct {
     int32_t num_items;          /* work items of the attention kernel       */
     int32_t num_leaves;
     int32_t num_merge_entries;  /* partial results folded by the merge      */
-    int32_t chunk_pages;        /* split-K chunk length in pages            */
+    int32_t chunk_pages;        /* shortest split-K piece, in pages         */
     int64_t num_slots;          /* partial (o, m, l) rows in the workspace  */
     int64_t unique_tokens;      /* tokens of nodes some branch reads, once  */
     int64_t path_tokens;        /* sum over branches of their path tokens   */
     int32_t num_sms;            /* SM count the split targeted              */
     int32_t on_device;          /* 1 if decode can run on this plan         */
     int32_t num_ctas;           /* CTAs of the persistent attention kernel  */
-    int32_t num_empty_leaves;   /* branches whose whole path is empty       */
-    int32_t ctas_per_sm;        /* resident CTAs per SM the grid assumes    */
+    int32_t num_wide_ctas;      /* of which run the prefix pass             */
+    int32_t num_workers;        /* item lists: prefix CTAs + suffix warps   */
 } parason_plan_info;
 
 parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info);
@@ -212,18 +212,17 @@ parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info)
  *                            page_ids, page count, valid tokens in the last
  *                            page, first branch (index into the DFS branch
  *                            order), first node row, row count, kv head,
- *                            partial slot of node row 0
+ *                            partial slot of the item's first row
  *   PARASON_TABLE_DFS_LEAVES int32 [num_leaves]: branches in DFS order
- *   PARASON_TABLE_MERGE_PTR  int32 [num_leaves + 1]: CSR into the entries
- *   PARASON_TABLE_MERGE      int32 [num_merge_entries][2]: (base, stride);
- *                            q head h = j*g + r of the branch reads the
- *                            partial slot base + j*stride + r
- *   PARASON_TABLE_SCHEDULE_PTR int32 [num_ctas + 1]: CSR of the persistent
- *                            kernel's per-CTA item lists
- *   PARASON_TABLE_SCHEDULE   int32 [num_items]: item indices, CTA by CTA
- *   PARASON_TABLE_TARGETS    int32 [num_leaves][H_kv]: items whose rows
- *                            include (branch, kv head); the merge of that
- *                            pair runs when the last of them finishes
+ *   PARASON_TABLE_MERGE_PTR  int32 [num_leaves * H_kv + 1]: CSR into the
+ *                            entries, per (branch, kv head)
+ *   PARASON_TABLE_MERGE      int32 [num_merge_entries]: partial slot of the
+ *                            branch's first q head of the kv head; q head
+ *                            j*g + r reads slot entry + r
+ *   PARASON_TABLE_SCHEDULE_PTR int32 [num_workers + 1]: CSR of the persistent
+ *                            kernel's item lists: one list per prefix-pass
+ *                            CTA, then one per suffix-pass warp
+ *   PARASON_TABLE_SCHEDULE   int32 [num_items]: item indices, list by list
  * Returns PARASON_EINVAL if `bytes` is smaller than the table.
  */
 enum {
@@ -232,8 +231,7 @@ enum {
     PARASON_TABLE_MERGE_PTR = 2,
     PARASON_TABLE_MERGE = 3,
     PARASON_TABLE_SCHEDULE_PTR = 4,
-    PARASON_TABLE_SCHEDULE = 5,
-    PARASON_TABLE_TARGETS = 6
+    PARASON_TABLE_SCHEDULE = 5
 };
 parason_status parason_plan_export(parason_plan plan, int32_t table, void *dst, size_t bytes);
 

@@ -1,64 +1,84 @@
 // attn_bf16.cu -- fork-tree decode attention for bf16 KV on sm_103a.
 //
-// Persistent kernel, two CTAs per SM.  Each CTA runs a planner-made list of
-// work items back to back; an item is up to 64 stacked query rows (the
-// branches under one fork-tree node times the q heads of one kv head)
-// against one chunk of that node's pages.  A node's KV is read from HBM once
-// for all the rows stacked on it: this is what turns the shared prefix of many
-// Subtask/Trial branches (paper Sec. 3.1, 3.4) into one read.
+// One persistent launch, one CTA per SM, two roles (the planner decides how
+// many SMs each gets so that both finish together):
 //
-//   warp 4 (producer)   TMA: one 3-D box per (page, kv head) for K and for V,
-//                       128-byte swizzle, into a ring of single-page stages
-//                       that runs continuously across item boundaries, so the
-//                       next item's pages load during this item's epilogue.
-//   warps 0-3           tensor-core QK^T and PV with mma.sync m16n8k16 (bf16
-//                       in, fp32 accumulate) from ldmatrix fragments, online
-//                       softmax in registers with quad shuffles.  The warps
-//                       split the tile's rows (16 per warp) and, for small
-//                       tiles, the item's pages (page p to warp p % tgc).
+//  * prefix pass (CTAs [0, num_wide_ctas)): nodes that many branches share.
+//    Up to 128 query rows -- the branches under the node times the q heads
+//    of one kv head -- are stacked on one page stream: a producer warp moves
+//    each (page, kv head) of K and V by TMA (3-D box, 128-byte swizzle) into
+//    a shared ring, and 8 consumer warps of 16 rows each read it from shared
+//    memory.  The node's KV is read from HBM once for all its rows, which is
+//    what the shared prefix of Subtask/Trial branches buys (paper Sec. 3.1,
+//    3.4).
+//  * suffix pass (the other CTAs): nodes of at most 16 rows (a branch's own
+//    suffix).  Each of the 8 warps is an independent worker with its own
+//    TMA ring and its own balanced list of items (split-K pieces of
+//    suffixes): no CTA barrier, no cross-warp combine.
 //
-// Epilogue of an item: the warps of a row group combine through shared memory
-// and write the item's partial (o, m, l) rows; then the item is counted into
-// every (branch, kv head) it feeds, and the item that completes a pair runs
-// that pair's log-sum-exp merge (merge_epilogue.cuh) -- no second kernel.
+// Both roles use tensor-core QK^T and PV (mma.sync m16n8k16, bf16 in, fp32
+// accumulate) from ldmatrix fragments and an online softmax in registers with
+// quad shuffles, and write a partial (o, m, l) per item row.  The merge kernel
+// (merge.cu) folds the partials of every branch's path afterwards; it is
+// launched as a programmatic dependent of this grid.
 //
-// Scores are kept in the log2 domain: x = sm_scale*log2(e)*<q,k>, so the
+// Scores are kept in the log2 domain: x = sm_scale*log2(e)*<q,k>, so a
 // partial is m = max x, l = sum 2^(x-m), o = sum 2^(x-m) v (unnormalised).
 #include "device_common.cuh"
-#include "merge_epilogue.cuh"
 
 namespace parason {
 namespace {
 
-constexpr int kConsumerWarps = 4;
+constexpr int kConsumerWarps = 8;
 constexpr int kConsumerThreads = kConsumerWarps * 32;
-constexpr int kThreads = kConsumerThreads + 32;
-constexpr int kCtasPerSm = 2;
+constexpr int kThreads = kConsumerThreads + 32;            // + producer warp
 constexpr long long kDrainLimitNs = 1000000000LL;
-// shared memory one CTA may use when two share an SM (228 KB per SM, 1 KB
-// reserved per CTA, a little static shared memory)
-constexpr int kCtaSmemBudget = (228 * 1024) / kCtasPerSm - 1024 - 512;
+constexpr int kSmemBudget = 220 * 1024;                    // dynamic, one CTA per SM
 
 template <int D>
-struct Bf16Shape {
-    static constexpr int kPageBytes = kPageSize * D * 2;        // one page of one kv head
-    static constexpr int kSeg = D * 2 / 128;                     // 128-byte rows per token
-    static constexpr int kStageBytes = 2 * kPageBytes;           // K and V of one page
-    // combine scratch: [warp][16 rows][D/2 + 8] floats (two column halves)
+struct Shape {
+    static constexpr int kPageBytes = kPageSize * D * 2;   // one page of one kv head
+    // a page lands as kSeg column blocks of 16 tokens x 128 bytes, so that 8
+    // consecutive tokens hit 8 different 128-byte swizzle rows
+    static constexpr int kSeg = D * 2 / 128;
+    static constexpr int kSegBytes = kPageSize * 128;
+    static constexpr int kStageBytes = 2 * kPageBytes;      // K and V of one page
+
+    // suffix pass: a private ring per warp
+    static constexpr int kWarpStages = (192 * 1024) / (kConsumerWarps * kStageBytes);
+    static constexpr int kWarpRingBytes = kWarpStages * kStageBytes;
+    static constexpr int kNarrowBytes = kConsumerWarps * kWarpRingBytes;
+    static constexpr int kNarrowBars = kConsumerWarps * kWarpStages;
+
+    // prefix pass: one ring + combine scratch [warp][16 rows][D/2 + 8] floats
     static constexpr int kHalf = D / 2;
     static constexpr int kScratchStride = kHalf + 8;
-    static constexpr int kCombineBytes = kConsumerWarps * 16 * (kScratchStride * 4 + 8);
-    static constexpr int kScratchBytes =
-        kCombineBytes > dev::kMergeStageBytes ? kCombineBytes : dev::kMergeStageBytes;
-    static constexpr int kBarBytesMax = 2 * 64 * 8;
-    static constexpr int kStages =
-        (kCtaSmemBudget - kScratchBytes - kBarBytesMax - 1024) / kStageBytes;
-    static constexpr int kRingBytes = kStages * kStageBytes;
-    static constexpr int kBarBytes = 2 * kStages * 8;
-    static constexpr int kSmemBytes = kRingBytes + kScratchBytes + kBarBytes + 1024;
-    static_assert(kStages >= 4 && kStages <= 64, "ring depth");
-    static_assert(kSmemBytes <= kCtaSmemBudget, "two CTAs per SM must fit");
+    static constexpr int kScratchBytes = kConsumerWarps * 16 * (kScratchStride * 4 + 8);
+    static constexpr int kWideStages = (kNarrowBytes - kScratchBytes) / kStageBytes;
+    static constexpr int kWideRingBytes = kWideStages * kStageBytes;
+    static constexpr int kWideBars = 2 * kWideStages;
+
+    static constexpr int kBars = kNarrowBars > kWideBars ? kNarrowBars : kWideBars;
+    static constexpr int kBodyBytes =
+        kNarrowBytes > kWideRingBytes + kScratchBytes ? kNarrowBytes : kWideRingBytes + kScratchBytes;
+    static constexpr int kSmemBytes = kBodyBytes + kBars * 8 + 1024;   // + alignment slack
+    static_assert(kWarpStages >= 2, "suffix ring depth");
+    static_assert(kWideStages >= 4, "prefix ring depth");
+    static_assert(kSmemBytes <= kSmemBudget, "shared memory budget");
 };
+
+// K then V of one (page, kv head) into a stage: one TMA box {64 columns, 1
+// block, 16 tokens} per column block and tensor.
+template <int D>
+__device__ __forceinline__ void load_page(uint32_t dst, const CUtensorMap *tmap_k,
+                                          const CUtensorMap *tmap_v, int row, uint32_t bar) {
+    using S = Shape<D>;
+#pragma unroll
+    for (int sg = 0; sg < S::kSeg; ++sg) {
+        dev::tma_load_3d(dst + sg * S::kSegBytes, tmap_k, 0, sg, row, bar);
+        dev::tma_load_3d(dst + S::kPageBytes + sg * S::kSegBytes, tmap_v, 0, sg, row, bar);
+    }
+}
 
 // Online-softmax state of one warp: 16 rows, thread holds rows gid, gid+8.
 template <int D>
@@ -68,12 +88,20 @@ struct WarpState {
     float l[2];
 };
 
+template <int D>
+__device__ __forceinline__ void reset(WarpState<D> &st) {
+#pragma unroll
+    for (int dt = 0; dt < D / 8; ++dt) st.o[dt][0] = st.o[dt][1] = st.o[dt][2] = st.o[dt][3] = 0.f;
+    st.m[0] = st.m[1] = -INFINITY;
+    st.l[0] = st.l[1] = 0.f;
+}
+
 // One 16-token page: S = Q K^T, online softmax, O += P V.
 template <int D>
 __device__ __forceinline__ void page_step(uint32_t kbase, uint32_t vbase, int valid,
                                           const uint32_t (&qa)[D / 16][4], WarpState<D> &st,
                                           float scale_log2, int lane) {
-    using S = Bf16Shape<D>;
+    using S = Shape<D>;
     const int tig = lane & 3;
     const int mi = lane >> 3, r8 = lane & 7;
 
@@ -85,9 +113,9 @@ __device__ __forceinline__ void page_step(uint32_t kbase, uint32_t vbase, int va
 #pragma unroll
         for (int ks = 0; ks < D / 16; ++ks) {
             const int dch = 2 * ks + (mi & 1);
-            const uint32_t row = tok * S::kSeg + (dch >> 3);
             uint32_t b00, b01, b10, b11;
-            dev::ldsm_x4(kbase + dev::swz128(row, dch & 7), b00, b01, b10, b11);
+            dev::ldsm_x4(kbase + (dch >> 3) * S::kSegBytes + dev::swz128(tok, dch & 7), b00, b01,
+                         b10, b11);
             if (ks < D / 32) {
                 dev::mma_bf16_16816(sc[0], qa[ks], b00, b01);
                 dev::mma_bf16_16816(sc[1], qa[ks], b10, b11);
@@ -117,7 +145,7 @@ __device__ __forceinline__ void page_step(uint32_t kbase, uint32_t vbase, int va
     mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
     mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
     mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-    // token 0 of every page in a chunk is valid, so mx0/mx1 are finite
+    // token 0 of every page of an item is valid, so mx0/mx1 are finite
     const float mn0 = fmaxf(st.m[0], mx0), mn1 = fmaxf(st.m[1], mx1);
     const float al0 = dev::fast_exp2(st.m[0] - mn0), al1 = dev::fast_exp2(st.m[1] - mn1);
     st.m[0] = mn0;
@@ -155,9 +183,9 @@ __device__ __forceinline__ void page_step(uint32_t kbase, uint32_t vbase, int va
 #pragma unroll
     for (int dt = 0; dt < D / 8; dt += 2) {
         const int dch = dt + (mi >> 1);
-        const uint32_t row = vtok * S::kSeg + (dch >> 3);
         uint32_t v0, v1, v2, v3;
-        dev::ldsm_x4_trans(vbase + dev::swz128(row, dch & 7), v0, v1, v2, v3);
+        dev::ldsm_x4_trans(vbase + (dch >> 3) * S::kSegBytes + dev::swz128(vtok, dch & 7), v0, v1,
+                           v2, v3);
         v0 &= keep_lo;
         v1 &= keep_hi;
         v2 &= keep_lo;
@@ -167,7 +195,7 @@ __device__ __forceinline__ void page_step(uint32_t kbase, uint32_t vbase, int va
     }
 }
 
-// Q fragments (A operand, row-major 16 x D) for rows rg*16 + {gid, gid+8}.
+// Q fragments (A operand, row-major 16 x D) for tile rows rg*16 + {gid, gid+8}.
 template <int D>
 __device__ __forceinline__ void load_q_fragments(const AttnArgs &a, const WorkItem &it, int rg,
                                                  int lane, uint32_t (&qa)[D / 16][4]) {
@@ -194,238 +222,323 @@ __device__ __forceinline__ void load_q_fragments(const AttnArgs &a, const WorkIt
         }
 }
 
-// Write the partial (o, m, l) of an item: straight from registers when each
-// warp owns its rows, else combining the warps of a row group through shared
-// memory, one column half at a time.
+// A warp that owns rows rg*16 .. rg*16+15 of an item writes their partials
+// straight from registers.
 template <int D>
-__device__ __forceinline__ void write_partials(const AttnArgs &a, const WorkItem &it,
-                                               WarpState<D> &st, int tgc, int rg, int warp,
-                                               int lane, float *sc_o, float2 *sc_ml) {
-    using S = Bf16Shape<D>;
+__device__ __forceinline__ void store_warp_partials(const AttnArgs &a, const WorkItem &it,
+                                                    WarpState<D> &st, int rg, int lane) {
     const int gid = lane >> 2, tig = lane & 3;
     st.l[0] += __shfl_xor_sync(0xffffffffu, st.l[0], 1);
     st.l[0] += __shfl_xor_sync(0xffffffffu, st.l[0], 2);
     st.l[1] += __shfl_xor_sync(0xffffffffu, st.l[1], 1);
     st.l[1] += __shfl_xor_sync(0xffffffffu, st.l[1], 2);
-    if (tgc == 1) {
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int r = rg * 16 + gid + 8 * h;
-            if (r >= it.nrows) continue;
-            const int64_t slot = static_cast<int64_t>(it.slot_base) + it.row0 + r;
-            float *dst = a.part_o + slot * D;
+    for (int h = 0; h < 2; ++h) {
+        const int r = rg * 16 + gid + 8 * h;
+        if (r >= it.nrows) continue;
+        const int64_t slot = static_cast<int64_t>(it.slot_base) + r;
+        float *dst = a.part_o + slot * D;
 #pragma unroll
-            for (int dt = 0; dt < D / 8; ++dt)
-                *reinterpret_cast<float2 *>(dst + dt * 8 + 2 * tig) =
-                    make_float2(st.o[dt][2 * h], st.o[dt][2 * h + 1]);
-            if (tig == 0) a.part_ml[slot] = make_float2(st.m[h], st.l[h]);
-        }
-        return;
-    }
-    const int tid = threadIdx.x;
-    if (tig == 0) {
-        sc_ml[warp * 16 + gid] = make_float2(st.m[0], st.l[0]);
-        sc_ml[warp * 16 + gid + 8] = make_float2(st.m[1], st.l[1]);
-    }
-    constexpr int kVec = S::kHalf / 4;
-#pragma unroll
-    for (int half = 0; half < 2; ++half) {
-        float *wo = sc_o + warp * 16 * S::kScratchStride;
-#pragma unroll
-        for (int dt = 0; dt < D / 16; ++dt) {
-            const int c = dt * 8 + 2 * tig;
-            const int src = half * (D / 16) + dt;
-            *reinterpret_cast<float2 *>(wo + gid * S::kScratchStride + c) =
-                make_float2(st.o[src][0], st.o[src][1]);
-            *reinterpret_cast<float2 *>(wo + (gid + 8) * S::kScratchStride + c) =
-                make_float2(st.o[src][2], st.o[src][3]);
-        }
-        dev::bar_sync<kConsumerThreads>(1);
-        for (int idx = tid; idx < it.nrows * kVec; idx += kConsumerThreads) {
-            const int r = idx / kVec, c4 = idx % kVec;
-            const int grp = r >> 4, rr = r & 15;
-            float M = -INFINITY;
-            for (int w = 0; w < tgc; ++w) M = fmaxf(M, sc_ml[(grp * tgc + w) * 16 + rr].x);
-            float L = 0.f;
-            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-            for (int w = 0; w < tgc; ++w) {
-                const int ww = grp * tgc + w;
-                const float2 ml = sc_ml[ww * 16 + rr];
-                const float sc = dev::fast_exp2(ml.x - M);
-                L += sc * ml.y;
-                const float4 v = *reinterpret_cast<const float4 *>(
-                    sc_o + (ww * 16 + rr) * S::kScratchStride + 4 * c4);
-                acc.x += sc * v.x;
-                acc.y += sc * v.y;
-                acc.z += sc * v.z;
-                acc.w += sc * v.w;
-            }
-            const int64_t slot = static_cast<int64_t>(it.slot_base) + it.row0 + r;
-            *reinterpret_cast<float4 *>(a.part_o + slot * D + half * S::kHalf + 4 * c4) = acc;
-            if (half == 0 && c4 == 0) a.part_ml[slot] = make_float2(M, L);
-        }
-        dev::bar_sync<kConsumerThreads>(1);
+        for (int dt = 0; dt < D / 8; ++dt)
+            *reinterpret_cast<float2 *>(dst + dt * 8 + 2 * tig) =
+                make_float2(st.o[dt][2 * h], st.o[dt][2 * h + 1]);
+        if (tig == 0) a.part_ml[slot] = make_float2(st.m[h], st.l[h]);
     }
 }
 
-// Persistent kernel: CTA c runs its planner-assigned items back to back.
-// Two CTAs of 5 warps per SM: 10 warps over 4 sub-partitions of 16K
-// registers allow at most 168 registers per thread.
-template <int D>
-__global__ void __launch_bounds__(kThreads, kCtasPerSm)
-    attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
-                     const __grid_constant__ CUtensorMap tmap_v, const AttnArgs a) {
-    using S = Bf16Shape<D>;
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = reinterpret_cast<uint8_t *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    const uint32_t ring = dev::smem_addr(smem);
-    uint8_t *scratch = smem + S::kRingBytes;
-    float *sc_o = reinterpret_cast<float *>(scratch);
-    float2 *sc_ml = reinterpret_cast<float2 *>(scratch + kConsumerWarps * 16 * S::kScratchStride * 4);
-    const uint32_t bar_full = dev::smem_addr(smem + S::kRingBytes + S::kScratchBytes);
-    const uint32_t bar_empty = bar_full + S::kStages * 8;
-    __shared__ int abort_flag;
-    __shared__ int merge_count;
-    __shared__ int merge_list[kMaxTileRows + 1];
-
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int i_begin = a.cta_ptr[blockIdx.x], i_end = a.cta_ptr[blockIdx.x + 1];
-    auto k_page = [&](int s) { return ring + s * S::kStageBytes; };
-    auto v_page = [&](int s) { return ring + s * S::kStageBytes + S::kPageBytes; };
-
-    if (threadIdx.x == 0) {
-        abort_flag = 0;
-        for (int s = 0; s < S::kStages; ++s) {
-            dev::mbar_init(bar_full + 8 * s, 1);
-            dev::mbar_init(bar_empty + 8 * s, kConsumerWarps);
-        }
-        dev::fence_mbar_init();
+// A worker's page stream, read by one whole warp: lane i holds entry
+// base + i of the window; row(q) returns entry q (q uniform over the warp,
+// nondecreasing), refilling the window with one coalesced load every 32.
+struct PageStream {
+    const int32_t *rows;
+    int size;
+    int base;
+    int win;
+    __device__ PageStream(const AttnArgs &a, int worker, int lane) {
+        const int s0 = a.stream_ptr[worker];
+        rows = a.stream_rows + s0;
+        size = a.stream_ptr[worker + 1] - s0;
+        base = 0;
+        win = rows[lane];                 // the stream array is padded by 32 entries
     }
-    __syncthreads();
+    __device__ __forceinline__ int row(int q, int lane) {
+        if (q >= base + 32) {
+            base = q & ~31;
+            win = rows[base + lane];
+        }
+        return __shfl_sync(0xffffffffu, win, q - base);
+    }
+};
+
+// ---------------------------------------------------------------------------
+// suffix pass: every warp streams its own item list through its own ring
+// ---------------------------------------------------------------------------
+template <int D>
+__device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
+                            const AttnArgs &a, uint32_t ring, uint32_t bars, int warp, int lane) {
+    using S = Shape<D>;
+    constexpr int NS = S::kWarpStages;
+    const int worker = a.num_wide_ctas + (blockIdx.x - a.num_wide_ctas) * kConsumerWarps + warp;
+    const int i_begin = a.sched_ptr[worker], i_end = a.sched_ptr[worker + 1];
+    if (i_begin >= i_end) return;
+    const uint32_t my_ring = ring + warp * S::kWarpRingBytes;
+    const uint32_t my_bar = bars + warp * NS * 8;
+
+    // the warp's page stream: TMA rows read 32 at a time by the whole warp
+    PageStream ps(a, worker, lane);
+    const bool skip_first = (a.debug_flags & PARASON_DEBUG_SKIP_FIRST_LOAD) && warp == 0;
+    int issued = 0;
+    auto issue_next = [&]() {
+        // whole warp (uniform): the stream position is the same in every lane
+        if (issued >= ps.size) return;
+        const int row = ps.row(issued, lane);
+        if (lane == 0 && !(skip_first && issued == 0)) {
+            const int s = issued % NS;
+            const uint32_t dst = my_ring + s * S::kStageBytes;
+            const uint32_t bar = my_bar + s * 8;
+            dev::mbar_arrive_expect_tx(bar, S::kStageBytes);
+            load_page<D>(dst, tmap_k, tmap_v, row, bar);
+        }
+        ++issued;
+    };
+    for (int i = 0; i < NS; ++i) issue_next();
+
+    int consumed = 0;
+    bool ok = true;
+    for (int ii = i_begin; ii < i_end && ok; ++ii) {
+        const WorkItem it = a.items[a.sched_items[ii]];
+        uint32_t qa[D / 16][4];
+        load_q_fragments<D>(a, it, 0, lane, qa);
+        WarpState<D> st;
+        reset<D>(st);
+        for (int pg = 0; pg < it.num_pages; ++pg, ++consumed) {
+            const int s = consumed % NS;
+            if (!dev::mbar_wait_bounded(my_bar + s * 8, (consumed / NS) & 1, a.wait_limit_ns,
+                                        nullptr)) {
+                ok = false;
+                break;
+            }
+            const int valid = (pg == it.num_pages - 1) ? it.last_valid : kPageSize;
+            page_step<D>(my_ring + s * S::kStageBytes, my_ring + s * S::kStageBytes + S::kPageBytes,
+                         valid, qa, st, a.scale_log2, lane);
+            // refill this slot: its ldmatrix reads are complete, since every MMA
+            // that consumed them has issued (in order) before this point
+            __syncwarp();
+            issue_next();
+        }
+        if (!ok) break;
+        store_warp_partials<D>(a, it, st, 0, lane);
+    }
+    if (!ok && lane == 0) dev::record_error(a.err, PARASON_ETIMEOUT, kSiteConsumerFull);
+    // copies still in flight must land before the CTA's shared memory goes
+    if (lane == 0) {
+        for (int q = consumed; q < issued; ++q) {
+            if (skip_first && q == 0) continue;
+            dev::mbar_wait_bounded(my_bar + (q % NS) * 8, (q / NS) & 1, kDrainLimitNs, nullptr);
+        }
+    }
+    __syncwarp();
+}
+
+// ---------------------------------------------------------------------------
+// prefix pass: up to 128 stacked rows share one page stream
+// ---------------------------------------------------------------------------
+template <int D>
+__device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
+                           const AttnArgs &a, uint8_t *smem, uint32_t ring, uint32_t bars,
+                           int warp, int lane, volatile int *abort_flag) {
+    using S = Shape<D>;
+    constexpr int NS = S::kWideStages;
+    const uint32_t bar_full = bars, bar_empty = bars + NS * 8;
+    const int i_begin = a.sched_ptr[blockIdx.x], i_end = a.sched_ptr[blockIdx.x + 1];
+    auto k_page = [&](int s) { return ring + s * S::kStageBytes; };
 
     if (warp == kConsumerWarps) {
         // ------------------------------------------------------------ producer
-        if (lane == 0) {
-            dev::prefetch_tensormap(&tmap_k);
-            dev::prefetch_tensormap(&tmap_v);
-            int last_issue[S::kStages];
-            for (int s = 0; s < S::kStages; ++s) last_issue[s] = -1;
-            int stage = 0;
-            bool ok = true;
-            for (int ii = i_begin; ii < i_end && ok; ++ii) {
-                const WorkItem it = a.items[a.cta_items[ii]];
-                for (int pg = 0; pg < it.num_pages; ++pg, ++stage) {
-                    const int s = stage % S::kStages;
-                    if (stage >= S::kStages &&
-                        !dev::mbar_wait_bounded(bar_empty + 8 * s, ((stage / S::kStages) - 1) & 1,
-                                                a.wait_limit_ns, &abort_flag)) {
-                        if (!abort_flag) {
-                            abort_flag = 1;
-                            dev::record_error(a.err, PARASON_ETIMEOUT, kSiteProducerEmpty);
-                        }
-                        ok = false;
-                        break;
+        // the whole warp walks the page stream; lane 0 waits and issues
+        PageStream ps(a, blockIdx.x, lane);
+        int last_issue[NS];
+        for (int s = 0; s < NS; ++s) last_issue[s] = -1;
+        const bool skip_first = a.debug_flags & PARASON_DEBUG_SKIP_FIRST_LOAD;
+        for (int stage = 0; stage < ps.size; ++stage) {
+            const int s = stage % NS;
+            int stop = 0;
+            if (lane == 0) {
+                if (stage >= NS && !dev::mbar_wait_bounded(bar_empty + 8 * s, ((stage / NS) - 1) & 1,
+                                                           a.wait_limit_ns, abort_flag)) {
+                    if (!*abort_flag) {
+                        *abort_flag = 1;
+                        dev::record_error(a.err, PARASON_ETIMEOUT, kSiteProducerEmpty);
                     }
-                    if (abort_flag) {
-                        ok = false;
-                        break;
-                    }
-                    if ((a.debug_flags & PARASON_DEBUG_SKIP_FIRST_LOAD) && stage == 0) continue;
-                    const int page = a.page_ids[it.page_pos + pg];
-                    const int row = (page * a.num_kv_heads + it.kv_head) * kPageSize;
-                    dev::mbar_arrive_expect_tx(bar_full + 8 * s, S::kStageBytes);
-                    dev::tma_load_3d(k_page(s), &tmap_k, 0, 0, row, bar_full + 8 * s);
-                    dev::tma_load_3d(v_page(s), &tmap_v, 0, 0, row, bar_full + 8 * s);
-                    last_issue[s] = stage;
+                    stop = 1;
+                } else if (*abort_flag) {
+                    stop = 1;
                 }
             }
-            // every copy this CTA issued must land before its shared memory goes
-            for (int s = 0; s < S::kStages; ++s)
-                if (last_issue[s] >= 0)
-                    dev::mbar_wait_bounded(bar_full + 8 * s, (last_issue[s] / S::kStages) & 1,
-                                           kDrainLimitNs, nullptr);
+            if (__shfl_sync(0xffffffffu, stop, 0)) break;
+            const int row = ps.row(stage, lane);
+            if (lane == 0 && !(skip_first && stage == 0)) {
+                dev::mbar_arrive_expect_tx(bar_full + 8 * s, S::kStageBytes);
+                load_page<D>(k_page(s), tmap_k, tmap_v, row, bar_full + 8 * s);
+                last_issue[s] = stage;
+            }
         }
+        // every copy this CTA issued must land before its shared memory goes
+        if (lane == 0)
+            for (int s = 0; s < NS; ++s)
+                if (last_issue[s] >= 0)
+                    dev::mbar_wait_bounded(bar_full + 8 * s, (last_issue[s] / NS) & 1, kDrainLimitNs,
+                                           nullptr);
         return;
     }
 
     // ---------------------------------------------------------------- consumers
-    const int tid = threadIdx.x;                     // 0 .. 127
-    if (blockIdx.x == 0 && a.num_empty_leaves > 0)
-        dev::write_empty_branches<D>(a, tid, kConsumerThreads);
-
+    uint8_t *scratch = smem + S::kWideRingBytes;
+    float *sc_o = reinterpret_cast<float *>(scratch);
+    float2 *sc_ml = reinterpret_cast<float2 *>(scratch + kConsumerWarps * 16 * S::kScratchStride * 4);
+    const int tid = threadIdx.x;
+    const int gid = lane >> 2, tig = lane & 3;
     int stage = 0;
     for (int ii = i_begin; ii < i_end; ++ii) {
-        const WorkItem it = a.items[a.cta_items[ii]];
-        const int rgc = it.nrows <= 16 ? 1 : (it.nrows <= 32 ? 2 : 4);
+        const WorkItem it = a.items[a.sched_items[ii]];
+        const int groups = (it.nrows + 15) >> 4;
+        const int rgc = groups <= 2 ? 2 : (groups <= 4 ? 4 : 8);
         const int tgc = kConsumerWarps / rgc;
         const int rg = warp / tgc, tg = warp % tgc;
+        const bool has_rows = rg * 16 < it.nrows;
 
         uint32_t qa[D / 16][4];
         load_q_fragments<D>(a, it, rg, lane, qa);
         WarpState<D> st;
-#pragma unroll
-        for (int dt = 0; dt < D / 8; ++dt)
-            st.o[dt][0] = st.o[dt][1] = st.o[dt][2] = st.o[dt][3] = 0.f;
-        st.m[0] = st.m[1] = -INFINITY;
-        st.l[0] = st.l[1] = 0.f;
+        reset<D>(st);
 
-        // page pg is processed by token-group warp pg % tgc of each row group;
-        // every warp waits for every page (which keeps the empty barrier's
-        // phases exact) and releases it
+        // page pg goes to token-group warp pg % tgc of each row group; every
+        // warp waits for every page (keeping the empty barrier's phases exact)
+        // and releases it
         bool ok = true;
         for (int pg = 0; pg < it.num_pages; ++pg, ++stage) {
-            const int s = stage % S::kStages;
-            if (!dev::mbar_wait_bounded(bar_full + 8 * s, (stage / S::kStages) & 1,
-                                        a.wait_limit_ns, &abort_flag)) {
+            const int s = stage % NS;
+            if (!dev::mbar_wait_bounded(bar_full + 8 * s, (stage / NS) & 1, a.wait_limit_ns,
+                                        abort_flag)) {
                 ok = false;
                 break;
             }
-            if (pg % tgc == tg) {
+            if (has_rows && pg % tgc == tg) {
                 const int valid = (pg == it.num_pages - 1) ? it.last_valid : kPageSize;
-                page_step<D>(k_page(s), v_page(s), valid, qa, st, a.scale_log2, lane);
+                page_step<D>(k_page(s), k_page(s) + S::kPageBytes, valid, qa, st, a.scale_log2,
+                             lane);
             }
             __syncwarp();
             if (lane == 0) dev::mbar_arrive(bar_empty + 8 * s);
         }
-        if (!ok && lane == 0 && !abort_flag) {
-            abort_flag = 1;
+        if (!ok && lane == 0 && !*abort_flag) {
+            *abort_flag = 1;
             dev::record_error(a.err, PARASON_ETIMEOUT, kSiteConsumerFull);
         }
         // one decision for all consumer warps, whatever the producer does meanwhile
-        if (dev::bar_sync_or<kConsumerThreads>(1, !ok || abort_flag)) break;
+        if (dev::bar_sync_or<kConsumerThreads>(1, !ok || *abort_flag)) break;
 
-        write_partials<D>(a, it, st, tgc, rg, warp, lane, sc_o, sc_ml);
-
-        // ------------------------------- count this item into its branches
-        __threadfence();
-        dev::bar_sync<kConsumerThreads>(1);
-        if (tid == 0) {
-            int n = 0;
-            const int pos_lo = it.row0 / a.group;
-            const int pos_hi = (it.row0 + it.nrows - 1) / a.group;
-            for (int pos = pos_lo; pos <= pos_hi; ++pos) {
-                const int b = a.dfs_leaf[it.leaf_lo + pos];
-                const int idx = b * a.num_kv_heads + it.kv_head;
-                if (atomicAdd(a.counters + idx, 1) == a.targets[idx] - 1) {
-                    a.counters[idx] = 0;           // ready for the next decode call
-                    merge_list[n++] = b;
-                }
-            }
-            __threadfence();
-            merge_count = n;
+        if (tgc == 1) {
+            if (has_rows) store_warp_partials<D>(a, it, st, rg, lane);
+            continue;
         }
-        dev::bar_sync<kConsumerThreads>(1);
-        for (int m = 0; m < merge_count; ++m)
-            dev::merge_branch_head<D, kConsumerThreads>(a, merge_list[m], it.kv_head, tid, scratch);
+        // combine the token-group warps of each row group, one column half at a time
+        st.l[0] += __shfl_xor_sync(0xffffffffu, st.l[0], 1);
+        st.l[0] += __shfl_xor_sync(0xffffffffu, st.l[0], 2);
+        st.l[1] += __shfl_xor_sync(0xffffffffu, st.l[1], 1);
+        st.l[1] += __shfl_xor_sync(0xffffffffu, st.l[1], 2);
+        if (tig == 0) {
+            sc_ml[warp * 16 + gid] = make_float2(st.m[0], st.l[0]);
+            sc_ml[warp * 16 + gid + 8] = make_float2(st.m[1], st.l[1]);
+        }
+        constexpr int kVec = S::kHalf / 4;
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            float *wo = sc_o + warp * 16 * S::kScratchStride;
+#pragma unroll
+            for (int dt = 0; dt < D / 16; ++dt) {
+                const int c = dt * 8 + 2 * tig;
+                const int src = half * (D / 16) + dt;
+                *reinterpret_cast<float2 *>(wo + gid * S::kScratchStride + c) =
+                    make_float2(st.o[src][0], st.o[src][1]);
+                *reinterpret_cast<float2 *>(wo + (gid + 8) * S::kScratchStride + c) =
+                    make_float2(st.o[src][2], st.o[src][3]);
+            }
+            dev::bar_sync<kConsumerThreads>(1);
+            for (int idx = tid; idx < it.nrows * kVec; idx += kConsumerThreads) {
+                const int r = idx / kVec, c4 = idx % kVec;
+                const int grp = r >> 4, rr = r & 15;
+                float M = -INFINITY;
+                for (int w = 0; w < tgc; ++w) M = fmaxf(M, sc_ml[(grp * tgc + w) * 16 + rr].x);
+                float L = 0.f;
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int w = 0; w < tgc; ++w) {
+                    const int ww = grp * tgc + w;
+                    const float2 ml = sc_ml[ww * 16 + rr];
+                    const float sc = dev::fast_exp2(ml.x - M);
+                    L += sc * ml.y;
+                    const float4 v = *reinterpret_cast<const float4 *>(
+                        sc_o + (ww * 16 + rr) * S::kScratchStride + 4 * c4);
+                    acc.x += sc * v.x;
+                    acc.y += sc * v.y;
+                    acc.z += sc * v.z;
+                    acc.w += sc * v.w;
+                }
+                const int64_t slot = static_cast<int64_t>(it.slot_base) + r;
+                *reinterpret_cast<float4 *>(a.part_o + slot * D + half * S::kHalf + 4 * c4) = acc;
+                if (half == 0 && c4 == 0) a.part_ml[slot] = make_float2(M, L);
+            }
+            dev::bar_sync<kConsumerThreads>(1);
+        }
     }
 }
 
-// Shared memory and carveout are set once per device; returns the number of
-// CTAs the hardware keeps resident per SM (the persistent grid's width).
+// One CTA per SM: 9 warps leave at most 168 registers per thread (three warps
+// on one sub-partition of 16K registers).
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
+                     const __grid_constant__ CUtensorMap tmap_v, const AttnArgs a) {
+    using S = Shape<D>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    const uint32_t ring = dev::smem_addr(smem);
+    const uint32_t bars = dev::smem_addr(smem + S::kBodyBytes);
+    __shared__ int abort_flag;
+    const bool wide = static_cast<int>(blockIdx.x) < a.num_wide_ctas;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        abort_flag = 0;
+        if (wide) {
+            for (int s = 0; s < S::kWideStages; ++s) {
+                dev::mbar_init(bars + 8 * s, 1);
+                dev::mbar_init(bars + 8 * (S::kWideStages + s), kConsumerWarps);
+            }
+        } else {
+            for (int s = 0; s < S::kNarrowBars; ++s) dev::mbar_init(bars + 8 * s, 1);
+        }
+        dev::fence_mbar_init();
+        dev::prefetch_tensormap(&tmap_k);
+        dev::prefetch_tensormap(&tmap_v);
+    }
+    __syncthreads();
+    // let the merge grid launch now; it waits for this grid to complete
+    if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+    if (wide) {
+        prefix_cta<D>(&tmap_k, &tmap_v, a, smem, ring, bars, warp, lane, &abort_flag);
+    } else if (warp < kConsumerWarps) {
+        suffix_warp<D>(&tmap_k, &tmap_v, a, ring, bars, warp, lane);
+    }
+}
+
+// Shared memory and carveout are set once per device; reports the number of
+// CTAs that fit per SM (the persistent grid needs one).
 template <int D>
 cudaError_t configure(int *ctas_per_sm) {
-    using S = Bf16Shape<D>;
+    using S = Shape<D>;
     static int configured_device = -1;
     static int resident = 0;
     int dev = 0;
@@ -451,7 +564,7 @@ cudaError_t configure(int *ctas_per_sm) {
 template <int D>
 cudaError_t launch(const AttnArgs &a, const CUtensorMap &tk, const CUtensorMap &tv,
                    cudaStream_t stream) {
-    using S = Bf16Shape<D>;
+    using S = Shape<D>;
     cudaError_t e = configure<D>(nullptr);
     if (e != cudaSuccess) return e;
     attn_bf16_kernel<D><<<a.num_ctas, kThreads, S::kSmemBytes, stream>>>(tk, tv, a);
@@ -468,7 +581,7 @@ cudaError_t attn_bf16_ctas_per_sm(int head_dim, int *ctas_per_sm) {
 
 cudaError_t launch_attn_bf16(const AttnArgs &a, const CUtensorMap &tk, const CUtensorMap &tv,
                              int head_dim, cudaStream_t stream) {
-    if (a.num_items <= 0) return cudaSuccess;
+    if (a.num_items <= 0 || a.num_ctas <= 0) return cudaSuccess;
     if (head_dim == 128) return launch<128>(a, tk, tv, stream);
     if (head_dim == 64) return launch<64>(a, tk, tv, stream);
     return cudaErrorNotSupported;

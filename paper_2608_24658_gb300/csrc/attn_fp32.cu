@@ -95,7 +95,7 @@ __global__ void __launch_bounds__(kWarps * 32)
             L += s * sc_ml[w][r].y;
             acc += s * sc_o[w][r][c];
         }
-        const int64_t slot = static_cast<int64_t>(it.slot_base) + it.row0 + r;
+        const int64_t slot = static_cast<int64_t>(it.slot_base) + r;
         a.part_o[slot * D + c] = acc;
         if (c == 0) a.part_ml[slot] = make_float2(M, L);
     }

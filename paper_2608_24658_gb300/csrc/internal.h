@@ -9,27 +9,28 @@
 
 namespace parason {
 
-// One unit of attention work: a tile of up to 64 query rows of one tree node
-// and one kv head, against one contiguous chunk of that node's pages.
+// One unit of attention work: a tile of query rows of one tree node and one
+// kv head, against a run of that node's pages.
 //
 // The rows of node n are its branches in DFS order times the g = H_q/H_kv
 // q heads of the kv head: node row r is branch dfs_leaf[leaf_lo + r / g],
-// q head kv_head * g + r % g.  The item writes the partial result (o, m, l)
-// of node row r to partial slot slot_base + r.
+// q head kv_head * g + r % g.  Tiles start at multiples of g.  The item
+// writes the partial result (o, m, l) of its row row0 + i to partial slot
+// slot_base + i.
 struct WorkItem {
-    int32_t page_pos;    // index in page_ids of the chunk's first page
-    int32_t num_pages;   // pages in the chunk (>= 1)
-    int32_t last_valid;  // valid tokens in the chunk's last page (1..16)
+    int32_t page_pos;    // index in page_ids of the item's first page
+    int32_t num_pages;   // pages in the item (>= 1)
+    int32_t last_valid;  // valid tokens in the item's last page (1..16)
     int32_t leaf_lo;     // DFS position of the node's first branch
     int32_t row0;        // first node row of this tile
-    int32_t nrows;       // rows in this tile (1..64)
+    int32_t nrows;       // rows in this tile (1..128)
     int32_t kv_head;
-    int32_t slot_base;   // partial slot of node row 0 for (node, chunk, kv head)
+    int32_t slot_base;   // partial slot of the tile's first row
 };
 static_assert(sizeof(WorkItem) == 32, "WorkItem is a 32-byte device record");
 
 constexpr int kPageSize = 16;
-constexpr int kMaxTileRows = 64;
+constexpr int kMaxTileRows = 128;
 constexpr int kErrWords = 4;            // device error record: code, block, site, aux
 
 // Where a bounded wait gave up (error record word 2).
@@ -56,34 +57,29 @@ struct AttnArgs {
     int32_t group;
     float scale_log2;       // sm_scale * log2(e): x_t = scale_log2 * <q, k_t>
 
-    // persistent schedule: CTA c runs items cta_items[cta_ptr[c] .. cta_ptr[c+1])
-    const int32_t *cta_ptr;
-    const int32_t *cta_items;
+    // persistent schedule, CSR over workers: CTAs [0, num_wide_ctas) each run
+    // one list (prefix pass); every warp w of CTA c >= num_wide_ctas runs list
+    // num_wide_ctas + (c - num_wide_ctas) * 8 + w (suffix pass)
+    const int32_t *sched_ptr;
+    const int32_t *sched_items;
+    // worker w loads the pages of its items in order; their TMA rows
+    // (page * H_kv + kv head) * 16 are stream_rows[stream_ptr[w] ...]
+    const int32_t *stream_ptr;
+    const int32_t *stream_rows;
     int32_t num_ctas;
-
-    // fused merge: the CTA whose item brings counters[b * H_kv + j] to
-    // targets[b * H_kv + j] merges branch b, kv head j into out / lse and
-    // sets the counter back to 0
-    int32_t *counters;
-    const int32_t *targets;
-    const int32_t *merge_ptr;
-    const int2 *merge_ent;
-    void *out;
-    float *lse;
-    const int32_t *empty_leaves;    // branches whose whole path is empty
-    int32_t num_empty_leaves;
-    int32_t num_leaves;
+    int32_t num_wide_ctas;
 };
 
 struct MergeArgs {
-    const int32_t *merge_ptr;   // [num_leaves + 1]
-    const int2 *merge_ent;      // (base, stride)
+    const int32_t *merge_ptr;   // [num_leaves * H_kv + 1]
+    const int32_t *merge_ent;   // first partial slot of the branch's rows
     const float *part_o;
     const float2 *part_ml;
     void *out;
     float *lse;
     int32_t num_leaves;
     int32_t num_q_heads;
+    int32_t num_kv_heads;
     int32_t group;
 };
 
@@ -97,7 +93,8 @@ cudaError_t launch_attn_fp8(const AttnArgs &a, const CUtensorMap &tmap_k,
                             const CUtensorMap &tmap_v, int head_dim, cudaStream_t stream);
 cudaError_t launch_attn_fp32(const AttnArgs &a, const float *k_pages, const float *v_pages,
                              int head_dim, cudaStream_t stream);
-cudaError_t launch_merge(const MergeArgs &a, int head_dim, int mode, cudaStream_t stream);
+cudaError_t launch_merge(const MergeArgs &a, int head_dim, int mode, bool programmatic,
+                         cudaStream_t stream);
 cudaError_t launch_lse_merge(const void *o_a, const float *lse_a, const void *o_b,
                              const float *lse_b, void *o_out, float *lse_out, int64_t rows,
                              int head_dim, int mode, cudaStream_t stream);

@@ -84,38 +84,67 @@ __device__ __forceinline__ void load_in(const void *in, int64_t off, float (&v)[
     }
 }
 
-// one warp per (branch, q head)
+// One warp per (branch, q head).  Entries are taken 32 at a time: lane e
+// loads entry e's (m, l) (one round trip for all of them), the batch's max
+// and weights come from warp reductions, then every lane accumulates its
+// D/32 columns over the batch with independent loads.  Runs as a dependent
+// grid of the attention kernel: griddepcontrol.wait returns once that grid
+// has completed and its writes are visible.
 template <int D>
 __global__ void __launch_bounds__(kMergeThreads)
     tree_merge_kernel(const MergeArgs a, bool out_bf16) {
     constexpr int N = Vec<D>::N;
     const int64_t w = (static_cast<int64_t>(blockIdx.x) * kMergeThreads + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
-    if (w >= static_cast<int64_t>(a.num_leaves) * a.num_q_heads) return;
-    const int b = static_cast<int>(w / a.num_q_heads), h = static_cast<int>(w % a.num_q_heads);
+    const bool active = w < static_cast<int64_t>(a.num_leaves) * a.num_q_heads;
+    const int b = active ? static_cast<int>(w / a.num_q_heads) : 0;
+    const int h = active ? static_cast<int>(w % a.num_q_heads) : 0;
     const int j = h / a.group, r = h % a.group;
-    const int e0 = a.merge_ptr[b], e1 = a.merge_ptr[b + 1];
+    const int64_t pair = static_cast<int64_t>(b) * a.num_kv_heads + j;
+    // the merge lists are plan data: read them while the attention grid drains
+    const int e0 = active ? a.merge_ptr[pair] : 0, e1 = active ? a.merge_ptr[pair + 1] : 0;
+    int first_slot = (e0 + lane < e1) ? a.merge_ent[e0 + lane] + r : 0;
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (!active) return;
 
-    float M = -INFINITY;
-    for (int e = e0; e < e1; ++e) {
-        const int2 ent = a.merge_ent[e];
-        const int64_t slot = static_cast<int64_t>(ent.x) + static_cast<int64_t>(j) * ent.y + r;
-        M = fmaxf(M, a.part_ml[slot].x);
-    }
-    float L = 0.f;
+    float M = -INFINITY, L = 0.f;
     float acc[N];
 #pragma unroll
     for (int i = 0; i < N; ++i) acc[i] = 0.f;
-    for (int e = e0; e < e1; ++e) {
-        const int2 ent = a.merge_ent[e];
-        const int64_t slot = static_cast<int64_t>(ent.x) + static_cast<int64_t>(j) * ent.y + r;
-        const float2 ml = a.part_ml[slot];
-        const float sc = exp2f(ml.x - M);
-        L += sc * ml.y;
-        float v[N];
-        load_f32<N>(a.part_o + slot * D + lane * N, v);
+    for (int base = e0; base < e1; base += 32) {
+        const int e = base + lane;
+        const bool valid = e < e1;
+        int slot = 0;
+        float m = -INFINITY, l = 0.f;
+        if (valid) {
+            slot = base == e0 ? first_slot : a.merge_ent[e] + r;
+            const float2 ml = a.part_ml[slot];
+            m = ml.x;
+            l = ml.y;
+        }
+        float mb = m;
 #pragma unroll
-        for (int i = 0; i < N; ++i) acc[i] += sc * v[i];
+        for (int o = 16; o > 0; o >>= 1) mb = fmaxf(mb, __shfl_xor_sync(0xffffffffu, mb, o));
+        const float Mn = fmaxf(M, mb);             // finite: the batch has a valid entry
+        const float s_old = exp2f(M - Mn);
+        const float wgt = valid ? exp2f(m - Mn) : 0.f;
+        float lw = l * wgt;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) lw += __shfl_xor_sync(0xffffffffu, lw, o);
+        L = L * s_old + lw;
+#pragma unroll
+        for (int i = 0; i < N; ++i) acc[i] *= s_old;
+        const int cnt = min(32, e1 - base);
+#pragma unroll 8
+        for (int i = 0; i < cnt; ++i) {
+            const int si = __shfl_sync(0xffffffffu, slot, i);
+            const float wi = __shfl_sync(0xffffffffu, wgt, i);
+            float v[N];
+            load_f32<N>(a.part_o + static_cast<int64_t>(si) * D + lane * N, v);
+#pragma unroll
+            for (int k = 0; k < N; ++k) acc[k] += wi * v[k];
+        }
+        M = Mn;
     }
     const bool empty = !(L > 0.f);
     const float inv = empty ? 0.f : 1.f / L;
@@ -158,18 +187,25 @@ __global__ void __launch_bounds__(kMergeThreads)
 
 }  // namespace
 
-cudaError_t launch_merge(const MergeArgs &a, int head_dim, int mode, cudaStream_t stream) {
+cudaError_t launch_merge(const MergeArgs &a, int head_dim, int mode, bool programmatic,
+                         cudaStream_t stream) {
     const int64_t warps = static_cast<int64_t>(a.num_leaves) * a.num_q_heads;
     if (warps == 0) return cudaSuccess;
     const int64_t blocks = (warps * 32 + kMergeThreads - 1) / kMergeThreads;
     const bool bf16 = mode != PARASON_FP32;
-    if (head_dim == 128)
-        tree_merge_kernel<128><<<static_cast<unsigned>(blocks), kMergeThreads, 0, stream>>>(a, bf16);
-    else if (head_dim == 64)
-        tree_merge_kernel<64><<<static_cast<unsigned>(blocks), kMergeThreads, 0, stream>>>(a, bf16);
-    else
-        return cudaErrorNotSupported;
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(blocks));
+    cfg.blockDim = dim3(kMergeThreads);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = programmatic ? 1 : 0;
+    if (head_dim == 128) return cudaLaunchKernelEx(&cfg, tree_merge_kernel<128>, a, bf16);
+    if (head_dim == 64) return cudaLaunchKernelEx(&cfg, tree_merge_kernel<64>, a, bf16);
+    return cudaErrorNotSupported;
 }
 
 cudaError_t launch_lse_merge(const void *o_a, const float *lse_a, const void *o_b,

@@ -29,26 +29,32 @@ using parason::WorkItem;
 
 namespace {
 
-constexpr int kMinChunkPages = 8;
-constexpr int kItemsPerSm = 8;          // 2 persistent CTAs x ~4 items each
-constexpr int kDefaultCtasPerSm = 2;    // persistent attention CTAs per SM (host plans)
+constexpr int kNarrowRows = 16;         // nodes with at most this many rows: suffix pass
+constexpr int kNarrowWarps = 8;         // autonomous warps per suffix-pass CTA
+constexpr int kMinPiecePages = 4;       // no split leaves a piece shorter than this
+constexpr int kFp32ChunkPages = 32;
+constexpr double kWideGroupPageCost = 1.0;   // one 16-row group of one page, in suffix pages
 constexpr int64_t kDefaultWaitNs = 2000000000LL;
 constexpr size_t kAlign = 256;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// Relative time of an item: its pages, weighted by the MMA work of wide tiles
-// (every consumer warp of a 64-row tile reads every page).
-int64_t item_cost(const WorkItem &it) {
-    const int64_t rgc = it.nrows <= 16 ? 1 : (it.nrows <= 32 ? 2 : 4);
-    return static_cast<int64_t>(it.num_pages) * (3 + rgc);
+// Time of one page of a prefix-pass tile relative to one page of the suffix
+// pass on the same SM.  The suffix pass runs 8 pages at once (one per warp);
+// a prefix tile runs one 16-row MMA group of the page per warp, so a page of
+// a tile with G groups costs G suffix pages of warp time.
+double wide_page_cost(int32_t rows) {
+    const double groups = (rows + 15) / 16;
+    return std::max(1.0, groups * kWideGroupPageCost);
 }
 
-int tile_rows_for(int32_t rows, int32_t mode) {
-    if (mode == PARASON_FP32) return 16;
-    if (rows <= 16) return 16;
-    if (rows <= 32) return 32;
-    return 64;
+// Rows of one tile: a multiple of g (so a branch's rows never straddle two
+// tiles) of at most 16 (fp32 mode and the suffix pass) or 128 (prefix pass).
+int32_t tile_rows_for(int32_t rows, int32_t g, int32_t mode) {
+    const int32_t cap = (mode == PARASON_FP32 || rows <= kNarrowRows) ? 16 : 128;
+    if (g > cap) return 0;
+    const int32_t t = (cap / g) * g;
+    return std::min(t, ((rows + g - 1) / g) * g);
 }
 
 }  // namespace
@@ -60,17 +66,18 @@ struct parason_plan_s {
     int32_t num_leaves = 0;
     int64_t num_phys = 0;
     int32_t num_sms = 152;
-    int32_t ctas_per_sm = kDefaultCtasPerSm;
-    int32_t chunk_pages = kMinChunkPages;
+    int32_t chunk_pages = kMinPiecePages;
     std::vector<WorkItem> items;
     std::vector<int32_t> page_ids;
     std::vector<int32_t> dfs_leaf;
     std::vector<int32_t> merge_ptr;
-    std::vector<int32_t> merge_ent;   // pairs (base, stride)
-    std::vector<int32_t> cta_ptr;     // persistent schedule (CSR over CTAs)
-    std::vector<int32_t> cta_items;
-    std::vector<int32_t> targets;     // items per (branch, kv head)
-    std::vector<int32_t> empty_leaves;
+    std::vector<int32_t> merge_ent;   // first partial slot of the branch's rows
+    std::vector<int32_t> sched_ptr;   // persistent schedule, CSR over workers:
+    std::vector<int32_t> sched_items; // wide CTAs first, then narrow warps
+    std::vector<int32_t> stream_ptr;  // per worker: start of its page stream
+    std::vector<int32_t> stream_rows; // TMA row of every page, worker by worker
+    int32_t num_ctas = 0;
+    int32_t num_wide_ctas = 0;
     int64_t num_slots = 0;
     int64_t unique_tokens = 0;
     int64_t path_tokens = 0;
@@ -83,12 +90,11 @@ struct parason_plan_s {
     int32_t *d_page_ids = nullptr;
     int32_t *d_dfs_leaf = nullptr;
     int32_t *d_merge_ptr = nullptr;
-    int2 *d_merge_ent = nullptr;
-    int32_t *d_cta_ptr = nullptr;
-    int32_t *d_cta_items = nullptr;
-    int32_t *d_counters = nullptr;
-    int32_t *d_targets = nullptr;
-    int32_t *d_empty = nullptr;
+    int32_t *d_merge_ent = nullptr;
+    int32_t *d_sched_ptr = nullptr;
+    int32_t *d_sched_items = nullptr;
+    int32_t *d_stream_ptr = nullptr;
+    int32_t *d_stream_rows = nullptr;
     int32_t *d_err = nullptr;
     uint32_t debug_flags = 0;
     int64_t wait_limit_ns = kDefaultWaitNs;
@@ -129,7 +135,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                           const int32_t *parent, const int32_t *node_len,
                           const int32_t *node_page_ptr, const int32_t *page_ids,
                           int32_t num_leaves, const int32_t *leaf_node,
-                          int64_t num_phys, int32_t num_sms, int32_t ctas_per_sm) {
+                          int64_t num_phys, int32_t num_sms) {
     parason_status st = validate_config(cfg);
     if (st != PARASON_OK) return st;
     if (num_nodes < 0 || num_leaves < 0 || num_phys < 0) return PARASON_EINVAL;
@@ -145,7 +151,6 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     p->num_leaves = num_leaves;
     p->num_phys = num_phys;
     p->num_sms = num_sms > 0 ? num_sms : 152;
-    p->ctas_per_sm = ctas_per_sm > 0 ? ctas_per_sm : kDefaultCtasPerSm;
 
     // tree and page table
     if (num_nodes > 0 && node_page_ptr[0] != 0) return PARASON_EINVAL;
@@ -210,131 +215,192 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     p->dfs_leaf.assign(num_leaves, -1);
     for (int32_t b = 0; b < num_leaves; ++b) p->dfs_leaf[lo[leaf_node[b]]] = b;
 
+    // ------------------------------------------------------------------
     // work decomposition
+    //
+    // A run is (node, kv head, row tile) over all of the node's pages.  Runs
+    // are cut into items along pages; every item owns `nrows` consecutive
+    // partial slots.  Row tiles start at multiples of g, so each branch's g
+    // rows of a node sit in one tile.
     const int32_t mode = cfg->mode;
-    int64_t units = 0;
+    struct Run {
+        int32_t node, head, row0, nrows;
+        int64_t pages;
+        double cost_per_page;
+        bool wide;
+    };
+    std::vector<Run> runs;
+    int64_t narrow_pages = 0;
+    double wide_cost = 0.0;
     for (int32_t n = 0; n < num_nodes; ++n) {
         if (cnt[n] == 0 || node_len[n] == 0) continue;
-        const int64_t R = cnt[n] * g;
-        const int rt = tile_rows_for(static_cast<int32_t>(std::min<int64_t>(R, 1 << 20)), mode);
-        units += static_cast<int64_t>(node_page_ptr[n + 1] - node_page_ptr[n]) * H_kv *
-                 ((R + rt - 1) / rt);
         p->unique_tokens += node_len[n];
-    }
-    const int64_t target = static_cast<int64_t>(p->num_sms) * kItemsPerSm;
-    int64_t chunk = target > 0 ? (units + target - 1) / target : units;
-    chunk = std::max<int64_t>(chunk, kMinChunkPages);
-    p->chunk_pages = static_cast<int32_t>(std::min<int64_t>(chunk, INT32_MAX));
-
-    std::vector<int64_t> slot_first(num_nodes, -1);
-    std::vector<int32_t> nchunks(num_nodes, 0);
-    int64_t slots = 0;
-    std::vector<std::pair<int64_t, WorkItem>> keyed;
-    for (int32_t n = 0; n < num_nodes; ++n) {
-        if (cnt[n] == 0 || node_len[n] == 0) continue;
         const int64_t R = cnt[n] * g;
         if (R > INT32_MAX / 4) return PARASON_EUNSUPPORTED;
-        const int rt = tile_rows_for(static_cast<int32_t>(R), mode);
-        const int32_t P = node_page_ptr[n + 1] - node_page_ptr[n];
-        const int32_t nc = static_cast<int32_t>((P + chunk - 1) / chunk);
-        const int32_t base = P / nc, rem = P % nc;
-        nchunks[n] = nc;
-        slot_first[n] = slots;
-        int32_t pg = 0;
-        for (int32_t c = 0; c < nc; ++c) {
-            const int32_t np = base + (c < rem ? 1 : 0);
-            const bool has_last = (pg + np == P);
-            const int32_t last_valid =
-                has_last ? node_len[n] - (P - 1) * parason::kPageSize : parason::kPageSize;
-            for (int32_t j = 0; j < H_kv; ++j) {
-                const int64_t sb = slots + static_cast<int64_t>(c) * H_kv * R +
-                                   static_cast<int64_t>(j) * R;
-                for (int64_t r0 = 0; r0 < R; r0 += rt) {
-                    WorkItem it;
-                    it.page_pos = node_page_ptr[n] + pg;
-                    it.num_pages = np;
-                    it.last_valid = last_valid;
-                    it.leaf_lo = static_cast<int32_t>(lo[n]);
-                    it.row0 = static_cast<int32_t>(r0);
-                    it.nrows = static_cast<int32_t>(std::min<int64_t>(rt, R - r0));
-                    it.kv_head = j;
-                    if (sb > INT32_MAX) return PARASON_EUNSUPPORTED;
-                    it.slot_base = static_cast<int32_t>(sb);
-                    keyed.emplace_back(item_cost(it), it);
-                }
+        const int64_t P = node_page_ptr[n + 1] - node_page_ptr[n];
+        const int32_t rt = tile_rows_for(static_cast<int32_t>(std::min<int64_t>(R, 1 << 20)), g, mode);
+        if (rt <= 0) return PARASON_EUNSUPPORTED;
+        const bool wide = mode != PARASON_FP32 && R > kNarrowRows;
+        for (int32_t j = 0; j < H_kv; ++j)
+            for (int64_t r0 = 0; r0 < R; r0 += rt) {
+                Run run;
+                run.node = n;
+                run.head = j;
+                run.row0 = static_cast<int32_t>(r0);
+                run.nrows = static_cast<int32_t>(std::min<int64_t>(rt, R - r0));
+                run.pages = P;
+                run.wide = wide;
+                run.cost_per_page = wide ? wide_page_cost(run.nrows) : 1.0;
+                if (wide)
+                    wide_cost += run.cost_per_page * static_cast<double>(P);
+                else
+                    narrow_pages += P;
+                runs.push_back(run);
             }
-            pg += np;
-        }
-        slots += static_cast<int64_t>(nc) * H_kv * R;
-        if (slots > INT32_MAX) return PARASON_EUNSUPPORTED;
     }
-    // longest items first, so the tail of the grid is made of short ones
-    std::stable_sort(keyed.begin(), keyed.end(),
-                     [](const auto &a, const auto &b) { return a.first > b.first; });
+
+    // workers: wide CTAs (prefix pass) and narrow warps (suffix pass) of the
+    // persistent kernel; the fp32 kernel runs one item per CTA instead
+    int32_t n_wide = 0, n_narrow_ctas = 0;
+    if (mode != PARASON_FP32) {
+        const int32_t S = p->num_sms;
+        const double narrow_cost = static_cast<double>(narrow_pages);
+        // each role gets at least one CTA; the grid may exceed the SM count
+        // (CTAs of the persistent kernel never wait on one another)
+        if (wide_cost > 0 && narrow_cost > 0) {
+            n_wide = static_cast<int32_t>(std::lround(S * wide_cost / (wide_cost + narrow_cost)));
+            n_wide = std::min(std::max(n_wide, 1), std::max(S - 1, 1));
+        } else if (wide_cost > 0) {
+            n_wide = S;
+        }
+        n_narrow_ctas = narrow_cost > 0 ? std::max(S - n_wide, 1) : 0;
+    }
+    p->num_wide_ctas = n_wide;
+    p->num_ctas = n_wide + n_narrow_ctas;
+    const int64_t n_narrow_workers = static_cast<int64_t>(n_narrow_ctas) * kNarrowWarps;
+
+    // balanced contiguous partition of the runs of one role over its workers:
+    // worker k gets the pages whose cumulative cost falls in [k T/W, (k+1) T/W)
     p->items.clear();
-    p->items.reserve(keyed.size());
-    for (auto &kv : keyed) p->items.push_back(kv.second);
+    std::vector<int32_t> worker_of_item;
+    std::vector<int64_t> slot_of_item;
+    int64_t slots = 0;
+    auto emit = [&](const Run &run, int64_t pg0, int64_t np, int32_t worker) -> bool {
+        WorkItem it;
+        const int64_t P = run.pages;
+        it.page_pos = node_page_ptr[run.node] + static_cast<int32_t>(pg0);
+        it.num_pages = static_cast<int32_t>(np);
+        it.last_valid = (pg0 + np == P)
+                            ? node_len[run.node] - static_cast<int32_t>(P - 1) * parason::kPageSize
+                            : parason::kPageSize;
+        it.leaf_lo = static_cast<int32_t>(lo[run.node]);
+        it.row0 = run.row0;
+        it.nrows = run.nrows;
+        it.kv_head = run.head;
+        if (slots + run.nrows > INT32_MAX) return false;
+        it.slot_base = static_cast<int32_t>(slots);
+        slots += run.nrows;
+        p->items.push_back(it);
+        worker_of_item.push_back(worker);
+        return true;
+    };
+    auto partition = [&](bool wide_role, int64_t workers, int64_t worker0, int64_t min_chunk) -> bool {
+        double total = 0.0;
+        for (const Run &r : runs)
+            if (r.wide == wide_role) total += r.cost_per_page * static_cast<double>(r.pages);
+        if (total <= 0.0) return true;
+        const double share = total / static_cast<double>(std::max<int64_t>(workers, 1));
+        double acc = 0.0;                       // cost before the current page
+        for (const Run &r : runs) {
+            if (r.wide != wide_role) continue;
+            int64_t pg = 0;
+            while (pg < r.pages) {
+                int64_t k = std::min<int64_t>(workers - 1, static_cast<int64_t>(acc / share));
+                // pages of this run that fit before worker k's share ends
+                const int64_t left = r.pages - pg;
+                int64_t np = left;
+                if (k + 1 < workers) {
+                    const double fit = std::ceil(((k + 1) * share - acc) / r.cost_per_page - 1e-9);
+                    if (fit < static_cast<double>(left)) np = std::max<int64_t>(1, static_cast<int64_t>(fit));
+                }
+                // avoid crumbs: a piece shorter than min_chunk joins its neighbour
+                if (r.pages - (pg + np) < min_chunk) np = r.pages - pg;
+                np = std::min<int64_t>(np, r.pages - pg);
+                if (!emit(r, pg, np, static_cast<int32_t>(worker0 + k))) return false;
+                acc += r.cost_per_page * static_cast<double>(np);
+                pg += np;
+            }
+        }
+        return true;
+    };
+    if (mode == PARASON_FP32) {
+        // one item per CTA: chunks of about kFp32ChunkPages pages
+        for (const Run &r : runs) {
+            const int64_t nc = std::max<int64_t>(1, (r.pages + kFp32ChunkPages - 1) / kFp32ChunkPages);
+            const int64_t base = r.pages / nc, rem = r.pages % nc;
+            int64_t pg = 0;
+            for (int64_t c = 0; c < nc; ++c) {
+                const int64_t np = base + (c < rem ? 1 : 0);
+                if (!emit(r, pg, np, 0)) return PARASON_EUNSUPPORTED;
+                pg += np;
+            }
+        }
+    } else {
+        if (!partition(true, n_wide, 0, kMinPiecePages)) return PARASON_EUNSUPPORTED;
+        if (!partition(false, n_narrow_workers, n_wide, kMinPiecePages)) return PARASON_EUNSUPPORTED;
+    }
     if (p->items.size() > static_cast<size_t>(INT32_MAX)) return PARASON_EUNSUPPORTED;
     p->num_slots = slots;
 
-    // merge lists: every chunk of every node on the branch's path
-    p->merge_ptr.assign(num_leaves + 1, 0);
-    p->merge_ent.clear();
-    std::vector<int32_t> path;
-    for (int32_t b = 0; b < num_leaves; ++b) {
-        path.clear();
-        for (int32_t n = leaf_node[b]; n >= 0; n = parent[n]) path.push_back(n);
-        std::reverse(path.begin(), path.end());
-        const int64_t pos = lo[leaf_node[b]];
-        for (int32_t n : path) {
-            p->path_tokens += node_len[n];
-            if (nchunks[n] == 0) continue;
-            const int64_t R = cnt[n] * g;
-            for (int32_t c = 0; c < nchunks[n]; ++c) {
-                const int64_t base =
-                    slot_first[n] + static_cast<int64_t>(c) * H_kv * R + (pos - lo[n]) * g;
-                p->merge_ent.push_back(static_cast<int32_t>(base));
-                p->merge_ent.push_back(static_cast<int32_t>(R));
-            }
+    // schedule: worker lists in item order (each worker's items are one
+    // contiguous stretch of the partition)
+    const int64_t n_workers = mode == PARASON_FP32 ? 0 : n_wide + n_narrow_workers;
+    p->sched_ptr.assign(static_cast<size_t>(n_workers) + 1, 0);
+    p->sched_items.clear();
+    if (n_workers > 0) {
+        std::vector<int32_t> count(static_cast<size_t>(n_workers), 0);
+        for (int32_t w : worker_of_item) count[w]++;
+        for (int64_t w = 0; w < n_workers; ++w) p->sched_ptr[w + 1] = p->sched_ptr[w] + count[w];
+        p->sched_items.assign(p->items.size(), 0);
+        std::vector<int32_t> fill(p->sched_ptr.begin(), p->sched_ptr.end() - 1);
+        for (size_t i = 0; i < p->items.size(); ++i)
+            p->sched_items[fill[worker_of_item[i]]++] = static_cast<int32_t>(i);
+    }
+    // page streams: the TMA row (page * H_kv + kv head) * 16 of every page a
+    // worker loads, in the order it loads them
+    p->stream_ptr.assign(static_cast<size_t>(n_workers) + 1, 0);
+    p->stream_rows.clear();
+    for (int64_t w = 0; w < n_workers; ++w) {
+        for (int32_t k = p->sched_ptr[w]; k < p->sched_ptr[w + 1]; ++k) {
+            const WorkItem &it = p->items[p->sched_items[k]];
+            for (int32_t pg = 0; pg < it.num_pages; ++pg)
+                p->stream_rows.push_back((page_ids[it.page_pos + pg] * H_kv + it.kv_head) *
+                                         parason::kPageSize);
         }
-        p->merge_ptr[b + 1] = static_cast<int32_t>(p->merge_ent.size() / 2);
+        if (p->stream_rows.size() > static_cast<size_t>(INT32_MAX)) return PARASON_EUNSUPPORTED;
+        p->stream_ptr[w + 1] = static_cast<int32_t>(p->stream_rows.size());
     }
 
-    // items that feed each (branch, kv head), and branches with no item at all
-    p->targets.assign(static_cast<size_t>(num_leaves) * H_kv, 0);
+    // merge lists per (branch, kv head): the first of the branch's g partial
+    // slots in every item, on the branch's path, that covers its rows
+    std::vector<std::vector<int32_t>> ent(static_cast<size_t>(num_leaves) * H_kv);
     for (const WorkItem &it : p->items) {
         const int32_t pos_lo = it.row0 / g, pos_hi = (it.row0 + it.nrows - 1) / g;
         for (int32_t pos = pos_lo; pos <= pos_hi; ++pos) {
             const int32_t b = p->dfs_leaf[it.leaf_lo + pos];
-            p->targets[static_cast<size_t>(b) * H_kv + it.kv_head]++;
+            ent[static_cast<size_t>(b) * H_kv + it.kv_head].push_back(it.slot_base + pos * g -
+                                                                       it.row0);
         }
     }
-    p->empty_leaves.clear();
+    p->merge_ptr.assign(static_cast<size_t>(num_leaves) * H_kv + 1, 0);
+    p->merge_ent.clear();
+    for (size_t k = 0; k < ent.size(); ++k) {
+        p->merge_ent.insert(p->merge_ent.end(), ent[k].begin(), ent[k].end());
+        if (p->merge_ent.size() > static_cast<size_t>(INT32_MAX)) return PARASON_EUNSUPPORTED;
+        p->merge_ptr[k + 1] = static_cast<int32_t>(p->merge_ent.size());
+    }
     for (int32_t b = 0; b < num_leaves; ++b)
-        if (p->targets[static_cast<size_t>(b) * H_kv] == 0) p->empty_leaves.push_back(b);
-
-    // persistent schedule: longest item first onto the least loaded CTA
-    const int32_t n_items = static_cast<int32_t>(p->items.size());
-    const int32_t n_ctas =
-        std::max<int32_t>(1, std::min<int32_t>(p->num_sms * p->ctas_per_sm, n_items));
-    std::vector<std::vector<int32_t>> per(n_ctas);
-    {
-        using Load = std::pair<int64_t, int32_t>;
-        std::priority_queue<Load, std::vector<Load>, std::greater<Load>> heap;
-        for (int32_t c = 0; c < n_ctas; ++c) heap.emplace(0, c);
-        for (int32_t i = 0; i < n_items; ++i) {     // items are sorted by cost, longest first
-            Load l = heap.top();
-            heap.pop();
-            per[l.second].push_back(i);
-            heap.emplace(l.first + item_cost(p->items[i]), l.second);
-        }
-    }
-    p->cta_ptr.assign(n_ctas + 1, 0);
-    p->cta_items.clear();
-    for (int32_t c = 0; c < n_ctas; ++c) {
-        p->cta_items.insert(p->cta_items.end(), per[c].begin(), per[c].end());
-        p->cta_ptr[c + 1] = static_cast<int32_t>(p->cta_items.size());
-    }
+        for (int32_t n = leaf_node[b]; n >= 0; n = parent[n]) p->path_tokens += node_len[n];
     return PARASON_OK;
 }
 
@@ -349,16 +415,17 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     const size_t n_dfs = p->dfs_leaf.size() * sizeof(int32_t);
     const size_t n_mptr = p->merge_ptr.size() * sizeof(int32_t);
     const size_t n_ment = p->merge_ent.size() * sizeof(int32_t);
-    const size_t n_cptr = p->cta_ptr.size() * sizeof(int32_t);
-    const size_t n_citems = p->cta_items.size() * sizeof(int32_t);
-    const size_t n_targets = p->targets.size() * sizeof(int32_t);
-    const size_t n_empty = p->empty_leaves.size() * sizeof(int32_t);
+    const size_t n_sptr = p->sched_ptr.size() * sizeof(int32_t);
+    const size_t n_sitems = p->sched_items.size() * sizeof(int32_t);
+    const size_t n_stptr = p->stream_ptr.size() * sizeof(int32_t);
+    // page streams are read 32 entries past their end by whole warps: pad
+    const size_t n_strows = (p->stream_rows.size() + 32) * sizeof(int32_t);
     const size_t n_err = parason::kErrWords * sizeof(int32_t);
-    constexpr int kArrays = 11;
+    constexpr int kArrays = 10;
     size_t off[kArrays], total = 0;
-    // the last two (counters, error record) are zero-filled, not copied
-    const size_t sizes[kArrays] = {n_items, n_pages,   n_dfs,    n_mptr,    n_ment, n_cptr,
-                                   n_citems, n_targets, n_empty, n_targets, n_err};
+    // the last one (error record) is zero-filled, not copied
+    const size_t sizes[kArrays] = {n_items, n_pages,  n_dfs,   n_mptr,   n_ment,
+                                   n_sptr,  n_sitems, n_stptr, n_strows, n_err};
     for (int i = 0; i < kArrays; ++i) {
         off[i] = total;
         total = align_up(total + std::max<size_t>(sizes[i], 4), kAlign);
@@ -373,21 +440,20 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     p->d_page_ids = reinterpret_cast<int32_t *>(base + off[1]);
     p->d_dfs_leaf = reinterpret_cast<int32_t *>(base + off[2]);
     p->d_merge_ptr = reinterpret_cast<int32_t *>(base + off[3]);
-    p->d_merge_ent = reinterpret_cast<int2 *>(base + off[4]);
-    p->d_cta_ptr = reinterpret_cast<int32_t *>(base + off[5]);
-    p->d_cta_items = reinterpret_cast<int32_t *>(base + off[6]);
-    p->d_targets = reinterpret_cast<int32_t *>(base + off[7]);
-    p->d_empty = reinterpret_cast<int32_t *>(base + off[8]);
-    p->d_counters = reinterpret_cast<int32_t *>(base + off[9]);
-    p->d_err = reinterpret_cast<int32_t *>(base + off[10]);
+    p->d_merge_ent = reinterpret_cast<int32_t *>(base + off[4]);
+    p->d_sched_ptr = reinterpret_cast<int32_t *>(base + off[5]);
+    p->d_sched_items = reinterpret_cast<int32_t *>(base + off[6]);
+    p->d_stream_ptr = reinterpret_cast<int32_t *>(base + off[7]);
+    p->d_stream_rows = reinterpret_cast<int32_t *>(base + off[8]);
+    p->d_err = reinterpret_cast<int32_t *>(base + off[9]);
     const void *src[9] = {p->items.data(),     p->page_ids.data(),  p->dfs_leaf.data(),
-                          p->merge_ptr.data(), p->merge_ent.data(), p->cta_ptr.data(),
-                          p->cta_items.data(), p->targets.data(),   p->empty_leaves.data()};
-    if (n_targets > 0 && cudaMemsetAsync(p->d_counters, 0, n_targets, stream) != cudaSuccess)
-        return PARASON_ECUDA;
+                          p->merge_ptr.data(), p->merge_ent.data(), p->sched_ptr.data(),
+                          p->sched_items.data(), p->stream_ptr.data(), p->stream_rows.data()};
+    const size_t copy[9] = {n_items, n_pages, n_dfs, n_mptr, n_ment, n_sptr, n_sitems, n_stptr,
+                            p->stream_rows.size() * sizeof(int32_t)};
     for (int i = 0; i < 9; ++i) {
-        if (sizes[i] == 0) continue;
-        if (cudaMemcpyAsync(base + off[i], src[i], sizes[i], cudaMemcpyHostToDevice, stream) !=
+        if (copy[i] == 0) continue;
+        if (cudaMemcpyAsync(base + off[i], src[i], copy[i], cudaMemcpyHostToDevice, stream) !=
             cudaSuccess)
             return PARASON_ECUDA;
     }
@@ -416,7 +482,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 // KV pool [P, H_kv, 16, d] seen as rows of 128-byte segments:
 //   dim0 = 128 bytes of one segment (64 bf16 or 128 e4m3), dim1 = segment in
 //   the token row, dim2 = token row (page * H_kv + kv_head) * 16 + slot.
-// One box {seg, nseg, 16} is one page of one kv head; 128-byte swizzle.
+// One box {seg, 1, 16} is one 128-byte column block of one page of one kv
+// head (16 rows of 128 bytes, 128-byte swizzle).
 parason_status encode_kv_map(CUtensorMap *map, const void *pages, int64_t num_phys,
                              int32_t H_kv, int32_t head_dim, int32_t mode) {
     auto fn = encode_fn();
@@ -431,7 +498,7 @@ parason_status encode_kv_map(CUtensorMap *map, const void *pages, int64_t num_ph
     const cuuint64_t rows = static_cast<cuuint64_t>(num_phys) * H_kv * parason::kPageSize;
     cuuint64_t dims[3] = {static_cast<cuuint64_t>(seg_elems), static_cast<cuuint64_t>(nseg), rows};
     cuuint64_t strides[2] = {128, static_cast<cuuint64_t>(row_bytes)};
-    cuuint32_t box[3] = {static_cast<cuuint32_t>(seg_elems), static_cast<cuuint32_t>(nseg),
+    cuuint32_t box[3] = {static_cast<cuuint32_t>(seg_elems), 1u,
                          static_cast<cuuint32_t>(parason::kPageSize)};
     cuuint32_t estr[3] = {1, 1, 1};
     CUresult r = fn(map, dt, 3, const_cast<void *>(pages), dims, strides, box, estr,
@@ -470,7 +537,7 @@ parason_status parason_attn_plan_host(const parason_attn_config *cfg, int32_t nu
     parason_status st;
     try {
         st = build_host(p, cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves,
-                        leaf_node, num_physical_pages, num_sms, kDefaultCtasPerSm);
+                        leaf_node, num_physical_pages, num_sms);
     } catch (const std::bad_alloc &) {
         st = PARASON_ENOMEM;
     }
@@ -504,8 +571,8 @@ parason_status parason_attn_plan(const parason_attn_config *cfg, int32_t num_nod
         cudaGetLastError();
         return st != PARASON_OK ? st : PARASON_ECUDA;
     }
-    int ctas_per_sm = kDefaultCtasPerSm;
     if (cfg->mode != PARASON_FP32) {
+        int ctas_per_sm = 0;
         if (parason::attn_bf16_ctas_per_sm(cfg->head_dim, &ctas_per_sm) != cudaSuccess)
             return PARASON_ECUDA;
         if (ctas_per_sm < 1) return PARASON_EUNSUPPORTED;
@@ -514,7 +581,7 @@ parason_status parason_attn_plan(const parason_attn_config *cfg, int32_t num_nod
     if (!p) return PARASON_ENOMEM;
     try {
         st = build_host(p, cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves,
-                        leaf_node, num_physical_pages, sms, ctas_per_sm);
+                        leaf_node, num_physical_pages, sms);
     } catch (const std::bad_alloc &) {
         st = PARASON_ENOMEM;
     }
@@ -571,7 +638,6 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
 
     parason_status st = record_event(p, 0, stream);
     if (st != PARASON_OK) return st;
-    const bool fused = has_items && p->cfg.mode != PARASON_FP32;
     if (has_items) {
         parason::AttnArgs a{};
         a.items = p->d_items;
@@ -590,18 +656,12 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
         a.num_kv_heads = p->cfg.num_kv_heads;
         a.group = p->group;
         a.scale_log2 = sm_scale * 1.4426950408889634f;
-        a.cta_ptr = p->d_cta_ptr;
-        a.cta_items = p->d_cta_items;
-        a.num_ctas = static_cast<int32_t>(p->cta_ptr.size()) - 1;
-        a.counters = p->d_counters;
-        a.targets = p->d_targets;
-        a.merge_ptr = p->d_merge_ptr;
-        a.merge_ent = p->d_merge_ent;
-        a.out = out;
-        a.lse = lse;
-        a.empty_leaves = p->d_empty;
-        a.num_empty_leaves = static_cast<int32_t>(p->empty_leaves.size());
-        a.num_leaves = p->num_leaves;
+        a.sched_ptr = p->d_sched_ptr;
+        a.sched_items = p->d_sched_items;
+        a.stream_ptr = p->d_stream_ptr;
+        a.stream_rows = p->d_stream_rows;
+        a.num_ctas = p->num_ctas;
+        a.num_wide_ctas = p->num_wide_ctas;
         cudaError_t e;
         if (p->cfg.mode == PARASON_FP32) {
             e = parason::launch_attn_fp32(a, static_cast<const float *>(k_pages),
@@ -641,8 +701,11 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
     m.num_leaves = p->num_leaves;
     m.num_q_heads = p->cfg.num_q_heads;
     m.group = p->group;
-    if (!fused && parason::launch_merge(m, d, p->cfg.mode, stream) != cudaSuccess)
-        return PARASON_ECUDA;
+    m.num_kv_heads = p->cfg.num_kv_heads;
+    // programmatic dependent launch after the persistent kernel: the merge
+    // grid is launched while the attention grid drains, and waits for it
+    const bool pdl = has_items && p->cfg.mode != PARASON_FP32;
+    if (parason::launch_merge(m, d, p->cfg.mode, pdl, stream) != cudaSuccess) return PARASON_ECUDA;
     st = record_event(p, 2, stream);
     if (st != PARASON_OK) return st;
     if (p->timing_cap > 0 && p->timing_n < p->timing_cap) p->timing_n++;
@@ -673,11 +736,7 @@ parason_status parason_plan_check(parason_plan p, parason_stream_t stream) {
     if (cudaMemcpy(rec, p->d_err, sizeof rec, cudaMemcpyDeviceToHost) != cudaSuccess)
         return PARASON_ECUDA;
     if (rec[0] != 0) {
-        // an aborted launch leaves merge counters part-way: start them over
         if (cudaMemset(p->d_err, 0, sizeof rec) != cudaSuccess) return PARASON_ECUDA;
-        if (!p->targets.empty() &&
-            cudaMemset(p->d_counters, 0, p->targets.size() * sizeof(int32_t)) != cudaSuccess)
-            return PARASON_ECUDA;
         return rec[0] == PARASON_ETIMEOUT ? PARASON_ETIMEOUT : PARASON_ECUDA;
     }
     return PARASON_OK;
@@ -706,16 +765,16 @@ parason_status parason_plan_get_info(parason_plan p, parason_plan_info *info) {
     if (!p || !info) return PARASON_EINVAL;
     info->num_items = static_cast<int32_t>(p->items.size());
     info->num_leaves = p->num_leaves;
-    info->num_merge_entries = static_cast<int32_t>(p->merge_ent.size() / 2);
+    info->num_merge_entries = static_cast<int32_t>(p->merge_ent.size());
     info->chunk_pages = p->chunk_pages;
     info->num_slots = p->num_slots;
     info->unique_tokens = p->unique_tokens;
     info->path_tokens = p->path_tokens;
     info->num_sms = p->num_sms;
     info->on_device = p->on_device ? 1 : 0;
-    info->num_ctas = p->cta_ptr.empty() ? 0 : static_cast<int32_t>(p->cta_ptr.size()) - 1;
-    info->ctas_per_sm = p->ctas_per_sm;
-    info->num_empty_leaves = static_cast<int32_t>(p->empty_leaves.size());
+    info->num_ctas = p->num_ctas;
+    info->num_wide_ctas = p->num_wide_ctas;
+    info->num_workers = p->sched_ptr.empty() ? 0 : static_cast<int32_t>(p->sched_ptr.size()) - 1;
     return PARASON_OK;
 }
 
@@ -728,9 +787,8 @@ parason_status parason_plan_export(parason_plan p, int32_t table, void *dst, siz
     case PARASON_TABLE_DFS_LEAVES: src = p->dfs_leaf.data(); n = p->dfs_leaf.size() * 4; break;
     case PARASON_TABLE_MERGE_PTR: src = p->merge_ptr.data(); n = p->merge_ptr.size() * 4; break;
     case PARASON_TABLE_MERGE: src = p->merge_ent.data(); n = p->merge_ent.size() * 4; break;
-    case PARASON_TABLE_SCHEDULE_PTR: src = p->cta_ptr.data(); n = p->cta_ptr.size() * 4; break;
-    case PARASON_TABLE_SCHEDULE: src = p->cta_items.data(); n = p->cta_items.size() * 4; break;
-    case PARASON_TABLE_TARGETS: src = p->targets.data(); n = p->targets.size() * 4; break;
+    case PARASON_TABLE_SCHEDULE_PTR: src = p->sched_ptr.data(); n = p->sched_ptr.size() * 4; break;
+    case PARASON_TABLE_SCHEDULE: src = p->sched_items.data(); n = p->sched_items.size() * 4; break;
     default: return PARASON_EINVAL;
     }
     if (bytes < n || (n > 0 && !dst)) return PARASON_EINVAL;
@@ -783,8 +841,7 @@ parason_status parason_plan_read_timing(parason_plan p, float *attn_ms, float *m
 
 int32_t parason_plan_launches_per_decode(parason_plan p) {
     if (!p || p->num_leaves == 0) return 0;
-    if (p->items.empty()) return 1;                       // merge kernel only
-    return p->cfg.mode == PARASON_FP32 ? 2 : 1;           // bf16/fp8 merge is fused
+    return (p->items.empty() ? 0 : 1) + 1;                // attention, then merge
 }
 
 const char *parason_version(void) { return "0.1.0"; }
