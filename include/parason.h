@@ -99,6 +99,7 @@ typedef struct parason_plan_s *parason_plan;
  * parent out of range or not smaller than its child, a negative length, a
  * page count that is not ceil(len/page_size), a page id out of range or owned
  * twice, a leaf out of range, repeated or with children, or a NULL pointer.
+ * PARASON_EUNSUPPORTED for e4m3 KV with head_dim 64 (only 128 has a kernel).
  * PARASON_ENOMEM / PARASON_ECUDA if the metadata cannot be allocated or
  * copied.  On success *out owns host and device memory until
  * parason_plan_destroy.  The plan is immutable and may be used by any number

@@ -1,4 +1,4 @@
-// attn_bf16.cu -- fork-tree decode attention for bf16 KV on sm_103a.
+// attn_mma.cu -- fork-tree decode attention for bf16 or e4m3 KV on sm_103a.
 //
 // One persistent launch, one CTA per SM, two roles (the planner decides how
 // many SMs each gets so that both finish together):
@@ -6,24 +6,35 @@
 //  * prefix pass (CTAs [0, num_wide_ctas)): nodes that many branches share.
 //    Up to 128 query rows -- the branches under the node times the q heads
 //    of one kv head -- are stacked on one page stream: a producer warp moves
-//    each (page, kv head) of K and V by TMA (3-D box, 128-byte swizzle) into
-//    a shared ring, and 8 consumer warps of 16 rows each read it from shared
-//    memory.  The node's KV is read from HBM once for all its rows, which is
-//    what the shared prefix of Subtask/Trial branches buys (paper Sec. 3.1,
-//    3.4).
+//    each (page, kv head) of K and V by TMA (3-D boxes, 128-byte swizzle)
+//    into a shared ring, and 8 consumer warps of 16 rows each read it from
+//    shared memory.  The node's KV is read from HBM once for all its rows,
+//    which is what the shared prefix of Subtask/Trial branches buys (paper
+//    Sec. 3.1, 3.4).
 //  * suffix pass (the other CTAs): nodes of at most 16 rows (a branch's own
 //    suffix).  Each of the 8 warps is an independent worker with its own
 //    TMA ring and its own balanced list of items (split-K pieces of
 //    suffixes): no CTA barrier, no cross-warp combine.
 //
-// Both roles use tensor-core QK^T and PV (mma.sync m16n8k16, bf16 in, fp32
-// accumulate) from ldmatrix fragments and an online softmax in registers with
-// quad shuffles, and write a partial (o, m, l) per item row.  The merge kernel
-// (merge.cu) folds the partials of every branch's path afterwards; it is
-// launched as a programmatic dependent of this grid.
+// Both roles use tensor-core QK^T and PV (mma.sync m16n8k16, fp32
+// accumulate) and an online softmax in registers with quad shuffles, and
+// write a partial (o, m, l) per item row.  The merge kernel (merge.cu) folds
+// the partials of every branch's path; it is launched as a programmatic
+// dependent of this grid.
 //
-// Scores are kept in the log2 domain: x = sm_scale*log2(e)*<q,k>, so a
-// partial is m = max x, l = sum 2^(x-m), o = sum 2^(x-m) v (unnormalised).
+// KV formats:
+//  * bf16: fragments by ldmatrix (V transposed by ldmatrix.trans), bf16 MMA.
+//  * e4m3 (one fp32 scale per kv head for K and for V): 4- and 16-byte
+//    shared loads, every e4m3 pair widened to f16 exactly (cvt.rn.f16x2.
+//    e4m3x2), f16 MMA; q is widened from bf16 to f16 (exact for |q| in the
+//    f16 normal range).  The K scale joins the softmax scale, the V scale
+//    multiplies the partial o.  The fragment layouts permute d so that each
+//    thread's bytes are contiguous: QK^T takes d = 16ks + 4t + {0..3} for
+//    thread t of a quad, PV gives thread column c of n-tile n the output
+//    d = 16c + n.
+//
+// Scores are kept in the log2 domain: x = scale*log2(e)*<q,k>, so a partial
+// is m = max x, l = sum 2^(x-m), o = sum 2^(x-m) v (unnormalised).
 #include "device_common.cuh"
 
 namespace parason {
@@ -35,12 +46,20 @@ constexpr int kThreads = kConsumerThreads + 32;            // + producer warp
 constexpr long long kDrainLimitNs = 1000000000LL;
 constexpr int kSmemBudget = 220 * 1024;                    // dynamic, one CTA per SM
 
-template <int D>
+struct KvBf16 {
+    static constexpr int kElemBytes = 2;
+};
+struct KvE4m3 {
+    static constexpr int kElemBytes = 1;
+};
+
+template <int D, class KV>
 struct Shape {
-    static constexpr int kPageBytes = kPageSize * D * 2;   // one page of one kv head
+    static constexpr int kRowBytes = D * KV::kElemBytes;    // one token of one kv head
+    static constexpr int kPageBytes = kPageSize * kRowBytes; // one page of one kv head
     // a page lands as kSeg column blocks of 16 tokens x 128 bytes, so that 8
     // consecutive tokens hit 8 different 128-byte swizzle rows
-    static constexpr int kSeg = D * 2 / 128;
+    static constexpr int kSeg = kRowBytes / 128;
     static constexpr int kSegBytes = kPageSize * 128;
     static constexpr int kStageBytes = 2 * kPageBytes;      // K and V of one page
 
@@ -62,17 +81,18 @@ struct Shape {
     static constexpr int kBodyBytes =
         kNarrowBytes > kWideRingBytes + kScratchBytes ? kNarrowBytes : kWideRingBytes + kScratchBytes;
     static constexpr int kSmemBytes = kBodyBytes + kBars * 8 + 1024;   // + alignment slack
+    static_assert(kRowBytes % 128 == 0, "token rows are whole 128-byte blocks");
     static_assert(kWarpStages >= 2, "suffix ring depth");
     static_assert(kWideStages >= 4, "prefix ring depth");
     static_assert(kSmemBytes <= kSmemBudget, "shared memory budget");
 };
 
-// K then V of one (page, kv head) into a stage: one TMA box {64 columns, 1
+// K then V of one (page, kv head) into a stage: one TMA box {128 bytes, 1
 // block, 16 tokens} per column block and tensor.
-template <int D>
+template <int D, class KV>
 __device__ __forceinline__ void load_page(uint32_t dst, const CUtensorMap *tmap_k,
                                           const CUtensorMap *tmap_v, int row, uint32_t bar) {
-    using S = Shape<D>;
+    using S = Shape<D, KV>;
 #pragma unroll
     for (int sg = 0; sg < S::kSeg; ++sg) {
         dev::tma_load_3d(dst + sg * S::kSegBytes, tmap_k, 0, sg, row, bar);
@@ -96,41 +116,45 @@ __device__ __forceinline__ void reset(WarpState<D> &st) {
     st.l[0] = st.l[1] = 0.f;
 }
 
-// One 16-token page: S = Q K^T, online softmax, O += P V.
-template <int D>
-__device__ __forceinline__ void page_step(uint32_t kbase, uint32_t vbase, int valid,
-                                          const uint32_t (&qa)[D / 16][4], WarpState<D> &st,
-                                          float scale_log2, int lane) {
-    using S = Shape<D>;
-    const int tig = lane & 3;
-    const int mi = lane >> 3, r8 = lane & 7;
+// Output column of accumulator o[nt][e] of thread (gid, tig): its row is gid
+// (e < 2) or gid + 8, its column below.
+template <class KV>
+__device__ __forceinline__ int out_col(int nt, int e, int tig) {
+    if constexpr (KV::kElemBytes == 2)
+        return nt * 8 + 2 * tig + (e & 1);
+    else
+        return 16 * (2 * tig + (e & 1)) + nt;
+}
 
-    // two accumulator pairs (first and second half of d) halve the MMA chain
-    float sc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-    float sd[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-    {
-        const int tok = r8 + ((mi >> 1) << 3);
-#pragma unroll
-        for (int ks = 0; ks < D / 16; ++ks) {
-            const int dch = 2 * ks + (mi & 1);
-            uint32_t b00, b01, b10, b11;
-            dev::ldsm_x4(kbase + (dch >> 3) * S::kSegBytes + dev::swz128(tok, dch & 7), b00, b01,
-                         b10, b11);
-            if (ks < D / 32) {
-                dev::mma_bf16_16816(sc[0], qa[ks], b00, b01);
-                dev::mma_bf16_16816(sc[1], qa[ks], b10, b11);
-            } else {
-                dev::mma_bf16_16816(sd[0], qa[ks], b00, b01);
-                dev::mma_bf16_16816(sd[1], qa[ks], b10, b11);
-            }
-        }
-#pragma unroll
-        for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) sc[nt][e] += sd[nt][e];
-    }
+__device__ __forceinline__ uint32_t e4m3x2_to_f16x2(uint32_t two_bytes) {
+    uint32_t out;
+    asm("{\n\t.reg .b16 lo, hi;\n\t"
+        "mov.b32 {lo, hi}, %1;\n\t"
+        "cvt.rn.f16x2.e4m3x2 %0, lo;\n\t}"
+        : "=r"(out)
+        : "r"(two_bytes));
+    return out;
+}
 
-    // online softmax (log2 domain), rows gid (e = 0,1) and gid + 8 (e = 2,3)
+__device__ __forceinline__ uint32_t lds32(uint32_t addr) {
+    uint32_t v;
+    asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(addr));
+    return v;
+}
+
+// Online softmax over one page's scores s (two n-tiles of 8 tokens), then
+// rescale o; returns P packed as the A operand of the PV MMA.
+template <int D, class KV>
+__device__ __forceinline__ void softmax_page(const float (&sc)[2][4], int valid, float scale_log2,
+                                             WarpState<D> &st, int tig, uint32_t (&pa)[4]) {
     float x[2][4];
 #pragma unroll
     for (int nt = 0; nt < 2; ++nt)
@@ -167,36 +191,117 @@ __device__ __forceinline__ void page_step(uint32_t kbase, uint32_t vbase, int va
         st.o[dt][2] *= al1;
         st.o[dt][3] *= al1;
     }
-
-    // O += P V: P (16 rows x 16 tokens) straight from the S accumulators
-    const uint32_t pa[4] = {dev::pack_bf16(p[0][0], p[0][1]), dev::pack_bf16(p[0][2], p[0][3]),
-                            dev::pack_bf16(p[1][0], p[1][1]), dev::pack_bf16(p[1][2], p[1][3])};
-    // slots past the node's length may hold anything (NaN included): their
-    // P is 0, but 0 * NaN is NaN, so their V values are zeroed
-    uint32_t keep_lo = 0xffffffffu, keep_hi = 0xffffffffu;
-    if (valid < kPageSize) {
-        const int t0 = 2 * tig;
-        keep_lo = (t0 < valid ? 0x0000ffffu : 0u) | (t0 + 1 < valid ? 0xffff0000u : 0u);
-        keep_hi = (t0 + 8 < valid ? 0x0000ffffu : 0u) | (t0 + 9 < valid ? 0xffff0000u : 0u);
-    }
-    const int vtok = r8 + ((mi & 1) << 3);
-#pragma unroll
-    for (int dt = 0; dt < D / 8; dt += 2) {
-        const int dch = dt + (mi >> 1);
-        uint32_t v0, v1, v2, v3;
-        dev::ldsm_x4_trans(vbase + (dch >> 3) * S::kSegBytes + dev::swz128(vtok, dch & 7), v0, v1,
-                           v2, v3);
-        v0 &= keep_lo;
-        v1 &= keep_hi;
-        v2 &= keep_lo;
-        v3 &= keep_hi;
-        dev::mma_bf16_16816(st.o[dt], pa, v0, v1);
-        dev::mma_bf16_16816(st.o[dt + 1], pa, v2, v3);
+    if constexpr (KV::kElemBytes == 2) {
+        pa[0] = dev::pack_bf16(p[0][0], p[0][1]);
+        pa[1] = dev::pack_bf16(p[0][2], p[0][3]);
+        pa[2] = dev::pack_bf16(p[1][0], p[1][1]);
+        pa[3] = dev::pack_bf16(p[1][2], p[1][3]);
+    } else {
+        pa[0] = dev::pack_f16(p[0][0], p[0][1]);
+        pa[1] = dev::pack_f16(p[0][2], p[0][3]);
+        pa[2] = dev::pack_f16(p[1][0], p[1][1]);
+        pa[3] = dev::pack_f16(p[1][2], p[1][3]);
     }
 }
 
-// Q fragments (A operand, row-major 16 x D) for tile rows rg*16 + {gid, gid+8}.
-template <int D>
+// One 16-token page: S = Q K^T, online softmax, O += P V.
+template <int D, class KV>
+__device__ __forceinline__ void page_step(uint32_t kbase, uint32_t vbase, int valid,
+                                          const uint32_t (&qa)[D / 16][4], WarpState<D> &st,
+                                          float scale_log2, int lane) {
+    using S = Shape<D, KV>;
+    const int gid = lane >> 2, tig = lane & 3;
+    const int mi = lane >> 3, r8 = lane & 7;
+
+    // two accumulator pairs (first and second half of d) halve the MMA chain
+    float sc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+    float sd[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+    if constexpr (KV::kElemBytes == 2) {
+        const int tok = r8 + ((mi >> 1) << 3);
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+            const int dch = 2 * ks + (mi & 1);
+            uint32_t b00, b01, b10, b11;
+            dev::ldsm_x4(kbase + (dch >> 3) * S::kSegBytes + dev::swz128(tok, dch & 7), b00, b01,
+                         b10, b11);
+            float(&acc)[2][4] = ks < D / 32 ? sc : sd;
+            dev::mma_bf16_16816(acc[0], qa[ks], b00, b01);
+            dev::mma_bf16_16816(acc[1], qa[ks], b10, b11);
+        }
+    } else {
+        // thread (gid, tig) reads bytes 4tig..4tig+3 of 16-byte chunk ks of token gid
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+            float(&acc)[2][4] = ks < D / 32 ? sc : sd;
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) {
+                const uint32_t w = lds32(kbase + dev::swz128(nt * 8 + gid, ks) + 4 * tig);
+                dev::mma_f16_16816(acc[nt], qa[ks], e4m3x2_to_f16x2(w), e4m3x2_to_f16x2(w >> 16));
+            }
+        }
+    }
+#pragma unroll
+    for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) sc[nt][e] += sd[nt][e];
+
+    uint32_t pa[4];
+    softmax_page<D, KV>(sc, valid, scale_log2, st, tig, pa);
+
+    if constexpr (KV::kElemBytes == 2) {
+        // slots past the node's length may hold anything (NaN included): their
+        // P is 0, but 0 * NaN is NaN, so their V values are zeroed
+        uint32_t keep_lo = 0xffffffffu, keep_hi = 0xffffffffu;
+        if (valid < kPageSize) {
+            const int t0 = 2 * tig;
+            keep_lo = (t0 < valid ? 0x0000ffffu : 0u) | (t0 + 1 < valid ? 0xffff0000u : 0u);
+            keep_hi = (t0 + 8 < valid ? 0x0000ffffu : 0u) | (t0 + 9 < valid ? 0xffff0000u : 0u);
+        }
+        const int vtok = r8 + ((mi & 1) << 3);
+#pragma unroll
+        for (int dt = 0; dt < D / 8; dt += 2) {
+            const int dch = dt + (mi >> 1);
+            uint32_t v0, v1, v2, v3;
+            dev::ldsm_x4_trans(vbase + (dch >> 3) * S::kSegBytes + dev::swz128(vtok, dch & 7), v0,
+                               v1, v2, v3);
+            v0 &= keep_lo;
+            v1 &= keep_hi;
+            v2 &= keep_lo;
+            v3 &= keep_hi;
+            dev::mma_bf16_16816(st.o[dt], pa, v0, v1);
+            dev::mma_bf16_16816(st.o[dt + 1], pa, v2, v3);
+        }
+    } else {
+        // thread gid owns output columns 16gid .. 16gid+15: one 16-byte chunk
+        // of each of its four tokens 2tig, 2tig+1, 2tig+8, 2tig+9
+        static_assert(D == 128, "e4m3 KV path is written for head_dim 128");
+        const int t0 = 2 * tig;
+        uint4 va = lds128(vbase + dev::swz128(t0, gid));
+        uint4 vb = lds128(vbase + dev::swz128(t0 + 1, gid));
+        uint4 vc = lds128(vbase + dev::swz128(t0 + 8, gid));
+        uint4 vd = lds128(vbase + dev::swz128(t0 + 9, gid));
+        if (valid < kPageSize) {
+            const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+            if (t0 >= valid) va = z;
+            if (t0 + 1 >= valid) vb = z;
+            if (t0 + 8 >= valid) vc = z;
+            if (t0 + 9 >= valid) vd = z;
+        }
+        const uint32_t wa[4] = {va.x, va.y, va.z, va.w}, wb[4] = {vb.x, vb.y, vb.z, vb.w};
+        const uint32_t wc[4] = {vc.x, vc.y, vc.z, vc.w}, wd[4] = {vd.x, vd.y, vd.z, vd.w};
+#pragma unroll
+        for (int nt = 0; nt < 16; ++nt) {
+            const uint32_t sel = (nt & 3) | ((4 + (nt & 3)) << 4);   // byte nt of x, byte nt of y
+            const uint32_t lo = __byte_perm(wa[nt >> 2], wb[nt >> 2], sel);
+            const uint32_t hi = __byte_perm(wc[nt >> 2], wd[nt >> 2], sel);
+            dev::mma_f16_16816(st.o[nt], pa, e4m3x2_to_f16x2(lo), e4m3x2_to_f16x2(hi));
+        }
+    }
+}
+
+// Q fragments (A operand, row-major 16 x D) for tile rows rg*16 + {gid, gid+8}:
+// bf16 as stored, or widened to f16 with d permuted as the e4m3 QK^T wants.
+template <int D, class KV>
 __device__ __forceinline__ void load_q_fragments(const AttnArgs &a, const WorkItem &it, int rg,
                                                  int lane, uint32_t (&qa)[D / 16][4]) {
     const int gid = lane >> 2, tig = lane & 3;
@@ -216,17 +321,37 @@ __device__ __forceinline__ void load_q_fragments(const AttnArgs &a, const WorkIt
     for (int ks = 0; ks < D / 16; ++ks)
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-            const int c0 = ks * 16 + 2 * tig;
-            qa[ks][h] = qrow[h] ? *reinterpret_cast<const uint32_t *>(qrow[h] + c0) : 0u;
-            qa[ks][2 + h] = qrow[h] ? *reinterpret_cast<const uint32_t *>(qrow[h] + c0 + 8) : 0u;
+            if constexpr (KV::kElemBytes == 2) {
+                const int c0 = ks * 16 + 2 * tig;
+                qa[ks][h] = qrow[h] ? *reinterpret_cast<const uint32_t *>(qrow[h] + c0) : 0u;
+                qa[ks][2 + h] = qrow[h] ? *reinterpret_cast<const uint32_t *>(qrow[h] + c0 + 8) : 0u;
+            } else {
+                uint2 u = make_uint2(0u, 0u);
+                if (qrow[h]) u = *reinterpret_cast<const uint2 *>(qrow[h] + ks * 16 + 4 * tig);
+                const __nv_bfloat162 p0 = *reinterpret_cast<const __nv_bfloat162 *>(&u.x);
+                const __nv_bfloat162 p1 = *reinterpret_cast<const __nv_bfloat162 *>(&u.y);
+                qa[ks][h] = dev::pack_f16(__low2float(p0), __high2float(p0));
+                qa[ks][2 + h] = dev::pack_f16(__low2float(p1), __high2float(p1));
+            }
         }
+}
+
+// Softmax scale of an item and the factor of its partial o (the kv head's
+// e4m3 scales for K and V; 1 for bf16).
+template <class KV>
+__device__ __forceinline__ float2 item_scales(const AttnArgs &a, const WorkItem &it) {
+    if constexpr (KV::kElemBytes == 2)
+        return make_float2(a.scale_log2, 1.f);
+    else
+        return make_float2(a.scale_log2 * a.k_scale[it.kv_head], a.v_scale[it.kv_head]);
 }
 
 // A warp that owns rows rg*16 .. rg*16+15 of an item writes their partials
 // straight from registers.
-template <int D>
+template <int D, class KV>
 __device__ __forceinline__ void store_warp_partials(const AttnArgs &a, const WorkItem &it,
-                                                    WarpState<D> &st, int rg, int lane) {
+                                                    WarpState<D> &st, int rg, int lane,
+                                                    float o_scale) {
     const int gid = lane >> 2, tig = lane & 3;
     st.l[0] += __shfl_xor_sync(0xffffffffu, st.l[0], 1);
     st.l[0] += __shfl_xor_sync(0xffffffffu, st.l[0], 2);
@@ -239,9 +364,15 @@ __device__ __forceinline__ void store_warp_partials(const AttnArgs &a, const Wor
         const int64_t slot = static_cast<int64_t>(it.slot_base) + r;
         float *dst = a.part_o + slot * D;
 #pragma unroll
-        for (int dt = 0; dt < D / 8; ++dt)
-            *reinterpret_cast<float2 *>(dst + dt * 8 + 2 * tig) =
-                make_float2(st.o[dt][2 * h], st.o[dt][2 * h + 1]);
+        for (int dt = 0; dt < D / 8; ++dt) {
+            if constexpr (KV::kElemBytes == 2) {
+                *reinterpret_cast<float2 *>(dst + dt * 8 + 2 * tig) =
+                    make_float2(st.o[dt][2 * h], st.o[dt][2 * h + 1]);
+            } else {
+                dst[out_col<KV>(dt, 0, tig)] = st.o[dt][2 * h] * o_scale;
+                dst[out_col<KV>(dt, 1, tig)] = st.o[dt][2 * h + 1] * o_scale;
+            }
+        }
         if (tig == 0) a.part_ml[slot] = make_float2(st.m[h], st.l[h]);
     }
 }
@@ -273,10 +404,10 @@ struct PageStream {
 // ---------------------------------------------------------------------------
 // suffix pass: every warp streams its own item list through its own ring
 // ---------------------------------------------------------------------------
-template <int D>
+template <int D, class KV>
 __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
                             const AttnArgs &a, uint32_t ring, uint32_t bars, int warp, int lane) {
-    using S = Shape<D>;
+    using S = Shape<D, KV>;
     constexpr int NS = S::kWarpStages;
     const int worker = a.num_wide_ctas + (blockIdx.x - a.num_wide_ctas) * kConsumerWarps + warp;
     const int i_begin = a.sched_ptr[worker], i_end = a.sched_ptr[worker + 1];
@@ -294,10 +425,9 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
         const int row = ps.row(issued, lane);
         if (lane == 0 && !(skip_first && issued == 0)) {
             const int s = issued % NS;
-            const uint32_t dst = my_ring + s * S::kStageBytes;
             const uint32_t bar = my_bar + s * 8;
             dev::mbar_arrive_expect_tx(bar, S::kStageBytes);
-            load_page<D>(dst, tmap_k, tmap_v, row, bar);
+            load_page<D, KV>(my_ring + s * S::kStageBytes, tmap_k, tmap_v, row, bar);
         }
         ++issued;
     };
@@ -307,8 +437,9 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
     bool ok = true;
     for (int ii = i_begin; ii < i_end && ok; ++ii) {
         const WorkItem it = a.items[a.sched_items[ii]];
+        const float2 scl = item_scales<KV>(a, it);
         uint32_t qa[D / 16][4];
-        load_q_fragments<D>(a, it, 0, lane, qa);
+        load_q_fragments<D, KV>(a, it, 0, lane, qa);
         WarpState<D> st;
         reset<D>(st);
         for (int pg = 0; pg < it.num_pages; ++pg, ++consumed) {
@@ -319,15 +450,16 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
                 break;
             }
             const int valid = (pg == it.num_pages - 1) ? it.last_valid : kPageSize;
-            page_step<D>(my_ring + s * S::kStageBytes, my_ring + s * S::kStageBytes + S::kPageBytes,
-                         valid, qa, st, a.scale_log2, lane);
-            // refill this slot: its ldmatrix reads are complete, since every MMA
-            // that consumed them has issued (in order) before this point
+            page_step<D, KV>(my_ring + s * S::kStageBytes,
+                             my_ring + s * S::kStageBytes + S::kPageBytes, valid, qa, st, scl.x,
+                             lane);
+            // refill this slot: its shared-memory reads are complete, since
+            // every MMA that consumed them has issued (in order) before this point
             __syncwarp();
             issue_next();
         }
         if (!ok) break;
-        store_warp_partials<D>(a, it, st, 0, lane);
+        store_warp_partials<D, KV>(a, it, st, 0, lane, scl.y);
     }
     if (!ok && lane == 0) dev::record_error(a.err, PARASON_ETIMEOUT, kSiteConsumerFull);
     // copies still in flight must land before the CTA's shared memory goes
@@ -343,11 +475,11 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
 // ---------------------------------------------------------------------------
 // prefix pass: up to 128 stacked rows share one page stream
 // ---------------------------------------------------------------------------
-template <int D>
+template <int D, class KV>
 __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
                            const AttnArgs &a, uint8_t *smem, uint32_t ring, uint32_t bars,
                            int warp, int lane, volatile int *abort_flag) {
-    using S = Shape<D>;
+    using S = Shape<D, KV>;
     constexpr int NS = S::kWideStages;
     const uint32_t bar_full = bars, bar_empty = bars + NS * 8;
     const int i_begin = a.sched_ptr[blockIdx.x], i_end = a.sched_ptr[blockIdx.x + 1];
@@ -379,7 +511,7 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
             const int row = ps.row(stage, lane);
             if (lane == 0 && !(skip_first && stage == 0)) {
                 dev::mbar_arrive_expect_tx(bar_full + 8 * s, S::kStageBytes);
-                load_page<D>(k_page(s), tmap_k, tmap_v, row, bar_full + 8 * s);
+                load_page<D, KV>(k_page(s), tmap_k, tmap_v, row, bar_full + 8 * s);
                 last_issue[s] = stage;
             }
         }
@@ -401,6 +533,7 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
     int stage = 0;
     for (int ii = i_begin; ii < i_end; ++ii) {
         const WorkItem it = a.items[a.sched_items[ii]];
+        const float2 scl = item_scales<KV>(a, it);
         const int groups = (it.nrows + 15) >> 4;
         const int rgc = groups <= 2 ? 2 : (groups <= 4 ? 4 : 8);
         const int tgc = kConsumerWarps / rgc;
@@ -408,7 +541,7 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
         const bool has_rows = rg * 16 < it.nrows;
 
         uint32_t qa[D / 16][4];
-        load_q_fragments<D>(a, it, rg, lane, qa);
+        load_q_fragments<D, KV>(a, it, rg, lane, qa);
         WarpState<D> st;
         reset<D>(st);
 
@@ -425,8 +558,7 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
             }
             if (has_rows && pg % tgc == tg) {
                 const int valid = (pg == it.num_pages - 1) ? it.last_valid : kPageSize;
-                page_step<D>(k_page(s), k_page(s) + S::kPageBytes, valid, qa, st, a.scale_log2,
-                             lane);
+                page_step<D, KV>(k_page(s), k_page(s) + S::kPageBytes, valid, qa, st, scl.x, lane);
             }
             __syncwarp();
             if (lane == 0) dev::mbar_arrive(bar_empty + 8 * s);
@@ -439,7 +571,7 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
         if (dev::bar_sync_or<kConsumerThreads>(1, !ok || *abort_flag)) break;
 
         if (tgc == 1) {
-            if (has_rows) store_warp_partials<D>(a, it, st, rg, lane);
+            if (has_rows) store_warp_partials<D, KV>(a, it, st, rg, lane, scl.y);
             continue;
         }
         // combine the token-group warps of each row group, one column half at a time
@@ -456,14 +588,14 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
         for (int half = 0; half < 2; ++half) {
             float *wo = sc_o + warp * 16 * S::kScratchStride;
 #pragma unroll
-            for (int dt = 0; dt < D / 16; ++dt) {
-                const int c = dt * 8 + 2 * tig;
-                const int src = half * (D / 16) + dt;
-                *reinterpret_cast<float2 *>(wo + gid * S::kScratchStride + c) =
-                    make_float2(st.o[src][0], st.o[src][1]);
-                *reinterpret_cast<float2 *>(wo + (gid + 8) * S::kScratchStride + c) =
-                    make_float2(st.o[src][2], st.o[src][3]);
-            }
+            for (int dt = 0; dt < D / 8; ++dt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int col = out_col<KV>(dt, e, tig);
+                    if (col / S::kHalf == half)
+                        wo[(gid + 8 * (e >> 1)) * S::kScratchStride + col % S::kHalf] =
+                            st.o[dt][e] * scl.y;
+                }
             dev::bar_sync<kConsumerThreads>(1);
             for (int idx = tid; idx < it.nrows * kVec; idx += kConsumerThreads) {
                 const int r = idx / kVec, c4 = idx % kVec;
@@ -495,11 +627,11 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
 
 // One CTA per SM: 9 warps leave at most 168 registers per thread (three warps
 // on one sub-partition of 16K registers).
-template <int D>
+template <int D, class KV>
 __global__ void __launch_bounds__(kThreads, 1)
-    attn_bf16_kernel(const __grid_constant__ CUtensorMap tmap_k,
-                     const __grid_constant__ CUtensorMap tmap_v, const AttnArgs a) {
-    using S = Shape<D>;
+    attn_kernel(const __grid_constant__ CUtensorMap tmap_k,
+                const __grid_constant__ CUtensorMap tmap_v, const AttnArgs a) {
+    using S = Shape<D, KV>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -528,31 +660,30 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     if (wide) {
-        prefix_cta<D>(&tmap_k, &tmap_v, a, smem, ring, bars, warp, lane, &abort_flag);
+        prefix_cta<D, KV>(&tmap_k, &tmap_v, a, smem, ring, bars, warp, lane, &abort_flag);
     } else if (warp < kConsumerWarps) {
-        suffix_warp<D>(&tmap_k, &tmap_v, a, ring, bars, warp, lane);
+        suffix_warp<D, KV>(&tmap_k, &tmap_v, a, ring, bars, warp, lane);
     }
 }
 
 // Shared memory and carveout are set once per device; reports the number of
 // CTAs that fit per SM (the persistent grid needs one).
-template <int D>
+template <int D, class KV>
 cudaError_t configure(int *ctas_per_sm) {
-    using S = Shape<D>;
+    using S = Shape<D, KV>;
     static int configured_device = -1;
     static int resident = 0;
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (configured_device != dev) {
-        e = cudaFuncSetAttribute(attn_bf16_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(attn_kernel<D, KV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  S::kSmemBytes);
         if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(attn_bf16_kernel<D>,
-                                 cudaFuncAttributePreferredSharedMemoryCarveout,
+        e = cudaFuncSetAttribute(attn_kernel<D, KV>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                  cudaSharedmemCarveoutMaxShared);
         if (e != cudaSuccess) return e;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&resident, attn_bf16_kernel<D>, kThreads,
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&resident, attn_kernel<D, KV>, kThreads,
                                                           S::kSmemBytes);
         if (e != cudaSuccess) return e;
         configured_device = dev;
@@ -561,29 +692,38 @@ cudaError_t configure(int *ctas_per_sm) {
     return cudaSuccess;
 }
 
-template <int D>
+template <int D, class KV>
 cudaError_t launch(const AttnArgs &a, const CUtensorMap &tk, const CUtensorMap &tv,
                    cudaStream_t stream) {
-    using S = Shape<D>;
-    cudaError_t e = configure<D>(nullptr);
+    using S = Shape<D, KV>;
+    cudaError_t e = configure<D, KV>(nullptr);
     if (e != cudaSuccess) return e;
-    attn_bf16_kernel<D><<<a.num_ctas, kThreads, S::kSmemBytes, stream>>>(tk, tv, a);
+    attn_kernel<D, KV><<<a.num_ctas, kThreads, S::kSmemBytes, stream>>>(tk, tv, a);
     return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t attn_bf16_ctas_per_sm(int head_dim, int *ctas_per_sm) {
-    if (head_dim == 128) return configure<128>(ctas_per_sm);
-    if (head_dim == 64) return configure<64>(ctas_per_sm);
+cudaError_t attn_mma_ctas_per_sm(int head_dim, int mode, int *ctas_per_sm) {
+    if (mode == PARASON_FP8_E4M3_KV)
+        return head_dim == 128 ? configure<128, KvE4m3>(ctas_per_sm) : cudaErrorNotSupported;
+    if (head_dim == 128) return configure<128, KvBf16>(ctas_per_sm);
+    if (head_dim == 64) return configure<64, KvBf16>(ctas_per_sm);
     return cudaErrorNotSupported;
 }
 
 cudaError_t launch_attn_bf16(const AttnArgs &a, const CUtensorMap &tk, const CUtensorMap &tv,
                              int head_dim, cudaStream_t stream) {
     if (a.num_items <= 0 || a.num_ctas <= 0) return cudaSuccess;
-    if (head_dim == 128) return launch<128>(a, tk, tv, stream);
-    if (head_dim == 64) return launch<64>(a, tk, tv, stream);
+    if (head_dim == 128) return launch<128, KvBf16>(a, tk, tv, stream);
+    if (head_dim == 64) return launch<64, KvBf16>(a, tk, tv, stream);
+    return cudaErrorNotSupported;
+}
+
+cudaError_t launch_attn_fp8(const AttnArgs &a, const CUtensorMap &tk, const CUtensorMap &tv,
+                            int head_dim, cudaStream_t stream) {
+    if (a.num_items <= 0 || a.num_ctas <= 0) return cudaSuccess;
+    if (head_dim == 128) return launch<128, KvE4m3>(a, tk, tv, stream);
     return cudaErrorNotSupported;
 }
 

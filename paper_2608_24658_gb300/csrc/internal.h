@@ -83,8 +83,9 @@ struct MergeArgs {
     int32_t group;
 };
 
-// Resident CTAs per SM of the persistent attention kernel (sets its attributes).
-cudaError_t attn_bf16_ctas_per_sm(int head_dim, int *ctas_per_sm);
+// Resident CTAs per SM of the persistent attention kernel of a mode (sets its
+// attributes); cudaErrorNotSupported for a shape it has no kernel for.
+cudaError_t attn_mma_ctas_per_sm(int head_dim, int mode, int *ctas_per_sm);
 
 // Kernel launchers; each returns the launch's cudaError_t.
 cudaError_t launch_attn_bf16(const AttnArgs &a, const CUtensorMap &tmap_k,

@@ -128,6 +128,7 @@ parason_status validate_config(const parason_attn_config *cfg) {
         cfg->mode != PARASON_FP8_E4M3_KV)
         return PARASON_EINVAL;
     if (!(cfg->sm_scale >= 0.0f) || !std::isfinite(cfg->sm_scale)) return PARASON_EINVAL;
+    if (cfg->mode == PARASON_FP8_E4M3_KV && cfg->head_dim != 128) return PARASON_EUNSUPPORTED;
     return PARASON_OK;
 }
 
@@ -573,8 +574,9 @@ parason_status parason_attn_plan(const parason_attn_config *cfg, int32_t num_nod
     }
     if (cfg->mode != PARASON_FP32) {
         int ctas_per_sm = 0;
-        if (parason::attn_bf16_ctas_per_sm(cfg->head_dim, &ctas_per_sm) != cudaSuccess)
-            return PARASON_ECUDA;
+        const cudaError_t e = parason::attn_mma_ctas_per_sm(cfg->head_dim, cfg->mode, &ctas_per_sm);
+        if (e == cudaErrorNotSupported) return PARASON_EUNSUPPORTED;
+        if (e != cudaSuccess) return PARASON_ECUDA;
         if (ctas_per_sm < 1) return PARASON_EUNSUPPORTED;
     }
     auto *p = new (std::nothrow) parason_plan_s();

@@ -146,3 +146,12 @@ def test_lse_merge_argument_checks(lib):
     assert lib.parason_lse_merge(None, None, None, None, None, None, 4, 128, 0, None) == _lib.EINVAL
     assert lib.parason_lse_merge(None, None, None, None, None, None, 4, 96, 0, None) == _lib.EINVAL
     assert lib.parason_lse_merge(None, None, None, None, None, None, 4, 128, 7, None) == _lib.EINVAL
+
+
+def test_fp8_head_dim_64_unsupported(lib):
+    tree = W.figure3_tree(values=False)          # head_dim 64
+    f = _fields(tree)
+    f["mode"] = "fp8"
+    with pytest.raises(ParasonError) as e:
+        Plan(host_only=True, **f)
+    assert e.value.status == _lib.EUNSUPPORTED
