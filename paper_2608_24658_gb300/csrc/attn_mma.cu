@@ -36,6 +36,7 @@
 // Scores are kept in the log2 domain: x = scale*log2(e)*<q,k>, so a partial
 // is m = max x, l = sum 2^(x-m), o = sum 2^(x-m) v (unnormalised).
 #include "device_common.cuh"
+#include "tcgen05.cuh"
 
 namespace parason {
 namespace {
@@ -85,6 +86,7 @@ struct Shape {
     static_assert(kWarpStages >= 2, "suffix ring depth");
     static_assert(kWideStages >= 4, "prefix ring depth");
     static_assert(kSmemBytes <= kSmemBudget, "shared memory budget");
+    static_assert(kBars >= 16, "room for the tcgen05 prefix tile's barriers");
 };
 
 // K then V of one (page, kv head) into a stage: one TMA box {128 bytes, 1
@@ -625,6 +627,355 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
     }
 }
 
+
+// ---------------------------------------------------------------------------
+// prefix pass on tcgen05 (bf16 KV, head_dim 128): a tile of up to 128 stacked
+// rows against 64-token blocks (4 pages) of the node's pages
+//
+//   warp 8      producer: TMA of K and V, a block per ring stage; pages past
+//               the item's end are loaded from an out-of-range row, which
+//               TMA fills with zeros
+//   warp 4      MMA issuer (one thread): S = Q K^T (M 128, N 64, K 128) into
+//               one of two TMEM buffers, then O += P V (M 128, N 128, K 64)
+//               into the TMEM accumulator; tcgen05.commit releases the ring
+//               stage and signals completion
+//   warps 0-3   softmax: thread r owns row r (TMEM lane r); online softmax in
+//               the log2 domain with a lazy rescale of O (only when a row's
+//               max grows by more than 2^8); P goes to shared memory as the
+//               A operand of PV; at the end of an item the row's O, m, l
+//               become its partial
+//
+// Shared memory: ring [4][K: 2 col blocks x 64 tokens x 128 B | V: same],
+// Q tile [2 col blocks][128 rows][128 B], P [2][128 rows][128 B]; all 128-byte
+// swizzled, so the MMA reads them through SW128 descriptors (K-major for Q, K
+// and P; MN-major for V).
+// ---------------------------------------------------------------------------
+constexpr int kTcRows = 128;
+constexpr int kTcBlockPages = 4;
+constexpr int kTcBlockTokens = kTcBlockPages * kPageSize;    // 64
+constexpr int kTcStages = 4;
+constexpr int kTcColBlockBytes = kTcBlockTokens * 128;        // 8 KB: 64 tokens x 128 B
+constexpr int kTcKBytes = 2 * kTcColBlockBytes;               // d = 128: two column blocks
+constexpr int kTcStageBytes = 2 * kTcKBytes;                  // K + V
+constexpr int kTcRingBytes = kTcStages * kTcStageBytes;       // 128 KB
+constexpr int kTcQBytes = 2 * kTcRows * 128;                  // 32 KB
+constexpr int kTcPBytes = kTcRows * 128;                      // 16 KB per buffer
+constexpr int kTcBodyBytes = kTcRingBytes + kTcQBytes + 2 * kTcPBytes;
+constexpr int kTcTmemCols = 256;                              // O 128 + S 2 x 64
+constexpr float kTcRescaleLog2 = 8.f;                         // lazy rescale threshold
+static_assert(kTcBodyBytes <= Shape<128, KvBf16>::kBodyBytes, "tcgen05 tile fits the CTA's memory");
+// barrier slots (8 bytes each) in the CTA's barrier area
+enum TcBar : int {
+    kBarKvFull = 0,      // [4] producer -> MMA
+    kBarKvEmpty = 4,     // [4] MMA commit -> producer
+    kBarSFull = 8,       // [2] MMA commit -> softmax
+    kBarPFull = 10,      // [2] softmax (128 arrivals) -> MMA
+    kBarPvDone = 12,     // [2] MMA commit -> softmax
+    kBarQReady = 14,     // softmax (128 arrivals) -> MMA
+    kBarDrain = 15,      // MMA commit -> MMA thread, before TMEM is freed
+    kTcBars = 16
+};
+
+__device__ __forceinline__ bool tc_wait(uint32_t bar, uint32_t parity, long long limit,
+                                        volatile int *abort) {
+    return dev::mbar_wait_bounded(bar, parity, limit, abort);
+}
+
+// one warp: lane 0 waits, the warp agrees on the outcome
+__device__ __forceinline__ bool tc_warp_wait(uint32_t bar, uint32_t parity, long long limit,
+                                             volatile int *abort, int lane) {
+    int ok = 1;
+    if (lane == 0) ok = tc_wait(bar, parity, limit, abort) ? 1 : 0;
+    return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+
+__device__ __forceinline__ void tc_fail(const AttnArgs &a, volatile int *abort, int site) {
+    if (!*abort) {
+        *abort = 1;
+        dev::record_error(a.err, PARASON_ETIMEOUT, site);
+    }
+}
+
+template <int D>
+__device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
+                              const AttnArgs &a, uint8_t *smem, uint32_t bars, uint32_t tmem,
+                              int warp, int lane, volatile int *abort_flag) {
+    static_assert(D == 128, "the tcgen05 prefix tile is written for head_dim 128");
+    const uint32_t ring = dev::smem_addr(smem);
+    const uint32_t sq = ring + kTcRingBytes;
+    const uint32_t sp = sq + kTcQBytes;
+    auto bar = [&](int i) { return bars + 8u * static_cast<uint32_t>(i); };
+    const int i_begin = a.sched_ptr[blockIdx.x], i_end = a.sched_ptr[blockIdx.x + 1];
+
+    if (warp == kConsumerWarps) {
+        // ------------------------------------------------------------ producer
+        PageStream ps(a, blockIdx.x, lane);
+        const bool skip_first = a.debug_flags & PARASON_DEBUG_SKIP_FIRST_LOAD;
+        int last_issue[kTcStages];
+        for (int s = 0; s < kTcStages; ++s) last_issue[s] = -1;
+        int q = 0, blk = 0;
+        bool ok = true;
+        for (int ii = i_begin; ii < i_end && ok; ++ii) {
+            const WorkItem it = a.items[a.sched_items[ii]];
+            const int nb = (it.num_pages + kTcBlockPages - 1) / kTcBlockPages;
+            for (int bi = 0; bi < nb; ++bi, ++blk) {
+                const int s = blk % kTcStages;
+                if (blk >= kTcStages &&
+                    !tc_warp_wait(bar(kBarKvEmpty + s), ((blk / kTcStages) - 1) & 1,
+                                  a.wait_limit_ns, abort_flag, lane)) {
+                    if (lane == 0) tc_fail(a, abort_flag, kSiteProducerEmpty);
+                    ok = false;
+                    break;
+                }
+                int rows[kTcBlockPages];
+#pragma unroll
+                for (int j = 0; j < kTcBlockPages; ++j) {
+                    const int pg = bi * kTcBlockPages + j;
+                    rows[j] = pg < it.num_pages ? ps.row(q++, lane) : a.kv_rows;   // kv_rows: zero fill
+                }
+                if (lane == 0 && !(skip_first && blk == 0)) {
+                    const uint32_t st = ring + s * kTcStageBytes;
+                    const uint32_t fb = bar(kBarKvFull + s);
+                    dev::mbar_arrive_expect_tx(fb, kTcStageBytes);
+#pragma unroll
+                    for (int j = 0; j < kTcBlockPages; ++j)
+#pragma unroll
+                        for (int cb = 0; cb < 2; ++cb) {
+                            const uint32_t off = cb * kTcColBlockBytes + j * kPageSize * 128;
+                            dev::tma_load_3d(st + off, tmap_k, 0, cb, rows[j], fb);
+                            dev::tma_load_3d(st + kTcKBytes + off, tmap_v, 0, cb, rows[j], fb);
+                        }
+                    last_issue[s] = blk;
+                }
+            }
+        }
+        if (lane == 0)
+            for (int s = 0; s < kTcStages; ++s)
+                if (last_issue[s] >= 0)
+                    dev::mbar_wait_bounded(bar(kBarKvFull + s), (last_issue[s] / kTcStages) & 1,
+                                           kDrainLimitNs, nullptr);
+    } else if (warp == 4) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t tO = tmem, tS0 = tmem + 128;
+            constexpr uint32_t kIdS = tc::idesc_bf16_f32(kTcRows, kTcBlockTokens, false);
+            constexpr uint32_t kIdPV = tc::idesc_bf16_f32(kTcRows, D, true);
+            auto issue_s = [&](int b) {
+                const uint32_t st = ring + (b % kTcStages) * kTcStageBytes;
+                const uint32_t tS = tS0 + 64u * (b & 1);
+#pragma unroll
+                for (int ks = 0; ks < D / 16; ++ks) {
+                    const uint32_t cb = ks >> 2, kk = ks & 3;
+                    const uint64_t ad = tc::smem_desc_sw128(sq + cb * (kTcRows * 128) + kk * 32, 16, 1024);
+                    const uint64_t bd = tc::smem_desc_sw128(st + cb * kTcColBlockBytes + kk * 32, 16, 1024);
+                    tc::mma_bf16(tS, ad, bd, kIdS, ks > 0);
+                }
+                tc::commit(bar(kBarSFull + (b & 1)));
+            };
+            int blk = 0, item = 0;
+            bool ok = true;
+            for (int ii = i_begin; ii < i_end && ok; ++ii, ++item) {
+                const WorkItem it = a.items[a.sched_items[ii]];
+                const int nb = (it.num_pages + kTcBlockPages - 1) / kTcBlockPages;
+                if (!tc_wait(bar(kBarQReady), item & 1, a.wait_limit_ns, abort_flag) ||
+                    !tc_wait(bar(kBarKvFull + blk % kTcStages), (blk / kTcStages) & 1,
+                             a.wait_limit_ns, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc::fence_after_sync();
+                issue_s(blk);
+                for (int i = 0; i < nb; ++i) {
+                    const int b = blk + i;
+                    if (i + 1 < nb) {
+                        if (!tc_wait(bar(kBarKvFull + (b + 1) % kTcStages), ((b + 1) / kTcStages) & 1,
+                                     a.wait_limit_ns, abort_flag)) {
+                            ok = false;
+                            break;
+                        }
+                        issue_s(b + 1);
+                    }
+                    if (!tc_wait(bar(kBarPFull + (b & 1)), (b >> 1) & 1, a.wait_limit_ns, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc::fence_after_sync();
+                    const uint32_t vst = ring + (b % kTcStages) * kTcStageBytes + kTcKBytes;
+                    const uint32_t pb = sp + (b & 1) * kTcPBytes;
+#pragma unroll
+                    for (int kk = 0; kk < kTcBlockTokens / 16; ++kk) {
+                        const uint64_t ad = tc::smem_desc_sw128(pb + kk * 32, 16, 1024);
+                        const uint64_t bd = tc::smem_desc_sw128(vst + kk * 2048, kTcColBlockBytes, 1024);
+                        tc::mma_bf16(tO, ad, bd, kIdPV, i > 0 || kk > 0);
+                    }
+                    tc::commit(bar(kBarKvEmpty + b % kTcStages));
+                    tc::commit(bar(kBarPvDone + (b & 1)));
+                }
+                blk += nb;
+            }
+            if (!ok) tc_fail(a, abort_flag, kSiteConsumerFull);
+            // every MMA must finish before TMEM is freed
+            tc::commit(bar(kBarDrain));
+            dev::mbar_wait_bounded(bar(kBarDrain), 0, kDrainLimitNs, nullptr);
+        }
+    } else if (warp < 4) {
+        // ------------------------------------------------------------ softmax
+        const int r = threadIdx.x;                       // tile row == TMEM lane
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+        const uint32_t tO = lane_base, tS0 = lane_base + 128;
+        int blk = 0;
+        for (int ii = i_begin; ii < i_end; ++ii) {
+            const WorkItem it = a.items[a.sched_items[ii]];
+            const int nb = (it.num_pages + kTcBlockPages - 1) / kTcBlockPages;
+            const int tokens = (it.num_pages - 1) * kPageSize + it.last_valid;
+
+            // Q row r of the tile into the swizzled Q tile (zeros past nrows)
+            {
+                uint4 qv[16];
+                if (r < it.nrows) {
+                    const int nr = it.row0 + r;
+                    const int leaf = a.dfs_leaf[it.leaf_lo + nr / a.group];
+                    const int head = it.kv_head * a.group + nr % a.group;
+                    const uint4 *src = reinterpret_cast<const uint4 *>(
+                        static_cast<const __nv_bfloat16 *>(a.q) +
+                        (static_cast<int64_t>(leaf) * a.num_q_heads + head) * D);
+#pragma unroll
+                    for (int c = 0; c < 16; ++c) qv[c] = src[c];
+                } else {
+#pragma unroll
+                    for (int c = 0; c < 16; ++c) qv[c] = make_uint4(0u, 0u, 0u, 0u);
+                }
+#pragma unroll
+                for (int c = 0; c < 16; ++c) {
+                    const uint32_t dst = sq + (c >> 3) * (kTcRows * 128) + r * 128 +
+                                         (((c & 7) ^ (r & 7)) << 4);
+                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst),
+                                 "r"(qv[c].x), "r"(qv[c].y), "r"(qv[c].z), "r"(qv[c].w)
+                                 : "memory");
+                }
+                tc::fence_proxy_async_smem();
+                dev::mbar_arrive(bar(kBarQReady));
+            }
+
+            float m_use = -INFINITY, l = 0.f;
+            bool ok = true;
+            for (int i = 0; i < nb; ++i) {
+                const int b = blk + i;
+                const int valid = min(kTcBlockTokens, tokens - i * kTcBlockTokens);
+                if (!tc_warp_wait(bar(kBarSFull + (b & 1)), (b >> 1) & 1, a.wait_limit_ns, abort_flag,
+                                  lane)) {
+                    ok = false;
+                    break;
+                }
+                tc::fence_after_sync();
+                uint32_t sr[2][32];
+                tc::ld32(tS0 + 64u * (b & 1), sr[0]);
+                tc::ld32(tS0 + 64u * (b & 1) + 32, sr[1]);
+                tc::wait_ld();
+                float x[64];
+                float mb = -INFINITY;
+#pragma unroll
+                for (int j = 0; j < 64; ++j) {
+                    x[j] = j < valid ? __uint_as_float(sr[j >> 5][j & 31]) * a.scale_log2 : -INFINITY;
+                    mb = fmaxf(mb, x[j]);
+                }
+                // this P buffer was read by PV(b - 2)
+                if (b >= 2 && !tc_warp_wait(bar(kBarPvDone + (b & 1)), ((b - 2) >> 1) & 1,
+                                            a.wait_limit_ns, abort_flag, lane)) {
+                    ok = false;
+                    break;
+                }
+                if (i == 0) {
+                    m_use = mb;
+                } else if (__any_sync(0xffffffffu, mb > m_use + kTcRescaleLog2)) {
+                    // O must hold PV(b - 1) before it is rescaled
+                    if (!tc_warp_wait(bar(kBarPvDone + ((b - 1) & 1)), ((b - 1) >> 1) & 1,
+                                      a.wait_limit_ns, abort_flag, lane)) {
+                        ok = false;
+                        break;
+                    }
+                    tc::fence_after_sync();
+                    const float m_new = fmaxf(m_use, mb);
+                    const float alpha = dev::fast_exp2(m_use - m_new);
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) {
+                        uint32_t ov[32];
+                        tc::ld32(tO + 32 * c, ov);
+                        tc::wait_ld();
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) ov[j] = __float_as_uint(__uint_as_float(ov[j]) * alpha);
+                        tc::st32(tO + 32 * c, ov);
+                    }
+                    tc::wait_st();
+                    l *= alpha;
+                    m_use = m_new;
+                }
+                // P = 2^(x - m) as bf16, row r of the swizzled P tile
+                const uint32_t pb = sp + (b & 1) * kTcPBytes + r * 128;
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    uint32_t w[4];
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const float p0 = dev::fast_exp2(x[8 * c + 2 * k] - m_use);
+                        const float p1 = dev::fast_exp2(x[8 * c + 2 * k + 1] - m_use);
+                        l += p0 + p1;
+                        w[k] = dev::pack_bf16(p0, p1);
+                    }
+                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(pb + ((c ^ (r & 7)) << 4)),
+                                 "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
+                                 : "memory");
+                }
+                // V rows past the item's last token may hold anything (NaN
+                // included); P is 0 there but 0 * NaN is NaN, so zero them
+                if (valid < kTcBlockTokens) {
+                    const uint32_t vst = ring + (b % kTcStages) * kTcStageBytes + kTcKBytes;
+                    const int n16 = (kTcBlockTokens - valid) * 2 * 8;     // 16-byte chunks
+                    for (int k = r; k < n16; k += kTcRows) {
+                        const int t = valid + k / 16, cb = (k / 8) & 1, c = k & 7;
+                        asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
+                                         vst + cb * kTcColBlockBytes + t * 128 + (c << 4)),
+                                     "r"(0u)
+                                     : "memory");
+                    }
+                }
+                tc::fence_proxy_async_smem();
+                tc::fence_before_sync();
+                dev::mbar_arrive(bar(kBarPFull + (b & 1)));
+            }
+            if (!ok) {
+                if (lane == 0) tc_fail(a, abort_flag, kSiteConsumerFull);
+                break;
+            }
+            // epilogue: O of the item's last PV, normalised by the merge later
+            const int bl = blk + nb - 1;
+            if (!tc_warp_wait(bar(kBarPvDone + (bl & 1)), (bl >> 1) & 1, a.wait_limit_ns, abort_flag,
+                              lane)) {
+                if (lane == 0) tc_fail(a, abort_flag, kSiteConsumerFull);
+                break;
+            }
+            tc::fence_after_sync();
+            float *dst = a.part_o + (static_cast<int64_t>(it.slot_base) + r) * D;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t ov[32];
+                tc::ld32(tO + 32 * c, ov);
+                tc::wait_ld();
+                if (r < it.nrows) {
+#pragma unroll
+                    for (int j = 0; j < 32; j += 4)
+                        *reinterpret_cast<float4 *>(dst + 32 * c + j) =
+                            make_float4(__uint_as_float(ov[j]), __uint_as_float(ov[j + 1]),
+                                        __uint_as_float(ov[j + 2]), __uint_as_float(ov[j + 3]));
+                }
+            }
+            if (r < it.nrows) a.part_ml[static_cast<int64_t>(it.slot_base) + r] = make_float2(m_use, l);
+            tc::fence_before_sync();
+            blk += nb;
+        }
+    }
+}
+
 // One CTA per SM: 9 warps leave at most 168 registers per thread (three warps
 // on one sub-partition of 16K registers).
 template <int D, class KV>
@@ -641,9 +992,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool wide = static_cast<int>(blockIdx.x) < a.num_wide_ctas;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
+    // the prefix pass of bf16 KV at head_dim 128 runs on tcgen05
+    constexpr bool kTcPrefix = (D == 128) && (KV::kElemBytes == 2);
+    __shared__ uint32_t tmem_base;
     if (threadIdx.x == 0) {
         abort_flag = 0;
-        if (wide) {
+        if (wide && kTcPrefix) {
+            for (int i = 0; i < kTcBars; ++i)
+                dev::mbar_init(bars + 8 * i, (i == kBarPFull || i == kBarPFull + 1 || i == kBarQReady)
+                                                 ? kTcRows
+                                                 : 1);
+        } else if (wide) {
             for (int s = 0; s < S::kWideStages; ++s) {
                 dev::mbar_init(bars + 8 * s, 1);
                 dev::mbar_init(bars + 8 * (S::kWideStages + s), kConsumerWarps);
@@ -655,12 +1014,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         dev::prefetch_tensormap(&tmap_k);
         dev::prefetch_tensormap(&tmap_v);
     }
+    if constexpr (kTcPrefix) {
+        if (wide && warp == 4) tc::alloc<kTcTmemCols>(dev::smem_addr(&tmem_base));
+        tc::fence_before_sync();
+    }
     __syncthreads();
     // let the merge grid launch now; it waits for this grid to complete
     if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     if (wide) {
-        prefix_cta<D, KV>(&tmap_k, &tmap_v, a, smem, ring, bars, warp, lane, &abort_flag);
+        if constexpr (kTcPrefix) {
+            tc::fence_after_sync();
+            prefix_cta_tc<D>(&tmap_k, &tmap_v, a, smem, bars, tmem_base, warp, lane, &abort_flag);
+            tc::fence_before_sync();
+            __syncthreads();
+            tc::fence_after_sync();
+            if (warp == 4) tc::dealloc<kTcTmemCols>(tmem_base);
+        } else {
+            prefix_cta<D, KV>(&tmap_k, &tmap_v, a, smem, ring, bars, warp, lane, &abort_flag);
+        }
     } else if (warp < kConsumerWarps) {
         suffix_warp<D, KV>(&tmap_k, &tmap_v, a, ring, bars, warp, lane);
     }

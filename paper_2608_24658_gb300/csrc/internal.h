@@ -68,6 +68,8 @@ struct AttnArgs {
     const int32_t *stream_rows;
     int32_t num_ctas;
     int32_t num_wide_ctas;
+    int32_t kv_rows;        // rows of the KV tensor maps (pages * H_kv * 16); a
+                            // TMA box starting there is out of range: zeros
 };
 
 struct MergeArgs {

@@ -34,6 +34,7 @@ constexpr int kNarrowWarps = 8;         // autonomous warps per suffix-pass CTA
 constexpr int kMinPiecePages = 4;       // no split leaves a piece shorter than this
 constexpr int kFp32ChunkPages = 32;
 constexpr double kWideGroupPageCost = 1.0;   // one 16-row group of one page, in suffix pages
+constexpr double kTcPageCost = 2.2;          // one page of a tcgen05 prefix tile (measured)
 constexpr int64_t kDefaultWaitNs = 2000000000LL;
 constexpr size_t kAlign = 256;
 
@@ -43,7 +44,11 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // pass on the same SM.  The suffix pass runs 8 pages at once (one per warp);
 // a prefix tile runs one 16-row MMA group of the page per warp, so a page of
 // a tile with G groups costs G suffix pages of warp time.
-double wide_page_cost(int32_t rows) {
+//
+// The bf16 prefix tile at head_dim 128 runs on tcgen05: one 128-row MMA per
+// 64 tokens, so its pages cost about a suffix page each.
+double wide_page_cost(int32_t rows, bool tensor_core_tile) {
+    if (tensor_core_tile) return kTcPageCost;
     const double groups = (rows + 15) / 16;
     return std::max(1.0, groups * kWideGroupPageCost);
 }
@@ -251,7 +256,9 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                 run.nrows = static_cast<int32_t>(std::min<int64_t>(rt, R - r0));
                 run.pages = P;
                 run.wide = wide;
-                run.cost_per_page = wide ? wide_page_cost(run.nrows) : 1.0;
+                run.cost_per_page =
+                    wide ? wide_page_cost(run.nrows, mode == PARASON_BF16 && cfg->head_dim == 128)
+                         : 1.0;
                 if (wide)
                     wide_cost += run.cost_per_page * static_cast<double>(P);
                 else
@@ -664,6 +671,7 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
         a.stream_rows = p->d_stream_rows;
         a.num_ctas = p->num_ctas;
         a.num_wide_ctas = p->num_wide_ctas;
+        a.kv_rows = static_cast<int32_t>(p->num_phys * p->cfg.num_kv_heads * parason::kPageSize);
         cudaError_t e;
         if (p->cfg.mode == PARASON_FP32) {
             e = parason::launch_attn_fp32(a, static_cast<const float *>(k_pages),
