@@ -201,8 +201,9 @@ typedef struct {
     int32_t num_sms;            /* SM count the split targeted              */
     int32_t on_device;          /* 1 if decode can run on this plan         */
     int32_t num_ctas;           /* CTAs of the persistent attention kernel  */
-    int32_t num_wide_ctas;      /* of which run the prefix pass             */
-    int32_t num_workers;        /* item lists: prefix CTAs + suffix warps   */
+    int32_t num_wide_ctas;      /* of which start on the prefix pass        */
+    int32_t num_wide_items;     /* prefix-pass items (tiles x pieces)       */
+    int32_t num_narrow_items;   /* suffix-pass items                        */
 } parason_plan_info;
 
 parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info);
@@ -220,10 +221,10 @@ parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info)
  *   PARASON_TABLE_MERGE      int32 [num_merge_entries]: partial slot of the
  *                            branch's first q head of the kv head; q head
  *                            j*g + r reads slot entry + r
- *   PARASON_TABLE_SCHEDULE_PTR int32 [num_workers + 1]: CSR of the persistent
- *                            kernel's item lists: one list per prefix-pass
- *                            CTA, then one per suffix-pass warp
- *   PARASON_TABLE_SCHEDULE   int32 [num_items]: item indices, list by list
+ *   PARASON_TABLE_WIDE_QUEUE int32 [num_wide_items]: prefix-pass items in the
+ *                            order the kernel's prefix CTAs pull them
+ *   PARASON_TABLE_NARROW_QUEUE int32 [num_narrow_items]: suffix-pass items in
+ *                            the order the kernel's warps pull them
  * Returns PARASON_EINVAL if `bytes` is smaller than the table.
  */
 enum {
@@ -231,8 +232,8 @@ enum {
     PARASON_TABLE_DFS_LEAVES = 1,
     PARASON_TABLE_MERGE_PTR = 2,
     PARASON_TABLE_MERGE = 3,
-    PARASON_TABLE_SCHEDULE_PTR = 4,
-    PARASON_TABLE_SCHEDULE = 5
+    PARASON_TABLE_WIDE_QUEUE = 4,
+    PARASON_TABLE_NARROW_QUEUE = 5
 };
 parason_status parason_plan_export(parason_plan plan, int32_t table, void *dst, size_t bytes);
 

@@ -13,8 +13,8 @@ LIB_PATH = os.path.join(_HERE, "_build", "libparason.so")
 
 OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EUNSUPPORTED = range(6)
 MODES = {"bf16": 0, "fp32": 1, "fp8": 2}
-(TABLE_ITEMS, TABLE_DFS_LEAVES, TABLE_MERGE_PTR, TABLE_MERGE, TABLE_SCHEDULE_PTR,
- TABLE_SCHEDULE) = range(6)
+(TABLE_ITEMS, TABLE_DFS_LEAVES, TABLE_MERGE_PTR, TABLE_MERGE, TABLE_WIDE_QUEUE,
+ TABLE_NARROW_QUEUE) = range(6)
 DEBUG_SKIP_FIRST_LOAD = 1
 
 # every function include/parason.h declares, with (restype, argtypes)
@@ -37,7 +37,8 @@ class PlanInfo(ctypes.Structure):
                 ("num_slots", ctypes.c_int64), ("unique_tokens", ctypes.c_int64),
                 ("path_tokens", ctypes.c_int64), ("num_sms", ctypes.c_int32),
                 ("on_device", ctypes.c_int32), ("num_ctas", ctypes.c_int32),
-                ("num_wide_ctas", ctypes.c_int32), ("num_workers", ctypes.c_int32)]
+                ("num_wide_ctas", ctypes.c_int32), ("num_wide_items", ctypes.c_int32),
+                ("num_narrow_items", ctypes.c_int32)]
 
 
 SIGNATURES = {

@@ -125,8 +125,8 @@ class Plan:
                  _lib.TABLE_DFS_LEAVES: (inf["num_leaves"],),
                  _lib.TABLE_MERGE_PTR: (inf["num_leaves"] * self.num_kv_heads + 1,),
                  _lib.TABLE_MERGE: (inf["num_merge_entries"],),
-                 _lib.TABLE_SCHEDULE_PTR: (inf["num_workers"] + 1,),
-                 _lib.TABLE_SCHEDULE: (inf["num_items"] if inf["num_workers"] else 0,)}[table]
+                 _lib.TABLE_WIDE_QUEUE: (inf["num_wide_items"],),
+                 _lib.TABLE_NARROW_QUEUE: (inf["num_narrow_items"],)}[table]
         buf = np.zeros(shape, dtype=np.int32)
         check(_lib.load().parason_plan_export(self.handle, table, _ptr(buf), buf.nbytes),
               "plan_export")

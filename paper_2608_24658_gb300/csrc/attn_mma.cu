@@ -46,6 +46,8 @@ constexpr int kConsumerThreads = kConsumerWarps * 32;
 constexpr int kThreads = kConsumerThreads + 32;            // + producer warp
 constexpr long long kDrainLimitNs = 1000000000LL;
 constexpr int kSmemBudget = 220 * 1024;                    // dynamic, one CTA per SM
+constexpr int kIdSlots = 8;      // prefix-pass item ids in flight from producer to consumers
+constexpr int kGrabSlots = 8;    // suffix-pass item ids a warp has pulled but not finished
 
 struct KvBf16 {
     static constexpr int kElemBytes = 2;
@@ -78,7 +80,10 @@ struct Shape {
     static constexpr int kWideRingBytes = kWideStages * kStageBytes;
     static constexpr int kWideBars = 2 * kWideStages;
 
-    static constexpr int kBars = kNarrowBars > kWideBars ? kNarrowBars : kWideBars;
+    // + kIdSlots item-id barriers of the prefix pass, + the tcgen05 tile's 16
+    static constexpr int kWideAll = kWideBars + kIdSlots;
+    static constexpr int kBars0 = kNarrowBars > kWideAll ? kNarrowBars : kWideAll;
+    static constexpr int kBars = kBars0 > 16 + kIdSlots ? kBars0 : 16 + kIdSlots;
     static constexpr int kBodyBytes =
         kNarrowBytes > kWideRingBytes + kScratchBytes ? kNarrowBytes : kWideRingBytes + kScratchBytes;
     static constexpr int kSmemBytes = kBodyBytes + kBars * 8 + 1024;   // + alignment slack
@@ -86,7 +91,7 @@ struct Shape {
     static_assert(kWarpStages >= 2, "suffix ring depth");
     static_assert(kWideStages >= 4, "prefix ring depth");
     static_assert(kSmemBytes <= kSmemBudget, "shared memory budget");
-    static_assert(kBars >= 16, "room for the tcgen05 prefix tile's barriers");
+
 };
 
 // K then V of one (page, kv head) into a stage: one TMA box {128 bytes, 1
@@ -379,66 +384,89 @@ __device__ __forceinline__ void store_warp_partials(const AttnArgs &a, const Wor
     }
 }
 
-// A worker's page stream, read by one whole warp: lane i holds entry
-// base + i of the window; row(q) returns entry q (q uniform over the warp,
-// nondecreasing), refilling the window with one coalesced load every 32.
-struct PageStream {
-    const int32_t *rows;
-    int size;
-    int base;
-    int win;
-    __device__ PageStream(const AttnArgs &a, int worker, int lane) {
-        const int s0 = a.stream_ptr[worker];
-        rows = a.stream_rows + s0;
-        size = a.stream_ptr[worker + 1] - s0;
-        base = 0;
-        win = rows[lane];                 // the stream array is padded by 32 entries
+// Work queues.  A queue position is taken with one atomicAdd; the merge
+// kernel rewinds both counters after every launch.
+__device__ __forceinline__ int pull(const AttnArgs &a, int which, int lane) {
+    int id = -1;
+    if (lane == 0) {
+        const int k = atomicAdd(a.queue_next + which, 1);
+        const int n = which == 0 ? a.num_wide_items : a.num_narrow_items;
+        if (k < n) id = (which == 0 ? a.wide_queue : a.narrow_queue)[k];
     }
-    __device__ __forceinline__ int row(int q, int lane) {
-        if (q >= base + 32) {
-            base = q & ~31;
-            win = rows[base + lane];
+    return __shfl_sync(0xffffffffu, id, 0);
+}
+
+// The TMA rows of one item's pages, read by one whole warp 32 at a time: lane
+// i holds row base + i; row(pg) returns the row of page pg (pg uniform over
+// the warp, nondecreasing within an item).
+struct ItemRows {
+    const int32_t *rows = nullptr;
+    int base = -1;
+    int win = 0;
+    __device__ void start(const AttnArgs &a, int item) {
+        rows = a.stream_rows + a.item_rows[item];
+        base = -1;
+    }
+    __device__ __forceinline__ int row(int pg, int lane) {
+        if (base < 0 || pg >= base + 32) {
+            base = pg & ~31;
+            win = rows[base + lane];        // the row array is padded by 32 entries
         }
-        return __shfl_sync(0xffffffffu, win, q - base);
+        return __shfl_sync(0xffffffffu, win, pg - base);
     }
 };
 
 // ---------------------------------------------------------------------------
-// suffix pass: every warp streams its own item list through its own ring
+// suffix pass: every warp pulls items from the suffix queue and streams their
+// pages through its own ring
 // ---------------------------------------------------------------------------
 template <int D, class KV>
 __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
-                            const AttnArgs &a, uint32_t ring, uint32_t bars, int warp, int lane) {
+                            const AttnArgs &a, uint32_t ring, uint32_t bars, int warp, int lane,
+                            volatile int *ids) {
     using S = Shape<D, KV>;
     constexpr int NS = S::kWarpStages;
-    const int worker = a.num_wide_ctas + (blockIdx.x - a.num_wide_ctas) * kConsumerWarps + warp;
-    const int i_begin = a.sched_ptr[worker], i_end = a.sched_ptr[worker + 1];
-    if (i_begin >= i_end) return;
     const uint32_t my_ring = ring + warp * S::kWarpRingBytes;
     const uint32_t my_bar = bars + warp * NS * 8;
+    const bool skip_first = (a.debug_flags & PARASON_DEBUG_SKIP_FIRST_LOAD) && warp == 0 &&
+                            static_cast<int>(blockIdx.x) >= a.num_wide_ctas;
 
-    // the warp's page stream: TMA rows read 32 at a time by the whole warp
-    PageStream ps(a, worker, lane);
-    const bool skip_first = (a.debug_flags & PARASON_DEBUG_SKIP_FIRST_LOAD) && warp == 0;
-    int issued = 0;
+    // issue side (whole warp, uniform): pulls items as its page cursor needs them
+    int pulled = 0, iss_pg = 0, iss_np = 0, issued = 0;
+    bool iss_done = false;
+    ItemRows rows;
     auto issue_next = [&]() {
-        // whole warp (uniform): the stream position is the same in every lane
-        if (issued >= ps.size) return;
-        const int row = ps.row(issued, lane);
+        if (iss_done) return;
+        while (iss_pg >= iss_np) {
+            const int id = pull(a, 1, lane);
+            if (id < 0) {
+                iss_done = true;
+                return;
+            }
+            if (lane == 0) ids[pulled % kGrabSlots] = id;
+            ++pulled;
+            iss_np = a.items[id].num_pages;
+            iss_pg = 0;
+            rows.start(a, id);
+        }
+        const int row = rows.row(iss_pg, lane);
         if (lane == 0 && !(skip_first && issued == 0)) {
             const int s = issued % NS;
             const uint32_t bar = my_bar + s * 8;
             dev::mbar_arrive_expect_tx(bar, S::kStageBytes);
             load_page<D, KV>(my_ring + s * S::kStageBytes, tmap_k, tmap_v, row, bar);
         }
+        ++iss_pg;
         ++issued;
     };
     for (int i = 0; i < NS; ++i) issue_next();
 
+    // consume side: the pulled items in order
     int consumed = 0;
     bool ok = true;
-    for (int ii = i_begin; ii < i_end && ok; ++ii) {
-        const WorkItem it = a.items[a.sched_items[ii]];
+    for (int k = 0; consumed < issued && ok; ++k) {
+        __syncwarp();
+        const WorkItem it = a.items[ids[k % kGrabSlots]];
         const float2 scl = item_scales<KV>(a, it);
         uint32_t qa[D / 16][4];
         load_q_fragments<D, KV>(a, it, 0, lane, qa);
@@ -474,47 +502,79 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
     __syncwarp();
 }
 
+// Prefix pass: the producer warp pulls items and hands their ids to the
+// consumer warps through kIdSlots shared slots, each with an mbarrier (id -1
+// ends the queue).  The producer is never more than a few items ahead of the
+// slowest consumer (it waits for ring stages they release), so the slots
+// are never overwritten before they are read.
+__device__ __forceinline__ void publish_id(volatile int *slots, uint32_t id_bars, int k, int id) {
+    slots[k % kIdSlots] = id;
+    dev::mbar_arrive(id_bars + 8 * (k % kIdSlots));
+}
+
+__device__ __forceinline__ int take_id(const volatile int *slots, uint32_t id_bars, int k,
+                                       long long limit, volatile int *abort, bool *ok) {
+    if (!dev::mbar_wait_bounded(id_bars + 8 * (k % kIdSlots), (k / kIdSlots) & 1, limit, abort)) {
+        *ok = false;
+        return -1;
+    }
+    return slots[k % kIdSlots];
+}
+
 // ---------------------------------------------------------------------------
 // prefix pass: up to 128 stacked rows share one page stream
 // ---------------------------------------------------------------------------
 template <int D, class KV>
 __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
                            const AttnArgs &a, uint8_t *smem, uint32_t ring, uint32_t bars,
-                           int warp, int lane, volatile int *abort_flag) {
+                           int warp, int lane, volatile int *abort_flag, volatile int *id_slots) {
     using S = Shape<D, KV>;
     constexpr int NS = S::kWideStages;
     const uint32_t bar_full = bars, bar_empty = bars + NS * 8;
-    const int i_begin = a.sched_ptr[blockIdx.x], i_end = a.sched_ptr[blockIdx.x + 1];
+    const uint32_t id_bars = bars + 2 * NS * 8;
     auto k_page = [&](int s) { return ring + s * S::kStageBytes; };
 
     if (warp == kConsumerWarps) {
         // ------------------------------------------------------------ producer
-        // the whole warp walks the page stream; lane 0 waits and issues
-        PageStream ps(a, blockIdx.x, lane);
+        // the whole warp pulls items and walks their pages; lane 0 waits and issues
         int last_issue[NS];
         for (int s = 0; s < NS; ++s) last_issue[s] = -1;
         const bool skip_first = a.debug_flags & PARASON_DEBUG_SKIP_FIRST_LOAD;
-        for (int stage = 0; stage < ps.size; ++stage) {
-            const int s = stage % NS;
-            int stop = 0;
-            if (lane == 0) {
-                if (stage >= NS && !dev::mbar_wait_bounded(bar_empty + 8 * s, ((stage / NS) - 1) & 1,
-                                                           a.wait_limit_ns, abort_flag)) {
-                    if (!*abort_flag) {
-                        *abort_flag = 1;
-                        dev::record_error(a.err, PARASON_ETIMEOUT, kSiteProducerEmpty);
+        int stage = 0;
+        bool go = true;
+        for (int k = 0; go; ++k) {
+            const int id = *abort_flag ? -1 : pull(a, 0, lane);
+            if (lane == 0) publish_id(id_slots, id_bars, k, id);
+            if (id < 0) break;
+            ItemRows rows;
+            rows.start(a, id);
+            const int np = a.items[id].num_pages;
+            for (int pg = 0; pg < np; ++pg, ++stage) {
+                const int s = stage % NS;
+                int stop = 0;
+                if (lane == 0) {
+                    if (stage >= NS && !dev::mbar_wait_bounded(bar_empty + 8 * s,
+                                                               ((stage / NS) - 1) & 1,
+                                                               a.wait_limit_ns, abort_flag)) {
+                        if (!*abort_flag) {
+                            *abort_flag = 1;
+                            dev::record_error(a.err, PARASON_ETIMEOUT, kSiteProducerEmpty);
+                        }
+                        stop = 1;
+                    } else if (*abort_flag) {
+                        stop = 1;
                     }
-                    stop = 1;
-                } else if (*abort_flag) {
-                    stop = 1;
                 }
-            }
-            if (__shfl_sync(0xffffffffu, stop, 0)) break;
-            const int row = ps.row(stage, lane);
-            if (lane == 0 && !(skip_first && stage == 0)) {
-                dev::mbar_arrive_expect_tx(bar_full + 8 * s, S::kStageBytes);
-                load_page<D, KV>(k_page(s), tmap_k, tmap_v, row, bar_full + 8 * s);
-                last_issue[s] = stage;
+                if (__shfl_sync(0xffffffffu, stop, 0)) {
+                    go = false;
+                    break;
+                }
+                const int row = rows.row(pg, lane);
+                if (lane == 0 && !(skip_first && stage == 0)) {
+                    dev::mbar_arrive_expect_tx(bar_full + 8 * s, S::kStageBytes);
+                    load_page<D, KV>(k_page(s), tmap_k, tmap_v, row, bar_full + 8 * s);
+                    last_issue[s] = stage;
+                }
             }
         }
         // every copy this CTA issued must land before its shared memory goes
@@ -533,8 +593,11 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
     const int tid = threadIdx.x;
     const int gid = lane >> 2, tig = lane & 3;
     int stage = 0;
-    for (int ii = i_begin; ii < i_end; ++ii) {
-        const WorkItem it = a.items[a.sched_items[ii]];
+    for (int k = 0;; ++k) {
+        bool got = true;
+        const int id = take_id(id_slots, id_bars, k, a.wait_limit_ns, abort_flag, &got);
+        if (dev::bar_sync_or<kConsumerThreads>(1, !got || id < 0)) break;
+        const WorkItem it = a.items[id];
         const float2 scl = item_scales<KV>(a, it);
         const int groups = (it.nrows + 15) >> 4;
         const int rgc = groups <= 2 ? 2 : (groups <= 4 ? 4 : 8);
@@ -699,24 +762,29 @@ __device__ __forceinline__ void tc_fail(const AttnArgs &a, volatile int *abort, 
 template <int D>
 __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
                               const AttnArgs &a, uint8_t *smem, uint32_t bars, uint32_t tmem,
-                              int warp, int lane, volatile int *abort_flag) {
+                              int warp, int lane, volatile int *abort_flag, volatile int *id_slots) {
     static_assert(D == 128, "the tcgen05 prefix tile is written for head_dim 128");
     const uint32_t ring = dev::smem_addr(smem);
     const uint32_t sq = ring + kTcRingBytes;
     const uint32_t sp = sq + kTcQBytes;
     auto bar = [&](int i) { return bars + 8u * static_cast<uint32_t>(i); };
-    const int i_begin = a.sched_ptr[blockIdx.x], i_end = a.sched_ptr[blockIdx.x + 1];
+    const uint32_t id_bars = bar(kTcBars);
 
     if (warp == kConsumerWarps) {
         // ------------------------------------------------------------ producer
-        PageStream ps(a, blockIdx.x, lane);
         const bool skip_first = a.debug_flags & PARASON_DEBUG_SKIP_FIRST_LOAD;
         int last_issue[kTcStages];
         for (int s = 0; s < kTcStages; ++s) last_issue[s] = -1;
-        int q = 0, blk = 0;
+        int blk = 0;
         bool ok = true;
-        for (int ii = i_begin; ii < i_end && ok; ++ii) {
-            const WorkItem it = a.items[a.sched_items[ii]];
+        for (int k = 0; ok; ++k) {
+            const int id = *abort_flag ? -1 : pull(a, 0, lane);
+            if (lane == 0) publish_id(id_slots, id_bars, k, id);
+            if (id < 0) break;
+            const WorkItem it = a.items[id];
+            ItemRows ps;
+            ps.start(a, id);
+            int q = 0;
             const int nb = (it.num_pages + kTcBlockPages - 1) / kTcBlockPages;
             for (int bi = 0; bi < nb; ++bi, ++blk) {
                 const int s = blk % kTcStages;
@@ -772,10 +840,12 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                 }
                 tc::commit(bar(kBarSFull + (b & 1)));
             };
-            int blk = 0, item = 0;
+            int blk = 0;
             bool ok = true;
-            for (int ii = i_begin; ii < i_end && ok; ++ii, ++item) {
-                const WorkItem it = a.items[a.sched_items[ii]];
+            for (int item = 0; ok; ++item) {
+                const int id = take_id(id_slots, id_bars, item, a.wait_limit_ns, abort_flag, &ok);
+                if (id < 0) break;
+                const WorkItem it = a.items[id];
                 const int nb = (it.num_pages + kTcBlockPages - 1) / kTcBlockPages;
                 if (!tc_wait(bar(kBarQReady), item & 1, a.wait_limit_ns, abort_flag) ||
                     !tc_wait(bar(kBarKvFull + blk % kTcStages), (blk / kTcStages) & 1,
@@ -824,8 +894,17 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(warp * 32) << 16);
         const uint32_t tO = lane_base, tS0 = lane_base + 128;
         int blk = 0;
-        for (int ii = i_begin; ii < i_end; ++ii) {
-            const WorkItem it = a.items[a.sched_items[ii]];
+        for (int item = 0;; ++item) {
+            int id = -1;
+            if (lane == 0) {
+                bool got = true;
+                id = take_id(id_slots, id_bars, item, a.wait_limit_ns, abort_flag, &got);
+                if (!got) id = -2;
+            }
+            id = __shfl_sync(0xffffffffu, id, 0);
+            if (id == -2 && lane == 0) tc_fail(a, abort_flag, kSiteConsumerFull);
+            if (id < 0) break;
+            const WorkItem it = a.items[id];
             const int nb = (it.num_pages + kTcBlockPages - 1) / kTcBlockPages;
             const int tokens = (it.num_pages - 1) * kPageSize + it.last_valid;
 
@@ -989,11 +1068,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t ring = dev::smem_addr(smem);
     const uint32_t bars = dev::smem_addr(smem + S::kBodyBytes);
     __shared__ int abort_flag;
+    __shared__ int id_slots[kIdSlots];                        // prefix-pass item ids
+    __shared__ int grab_ids[kConsumerWarps][kGrabSlots];      // suffix-pass item ids per warp
     const bool wide = static_cast<int>(blockIdx.x) < a.num_wide_ctas;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     // the prefix pass of bf16 KV at head_dim 128 runs on tcgen05
     constexpr bool kTcPrefix = (D == 128) && (KV::kElemBytes == 2);
+    constexpr int kPrefixBars = kTcPrefix ? kTcBars + kIdSlots : 2 * S::kWideStages + kIdSlots;
+    auto init_suffix_barriers = [&]() {
+        for (int s = 0; s < S::kNarrowBars; ++s) dev::mbar_init(bars + 8 * s, 1);
+    };
     __shared__ uint32_t tmem_base;
     if (threadIdx.x == 0) {
         abort_flag = 0;
@@ -1002,13 +1087,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 dev::mbar_init(bars + 8 * i, (i == kBarPFull || i == kBarPFull + 1 || i == kBarQReady)
                                                  ? kTcRows
                                                  : 1);
+            for (int i = 0; i < kIdSlots; ++i) dev::mbar_init(bars + 8 * (kTcBars + i), 1);
         } else if (wide) {
             for (int s = 0; s < S::kWideStages; ++s) {
                 dev::mbar_init(bars + 8 * s, 1);
                 dev::mbar_init(bars + 8 * (S::kWideStages + s), kConsumerWarps);
             }
+            for (int i = 0; i < kIdSlots; ++i) dev::mbar_init(bars + 8 * (2 * S::kWideStages + i), 1);
         } else {
-            for (int s = 0; s < S::kNarrowBars; ++s) dev::mbar_init(bars + 8 * s, 1);
+            init_suffix_barriers();
         }
         dev::fence_mbar_init();
         dev::prefetch_tensormap(&tmap_k);
@@ -1025,17 +1112,30 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (wide) {
         if constexpr (kTcPrefix) {
             tc::fence_after_sync();
-            prefix_cta_tc<D>(&tmap_k, &tmap_v, a, smem, bars, tmem_base, warp, lane, &abort_flag);
+            prefix_cta_tc<D>(&tmap_k, &tmap_v, a, smem, bars, tmem_base, warp, lane, &abort_flag,
+                             id_slots);
             tc::fence_before_sync();
             __syncthreads();
             tc::fence_after_sync();
             if (warp == 4) tc::dealloc<kTcTmemCols>(tmem_base);
         } else {
-            prefix_cta<D, KV>(&tmap_k, &tmap_v, a, smem, ring, bars, warp, lane, &abort_flag);
+            prefix_cta<D, KV>(&tmap_k, &tmap_v, a, smem, ring, bars, warp, lane, &abort_flag,
+                              id_slots);
         }
-    } else if (warp < kConsumerWarps) {
-        suffix_warp<D, KV>(&tmap_k, &tmap_v, a, ring, bars, warp, lane);
+        // the prefix queue is empty: this CTA joins the suffix queue with the
+        // same shared memory (every copy it issued has landed)
+        __syncthreads();
+        if (abort_flag) return;
+        if (threadIdx.x == 0) {
+            for (int i = 0; i < kPrefixBars; ++i)
+                asm volatile("mbarrier.inval.shared::cta.b64 [%0];" ::"r"(bars + 8 * i) : "memory");
+            init_suffix_barriers();
+            dev::fence_mbar_init();
+        }
+        __syncthreads();
     }
+    if (warp < kConsumerWarps)
+        suffix_warp<D, KV>(&tmap_k, &tmap_v, a, ring, bars, warp, lane, grab_ids[warp]);
 }
 
 // Shared memory and carveout are set once per device; reports the number of

@@ -57,14 +57,18 @@ struct AttnArgs {
     int32_t group;
     float scale_log2;       // sm_scale * log2(e): x_t = scale_log2 * <q, k_t>
 
-    // persistent schedule, CSR over workers: CTAs [0, num_wide_ctas) each run
-    // one list (prefix pass); every warp w of CTA c >= num_wide_ctas runs list
-    // num_wide_ctas + (c - num_wide_ctas) * 8 + w (suffix pass)
-    const int32_t *sched_ptr;
-    const int32_t *sched_items;
-    // worker w loads the pages of its items in order; their TMA rows
-    // (page * H_kv + kv head) * 16 are stream_rows[stream_ptr[w] ...]
-    const int32_t *stream_ptr;
+    // dynamic schedule: CTAs [0, num_wide_ctas) pull prefix-pass items from
+    // wide_queue and then suffix-pass items; every warp of the other CTAs
+    // pulls suffix-pass items from narrow_queue.  queue_next[0] / [1] are the
+    // next positions (zero at launch; the merge kernel zeroes them again).
+    const int32_t *wide_queue;
+    const int32_t *narrow_queue;
+    int32_t num_wide_items;
+    int32_t num_narrow_items;
+    int32_t *queue_next;
+    // TMA rows (page * H_kv + kv head) * 16 of item i's pages:
+    // stream_rows[item_rows[i] ...]
+    const int32_t *item_rows;
     const int32_t *stream_rows;
     int32_t num_ctas;
     int32_t num_wide_ctas;
@@ -83,6 +87,7 @@ struct MergeArgs {
     int32_t num_q_heads;
     int32_t num_kv_heads;
     int32_t group;
+    int32_t *queue_next;        // zeroed for the next launch
 };
 
 // Resident CTAs per SM of the persistent attention kernel of a mode (sets its

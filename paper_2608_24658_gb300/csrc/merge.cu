@@ -105,6 +105,11 @@ __global__ void __launch_bounds__(kMergeThreads)
     const int e0 = active ? a.merge_ptr[pair] : 0, e1 = active ? a.merge_ptr[pair + 1] : 0;
     int first_slot = (e0 + lane < e1) ? a.merge_ent[e0 + lane] + r : 0;
     asm volatile("griddepcontrol.wait;" ::: "memory");
+    // the attention grid is complete: rewind its work queues for the next call
+    if (blockIdx.x == 0 && threadIdx.x == 0 && a.queue_next) {
+        a.queue_next[0] = 0;
+        a.queue_next[1] = 0;
+    }
     if (!active) return;
 
     float M = -INFINITY, L = 0.f;
@@ -134,15 +139,22 @@ __global__ void __launch_bounds__(kMergeThreads)
         L = L * s_old + lw;
 #pragma unroll
         for (int i = 0; i < N; ++i) acc[i] *= s_old;
+        // partial rows are requested 8 at a time before any of them is used
         const int cnt = min(32, e1 - base);
-#pragma unroll 8
-        for (int i = 0; i < cnt; ++i) {
-            const int si = __shfl_sync(0xffffffffu, slot, i);
-            const float wi = __shfl_sync(0xffffffffu, wgt, i);
-            float v[N];
-            load_f32<N>(a.part_o + static_cast<int64_t>(si) * D + lane * N, v);
+        for (int i0 = 0; i0 < cnt; i0 += 8) {
+            float v[8][N];
 #pragma unroll
-            for (int k = 0; k < N; ++k) acc[k] += wi * v[k];
+            for (int i = 0; i < 8; ++i) {
+                const int si = __shfl_sync(0xffffffffu, slot, (i0 + i) & 31);
+                if (i0 + i < cnt) load_f32<N>(a.part_o + static_cast<int64_t>(si) * D + lane * N, v[i]);
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const float wi = __shfl_sync(0xffffffffu, wgt, (i0 + i) & 31);
+                if (i0 + i < cnt)
+#pragma unroll
+                    for (int k = 0; k < N; ++k) acc[k] += wi * v[i][k];
+            }
         }
         M = Mn;
     }

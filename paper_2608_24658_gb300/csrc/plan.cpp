@@ -31,7 +31,10 @@ namespace {
 
 constexpr int kNarrowRows = 16;         // nodes with at most this many rows: suffix pass
 constexpr int kNarrowWarps = 8;         // autonomous warps per suffix-pass CTA
-constexpr int kMinPiecePages = 4;       // no split leaves a piece shorter than this
+constexpr int kMinPiecePages = 8;       // suffix-pass pieces are at least this long
+constexpr int kMaxPiecePages = 128;     // and at most this long
+constexpr int kWideBlockPages = 4;      // prefix pieces are whole 64-token blocks
+constexpr double kWideProvision = 1.15; // prefix CTAs relative to the cost model
 constexpr int kFp32ChunkPages = 32;
 constexpr double kWideGroupPageCost = 1.0;   // one 16-row group of one page, in suffix pages
 constexpr double kTcPageCost = 2.2;          // one page of a tcgen05 prefix tile (measured)
@@ -71,16 +74,16 @@ struct parason_plan_s {
     int32_t num_leaves = 0;
     int64_t num_phys = 0;
     int32_t num_sms = 152;
-    int32_t chunk_pages = kMinPiecePages;
+    int32_t chunk_pages = kMinPiecePages;   // reported shortest piece
     std::vector<WorkItem> items;
     std::vector<int32_t> page_ids;
     std::vector<int32_t> dfs_leaf;
     std::vector<int32_t> merge_ptr;
     std::vector<int32_t> merge_ent;   // first partial slot of the branch's rows
-    std::vector<int32_t> sched_ptr;   // persistent schedule, CSR over workers:
-    std::vector<int32_t> sched_items; // wide CTAs first, then narrow warps
-    std::vector<int32_t> stream_ptr;  // per worker: start of its page stream
-    std::vector<int32_t> stream_rows; // TMA row of every page, worker by worker
+    std::vector<int32_t> wide_queue;   // prefix-pass items, in pull order
+    std::vector<int32_t> narrow_queue; // suffix-pass items, in pull order
+    std::vector<int32_t> item_rows;    // per item: start of its page rows
+    std::vector<int32_t> stream_rows;  // TMA row of every page, item by item
     int32_t num_ctas = 0;
     int32_t num_wide_ctas = 0;
     int64_t num_slots = 0;
@@ -96,10 +99,11 @@ struct parason_plan_s {
     int32_t *d_dfs_leaf = nullptr;
     int32_t *d_merge_ptr = nullptr;
     int32_t *d_merge_ent = nullptr;
-    int32_t *d_sched_ptr = nullptr;
-    int32_t *d_sched_items = nullptr;
-    int32_t *d_stream_ptr = nullptr;
+    int32_t *d_wide_queue = nullptr;
+    int32_t *d_narrow_queue = nullptr;
+    int32_t *d_item_rows = nullptr;
     int32_t *d_stream_rows = nullptr;
+    int32_t *d_queue_next = nullptr;   // 2 counters, zeroed by the merge kernel
     int32_t *d_err = nullptr;
     uint32_t debug_flags = 0;
     int64_t wait_limit_ns = kDefaultWaitNs;
@@ -267,16 +271,18 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
             }
     }
 
-    // workers: wide CTAs (prefix pass) and narrow warps (suffix pass) of the
-    // persistent kernel; the fp32 kernel runs one item per CTA instead
+    // CTAs of the persistent kernel: the first n_wide start on the prefix
+    // queue and join the suffix queue when it runs dry, the others run the
+    // suffix queue only.  Prefix CTAs are over-provisioned on purpose: spare
+    // prefix capacity turns into suffix work, a prefix shortfall would be the
+    // tail.  The fp32 kernel runs one item per CTA instead.
     int32_t n_wide = 0, n_narrow_ctas = 0;
     if (mode != PARASON_FP32) {
         const int32_t S = p->num_sms;
         const double narrow_cost = static_cast<double>(narrow_pages);
-        // each role gets at least one CTA; the grid may exceed the SM count
-        // (CTAs of the persistent kernel never wait on one another)
         if (wide_cost > 0 && narrow_cost > 0) {
-            n_wide = static_cast<int32_t>(std::lround(S * wide_cost / (wide_cost + narrow_cost)));
+            n_wide = static_cast<int32_t>(
+                std::ceil(kWideProvision * S * wide_cost / (wide_cost + narrow_cost)));
             n_wide = std::min(std::max(n_wide, 1), std::max(S - 1, 1));
         } else if (wide_cost > 0) {
             n_wide = S;
@@ -285,15 +291,15 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     }
     p->num_wide_ctas = n_wide;
     p->num_ctas = n_wide + n_narrow_ctas;
-    const int64_t n_narrow_workers = static_cast<int64_t>(n_narrow_ctas) * kNarrowWarps;
 
-    // balanced contiguous partition of the runs of one role over its workers:
-    // worker k gets the pages whose cumulative cost falls in [k T/W, (k+1) T/W)
+    // Items: every run cut into pieces of at most `chunk` pages (the prefix
+    // pass in whole 64-token blocks).  Each role's pieces form a queue,
+    // longest first, that the kernel's workers pull from at run time; the
+    // pieces are short enough that the last ones to be pulled end together.
     p->items.clear();
-    std::vector<int32_t> worker_of_item;
-    std::vector<int64_t> slot_of_item;
     int64_t slots = 0;
-    auto emit = [&](const Run &run, int64_t pg0, int64_t np, int32_t worker) -> bool {
+    std::vector<std::pair<int64_t, int32_t>> wide_q, narrow_q;   // (pages, item)
+    auto emit = [&](const Run &run, int64_t pg0, int64_t np) -> bool {
         WorkItem it;
         const int64_t P = run.pages;
         it.page_pos = node_page_ptr[run.node] + static_cast<int32_t>(pg0);
@@ -308,85 +314,68 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         if (slots + run.nrows > INT32_MAX) return false;
         it.slot_base = static_cast<int32_t>(slots);
         slots += run.nrows;
+        const int32_t id = static_cast<int32_t>(p->items.size());
         p->items.push_back(it);
-        worker_of_item.push_back(worker);
+        (run.wide ? wide_q : narrow_q).emplace_back(np, id);
         return true;
     };
-    auto partition = [&](bool wide_role, int64_t workers, int64_t worker0, int64_t min_chunk) -> bool {
-        double total = 0.0;
-        for (const Run &r : runs)
-            if (r.wide == wide_role) total += r.cost_per_page * static_cast<double>(r.pages);
-        if (total <= 0.0) return true;
-        const double share = total / static_cast<double>(std::max<int64_t>(workers, 1));
-        double acc = 0.0;                       // cost before the current page
-        for (const Run &r : runs) {
-            if (r.wide != wide_role) continue;
-            int64_t pg = 0;
-            while (pg < r.pages) {
-                int64_t k = std::min<int64_t>(workers - 1, static_cast<int64_t>(acc / share));
-                // pages of this run that fit before worker k's share ends
-                const int64_t left = r.pages - pg;
-                int64_t np = left;
-                if (k + 1 < workers) {
-                    const double fit = std::ceil(((k + 1) * share - acc) / r.cost_per_page - 1e-9);
-                    if (fit < static_cast<double>(left)) np = std::max<int64_t>(1, static_cast<int64_t>(fit));
-                }
-                // avoid crumbs: a piece shorter than min_chunk joins its neighbour
-                if (r.pages - (pg + np) < min_chunk) np = r.pages - pg;
-                np = std::min<int64_t>(np, r.pages - pg);
-                if (!emit(r, pg, np, static_cast<int32_t>(worker0 + k))) return false;
-                acc += r.cost_per_page * static_cast<double>(np);
-                pg += np;
-            }
-        }
+    auto cut = [&](const Run &r, int64_t chunk, int64_t align) -> bool {
+        chunk = std::max<int64_t>(align, chunk / align * align);
+        const int64_t n = (r.pages + chunk - 1) / chunk;
+        // equal pieces (multiples of `align` except the last)
+        int64_t per = (r.pages + n - 1) / n;
+        per = (per + align - 1) / align * align;
+        for (int64_t pg = 0; pg < r.pages; pg += per)
+            if (!emit(r, pg, std::min(per, r.pages - pg))) return false;
         return true;
     };
     if (mode == PARASON_FP32) {
-        // one item per CTA: chunks of about kFp32ChunkPages pages
-        for (const Run &r : runs) {
-            const int64_t nc = std::max<int64_t>(1, (r.pages + kFp32ChunkPages - 1) / kFp32ChunkPages);
-            const int64_t base = r.pages / nc, rem = r.pages % nc;
-            int64_t pg = 0;
-            for (int64_t c = 0; c < nc; ++c) {
-                const int64_t np = base + (c < rem ? 1 : 0);
-                if (!emit(r, pg, np, 0)) return PARASON_EUNSUPPORTED;
-                pg += np;
-            }
-        }
+        for (const Run &r : runs)
+            if (!cut(r, kFp32ChunkPages, 1)) return PARASON_EUNSUPPORTED;
     } else {
-        if (!partition(true, n_wide, 0, kMinPiecePages)) return PARASON_EUNSUPPORTED;
-        if (!partition(false, n_narrow_workers, n_wide, kMinPiecePages)) return PARASON_EUNSUPPORTED;
+        const int64_t total_warps = static_cast<int64_t>(p->num_sms) * kNarrowWarps;
+        const int64_t narrow_chunk = std::min<int64_t>(
+            kMaxPiecePages,
+            std::max<int64_t>(kMinPiecePages, narrow_pages / std::max<int64_t>(1, total_warps * 3)));
+        int64_t wide_pages = 0;
+        for (const Run &r : runs)
+            if (r.wide) wide_pages += r.pages;
+        const int64_t wide_chunk = std::min<int64_t>(
+            kMaxPiecePages,
+            std::max<int64_t>(kWideBlockPages,
+                              wide_pages / std::max<int64_t>(1, static_cast<int64_t>(n_wide) * 3)));
+        for (const Run &r : runs)
+            if (!cut(r, r.wide ? wide_chunk : narrow_chunk, r.wide ? kWideBlockPages : 1))
+                return PARASON_EUNSUPPORTED;
     }
     if (p->items.size() > static_cast<size_t>(INT32_MAX)) return PARASON_EUNSUPPORTED;
     p->num_slots = slots;
 
-    // schedule: worker lists in item order (each worker's items are one
-    // contiguous stretch of the partition)
-    const int64_t n_workers = mode == PARASON_FP32 ? 0 : n_wide + n_narrow_workers;
-    p->sched_ptr.assign(static_cast<size_t>(n_workers) + 1, 0);
-    p->sched_items.clear();
-    if (n_workers > 0) {
-        std::vector<int32_t> count(static_cast<size_t>(n_workers), 0);
-        for (int32_t w : worker_of_item) count[w]++;
-        for (int64_t w = 0; w < n_workers; ++w) p->sched_ptr[w + 1] = p->sched_ptr[w] + count[w];
-        p->sched_items.assign(p->items.size(), 0);
-        std::vector<int32_t> fill(p->sched_ptr.begin(), p->sched_ptr.end() - 1);
-        for (size_t i = 0; i < p->items.size(); ++i)
-            p->sched_items[fill[worker_of_item[i]]++] = static_cast<int32_t>(i);
+    // queues, longest piece first (ties in item order)
+    auto order = [](std::vector<std::pair<int64_t, int32_t>> &q, std::vector<int32_t> &out) {
+        std::stable_sort(q.begin(), q.end(),
+                         [](const auto &a, const auto &b) { return a.first > b.first; });
+        out.clear();
+        for (auto &e : q) out.push_back(e.second);
+    };
+    order(wide_q, p->wide_queue);
+    order(narrow_q, p->narrow_queue);
+    if (mode == PARASON_FP32) {        // one CTA per item, no queues
+        p->wide_queue.clear();
+        p->narrow_queue.clear();
     }
-    // page streams: the TMA row (page * H_kv + kv head) * 16 of every page a
-    // worker loads, in the order it loads them
-    p->stream_ptr.assign(static_cast<size_t>(n_workers) + 1, 0);
+
+    // page streams: the TMA row (page * H_kv + kv head) * 16 of every page of
+    // every item, item by item
+    p->item_rows.assign(p->items.size() + 1, 0);
     p->stream_rows.clear();
-    for (int64_t w = 0; w < n_workers; ++w) {
-        for (int32_t k = p->sched_ptr[w]; k < p->sched_ptr[w + 1]; ++k) {
-            const WorkItem &it = p->items[p->sched_items[k]];
-            for (int32_t pg = 0; pg < it.num_pages; ++pg)
-                p->stream_rows.push_back((page_ids[it.page_pos + pg] * H_kv + it.kv_head) *
-                                         parason::kPageSize);
-        }
+    for (size_t i = 0; i < p->items.size(); ++i) {
+        const WorkItem &it = p->items[i];
+        for (int32_t pg = 0; pg < it.num_pages; ++pg)
+            p->stream_rows.push_back((page_ids[it.page_pos + pg] * H_kv + it.kv_head) *
+                                     parason::kPageSize);
         if (p->stream_rows.size() > static_cast<size_t>(INT32_MAX)) return PARASON_EUNSUPPORTED;
-        p->stream_ptr[w + 1] = static_cast<int32_t>(p->stream_rows.size());
+        p->item_rows[i + 1] = static_cast<int32_t>(p->stream_rows.size());
     }
 
     // merge lists per (branch, kv head): the first of the branch's g partial
@@ -423,17 +412,18 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     const size_t n_dfs = p->dfs_leaf.size() * sizeof(int32_t);
     const size_t n_mptr = p->merge_ptr.size() * sizeof(int32_t);
     const size_t n_ment = p->merge_ent.size() * sizeof(int32_t);
-    const size_t n_sptr = p->sched_ptr.size() * sizeof(int32_t);
-    const size_t n_sitems = p->sched_items.size() * sizeof(int32_t);
-    const size_t n_stptr = p->stream_ptr.size() * sizeof(int32_t);
-    // page streams are read 32 entries past their end by whole warps: pad
+    const size_t n_wq = p->wide_queue.size() * sizeof(int32_t);
+    const size_t n_nq = p->narrow_queue.size() * sizeof(int32_t);
+    const size_t n_irows = p->item_rows.size() * sizeof(int32_t);
+    // page rows are read 32 entries past their end by whole warps: pad
     const size_t n_strows = (p->stream_rows.size() + 32) * sizeof(int32_t);
+    const size_t n_qnext = 2 * sizeof(int32_t);
     const size_t n_err = parason::kErrWords * sizeof(int32_t);
-    constexpr int kArrays = 10;
+    constexpr int kArrays = 11;
     size_t off[kArrays], total = 0;
-    // the last one (error record) is zero-filled, not copied
-    const size_t sizes[kArrays] = {n_items, n_pages,  n_dfs,   n_mptr,   n_ment,
-                                   n_sptr,  n_sitems, n_stptr, n_strows, n_err};
+    // the last two (queue counters, error record) are zero-filled, not copied
+    const size_t sizes[kArrays] = {n_items, n_pages,  n_dfs,    n_mptr,  n_ment, n_wq,
+                                   n_nq,    n_irows,  n_strows, n_qnext, n_err};
     for (int i = 0; i < kArrays; ++i) {
         off[i] = total;
         total = align_up(total + std::max<size_t>(sizes[i], 4), kAlign);
@@ -449,15 +439,16 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     p->d_dfs_leaf = reinterpret_cast<int32_t *>(base + off[2]);
     p->d_merge_ptr = reinterpret_cast<int32_t *>(base + off[3]);
     p->d_merge_ent = reinterpret_cast<int32_t *>(base + off[4]);
-    p->d_sched_ptr = reinterpret_cast<int32_t *>(base + off[5]);
-    p->d_sched_items = reinterpret_cast<int32_t *>(base + off[6]);
-    p->d_stream_ptr = reinterpret_cast<int32_t *>(base + off[7]);
+    p->d_wide_queue = reinterpret_cast<int32_t *>(base + off[5]);
+    p->d_narrow_queue = reinterpret_cast<int32_t *>(base + off[6]);
+    p->d_item_rows = reinterpret_cast<int32_t *>(base + off[7]);
     p->d_stream_rows = reinterpret_cast<int32_t *>(base + off[8]);
-    p->d_err = reinterpret_cast<int32_t *>(base + off[9]);
-    const void *src[9] = {p->items.data(),     p->page_ids.data(),  p->dfs_leaf.data(),
-                          p->merge_ptr.data(), p->merge_ent.data(), p->sched_ptr.data(),
-                          p->sched_items.data(), p->stream_ptr.data(), p->stream_rows.data()};
-    const size_t copy[9] = {n_items, n_pages, n_dfs, n_mptr, n_ment, n_sptr, n_sitems, n_stptr,
+    p->d_queue_next = reinterpret_cast<int32_t *>(base + off[9]);
+    p->d_err = reinterpret_cast<int32_t *>(base + off[10]);
+    const void *src[9] = {p->items.data(),      p->page_ids.data(),    p->dfs_leaf.data(),
+                          p->merge_ptr.data(),  p->merge_ent.data(),   p->wide_queue.data(),
+                          p->narrow_queue.data(), p->item_rows.data(), p->stream_rows.data()};
+    const size_t copy[9] = {n_items, n_pages, n_dfs, n_mptr, n_ment, n_wq, n_nq, n_irows,
                             p->stream_rows.size() * sizeof(int32_t)};
     for (int i = 0; i < 9; ++i) {
         if (copy[i] == 0) continue;
@@ -466,6 +457,7 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
             return PARASON_ECUDA;
     }
     if (cudaMemsetAsync(p->d_err, 0, n_err, stream) != cudaSuccess) return PARASON_ECUDA;
+    if (cudaMemsetAsync(p->d_queue_next, 0, n_qnext, stream) != cudaSuccess) return PARASON_ECUDA;
     // the host vectors are pageable: make sure the copies have consumed them
     // before the caller can free its own arrays (ours stay alive anyway)
     if (cudaStreamSynchronize(stream) != cudaSuccess) return PARASON_ECUDA;
@@ -665,10 +657,13 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
         a.num_kv_heads = p->cfg.num_kv_heads;
         a.group = p->group;
         a.scale_log2 = sm_scale * 1.4426950408889634f;
-        a.sched_ptr = p->d_sched_ptr;
-        a.sched_items = p->d_sched_items;
-        a.stream_ptr = p->d_stream_ptr;
+        a.wide_queue = p->d_wide_queue;
+        a.narrow_queue = p->d_narrow_queue;
+        a.num_wide_items = static_cast<int32_t>(p->wide_queue.size());
+        a.num_narrow_items = static_cast<int32_t>(p->narrow_queue.size());
+        a.item_rows = p->d_item_rows;
         a.stream_rows = p->d_stream_rows;
+        a.queue_next = p->d_queue_next;
         a.num_ctas = p->num_ctas;
         a.num_wide_ctas = p->num_wide_ctas;
         a.kv_rows = static_cast<int32_t>(p->num_phys * p->cfg.num_kv_heads * parason::kPageSize);
@@ -712,6 +707,7 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
     m.num_q_heads = p->cfg.num_q_heads;
     m.group = p->group;
     m.num_kv_heads = p->cfg.num_kv_heads;
+    m.queue_next = p->d_queue_next;
     // programmatic dependent launch after the persistent kernel: the merge
     // grid is launched while the attention grid drains, and waits for it
     const bool pdl = has_items && p->cfg.mode != PARASON_FP32;
@@ -747,6 +743,7 @@ parason_status parason_plan_check(parason_plan p, parason_stream_t stream) {
         return PARASON_ECUDA;
     if (rec[0] != 0) {
         if (cudaMemset(p->d_err, 0, sizeof rec) != cudaSuccess) return PARASON_ECUDA;
+        if (cudaMemset(p->d_queue_next, 0, 2 * sizeof(int32_t)) != cudaSuccess) return PARASON_ECUDA;
         return rec[0] == PARASON_ETIMEOUT ? PARASON_ETIMEOUT : PARASON_ECUDA;
     }
     return PARASON_OK;
@@ -784,7 +781,8 @@ parason_status parason_plan_get_info(parason_plan p, parason_plan_info *info) {
     info->on_device = p->on_device ? 1 : 0;
     info->num_ctas = p->num_ctas;
     info->num_wide_ctas = p->num_wide_ctas;
-    info->num_workers = p->sched_ptr.empty() ? 0 : static_cast<int32_t>(p->sched_ptr.size()) - 1;
+    info->num_wide_items = static_cast<int32_t>(p->wide_queue.size());
+    info->num_narrow_items = static_cast<int32_t>(p->narrow_queue.size());
     return PARASON_OK;
 }
 
@@ -797,8 +795,8 @@ parason_status parason_plan_export(parason_plan p, int32_t table, void *dst, siz
     case PARASON_TABLE_DFS_LEAVES: src = p->dfs_leaf.data(); n = p->dfs_leaf.size() * 4; break;
     case PARASON_TABLE_MERGE_PTR: src = p->merge_ptr.data(); n = p->merge_ptr.size() * 4; break;
     case PARASON_TABLE_MERGE: src = p->merge_ent.data(); n = p->merge_ent.size() * 4; break;
-    case PARASON_TABLE_SCHEDULE_PTR: src = p->sched_ptr.data(); n = p->sched_ptr.size() * 4; break;
-    case PARASON_TABLE_SCHEDULE: src = p->sched_items.data(); n = p->sched_items.size() * 4; break;
+    case PARASON_TABLE_WIDE_QUEUE: src = p->wide_queue.data(); n = p->wide_queue.size() * 4; break;
+    case PARASON_TABLE_NARROW_QUEUE: src = p->narrow_queue.data(); n = p->narrow_queue.size() * 4; break;
     default: return PARASON_EINVAL;
     }
     if (bytes < n || (n > 0 && !dst)) return PARASON_EINVAL;

@@ -94,24 +94,23 @@ def verify_plan(tree, plan):
             assert got == sorted(slots_of[(b, h)]), (b, h)
     assert info["unique_tokens"] == tree.unique_tokens()
     assert info["path_tokens"] == tree.path_tokens()
-    # persistent schedule: every item in exactly one worker list
-    sptr = plan.export(_lib.TABLE_SCHEDULE_PTR)
-    sched = plan.export(_lib.TABLE_SCHEDULE)
+    # work queues: every item in exactly one queue, longest first; prefix
+    # pieces belong to nodes with more than 16 rows
+    wq = plan.export(_lib.TABLE_WIDE_QUEUE)
+    nq = plan.export(_lib.TABLE_NARROW_QUEUE)
     if tree.mode == "fp32":
-        assert info["num_workers"] == 0
+        assert len(wq) == 0 and len(nq) == 0
     else:
-        assert sorted(sched.tolist()) == list(range(len(items)))
-        assert sptr[0] == 0 and sptr[-1] == len(items) and np.all(np.diff(sptr) >= 0)
-        n_wide = info["num_wide_ctas"]
-        assert info["num_workers"] == n_wide + (info["num_ctas"] - n_wide) * 8
+        assert sorted(wq.tolist() + nq.tolist()) == list(range(len(items)))
+        for q in (wq, nq):
+            pages = items[q, 1] if len(q) else np.zeros(0)
+            assert np.all(np.diff(pages) <= 0), "queue not longest first"
+        for i in wq:
+            assert len(under[int(owner[items[i][0]])]) * g > 16
+        for i in nq:
+            assert len(under[int(owner[items[i][0]])]) * g <= 16
         assert info["num_ctas"] <= max(info["num_sms"], 2)
-        for w in range(info["num_workers"]):
-            for i in sched[sptr[w]:sptr[w + 1]]:
-                wide_item = items[i][5] > 16 or (items[i][5] == 16 and False)
-                # prefix-pass CTAs run the tiles of nodes with more than 16 rows
-                n = int(owner[items[i][0]])
-                rows_of_node = len(under[n]) * g
-                assert (w < n_wide) == (rows_of_node > 16), (w, n_wide, rows_of_node)
+        assert (info["num_wide_ctas"] > 0) == (len(wq) > 0)
     return info
 
 
@@ -164,13 +163,10 @@ def test_plan_large_configs(idx):
         assert one[:, 1].sum() == sum(
             tree.node_page_ptr[n + 1] - tree.node_page_ptr[n]
             for n in range(tree.num_nodes) if tree.node_len[n] > 0)
-        # balanced suffix pass: every warp's page count within a few pages of the mean
-        sptr = plan.export(_lib.TABLE_SCHEDULE_PTR)
-        sched = plan.export(_lib.TABLE_SCHEDULE)
-        n_wide = info["num_wide_ctas"]
-        loads = [int(items[sched[sptr[w]:sptr[w + 1]], 1].sum())
-                 for w in range(n_wide, info["num_workers"])]
-        assert max(loads) - min(loads) <= 2 * 4 + 1, (min(loads), max(loads))
+        # suffix pieces are short against a warp's share of the suffix pages
+        nq = plan.export(_lib.TABLE_NARROW_QUEUE)
+        share = items[nq, 1].sum() / (info["num_sms"] * 8)
+        assert items[nq, 1].max() <= max(8, share / 2), (items[nq, 1].max(), share)
 
 
 def test_plan_deterministic():
