@@ -158,6 +158,43 @@ parason_status parason_attn_decode(parason_plan plan, const void *q, const void 
                                    void *workspace, size_t workspace_bytes,
                                    parason_stream_t stream);
 
+/* Scratch, in bytes, that parason_attn_decode_no_alloc holds per device. */
+#define PARASON_NO_ALLOC_SCRATCH_BYTES (64u << 20)
+
+/*
+ * parason_attn_decode without a caller workspace.  The paper has no
+ * counterpart: this is a library convenience for callers that cannot hand
+ * over device memory at decode time -- an engine whose HBM is fully
+ * committed to its KV page pool and fixed buffers, or a C host with no device
+ * allocator of its own.  The partial results go to a scratch array that is
+ * part of the library's device image: PARASON_NO_ALLOC_SCRATCH_BYTES (64 MiB)
+ * per device, reserved when the library's device code is loaded on that
+ * device.  Neither this call nor anything it calls allocates device memory.
+ *
+ * Arguments, layouts, results and errors are those of parason_attn_decode,
+ * plus:
+ *   - PARASON_EUNSUPPORTED if parason_plan_workspace_bytes(plan) exceeds
+ *     PARASON_NO_ALLOC_SCRATCH_BYTES (checked before anything else is
+ *     touched; such a plan needs parason_attn_decode with a workspace).
+ *     At head_dim 128 the scratch holds about 129,000 partial rows, e.g. a
+ *     Llama-3-8B step of 16 branches over a 2048-token prefix needs 7.2 MB.
+ *   - The first call on each device looks up the scratch's device address
+ *     (with that device current) and keeps it for the life of the process;
+ *     make that first call outside any stream capture.  The address is not
+ *     looked up again, so the device's primary context must not be reset
+ *     afterwards.
+ *   - Nothing in the scratch has to start at zero and nothing in it is kept
+ *     between calls: every partial row the merge reads is written earlier in
+ *     the same call.
+ *   - All calls on one device share the one scratch array, whatever their
+ *     plan or stream: two calls that overlap in time race on it and both
+ *     results are undefined.  Calls issued to a single stream never overlap.
+ */
+parason_status parason_attn_decode_no_alloc(parason_plan plan, const void *q,
+                                            const void *k_pages, const void *v_pages,
+                                            const float *k_scale, const float *v_scale,
+                                            void *out, float *lse, parason_stream_t stream);
+
 /*
  * Combine two attention results over disjoint key sets A and B (for example
  * two KV ranges of one branch, or a branch's context before and after a join)

@@ -16,6 +16,7 @@ MODES = {"bf16": 0, "fp32": 1, "fp8": 2}
 (TABLE_ITEMS, TABLE_DFS_LEAVES, TABLE_MERGE_PTR, TABLE_MERGE, TABLE_WIDE_QUEUE,
  TABLE_NARROW_QUEUE) = range(6)
 DEBUG_SKIP_FIRST_LOAD = 1
+NO_ALLOC_SCRATCH_BYTES = 64 << 20   # PARASON_NO_ALLOC_SCRATCH_BYTES
 
 # every function include/parason.h declares, with (restype, argtypes)
 _p = ctypes.c_void_p
@@ -48,6 +49,7 @@ SIGNATURES = {
                                               _i32, _p, _i64, _i32, _pp]),
     "parason_plan_workspace_bytes": (_sz, [_p]),
     "parason_attn_decode": (ctypes.c_int, [_p, _p, _p, _p, _p, _p, _p, _p, _p, _sz, _p]),
+    "parason_attn_decode_no_alloc": (ctypes.c_int, [_p, _p, _p, _p, _p, _p, _p, _p, _p]),
     "parason_lse_merge": (ctypes.c_int, [_p, _p, _p, _p, _p, _p, _i64, _i32, _i32, _p]),
     "parason_plan_check": (ctypes.c_int, [_p, _p]),
     "parason_plan_destroy": (None, [_p]),

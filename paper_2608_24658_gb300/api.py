@@ -177,6 +177,38 @@ class Plan:
         check(st, "parason_attn_decode")
         return out, lse
 
+    def decode_no_alloc(self, q: torch.Tensor, k_pages: torch.Tensor, v_pages: torch.Tensor,
+                        out: torch.Tensor, lse: Optional[torch.Tensor] = None, k_scale=None,
+                        v_scale=None, stream=None):
+        """``decode`` into caller-given ``out`` / ``lse`` with the library's fixed
+        per-device scratch instead of a workspace; returns (out, lse).  Calls on
+        one device must not overlap in time (they share the scratch)."""
+        L, Hq, Hkv, d = self.num_leaves, self.num_q_heads, self.num_kv_heads, self.head_dim
+        qd, kvd = _Q_DTYPES[self.mode], _KV_DTYPES[self.mode]
+        for name, t in (("q", q), ("out", out)):
+            if t.dtype != qd or tuple(t.shape) != (L, Hq, d) or not t.is_cuda or not t.is_contiguous():
+                raise ValueError(f"{name} must be a contiguous cuda {qd} tensor of shape {(L, Hq, d)}")
+        for name, t in (("k_pages", k_pages), ("v_pages", v_pages)):
+            if (t.dtype != kvd or t.dim() != 4 or tuple(t.shape[1:]) != (Hkv, 16, d)
+                    or t.shape[0] < self.num_physical_pages or not t.is_contiguous()
+                    or t.device != q.device):
+                raise ValueError(f"{name} must be a contiguous {kvd} tensor "
+                                 f"[>= {self.num_physical_pages}, {Hkv}, 16, {d}] on {q.device}")
+        if lse is not None and (lse.dtype != torch.float32 or tuple(lse.shape) != (L, Hq)
+                                or not lse.is_cuda or not lse.is_contiguous()):
+            raise ValueError(f"lse must be a contiguous cuda float32 tensor of shape {(L, Hq)}")
+        if self.mode == "fp8":
+            if k_scale is None or v_scale is None:
+                raise ValueError("fp8 mode needs k_scale and v_scale")
+            for s in (k_scale, v_scale):
+                if s.dtype != torch.float32 or s.numel() != Hkv or not s.is_cuda:
+                    raise ValueError(f"scales must be cuda float32 [{Hkv}]")
+        st = _lib.load().parason_attn_decode_no_alloc(
+            self.handle, _ptr(q), _ptr(k_pages), _ptr(v_pages), _ptr(k_scale), _ptr(v_scale),
+            _ptr(out), _ptr(lse), _stream_handle(stream))
+        check(st, "parason_attn_decode_no_alloc")
+        return out, lse
+
     def decode_tree(self, tree, **kw):
         """``decode`` with the tensors of a ``workloads.ForkTree``."""
         return self.decode(tree.q, tree.k_pages, tree.v_pages, k_scale=tree.k_scale,
