@@ -43,7 +43,10 @@ namespace {
 
 constexpr int kConsumerWarps = 8;
 constexpr int kConsumerThreads = kConsumerWarps * 32;
-constexpr int kThreads = kConsumerThreads + 32;            // + producer warp
+// 12 warps: the suffix pass runs 8 autonomous warps; the prefix pass on
+// tcgen05 uses 11 (softmax 4, epilogue 4, producer, MMA issuer, scheduler),
+// the one on mma.sync 9 (8 consumers and a producer)
+constexpr int kThreads = 12 * 32;
 constexpr long long kDrainLimitNs = 1000000000LL;
 constexpr int kSmemBudget = 220 * 1024;                    // dynamic, one CTA per SM
 constexpr int kIdSlots = 8;      // prefix-pass item ids in flight from producer to consumers
@@ -585,6 +588,7 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
                                            nullptr);
         return;
     }
+    if (warp > kConsumerWarps) return;
 
     // ---------------------------------------------------------------- consumers
     uint8_t *scratch = smem + S::kWideRingBytes;
@@ -695,49 +699,89 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
 // prefix pass on tcgen05 (bf16 KV, head_dim 128): a tile of up to 128 stacked
 // rows against 64-token blocks (4 pages) of the node's pages
 //
-//   warp 8      producer: TMA of K and V, a block per ring stage; pages past
+//   warp 10     scheduler: pulls items from the prefix queue and stages each
+//               one's metadata (the item, the TMA row of each page, the
+//               branch of each group of g rows) in one of kTcMeta shared
+//               slots, so that no other role waits on a dependent chain of
+//               global loads when it moves to the next item
+//   warp 8      producer: TMA of K and V, one block per ring stage; pages past
 //               the item's end are loaded from an out-of-range row, which
 //               TMA fills with zeros
-//   warp 4      MMA issuer (one thread): S = Q K^T (M 128, N 64, K 128) into
+//   warp 9      MMA issuer (one thread): S = Q K^T (M 128, N 64, K 128) into
 //               one of two TMEM buffers, then O += P V (M 128, N 128, K 64)
-//               into the TMEM accumulator; tcgen05.commit releases the ring
-//               stage and signals completion
+//               into the item's TMEM accumulator (two, alternating by item).
+//               A (Q or P) comes from TMEM, B (K or V) from shared memory.
+//               Blocks form one stream across items: S of a block is issued
+//               before PV of the block before it, item boundaries included.
+//               tcgen05.commit releases ring stages and signals completion.
 //   warps 0-3   softmax: thread r owns row r (TMEM lane r); online softmax in
 //               the log2 domain with a lazy rescale of O (only when a row's
-//               max grows by more than 2^8); P goes to shared memory as the
-//               A operand of PV; at the end of an item the row's O, m, l
-//               become its partial
+//               max grows by more than 2^8); P (bf16) overwrites the first 32
+//               columns of its S buffer, the A operand of PV; writes the
+//               row's (m, l) at the end of an item
+//   warps 4-7   epilogue: once an item's O is complete, stores its rows to the
+//               partials and loads the Q rows of the item two ahead into the
+//               TMEM Q buffer that item frees (Q of items 0 and 1 at start)
 //
-// Shared memory: ring [4][K: 2 col blocks x 64 tokens x 128 B | V: same],
-// Q tile [2 col blocks][128 rows][128 B], P [2][128 rows][128 B]; all 128-byte
-// swizzled, so the MMA reads them through SW128 descriptors (K-major for Q, K
-// and P; MN-major for V).
+// TMEM, 512 columns: O[2] at 0 and 128, S/P[2] at 256 and 320, Q[2] at 384
+// and 448.  Shared memory: the ring [6][K: 2 col blocks x 64 tokens x 128 B |
+// V: same], 128-byte swizzled (K-major descriptors for K, MN-major for V),
+// and the metadata slots.
 // ---------------------------------------------------------------------------
 constexpr int kTcRows = 128;
 constexpr int kTcBlockPages = 4;
 constexpr int kTcBlockTokens = kTcBlockPages * kPageSize;    // 64
-constexpr int kTcStages = 4;
+constexpr int kTcStages = 6;
 constexpr int kTcColBlockBytes = kTcBlockTokens * 128;        // 8 KB: 64 tokens x 128 B
 constexpr int kTcKBytes = 2 * kTcColBlockBytes;               // d = 128: two column blocks
 constexpr int kTcStageBytes = 2 * kTcKBytes;                  // K + V
-constexpr int kTcRingBytes = kTcStages * kTcStageBytes;       // 128 KB
-constexpr int kTcQBytes = 2 * kTcRows * 128;                  // 32 KB
-constexpr int kTcPBytes = kTcRows * 128;                      // 16 KB per buffer
-constexpr int kTcBodyBytes = kTcRingBytes + kTcQBytes + 2 * kTcPBytes;
-constexpr int kTcTmemCols = 256;                              // O 128 + S 2 x 64
+constexpr int kTcRingBytes = kTcStages * kTcStageBytes;       // 192 KB
+constexpr int kTcTmemCols = 512;
+constexpr uint32_t kTmemO = 0, kTmemS = 256, kTmemQ = 384;    // TMEM column bases
 constexpr float kTcRescaleLog2 = 8.f;                         // lazy rescale threshold
-static_assert(kTcBodyBytes <= Shape<128, KvBf16>::kBodyBytes, "tcgen05 tile fits the CTA's memory");
+constexpr int kTcMeta = 4;                                    // item metadata slots
+constexpr int kTcMetaPages = 128;                             // pages of one item at most
+constexpr int kTcSoftmaxWarps = 4;                            // warps 0-3
+constexpr int kTcEpilogueWarp = 4;                            // warps 4-7
+constexpr int kTcProducerWarp = 8;
+constexpr int kTcMmaWarp = 9;
+constexpr int kTcSchedulerWarp = 10;
+static_assert(kTcRingBytes <= Shape<128, KvBf16>::kBodyBytes, "tcgen05 ring fits the CTA's memory");
+static_assert(kTcSchedulerWarp < kThreads / 32, "every tcgen05 role has a warp");
+
+// Metadata of one prefix item, staged by the scheduler warp.
+struct TcMeta {
+    WorkItem it;
+    int32_t id;                      // -1: the queue is empty
+    int32_t pad[3];
+    int32_t rows[kTcMetaPages];      // TMA row of each page
+    int32_t leaves[kTcRows];         // branch of rows [g i, g i + g)
+};
+
 // barrier slots (8 bytes each) in the CTA's barrier area
 enum TcBar : int {
-    kBarKvFull = 0,      // [4] producer -> MMA
-    kBarKvEmpty = 4,     // [4] MMA commit -> producer
-    kBarSFull = 8,       // [2] MMA commit -> softmax
-    kBarPFull = 10,      // [2] softmax (128 arrivals) -> MMA
-    kBarPvDone = 12,     // [2] MMA commit -> softmax
-    kBarQReady = 14,     // softmax (128 arrivals) -> MMA
-    kBarDrain = 15,      // MMA commit -> MMA thread, before TMEM is freed
-    kTcBars = 16
+    kBarKvFull = 0,                          // [stages] producer -> MMA (TMA bytes)
+    kBarKvEmpty = kBarKvFull + kTcStages,    // [stages] MMA commit -> producer
+    kBarSFull = kBarKvEmpty + kTcStages,     // [2] MMA commit -> softmax
+    kBarPFull = kBarSFull + 2,               // [2] softmax (128 arrivals) -> MMA
+    kBarPvDone = kBarPFull + 2,              // [2] MMA commit -> softmax (before a rescale)
+    kBarQReady = kBarPvDone + 2,             // [2] epilogue (128 arrivals) -> MMA
+    kBarOFull = kBarQReady + 2,              // [2] MMA commit -> epilogue
+    kBarOEmpty = kBarOFull + 2,              // [2] epilogue (4 arrivals) -> MMA
+    kBarMetaFull = kBarOEmpty + 2,           // [kTcMeta] scheduler -> every role
+    kBarMetaEmpty = kBarMetaFull + kTcMeta,  // [kTcMeta] epilogue (4 arrivals) -> scheduler
+    kBarDrain = kBarMetaEmpty + kTcMeta,     // MMA commit -> MMA thread, before TMEM is freed
+    kTcBars
 };
+
+__host__ __device__ constexpr int tc_bar_count(int i) {
+    return (i == kBarPFull || i == kBarPFull + 1 || i == kBarQReady || i == kBarQReady + 1)
+               ? kTcRows
+               : ((i == kBarOEmpty || i == kBarOEmpty + 1 ||
+                   (i >= kBarMetaEmpty && i < kBarMetaEmpty + kTcMeta))
+                      ? 4
+                      : 1);
+}
 
 __device__ __forceinline__ bool tc_wait(uint32_t bar, uint32_t parity, long long limit,
                                         volatile int *abort) {
@@ -759,18 +803,54 @@ __device__ __forceinline__ void tc_fail(const AttnArgs &a, volatile int *abort, 
     }
 }
 
+__device__ __forceinline__ int tc_blocks(int num_pages) {
+    return (num_pages + kTcBlockPages - 1) / kTcBlockPages;
+}
+
 template <int D>
 __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
                               const AttnArgs &a, uint8_t *smem, uint32_t bars, uint32_t tmem,
-                              int warp, int lane, volatile int *abort_flag, volatile int *id_slots) {
+                              int warp, int lane, volatile int *abort_flag, TcMeta *meta) {
     static_assert(D == 128, "the tcgen05 prefix tile is written for head_dim 128");
     const uint32_t ring = dev::smem_addr(smem);
-    const uint32_t sq = ring + kTcRingBytes;
-    const uint32_t sp = sq + kTcQBytes;
     auto bar = [&](int i) { return bars + 8u * static_cast<uint32_t>(i); };
-    const uint32_t id_bars = bar(kTcBars);
+    const long long limit = a.wait_limit_ns;
 
-    if (warp == kConsumerWarps) {
+    if (warp == kTcSchedulerWarp) {
+        // ------------------------------------------------------------ scheduler
+        for (int k = 0;; ++k) {
+            const int s = k % kTcMeta;
+            if (k >= kTcMeta &&
+                !tc_warp_wait(bar(kBarMetaEmpty + s), ((k / kTcMeta) - 1) & 1, limit, abort_flag, lane)) {
+                if (lane == 0) tc_fail(a, abort_flag, kSiteProducerEmpty);
+                break;
+            }
+            int id = *abort_flag ? -1 : pull(a, 0, lane);
+            TcMeta &m = meta[s];
+            if (id >= 0) {
+                const WorkItem it = a.items[id];
+                if (it.num_pages <= 0 || it.num_pages > kTcMetaPages || it.nrows <= 0 ||
+                    it.nrows > kTcRows || it.row0 % a.group != 0) {
+                    if (lane == 0 && !*abort_flag) {
+                        *abort_flag = 1;
+                        dev::record_error(a.err, PARASON_EINVAL, kSiteBadItem);
+                    }
+                    id = -1;
+                } else {
+                    if (lane == 0) m.it = it;
+                    const int32_t *src = a.stream_rows + a.item_rows[id];
+                    for (int p = lane; p < it.num_pages; p += 32) m.rows[p] = src[p];
+                    const int nbr = (it.nrows + a.group - 1) / a.group;
+                    const int32_t *lv = a.dfs_leaf + it.leaf_lo + it.row0 / a.group;
+                    for (int i = lane; i < nbr; i += 32) m.leaves[i] = lv[i];
+                }
+            }
+            if (lane == 0) m.id = id;
+            __syncwarp();
+            if (lane == 0) dev::mbar_arrive(bar(kBarMetaFull + s));
+            if (id < 0) break;
+        }
+    } else if (warp == kTcProducerWarp) {
         // ------------------------------------------------------------ producer
         const bool skip_first = a.debug_flags & PARASON_DEBUG_SKIP_FIRST_LOAD;
         int last_issue[kTcStages];
@@ -778,178 +858,175 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
         int blk = 0;
         bool ok = true;
         for (int k = 0; ok; ++k) {
-            const int id = *abort_flag ? -1 : pull(a, 0, lane);
-            if (lane == 0) publish_id(id_slots, id_bars, k, id);
-            if (id < 0) break;
-            const WorkItem it = a.items[id];
-            ItemRows ps;
-            ps.start(a, id);
-            int q = 0;
-            const int nb = (it.num_pages + kTcBlockPages - 1) / kTcBlockPages;
+            const int ms = k % kTcMeta;
+            if (!tc_warp_wait(bar(kBarMetaFull + ms), (k / kTcMeta) & 1, limit, abort_flag, lane)) {
+                if (lane == 0) tc_fail(a, abort_flag, kSiteProducerEmpty);
+                break;
+            }
+            const TcMeta &m = meta[ms];
+            if (m.id < 0) break;
+            const int np = m.it.num_pages;
+            const int nb = tc_blocks(np);
             for (int bi = 0; bi < nb; ++bi, ++blk) {
                 const int s = blk % kTcStages;
                 if (blk >= kTcStages &&
-                    !tc_warp_wait(bar(kBarKvEmpty + s), ((blk / kTcStages) - 1) & 1,
-                                  a.wait_limit_ns, abort_flag, lane)) {
+                    !tc_warp_wait(bar(kBarKvEmpty + s), ((blk / kTcStages) - 1) & 1, limit, abort_flag,
+                                  lane)) {
                     if (lane == 0) tc_fail(a, abort_flag, kSiteProducerEmpty);
                     ok = false;
                     break;
-                }
-                int rows[kTcBlockPages];
-#pragma unroll
-                for (int j = 0; j < kTcBlockPages; ++j) {
-                    const int pg = bi * kTcBlockPages + j;
-                    rows[j] = pg < it.num_pages ? ps.row(q++, lane) : a.kv_rows;   // kv_rows: zero fill
                 }
                 if (lane == 0 && !(skip_first && blk == 0)) {
                     const uint32_t st = ring + s * kTcStageBytes;
                     const uint32_t fb = bar(kBarKvFull + s);
                     dev::mbar_arrive_expect_tx(fb, kTcStageBytes);
 #pragma unroll
-                    for (int j = 0; j < kTcBlockPages; ++j)
+                    for (int j = 0; j < kTcBlockPages; ++j) {
+                        const int pg = bi * kTcBlockPages + j;
+                        const int row = pg < np ? m.rows[pg] : a.kv_rows;   // kv_rows: zero fill
 #pragma unroll
                         for (int cb = 0; cb < 2; ++cb) {
                             const uint32_t off = cb * kTcColBlockBytes + j * kPageSize * 128;
-                            dev::tma_load_3d(st + off, tmap_k, 0, cb, rows[j], fb);
-                            dev::tma_load_3d(st + kTcKBytes + off, tmap_v, 0, cb, rows[j], fb);
+                            dev::tma_load_3d(st + off, tmap_k, 0, cb, row, fb);
+                            dev::tma_load_3d(st + kTcKBytes + off, tmap_v, 0, cb, row, fb);
                         }
+                    }
                     last_issue[s] = blk;
                 }
             }
         }
+        // every copy this CTA issued must land before its shared memory is reused
         if (lane == 0)
             for (int s = 0; s < kTcStages; ++s)
                 if (last_issue[s] >= 0)
                     dev::mbar_wait_bounded(bar(kBarKvFull + s), (last_issue[s] / kTcStages) & 1,
                                            kDrainLimitNs, nullptr);
-    } else if (warp == 4) {
+    } else if (warp == kTcMmaWarp) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
-            const uint32_t tO = tmem, tS0 = tmem + 128;
             constexpr uint32_t kIdS = tc::idesc_bf16_f32(kTcRows, kTcBlockTokens, false);
             constexpr uint32_t kIdPV = tc::idesc_bf16_f32(kTcRows, D, true);
-            auto issue_s = [&](int b) {
+            auto wait = [&](int i, int parity) {
+                return tc_wait(bar(i), static_cast<uint32_t>(parity & 1), limit, abort_flag);
+            };
+            // S(b) = Q(item k) K(b)^T into S buffer b & 1
+            auto issue_s = [&](int b, int k) {
                 const uint32_t st = ring + (b % kTcStages) * kTcStageBytes;
-                const uint32_t tS = tS0 + 64u * (b & 1);
+                const uint32_t tS = tmem + kTmemS + 64u * (b & 1);
+                const uint32_t tQ = tmem + kTmemQ + 64u * (k & 1);
 #pragma unroll
                 for (int ks = 0; ks < D / 16; ++ks) {
                     const uint32_t cb = ks >> 2, kk = ks & 3;
-                    const uint64_t ad = tc::smem_desc_sw128(sq + cb * (kTcRows * 128) + kk * 32, 16, 1024);
                     const uint64_t bd = tc::smem_desc_sw128(st + cb * kTcColBlockBytes + kk * 32, 16, 1024);
-                    tc::mma_bf16(tS, ad, bd, kIdS, ks > 0);
+                    tc::mma_bf16_tmem_a(tS, tQ + 8u * ks, bd, kIdS, ks > 0);
                 }
                 tc::commit(bar(kBarSFull + (b & 1)));
             };
-            int blk = 0;
-            bool ok = true;
-            for (int item = 0; ok; ++item) {
-                const int id = take_id(id_slots, id_bars, item, a.wait_limit_ns, abort_flag, &ok);
-                if (id < 0) break;
-                const WorkItem it = a.items[id];
-                const int nb = (it.num_pages + kTcBlockPages - 1) / kTcBlockPages;
-                if (!tc_wait(bar(kBarQReady), item & 1, a.wait_limit_ns, abort_flag) ||
-                    !tc_wait(bar(kBarKvFull + blk % kTcStages), (blk / kTcStages) & 1,
-                             a.wait_limit_ns, abort_flag)) {
-                    ok = false;
-                    break;
+            bool ok = wait(kBarMetaFull, 0);
+            bool have = ok && meta[0].id >= 0;
+            int k = 0, b = 0, blk0 = 0, nb = have ? tc_blocks(meta[0].it.num_pages) : 0;
+            if (have) {
+                ok = wait(kBarQReady, 0) && wait(kBarKvFull, 0);
+                if (ok) {
+                    tc::fence_after_sync();
+                    issue_s(0, 0);
                 }
-                tc::fence_after_sync();
-                issue_s(blk);
-                for (int i = 0; i < nb; ++i) {
-                    const int b = blk + i;
-                    if (i + 1 < nb) {
-                        if (!tc_wait(bar(kBarKvFull + (b + 1) % kTcStages), ((b + 1) / kTcStages) & 1,
-                                     a.wait_limit_ns, abort_flag)) {
-                            ok = false;
-                            break;
-                        }
-                        issue_s(b + 1);
-                    }
-                    if (!tc_wait(bar(kBarPFull + (b & 1)), (b >> 1) & 1, a.wait_limit_ns, abort_flag)) {
+            }
+            while (have && ok) {
+                const bool last = b == blk0 + nb - 1;
+                bool next = false;
+                int nb_next = 0;
+                if (!last) {
+                    if (!wait(kBarKvFull + (b + 1) % kTcStages, (b + 1) / kTcStages)) {
                         ok = false;
                         break;
                     }
                     tc::fence_after_sync();
-                    const uint32_t vst = ring + (b % kTcStages) * kTcStageBytes + kTcKBytes;
-                    const uint32_t pb = sp + (b & 1) * kTcPBytes;
-#pragma unroll
-                    for (int kk = 0; kk < kTcBlockTokens / 16; ++kk) {
-                        const uint64_t ad = tc::smem_desc_sw128(pb + kk * 32, 16, 1024);
-                        const uint64_t bd = tc::smem_desc_sw128(vst + kk * 2048, kTcColBlockBytes, 1024);
-                        tc::mma_bf16(tO, ad, bd, kIdPV, i > 0 || kk > 0);
+                    issue_s(b + 1, k);
+                } else {
+                    // first S of the next item before the last PV of this one
+                    const int s1 = (k + 1) % kTcMeta;
+                    if (!wait(kBarMetaFull + s1, (k + 1) / kTcMeta)) {
+                        ok = false;
+                        break;
                     }
-                    tc::commit(bar(kBarKvEmpty + b % kTcStages));
-                    tc::commit(bar(kBarPvDone + (b & 1)));
+                    if (meta[s1].id >= 0) {
+                        next = true;
+                        nb_next = tc_blocks(meta[s1].it.num_pages);
+                        if (!wait(kBarQReady + ((k + 1) & 1), (k + 1) >> 1) ||
+                            !wait(kBarKvFull + (b + 1) % kTcStages, (b + 1) / kTcStages)) {
+                            ok = false;
+                            break;
+                        }
+                        tc::fence_after_sync();
+                        issue_s(b + 1, k + 1);
+                    }
                 }
-                blk += nb;
+                if (!wait(kBarPFull + (b & 1), b >> 1)) {
+                    ok = false;
+                    break;
+                }
+                // the item's O buffer was last used by item k - 2: its epilogue must be done
+                if (b == blk0 && k >= 2 && !wait(kBarOEmpty + (k & 1), (k >> 1) - 1)) {
+                    ok = false;
+                    break;
+                }
+                tc::fence_after_sync();
+                const uint32_t tO = tmem + kTmemO + 128u * (k & 1);
+                const uint32_t tP = tmem + kTmemS + 64u * (b & 1);
+                const uint32_t vst = ring + (b % kTcStages) * kTcStageBytes + kTcKBytes;
+#pragma unroll
+                for (int kk = 0; kk < kTcBlockTokens / 16; ++kk) {
+                    const uint64_t bd = tc::smem_desc_sw128(vst + kk * 2048, kTcColBlockBytes, 1024);
+                    tc::mma_bf16_tmem_a(tO, tP + 8u * kk, bd, kIdPV, b > blk0 || kk > 0);
+                }
+                tc::commit(bar(kBarKvEmpty + b % kTcStages));
+                tc::commit(bar(kBarPvDone + (b & 1)));
+                if (last) {
+                    tc::commit(bar(kBarOFull + (k & 1)));
+                    if (!next) break;
+                    blk0 += nb;
+                    nb = nb_next;
+                    ++k;
+                }
+                ++b;
             }
             if (!ok) tc_fail(a, abort_flag, kSiteConsumerFull);
             // every MMA must finish before TMEM is freed
             tc::commit(bar(kBarDrain));
             dev::mbar_wait_bounded(bar(kBarDrain), 0, kDrainLimitNs, nullptr);
         }
-    } else if (warp < 4) {
+        __syncwarp();
+    } else if (warp < kTcSoftmaxWarps) {
         // ------------------------------------------------------------ softmax
         const int r = threadIdx.x;                       // tile row == TMEM lane
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-        const uint32_t tO = lane_base, tS0 = lane_base + 128;
         int blk = 0;
-        for (int item = 0;; ++item) {
-            int id = -1;
-            if (lane == 0) {
-                bool got = true;
-                id = take_id(id_slots, id_bars, item, a.wait_limit_ns, abort_flag, &got);
-                if (!got) id = -2;
+        for (int k = 0;; ++k) {
+            const int ms = k % kTcMeta;
+            if (!tc_warp_wait(bar(kBarMetaFull + ms), (k / kTcMeta) & 1, limit, abort_flag, lane)) {
+                if (lane == 0) tc_fail(a, abort_flag, kSiteConsumerFull);
+                break;
             }
-            id = __shfl_sync(0xffffffffu, id, 0);
-            if (id == -2 && lane == 0) tc_fail(a, abort_flag, kSiteConsumerFull);
-            if (id < 0) break;
-            const WorkItem it = a.items[id];
-            const int nb = (it.num_pages + kTcBlockPages - 1) / kTcBlockPages;
+            if (meta[ms].id < 0) break;
+            const WorkItem it = meta[ms].it;
+            const int nb = tc_blocks(it.num_pages);
             const int tokens = (it.num_pages - 1) * kPageSize + it.last_valid;
-
-            // Q row r of the tile into the swizzled Q tile (zeros past nrows)
-            {
-                uint4 qv[16];
-                if (r < it.nrows) {
-                    const int nr = it.row0 + r;
-                    const int leaf = a.dfs_leaf[it.leaf_lo + nr / a.group];
-                    const int head = it.kv_head * a.group + nr % a.group;
-                    const uint4 *src = reinterpret_cast<const uint4 *>(
-                        static_cast<const __nv_bfloat16 *>(a.q) +
-                        (static_cast<int64_t>(leaf) * a.num_q_heads + head) * D);
-#pragma unroll
-                    for (int c = 0; c < 16; ++c) qv[c] = src[c];
-                } else {
-#pragma unroll
-                    for (int c = 0; c < 16; ++c) qv[c] = make_uint4(0u, 0u, 0u, 0u);
-                }
-#pragma unroll
-                for (int c = 0; c < 16; ++c) {
-                    const uint32_t dst = sq + (c >> 3) * (kTcRows * 128) + r * 128 +
-                                         (((c & 7) ^ (r & 7)) << 4);
-                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst),
-                                 "r"(qv[c].x), "r"(qv[c].y), "r"(qv[c].z), "r"(qv[c].w)
-                                 : "memory");
-                }
-                tc::fence_proxy_async_smem();
-                dev::mbar_arrive(bar(kBarQReady));
-            }
-
+            const uint32_t tO = lane_base + kTmemO + 128u * (k & 1);
             float m_use = -INFINITY, l = 0.f;
             bool ok = true;
             for (int i = 0; i < nb; ++i) {
                 const int b = blk + i;
                 const int valid = min(kTcBlockTokens, tokens - i * kTcBlockTokens);
-                if (!tc_warp_wait(bar(kBarSFull + (b & 1)), (b >> 1) & 1, a.wait_limit_ns, abort_flag,
-                                  lane)) {
+                const uint32_t tS = lane_base + kTmemS + 64u * (b & 1);
+                if (!tc_warp_wait(bar(kBarSFull + (b & 1)), (b >> 1) & 1, limit, abort_flag, lane)) {
                     ok = false;
                     break;
                 }
                 tc::fence_after_sync();
                 uint32_t sr[2][32];
-                tc::ld32(tS0 + 64u * (b & 1), sr[0]);
-                tc::ld32(tS0 + 64u * (b & 1) + 32, sr[1]);
+                tc::ld32(tS, sr[0]);
+                tc::ld32(tS + 32, sr[1]);
                 tc::wait_ld();
                 float x[64];
                 float mb = -INFINITY;
@@ -958,18 +1035,12 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                     x[j] = j < valid ? __uint_as_float(sr[j >> 5][j & 31]) * a.scale_log2 : -INFINITY;
                     mb = fmaxf(mb, x[j]);
                 }
-                // this P buffer was read by PV(b - 2)
-                if (b >= 2 && !tc_warp_wait(bar(kBarPvDone + (b & 1)), ((b - 2) >> 1) & 1,
-                                            a.wait_limit_ns, abort_flag, lane)) {
-                    ok = false;
-                    break;
-                }
                 if (i == 0) {
                     m_use = mb;
                 } else if (__any_sync(0xffffffffu, mb > m_use + kTcRescaleLog2)) {
                     // O must hold PV(b - 1) before it is rescaled
-                    if (!tc_warp_wait(bar(kBarPvDone + ((b - 1) & 1)), ((b - 1) >> 1) & 1,
-                                      a.wait_limit_ns, abort_flag, lane)) {
+                    if (!tc_warp_wait(bar(kBarPvDone + ((b - 1) & 1)), ((b - 1) >> 1) & 1, limit,
+                                      abort_flag, lane)) {
                         ok = false;
                         break;
                     }
@@ -989,36 +1060,31 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                     l *= alpha;
                     m_use = m_new;
                 }
-                // P = 2^(x - m) as bf16, row r of the swizzled P tile
-                const uint32_t pb = sp + (b & 1) * kTcPBytes + r * 128;
+                // P = 2^(x - m) as bf16 pairs over the first 32 columns of S
+                uint32_t pw[32];
 #pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    uint32_t w[4];
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        const float p0 = dev::fast_exp2(x[8 * c + 2 * k] - m_use);
-                        const float p1 = dev::fast_exp2(x[8 * c + 2 * k + 1] - m_use);
-                        l += p0 + p1;
-                        w[k] = dev::pack_bf16(p0, p1);
-                    }
-                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(pb + ((c ^ (r & 7)) << 4)),
-                                 "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
-                                 : "memory");
+                for (int c = 0; c < 32; ++c) {
+                    const float p0 = dev::fast_exp2(x[2 * c] - m_use);
+                    const float p1 = dev::fast_exp2(x[2 * c + 1] - m_use);
+                    l += p0 + p1;
+                    pw[c] = dev::pack_bf16(p0, p1);
                 }
+                tc::st32(tS, pw);
+                tc::wait_st();
                 // V rows past the item's last token may hold anything (NaN
                 // included); P is 0 there but 0 * NaN is NaN, so zero them
                 if (valid < kTcBlockTokens) {
                     const uint32_t vst = ring + (b % kTcStages) * kTcStageBytes + kTcKBytes;
                     const int n16 = (kTcBlockTokens - valid) * 2 * 8;     // 16-byte chunks
-                    for (int k = r; k < n16; k += kTcRows) {
-                        const int t = valid + k / 16, cb = (k / 8) & 1, c = k & 7;
+                    for (int q = r; q < n16; q += kTcRows) {
+                        const int t = valid + q / 16, cb = (q / 8) & 1, c = q & 7;
                         asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
                                          vst + cb * kTcColBlockBytes + t * 128 + (c << 4)),
                                      "r"(0u)
                                      : "memory");
                     }
+                    tc::fence_proxy_async_smem();
                 }
-                tc::fence_proxy_async_smem();
                 tc::fence_before_sync();
                 dev::mbar_arrive(bar(kBarPFull + (b & 1)));
             }
@@ -1026,14 +1092,82 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                 if (lane == 0) tc_fail(a, abort_flag, kSiteConsumerFull);
                 break;
             }
-            // epilogue: O of the item's last PV, normalised by the merge later
-            const int bl = blk + nb - 1;
-            if (!tc_warp_wait(bar(kBarPvDone + (bl & 1)), (bl >> 1) & 1, a.wait_limit_ns, abort_flag,
+            if (r < it.nrows) a.part_ml[static_cast<int64_t>(it.slot_base) + r] = make_float2(m_use, l);
+            blk += nb;
+        }
+    } else if (warp >= kTcEpilogueWarp && warp < kTcEpilogueWarp + 4) {
+        // ------------------------------------------------------------ epilogue
+        const int quarter = warp - kTcEpilogueWarp;      // == warp % 4: its TMEM lanes
+        const int r = quarter * 32 + lane;
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+        bool ok = true;
+        // wait for slot k; true if it holds an item
+        auto has_item = [&](int k) {
+            if (!tc_warp_wait(bar(kBarMetaFull + k % kTcMeta), (k / kTcMeta) & 1, limit, abort_flag,
                               lane)) {
-                if (lane == 0) tc_fail(a, abort_flag, kSiteConsumerFull);
+                ok = false;
+                return false;
+            }
+            return meta[k % kTcMeta].id >= 0;
+        };
+        // Q row r of item k: global loads into registers ...
+        auto fetch_q = [&](int k, uint4 (&qv)[16]) {
+            const TcMeta &m = meta[k % kTcMeta];
+            if (r < m.it.nrows) {
+                const int leaf = m.leaves[r / a.group];
+                const int head = m.it.kv_head * a.group + r % a.group;
+                const uint4 *src = reinterpret_cast<const uint4 *>(
+                    static_cast<const __nv_bfloat16 *>(a.q) +
+                    (static_cast<int64_t>(leaf) * a.num_q_heads + head) * D);
+#pragma unroll
+                for (int c = 0; c < 16; ++c) qv[c] = src[c];
+            } else {
+#pragma unroll
+                for (int c = 0; c < 16; ++c) qv[c] = make_uint4(0u, 0u, 0u, 0u);
+            }
+        };
+        // ... then into TMEM Q buffer k & 1 (bf16 pairs, lane r)
+        auto put_q = [&](int k, const uint4 (&qv)[16]) {
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                uint32_t w[32];
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    w[4 * c] = qv[8 * h + c].x;
+                    w[4 * c + 1] = qv[8 * h + c].y;
+                    w[4 * c + 2] = qv[8 * h + c].z;
+                    w[4 * c + 3] = qv[8 * h + c].w;
+                }
+                tc::st32(lane_base + kTmemQ + 64u * (k & 1) + 32u * h, w);
+            }
+            tc::wait_st();
+            tc::fence_before_sync();
+            dev::mbar_arrive(bar(kBarQReady + (k & 1)));
+        };
+        bool has_k = has_item(0), has_k1 = false;
+        if (has_k) {
+            uint4 qv[16];
+            fetch_q(0, qv);
+            put_q(0, qv);
+            has_k1 = has_item(1);
+            if (has_k1) {
+                fetch_q(1, qv);
+                put_q(1, qv);
+            }
+        }
+        for (int k = 0; ok && has_k; ++k) {
+            const WorkItem it = meta[k % kTcMeta].it;
+            if (!tc_warp_wait(bar(kBarOFull + (k & 1)), (k >> 1) & 1, limit, abort_flag, lane)) {
+                ok = false;
                 break;
             }
             tc::fence_after_sync();
+            // item k's S MMAs are complete, so its Q buffer takes item k + 2's rows;
+            // their loads are in flight while O is stored
+            const bool has_k2 = has_k1 && has_item(k + 2);
+            uint4 qv[16];
+            if (has_k2) fetch_q(k + 2, qv);
+            const uint32_t tO = lane_base + kTmemO + 128u * (k & 1);
             float *dst = a.part_o + (static_cast<int64_t>(it.slot_base) + r) * D;
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
@@ -1048,14 +1182,21 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                                         __uint_as_float(ov[j + 2]), __uint_as_float(ov[j + 3]));
                 }
             }
-            if (r < it.nrows) a.part_ml[static_cast<int64_t>(it.slot_base) + r] = make_float2(m_use, l);
+            if (has_k2) put_q(k + 2, qv);
             tc::fence_before_sync();
-            blk += nb;
+            __syncwarp();
+            if (lane == 0) {
+                dev::mbar_arrive(bar(kBarOEmpty + (k & 1)));
+                dev::mbar_arrive(bar(kBarMetaEmpty + k % kTcMeta));
+            }
+            has_k = has_k1;
+            has_k1 = has_k2;
         }
+        if (!ok && lane == 0) tc_fail(a, abort_flag, kSiteConsumerFull);
     }
 }
 
-// One CTA per SM: 9 warps leave at most 168 registers per thread (three warps
+// One CTA per SM: 12 warps leave at most 168 registers per thread (three warps
 // on one sub-partition of 16K registers).
 template <int D, class KV>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -1075,7 +1216,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     // the prefix pass of bf16 KV at head_dim 128 runs on tcgen05
     constexpr bool kTcPrefix = (D == 128) && (KV::kElemBytes == 2);
-    constexpr int kPrefixBars = kTcPrefix ? kTcBars + kIdSlots : 2 * S::kWideStages + kIdSlots;
+    constexpr int kPrefixBars = kTcPrefix ? kTcBars : 2 * S::kWideStages + kIdSlots;
+    static_assert(!kTcPrefix || kTcBars <= S::kBars, "barrier area holds the tcgen05 barriers");
+    __shared__ TcMeta tc_meta[kTcPrefix ? kTcMeta : 1];
     auto init_suffix_barriers = [&]() {
         for (int s = 0; s < S::kNarrowBars; ++s) dev::mbar_init(bars + 8 * s, 1);
     };
@@ -1083,11 +1226,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         abort_flag = 0;
         if (wide && kTcPrefix) {
-            for (int i = 0; i < kTcBars; ++i)
-                dev::mbar_init(bars + 8 * i, (i == kBarPFull || i == kBarPFull + 1 || i == kBarQReady)
-                                                 ? kTcRows
-                                                 : 1);
-            for (int i = 0; i < kIdSlots; ++i) dev::mbar_init(bars + 8 * (kTcBars + i), 1);
+            for (int i = 0; i < kTcBars; ++i) dev::mbar_init(bars + 8 * i, tc_bar_count(i));
         } else if (wide) {
             for (int s = 0; s < S::kWideStages; ++s) {
                 dev::mbar_init(bars + 8 * s, 1);
@@ -1102,7 +1241,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         dev::prefetch_tensormap(&tmap_v);
     }
     if constexpr (kTcPrefix) {
-        if (wide && warp == 4) tc::alloc<kTcTmemCols>(dev::smem_addr(&tmem_base));
+        if (wide && warp == kTcMmaWarp) tc::alloc<kTcTmemCols>(dev::smem_addr(&tmem_base));
         tc::fence_before_sync();
     }
     __syncthreads();
@@ -1113,11 +1252,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         if constexpr (kTcPrefix) {
             tc::fence_after_sync();
             prefix_cta_tc<D>(&tmap_k, &tmap_v, a, smem, bars, tmem_base, warp, lane, &abort_flag,
-                             id_slots);
+                             tc_meta);
             tc::fence_before_sync();
             __syncthreads();
             tc::fence_after_sync();
-            if (warp == 4) tc::dealloc<kTcTmemCols>(tmem_base);
+            if (warp == kTcMmaWarp) tc::dealloc<kTcTmemCols>(tmem_base);
         } else {
             prefix_cta<D, KV>(&tmap_k, &tmap_v, a, smem, ring, bars, warp, lane, &abort_flag,
                               id_slots);

@@ -37,6 +37,7 @@ constexpr int kErrWords = 4;            // device error record: code, block, sit
 enum WaitSite : int32_t {
     kSiteConsumerFull = 1,
     kSiteProducerEmpty = 2,
+    kSiteBadItem = 3,        // an item the kernel cannot hold (planner contract broken)
 };
 
 struct AttnArgs {
