@@ -98,15 +98,27 @@ struct Shape {
 };
 
 // K then V of one (page, kv head) into a stage: one TMA box {128 bytes, 1
-// block, 16 tokens} per column block and tensor.
-template <int D, class KV>
+// block, 16 tokens} per column block and tensor.  A suffix page is read by
+// one item only, so its lines go first when L2 needs room (the partials
+// written meanwhile stay for the merge); a prefix page may be read again by
+// another row tile of its node and keeps the normal policy.
+template <int D, class KV, bool kReadOnce>
 __device__ __forceinline__ void load_page(uint32_t dst, const CUtensorMap *tmap_k,
                                           const CUtensorMap *tmap_v, int row, uint32_t bar) {
     using S = Shape<D, KV>;
+    if constexpr (kReadOnce) {
+        const uint64_t pol = dev::l2_evict_first_policy();
 #pragma unroll
-    for (int sg = 0; sg < S::kSeg; ++sg) {
-        dev::tma_load_3d(dst + sg * S::kSegBytes, tmap_k, 0, sg, row, bar);
-        dev::tma_load_3d(dst + S::kPageBytes + sg * S::kSegBytes, tmap_v, 0, sg, row, bar);
+        for (int sg = 0; sg < S::kSeg; ++sg) {
+            dev::tma_load_3d_hint(dst + sg * S::kSegBytes, tmap_k, 0, sg, row, bar, pol);
+            dev::tma_load_3d_hint(dst + S::kPageBytes + sg * S::kSegBytes, tmap_v, 0, sg, row, bar, pol);
+        }
+    } else {
+#pragma unroll
+        for (int sg = 0; sg < S::kSeg; ++sg) {
+            dev::tma_load_3d(dst + sg * S::kSegBytes, tmap_k, 0, sg, row, bar);
+            dev::tma_load_3d(dst + S::kPageBytes + sg * S::kSegBytes, tmap_v, 0, sg, row, bar);
+        }
     }
 }
 
@@ -457,7 +469,7 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
             const int s = issued % NS;
             const uint32_t bar = my_bar + s * 8;
             dev::mbar_arrive_expect_tx(bar, S::kStageBytes);
-            load_page<D, KV>(my_ring + s * S::kStageBytes, tmap_k, tmap_v, row, bar);
+            load_page<D, KV, true>(my_ring + s * S::kStageBytes, tmap_k, tmap_v, row, bar);
         }
         ++iss_pg;
         ++issued;
@@ -575,7 +587,7 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
                 const int row = rows.row(pg, lane);
                 if (lane == 0 && !(skip_first && stage == 0)) {
                     dev::mbar_arrive_expect_tx(bar_full + 8 * s, S::kStageBytes);
-                    load_page<D, KV>(k_page(s), tmap_k, tmap_v, row, bar_full + 8 * s);
+                    load_page<D, KV, false>(k_page(s), tmap_k, tmap_v, row, bar_full + 8 * s);
                     last_issue[s] = stage;
                 }
             }

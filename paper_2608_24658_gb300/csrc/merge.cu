@@ -84,45 +84,55 @@ __device__ __forceinline__ void load_in(const void *in, int64_t off, float (&v)[
     }
 }
 
-// One warp per (branch, q head).  Entries are taken 32 at a time: lane e
-// loads entry e's (m, l) (one round trip for all of them), the batch's max
-// and weights come from warp reductions, then every lane accumulates its
-// D/32 columns over the batch with independent loads.  Runs as a dependent
-// grid of the attention kernel: griddepcontrol.wait returns once that grid
-// has completed and its writes are visible.
-template <int D>
+// W warps per (branch, q head), 4 / W rows per CTA of 4 warps (W = 4 when
+// there are few rows, so that enough loads are in flight; 1 when there are
+// many).  Warp w of a row folds entries w, w + W, w + 2W, ... of the row's
+// list into its own (M_w, L_w, acc_w): lane e loads entry e's (m, l) (one
+// round trip for up to 32 entries), the pass's max and weights come from warp
+// reductions, then every lane accumulates its D/32 columns with the partial
+// rows requested 8 at a time.  The W results combine through shared memory
+// by the same rule.  Runs as a dependent grid of the attention kernel:
+// griddepcontrol.wait returns once that grid has completed and its writes
+// are visible.
+template <int D, int W>
 __global__ void __launch_bounds__(kMergeThreads)
     tree_merge_kernel(const MergeArgs a, bool out_bf16) {
     constexpr int N = Vec<D>::N;
-    const int64_t w = (static_cast<int64_t>(blockIdx.x) * kMergeThreads + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    const bool active = w < static_cast<int64_t>(a.num_leaves) * a.num_q_heads;
-    const int b = active ? static_cast<int>(w / a.num_q_heads) : 0;
-    const int h = active ? static_cast<int>(w % a.num_q_heads) : 0;
+    constexpr int kWarps = kMergeThreads / 32;
+    constexpr int kRowsPerCta = kWarps / W;
+    __shared__ float s_acc[W > 1 ? kWarps : 1][D];
+    __shared__ float s_m[kWarps], s_l[kWarps];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int w = warp % W;
+    const int64_t row = static_cast<int64_t>(blockIdx.x) * kRowsPerCta + warp / W;   // b * H_q + h
+    const bool active = row < static_cast<int64_t>(a.num_leaves) * a.num_q_heads;
+    const int b = active ? static_cast<int>(row / a.num_q_heads) : 0;
+    const int h = active ? static_cast<int>(row % a.num_q_heads) : 0;
     const int j = h / a.group, r = h % a.group;
     const int64_t pair = static_cast<int64_t>(b) * a.num_kv_heads + j;
     // the merge lists are plan data: read them while the attention grid drains
     const int e0 = active ? a.merge_ptr[pair] : 0, e1 = active ? a.merge_ptr[pair + 1] : 0;
-    int first_slot = (e0 + lane < e1) ? a.merge_ent[e0 + lane] + r : 0;
+    const int first_e = e0 + w + W * lane;
+    const int first_slot = first_e < e1 ? a.merge_ent[first_e] + r : 0;
     asm volatile("griddepcontrol.wait;" ::: "memory");
     // the attention grid is complete: rewind its work queues for the next call
     if (blockIdx.x == 0 && threadIdx.x == 0 && a.queue_next) {
         a.queue_next[0] = 0;
         a.queue_next[1] = 0;
     }
-    if (!active) return;
 
     float M = -INFINITY, L = 0.f;
     float acc[N];
 #pragma unroll
     for (int i = 0; i < N; ++i) acc[i] = 0.f;
-    for (int base = e0; base < e1; base += 32) {
-        const int e = base + lane;
+    // this warp's entries e0 + w + W * i, 32 per pass
+    for (int i0 = 0; e0 + w + W * i0 < e1; i0 += 32) {
+        const int e = e0 + w + W * (i0 + lane);
         const bool valid = e < e1;
         int slot = 0;
         float m = -INFINITY, l = 0.f;
         if (valid) {
-            slot = base == e0 ? first_slot : a.merge_ent[e] + r;
+            slot = i0 == 0 ? first_slot : a.merge_ent[e] + r;
             const float2 ml = a.part_ml[slot];
             m = ml.x;
             l = ml.y;
@@ -130,7 +140,7 @@ __global__ void __launch_bounds__(kMergeThreads)
         float mb = m;
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) mb = fmaxf(mb, __shfl_xor_sync(0xffffffffu, mb, o));
-        const float Mn = fmaxf(M, mb);             // finite: the batch has a valid entry
+        const float Mn = fmaxf(M, mb);             // finite: the pass has a valid entry
         const float s_old = exp2f(M - Mn);
         const float wgt = valid ? exp2f(m - Mn) : 0.f;
         float lw = l * wgt;
@@ -139,30 +149,56 @@ __global__ void __launch_bounds__(kMergeThreads)
         L = L * s_old + lw;
 #pragma unroll
         for (int i = 0; i < N; ++i) acc[i] *= s_old;
-        // partial rows are requested 8 at a time before any of them is used
-        const int cnt = min(32, e1 - base);
-        for (int i0 = 0; i0 < cnt; i0 += 8) {
+        const int cnt = min(32, (e1 - (e0 + w) + W - 1) / W - i0);
+        for (int k0 = 0; k0 < cnt; k0 += 8) {
             float v[8][N];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const int si = __shfl_sync(0xffffffffu, slot, (i0 + i) & 31);
-                if (i0 + i < cnt) load_f32<N>(a.part_o + static_cast<int64_t>(si) * D + lane * N, v[i]);
+            for (int k = 0; k < 8; ++k) {
+                const int si = __shfl_sync(0xffffffffu, slot, (k0 + k) & 31);
+                if (k0 + k < cnt) load_f32<N>(a.part_o + static_cast<int64_t>(si) * D + lane * N, v[k]);
             }
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const float wi = __shfl_sync(0xffffffffu, wgt, (i0 + i) & 31);
-                if (i0 + i < cnt)
+            for (int k = 0; k < 8; ++k) {
+                const float wk = __shfl_sync(0xffffffffu, wgt, (k0 + k) & 31);
+                if (k0 + k < cnt)
 #pragma unroll
-                    for (int k = 0; k < N; ++k) acc[k] += wi * v[i][k];
+                    for (int c = 0; c < N; ++c) acc[c] += wk * v[k][c];
             }
         }
         M = Mn;
     }
+    if constexpr (W > 1) {
+#pragma unroll
+        for (int c = 0; c < N; ++c) s_acc[warp][lane * N + c] = acc[c];
+        if (lane == 0) {
+            s_m[warp] = M;
+            s_l[warp] = L;
+        }
+        __syncthreads();
+        if (w != 0) return;
+        const int base = warp;                     // the row's first warp
+        float Mg = -INFINITY;
+#pragma unroll
+        for (int u = 0; u < W; ++u) Mg = fmaxf(Mg, s_m[base + u]);
+        L = 0.f;
+#pragma unroll
+        for (int c = 0; c < N; ++c) acc[c] = 0.f;
+        if (Mg != -INFINITY) {
+#pragma unroll
+            for (int u = 0; u < W; ++u) {
+                const float su = s_m[base + u] == -INFINITY ? 0.f : exp2f(s_m[base + u] - Mg);
+                L += s_l[base + u] * su;
+#pragma unroll
+                for (int c = 0; c < N; ++c) acc[c] += su * s_acc[base + u][lane * N + c];
+            }
+        }
+        M = Mg;
+    }
+    if (!active) return;
     const bool empty = !(L > 0.f);
     const float inv = empty ? 0.f : 1.f / L;
 #pragma unroll
-    for (int i = 0; i < N; ++i) acc[i] *= inv;
-    const int64_t row = static_cast<int64_t>(b) * a.num_q_heads + h;
+    for (int c = 0; c < N; ++c) acc[c] *= inv;
     store_out<N>(a.out, row * D + lane * N, acc, out_bf16);
     if (a.lse && lane == 0) a.lse[row] = empty ? -INFINITY : (M + log2f(L)) * kLn2;
 }
@@ -201,9 +237,12 @@ __global__ void __launch_bounds__(kMergeThreads)
 
 cudaError_t launch_merge(const MergeArgs &a, int head_dim, int mode, bool programmatic,
                          cudaStream_t stream) {
-    const int64_t warps = static_cast<int64_t>(a.num_leaves) * a.num_q_heads;
-    if (warps == 0) return cudaSuccess;
-    const int64_t blocks = (warps * 32 + kMergeThreads - 1) / kMergeThreads;
+    const int64_t rows = static_cast<int64_t>(a.num_leaves) * a.num_q_heads;
+    if (rows == 0) return cudaSuccess;
+    // warps per row: as many as keep the grid near 4096 warps, at most 4
+    const int W = rows * 4 <= 4096 ? 4 : (rows * 2 <= 4096 ? 2 : 1);
+    const int64_t blocks = (rows * W + kMergeThreads / 32 - 1) / (kMergeThreads / 32);
+    if (blocks > 0x7fffffff) return cudaErrorInvalidValue;
     const bool bf16 = mode != PARASON_FP32;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(blocks));
@@ -215,8 +254,16 @@ cudaError_t launch_merge(const MergeArgs &a, int head_dim, int mode, bool progra
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = programmatic ? 1 : 0;
-    if (head_dim == 128) return cudaLaunchKernelEx(&cfg, tree_merge_kernel<128>, a, bf16);
-    if (head_dim == 64) return cudaLaunchKernelEx(&cfg, tree_merge_kernel<64>, a, bf16);
+    if (head_dim == 128) {
+        if (W == 4) return cudaLaunchKernelEx(&cfg, tree_merge_kernel<128, 4>, a, bf16);
+        if (W == 2) return cudaLaunchKernelEx(&cfg, tree_merge_kernel<128, 2>, a, bf16);
+        return cudaLaunchKernelEx(&cfg, tree_merge_kernel<128, 1>, a, bf16);
+    }
+    if (head_dim == 64) {
+        if (W == 4) return cudaLaunchKernelEx(&cfg, tree_merge_kernel<64, 4>, a, bf16);
+        if (W == 2) return cudaLaunchKernelEx(&cfg, tree_merge_kernel<64, 2>, a, bf16);
+        return cudaLaunchKernelEx(&cfg, tree_merge_kernel<64, 1>, a, bf16);
+    }
     return cudaErrorNotSupported;
 }
 

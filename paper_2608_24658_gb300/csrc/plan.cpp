@@ -344,9 +344,25 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
             kMaxPiecePages,
             std::max<int64_t>(kWideBlockPages,
                               wide_pages / std::max<int64_t>(1, static_cast<int64_t>(n_wide) * 3)));
-        for (const Run &r : runs)
-            if (!cut(r, r.wide ? wide_chunk : narrow_chunk, r.wide ? kWideBlockPages : 1))
-                return PARASON_EUNSUPPORTED;
+        // The row tiles of one (node, kv head) read the same pages: their
+        // pieces are emitted piece by piece across the tiles, so that the
+        // queue hands out the copies of one page range together and all but
+        // the first read of each page come from L2.
+        for (size_t i = 0; i < runs.size();) {
+            size_t j = i + 1;
+            while (j < runs.size() && runs[j].node == runs[i].node && runs[j].head == runs[i].head) ++j;
+            const Run &r = runs[i];
+            const int64_t align = r.wide ? kWideBlockPages : 1;
+            int64_t chunk = r.wide ? wide_chunk : narrow_chunk;
+            chunk = std::max<int64_t>(align, chunk / align * align);
+            const int64_t n = (r.pages + chunk - 1) / chunk;
+            int64_t per = (r.pages + n - 1) / n;
+            per = (per + align - 1) / align * align;
+            for (int64_t pg = 0; pg < r.pages; pg += per)
+                for (size_t t = i; t < j; ++t)
+                    if (!emit(runs[t], pg, std::min(per, r.pages - pg))) return PARASON_EUNSUPPORTED;
+            i = j;
+        }
     }
     if (p->items.size() > static_cast<size_t>(INT32_MAX)) return PARASON_EUNSUPPORTED;
     p->num_slots = slots;
