@@ -399,15 +399,18 @@ __device__ __forceinline__ void store_warp_partials(const AttnArgs &a, const Wor
     }
 }
 
-// Work queues.  A queue position is taken with one atomicAdd; the merge
-// kernel rewinds both counters after every launch.
+// Work queues.  A queue position is taken with one atomicAdd; items are
+// numbered in pull order, so position k of the prefix queue is item k and
+// position k of the suffix queue item num_wide_items + k.  The merge kernel
+// rewinds both counters after every launch.
+__device__ __forceinline__ int queue_item(const AttnArgs &a, int which, int k) {
+    if (which == 0) return k < a.num_wide_items ? k : -1;
+    return k < a.num_narrow_items ? a.num_wide_items + k : -1;
+}
+
 __device__ __forceinline__ int pull(const AttnArgs &a, int which, int lane) {
     int id = -1;
-    if (lane == 0) {
-        const int k = atomicAdd(a.queue_next + which, 1);
-        const int n = which == 0 ? a.num_wide_items : a.num_narrow_items;
-        if (k < n) id = (which == 0 ? a.wide_queue : a.narrow_queue)[k];
-    }
+    if (lane == 0) id = queue_item(a, which, atomicAdd(a.queue_next + which, 1));
     return __shfl_sync(0xffffffffu, id, 0);
 }
 
@@ -438,7 +441,7 @@ struct ItemRows {
 template <int D, class KV>
 __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
                             const AttnArgs &a, uint32_t ring, uint32_t bars, int warp, int lane,
-                            volatile int *ids) {
+                            WorkItem *grab) {
     using S = Shape<D, KV>;
     constexpr int NS = S::kWarpStages;
     const uint32_t my_ring = ring + warp * S::kWarpRingBytes;
@@ -446,25 +449,64 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
     const bool skip_first = (a.debug_flags & PARASON_DEBUG_SKIP_FIRST_LOAD) && warp == 0 &&
                             static_cast<int>(blockIdx.x) >= a.num_wide_ctas;
 
-    // issue side (whole warp, uniform): pulls items as its page cursor needs them
+    // Issue side (whole warp, uniform).  The next item is fetched in steps
+    // spread over the current item's last pages -- claim a queue position,
+    // then read the item's record, then switch to it -- so that no step waits
+    // on the one before: the warp keeps streaming while they complete, and
+    // holds no more than one item beyond the one it is issuing.
+    constexpr int kFetchPages = 2;
     int pulled = 0, iss_pg = 0, iss_np = 0, issued = 0;
     bool iss_done = false;
-    ItemRows rows;
+    int fetch = 0;                   // 0: idle, 1: position claimed, 2: record requested
+    int claimed = 0;                 // lane 0: the claimed queue position
+    int nxt_id = -1;
+    int32_t nxt_w = 0;               // lane i: word i of the next item's record
+    int32_t cur_w = 0;               // lane i: word i of the current item's record
+    int rows_off = 0, win_base = -1;
+    int32_t win = 0;
+    auto fetch_step = [&]() {
+        if (fetch == 0) {
+            if (lane == 0) claimed = atomicAdd(a.queue_next + 1, 1);
+            fetch = 1;
+        } else if (fetch == 1) {
+            int id = -1;
+            if (lane == 0) id = queue_item(a, 1, claimed);
+            nxt_id = __shfl_sync(0xffffffffu, id, 0);
+            if (nxt_id >= 0) nxt_w = a.item_rec[static_cast<int64_t>(nxt_id) * kRecWords + lane];
+            fetch = 2;
+        }
+    };
+    // TMA row of page pg of the current item: from the record, then from the
+    // page stream 32 rows at a time (the stream is padded by 32 entries)
+    auto row_of = [&](int pg) {
+        if (pg < kRecRows) return __shfl_sync(0xffffffffu, cur_w, kRecRow0 + pg);
+        const int base = kRecRows + ((pg - kRecRows) & ~31);
+        if (base != win_base) {
+            win = a.stream_rows[rows_off + base + lane];
+            win_base = base;
+        }
+        return __shfl_sync(0xffffffffu, win, pg - base);
+    };
     auto issue_next = [&]() {
         if (iss_done) return;
+        if (iss_pg + kFetchPages >= iss_np) fetch_step();
         while (iss_pg >= iss_np) {
-            const int id = pull(a, 1, lane);
-            if (id < 0) {
+            while (fetch < 2) fetch_step();
+            if (nxt_id < 0) {
                 iss_done = true;
                 return;
             }
-            if (lane == 0) ids[pulled % kGrabSlots] = id;
-            ++pulled;
-            iss_np = a.items[id].num_pages;
+            cur_w = nxt_w;
+            fetch = 0;
+            iss_np = __shfl_sync(0xffffffffu, cur_w, 1);          // WorkItem::num_pages
+            rows_off = __shfl_sync(0xffffffffu, cur_w, kRecRowsOff);
+            win_base = -1;
             iss_pg = 0;
-            rows.start(a, id);
+            // hand the item to the consume side
+            if (lane < 8) reinterpret_cast<int32_t *>(grab + pulled % kGrabSlots)[lane] = cur_w;
+            ++pulled;
         }
-        const int row = rows.row(iss_pg, lane);
+        const int row = row_of(iss_pg);
         if (lane == 0 && !(skip_first && issued == 0)) {
             const int s = issued % NS;
             const uint32_t bar = my_bar + s * 8;
@@ -481,7 +523,7 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
     bool ok = true;
     for (int k = 0; consumed < issued && ok; ++k) {
         __syncwarp();
-        const WorkItem it = a.items[ids[k % kGrabSlots]];
+        const WorkItem it = grab[k % kGrabSlots];
         const float2 scl = item_scales<KV>(a, it);
         uint32_t qa[D / 16][4];
         load_q_fragments<D, KV>(a, it, 0, lane, qa);
@@ -1222,7 +1264,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t bars = dev::smem_addr(smem + S::kBodyBytes);
     __shared__ int abort_flag;
     __shared__ int id_slots[kIdSlots];                        // prefix-pass item ids
-    __shared__ int grab_ids[kConsumerWarps][kGrabSlots];      // suffix-pass item ids per warp
+    __shared__ WorkItem grab_items[kConsumerWarps][kGrabSlots];   // suffix-pass items per warp
     const bool wide = static_cast<int>(blockIdx.x) < a.num_wide_ctas;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -1286,7 +1328,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncthreads();
     }
     if (warp < kConsumerWarps)
-        suffix_warp<D, KV>(&tmap_k, &tmap_v, a, ring, bars, warp, lane, grab_ids[warp]);
+        suffix_warp<D, KV>(&tmap_k, &tmap_v, a, ring, bars, warp, lane, grab_items[warp]);
 }
 
 // Shared memory and carveout are set once per device; reports the number of

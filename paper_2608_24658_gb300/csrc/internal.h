@@ -30,6 +30,13 @@ struct WorkItem {
 static_assert(sizeof(WorkItem) == 32, "WorkItem is a 32-byte device record");
 
 constexpr int kPageSize = 16;
+
+// Suffix-warp item record: 32 words (one 128-byte line, word i read by lane
+// i): the WorkItem, the start of its page rows in the stream, its first rows.
+constexpr int kRecWords = 32;
+constexpr int kRecRowsOff = 8;
+constexpr int kRecRow0 = 9;
+constexpr int kRecRows = kRecWords - kRecRow0;   // 23
 constexpr int kMaxTileRows = 128;
 constexpr int kErrWords = 4;            // device error record: code, block, site, aux
 
@@ -58,12 +65,12 @@ struct AttnArgs {
     int32_t group;
     float scale_log2;       // sm_scale * log2(e): x_t = scale_log2 * <q, k_t>
 
-    // dynamic schedule: CTAs [0, num_wide_ctas) pull prefix-pass items from
-    // wide_queue and then suffix-pass items; every warp of the other CTAs
-    // pulls suffix-pass items from narrow_queue.  queue_next[0] / [1] are the
-    // next positions (zero at launch; the merge kernel zeroes them again).
-    const int32_t *wide_queue;
-    const int32_t *narrow_queue;
+    // dynamic schedule: items are numbered in pull order, prefix-pass items
+    // [0, num_wide_items) then suffix-pass items.  CTAs [0, num_wide_ctas)
+    // pull prefix-pass items and then suffix-pass items; every warp of the
+    // other CTAs pulls suffix-pass items.  queue_next[0] / [1] are the next
+    // positions (zero at launch; the merge kernel zeroes them again).
+    const int32_t *item_rec;        // kRecWords per item, items in pull order
     int32_t num_wide_items;
     int32_t num_narrow_items;
     int32_t *queue_next;

@@ -84,6 +84,7 @@ struct parason_plan_s {
     std::vector<int32_t> narrow_queue; // suffix-pass items, in pull order
     std::vector<int32_t> item_rows;    // per item: start of its page rows
     std::vector<int32_t> stream_rows;  // TMA row of every page, item by item
+    std::vector<int32_t> item_rec;     // kRecWords per item (suffix-warp record)
     int32_t num_ctas = 0;
     int32_t num_wide_ctas = 0;
     int64_t num_slots = 0;
@@ -99,8 +100,7 @@ struct parason_plan_s {
     int32_t *d_dfs_leaf = nullptr;
     int32_t *d_merge_ptr = nullptr;
     int32_t *d_merge_ent = nullptr;
-    int32_t *d_wide_queue = nullptr;
-    int32_t *d_narrow_queue = nullptr;
+    int32_t *d_item_rec = nullptr;
     int32_t *d_item_rows = nullptr;
     int32_t *d_stream_rows = nullptr;
     int32_t *d_queue_next = nullptr;   // 2 counters, zeroed by the merge kernel
@@ -379,6 +379,17 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     if (mode == PARASON_FP32) {        // one CTA per item, no queues
         p->wide_queue.clear();
         p->narrow_queue.clear();
+    } else {
+        // item ids in pull order: the prefix queue is items [0, W), the
+        // suffix queue items [W, W + N), so a pull needs no queue lookup
+        std::vector<WorkItem> sorted;
+        sorted.reserve(p->items.size());
+        for (int32_t id : p->wide_queue) sorted.push_back(p->items[id]);
+        for (int32_t id : p->narrow_queue) sorted.push_back(p->items[id]);
+        p->items.swap(sorted);
+        for (size_t k = 0; k < p->wide_queue.size(); ++k) p->wide_queue[k] = static_cast<int32_t>(k);
+        for (size_t k = 0; k < p->narrow_queue.size(); ++k)
+            p->narrow_queue[k] = static_cast<int32_t>(p->wide_queue.size() + k);
     }
 
     // page streams: the TMA row (page * H_kv + kv head) * 16 of every page of
@@ -392,6 +403,17 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                                      parason::kPageSize);
         if (p->stream_rows.size() > static_cast<size_t>(INT32_MAX)) return PARASON_EUNSUPPORTED;
         p->item_rows[i + 1] = static_cast<int32_t>(p->stream_rows.size());
+    }
+    // one 128-byte record per item for the suffix warps: the item, the start
+    // of its page rows in the stream, and its first page rows
+    p->item_rec.assign(p->items.size() * parason::kRecWords, 0);
+    for (size_t i = 0; i < p->items.size(); ++i) {
+        int32_t *rec = p->item_rec.data() + i * parason::kRecWords;
+        std::memcpy(rec, &p->items[i], sizeof(WorkItem));
+        rec[parason::kRecRowsOff] = p->item_rows[i];
+        const int32_t np = p->items[i].num_pages;
+        for (int32_t j = 0; j < std::min(np, parason::kRecRows); ++j)
+            rec[parason::kRecRow0 + j] = p->stream_rows[p->item_rows[i] + j];
     }
 
     // merge lists per (branch, kv head): the first of the branch's g partial
@@ -428,18 +450,17 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     const size_t n_dfs = p->dfs_leaf.size() * sizeof(int32_t);
     const size_t n_mptr = p->merge_ptr.size() * sizeof(int32_t);
     const size_t n_ment = p->merge_ent.size() * sizeof(int32_t);
-    const size_t n_wq = p->wide_queue.size() * sizeof(int32_t);
-    const size_t n_nq = p->narrow_queue.size() * sizeof(int32_t);
+    const size_t n_rec = p->item_rec.size() * sizeof(int32_t);
     const size_t n_irows = p->item_rows.size() * sizeof(int32_t);
     // page rows are read 32 entries past their end by whole warps: pad
     const size_t n_strows = (p->stream_rows.size() + 32) * sizeof(int32_t);
     const size_t n_qnext = 2 * sizeof(int32_t);
     const size_t n_err = parason::kErrWords * sizeof(int32_t);
-    constexpr int kArrays = 11;
+    constexpr int kArrays = 10;
     size_t off[kArrays], total = 0;
     // the last two (queue counters, error record) are zero-filled, not copied
-    const size_t sizes[kArrays] = {n_items, n_pages,  n_dfs,    n_mptr,  n_ment, n_wq,
-                                   n_nq,    n_irows,  n_strows, n_qnext, n_err};
+    const size_t sizes[kArrays] = {n_items, n_pages,  n_dfs,   n_mptr,  n_ment,
+                                   n_rec,   n_irows,  n_strows, n_qnext, n_err};
     for (int i = 0; i < kArrays; ++i) {
         off[i] = total;
         total = align_up(total + std::max<size_t>(sizes[i], 4), kAlign);
@@ -455,18 +476,17 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     p->d_dfs_leaf = reinterpret_cast<int32_t *>(base + off[2]);
     p->d_merge_ptr = reinterpret_cast<int32_t *>(base + off[3]);
     p->d_merge_ent = reinterpret_cast<int32_t *>(base + off[4]);
-    p->d_wide_queue = reinterpret_cast<int32_t *>(base + off[5]);
-    p->d_narrow_queue = reinterpret_cast<int32_t *>(base + off[6]);
-    p->d_item_rows = reinterpret_cast<int32_t *>(base + off[7]);
-    p->d_stream_rows = reinterpret_cast<int32_t *>(base + off[8]);
-    p->d_queue_next = reinterpret_cast<int32_t *>(base + off[9]);
-    p->d_err = reinterpret_cast<int32_t *>(base + off[10]);
-    const void *src[9] = {p->items.data(),      p->page_ids.data(),    p->dfs_leaf.data(),
-                          p->merge_ptr.data(),  p->merge_ent.data(),   p->wide_queue.data(),
-                          p->narrow_queue.data(), p->item_rows.data(), p->stream_rows.data()};
-    const size_t copy[9] = {n_items, n_pages, n_dfs, n_mptr, n_ment, n_wq, n_nq, n_irows,
+    p->d_item_rec = reinterpret_cast<int32_t *>(base + off[5]);
+    p->d_item_rows = reinterpret_cast<int32_t *>(base + off[6]);
+    p->d_stream_rows = reinterpret_cast<int32_t *>(base + off[7]);
+    p->d_queue_next = reinterpret_cast<int32_t *>(base + off[8]);
+    p->d_err = reinterpret_cast<int32_t *>(base + off[9]);
+    const void *src[8] = {p->items.data(),     p->page_ids.data(),  p->dfs_leaf.data(),
+                          p->merge_ptr.data(), p->merge_ent.data(), p->item_rec.data(),
+                          p->item_rows.data(), p->stream_rows.data()};
+    const size_t copy[8] = {n_items, n_pages, n_dfs, n_mptr, n_ment, n_rec, n_irows,
                             p->stream_rows.size() * sizeof(int32_t)};
-    for (int i = 0; i < 9; ++i) {
+    for (int i = 0; i < 8; ++i) {
         if (copy[i] == 0) continue;
         if (cudaMemcpyAsync(base + off[i], src[i], copy[i], cudaMemcpyHostToDevice, stream) !=
             cudaSuccess)
@@ -673,8 +693,7 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
         a.num_kv_heads = p->cfg.num_kv_heads;
         a.group = p->group;
         a.scale_log2 = sm_scale * 1.4426950408889634f;
-        a.wide_queue = p->d_wide_queue;
-        a.narrow_queue = p->d_narrow_queue;
+        a.item_rec = p->d_item_rec;
         a.num_wide_items = static_cast<int32_t>(p->wide_queue.size());
         a.num_narrow_items = static_cast<int32_t>(p->narrow_queue.size());
         a.item_rows = p->d_item_rows;
