@@ -458,7 +458,9 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
     int pulled = 0, iss_pg = 0, iss_np = 0, issued = 0;
     bool iss_done = false;
     int fetch = 0;                   // 0: idle, 1: position claimed, 2: record requested
-    int claimed = 0;                 // lane 0: the claimed queue position
+    // lane 0: the claimed queue position; a suffix CTA's warps own their first
+    const int own_first = static_cast<int>(blockIdx.x) - a.num_wide_ctas;
+    int claimed = own_first >= 0 ? own_first * kConsumerWarps + warp : -1;
     int nxt_id = -1;
     int32_t nxt_w = 0;               // lane i: word i of the next item's record
     int32_t cur_w = 0;               // lane i: word i of the current item's record
@@ -466,7 +468,7 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
     int32_t win = 0;
     auto fetch_step = [&]() {
         if (fetch == 0) {
-            if (lane == 0) claimed = atomicAdd(a.queue_next + 1, 1);
+            if (lane == 0 && (pulled > 0 || claimed < 0)) claimed = atomicAdd(a.queue_next + 1, 1);
             fetch = 1;
         } else if (fetch == 1) {
             int id = -1;
@@ -600,7 +602,10 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
         int stage = 0;
         bool go = true;
         for (int k = 0; go; ++k) {
-            const int id = *abort_flag ? -1 : pull(a, 0, lane);
+            // a prefix CTA owns position blockIdx.x of the prefix queue
+            const int id = *abort_flag ? -1
+                                       : (k == 0 ? queue_item(a, 0, static_cast<int>(blockIdx.x))
+                                                 : pull(a, 0, lane));
             if (lane == 0) publish_id(id_slots, id_bars, k, id);
             if (id < 0) break;
             ItemRows rows;
@@ -879,7 +884,10 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                 if (lane == 0) tc_fail(a, abort_flag, kSiteProducerEmpty);
                 break;
             }
-            int id = *abort_flag ? -1 : pull(a, 0, lane);
+            // a prefix CTA owns position blockIdx.x of the prefix queue
+            int id = *abort_flag ? -1
+                                 : (k == 0 ? queue_item(a, 0, static_cast<int>(blockIdx.x))
+                                           : pull(a, 0, lane));
             TcMeta &m = meta[s];
             if (id >= 0) {
                 const WorkItem it = a.items[id];

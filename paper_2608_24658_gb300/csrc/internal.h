@@ -69,7 +69,10 @@ struct AttnArgs {
     // [0, num_wide_items) then suffix-pass items.  CTAs [0, num_wide_ctas)
     // pull prefix-pass items and then suffix-pass items; every warp of the
     // other CTAs pulls suffix-pass items.  queue_next[0] / [1] are the next
-    // positions (zero at launch; the merge kernel zeroes them again).
+    // positions to claim.  The first claims need no atomic: position c of
+    // the prefix queue belongs to prefix CTA c, position 8 (c - W) + w of the
+    // suffix queue to warp w of suffix CTA c, so the counters start past
+    // them (queue_start; the merge kernel sets them back).
     const int32_t *item_rec;        // kRecWords per item, items in pull order
     int32_t num_wide_items;
     int32_t num_narrow_items;
@@ -95,7 +98,8 @@ struct MergeArgs {
     int32_t num_q_heads;
     int32_t num_kv_heads;
     int32_t group;
-    int32_t *queue_next;        // zeroed for the next launch
+    int32_t *queue_next;        // set back to queue_start for the next launch
+    int32_t queue_start[2];
 };
 
 // Resident CTAs per SM of the persistent attention kernel of a mode (sets its

@@ -117,8 +117,8 @@ __global__ void __launch_bounds__(kMergeThreads)
     asm volatile("griddepcontrol.wait;" ::: "memory");
     // the attention grid is complete: rewind its work queues for the next call
     if (blockIdx.x == 0 && threadIdx.x == 0 && a.queue_next) {
-        a.queue_next[0] = 0;
-        a.queue_next[1] = 0;
+        a.queue_next[0] = a.queue_start[0];
+        a.queue_next[1] = a.queue_start[1];
     }
 
     float M = -INFINITY, L = 0.f;

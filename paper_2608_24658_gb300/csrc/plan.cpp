@@ -103,7 +103,8 @@ struct parason_plan_s {
     int32_t *d_item_rec = nullptr;
     int32_t *d_item_rows = nullptr;
     int32_t *d_stream_rows = nullptr;
-    int32_t *d_queue_next = nullptr;   // 2 counters, zeroed by the merge kernel
+    int32_t *d_queue_next = nullptr;   // 2 counters, set back to queue_start by the merge kernel
+    int32_t queue_start[2] = {0, 0};   // positions past the ones CTAs own at launch
     int32_t *d_err = nullptr;
     uint32_t debug_flags = 0;
     int64_t wait_limit_ns = kDefaultWaitNs;
@@ -291,6 +292,10 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     }
     p->num_wide_ctas = n_wide;
     p->num_ctas = n_wide + n_narrow_ctas;
+    // the kernel's CTAs own the first positions of each queue (one per
+    // prefix CTA, one per warp of a suffix CTA); the counters start past them
+    p->queue_start[0] = n_wide;
+    p->queue_start[1] = n_narrow_ctas * kNarrowWarps;
 
     // Items: every run cut into pieces of at most `chunk` pages (the prefix
     // pass in whole 64-token blocks).  Each role's pieces form a queue,
@@ -493,7 +498,9 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
             return PARASON_ECUDA;
     }
     if (cudaMemsetAsync(p->d_err, 0, n_err, stream) != cudaSuccess) return PARASON_ECUDA;
-    if (cudaMemsetAsync(p->d_queue_next, 0, n_qnext, stream) != cudaSuccess) return PARASON_ECUDA;
+    if (cudaMemcpyAsync(p->d_queue_next, p->queue_start, n_qnext, cudaMemcpyHostToDevice, stream) !=
+        cudaSuccess)
+        return PARASON_ECUDA;
     // the host vectors are pageable: make sure the copies have consumed them
     // before the caller can free its own arrays (ours stay alive anyway)
     if (cudaStreamSynchronize(stream) != cudaSuccess) return PARASON_ECUDA;
@@ -743,6 +750,8 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
     m.group = p->group;
     m.num_kv_heads = p->cfg.num_kv_heads;
     m.queue_next = p->d_queue_next;
+    m.queue_start[0] = p->queue_start[0];
+    m.queue_start[1] = p->queue_start[1];
     // programmatic dependent launch after the persistent kernel: the merge
     // grid is launched while the attention grid drains, and waits for it
     const bool pdl = has_items && p->cfg.mode != PARASON_FP32;
@@ -778,7 +787,9 @@ parason_status parason_plan_check(parason_plan p, parason_stream_t stream) {
         return PARASON_ECUDA;
     if (rec[0] != 0) {
         if (cudaMemset(p->d_err, 0, sizeof rec) != cudaSuccess) return PARASON_ECUDA;
-        if (cudaMemset(p->d_queue_next, 0, 2 * sizeof(int32_t)) != cudaSuccess) return PARASON_ECUDA;
+        if (cudaMemcpy(p->d_queue_next, p->queue_start, 2 * sizeof(int32_t), cudaMemcpyHostToDevice) !=
+            cudaSuccess)
+            return PARASON_ECUDA;
         return rec[0] == PARASON_ETIMEOUT ? PARASON_ETIMEOUT : PARASON_ECUDA;
     }
     return PARASON_OK;
