@@ -41,8 +41,9 @@
 namespace parason {
 namespace {
 
-constexpr int kConsumerWarps = 8;
+constexpr int kConsumerWarps = 8;                          // prefix pass on mma.sync
 constexpr int kConsumerThreads = kConsumerWarps * 32;
+constexpr int kMaxSuffixWarps = 12;                        // suffix pass: warps per CTA, at most
 // 12 warps: the suffix pass runs 8 autonomous warps; the prefix pass on
 // tcgen05 uses 11 (softmax 4, epilogue 4, producer, MMA issuer, scheduler),
 // the one on mma.sync 9 (8 consumers and a producer)
@@ -69,11 +70,13 @@ struct Shape {
     static constexpr int kSegBytes = kPageSize * 128;
     static constexpr int kStageBytes = 2 * kPageBytes;      // K and V of one page
 
-    // suffix pass: a private ring per warp
-    static constexpr int kWarpStages = (192 * 1024) / (kConsumerWarps * kStageBytes);
+    // suffix pass: a private ring per warp.  An e4m3 page costs more issue
+    // per byte (widening to f16), so that pass runs more, shallower warps.
+    static constexpr int kSuffixWarps = KV::kElemBytes == 1 ? 12 : 8;
+    static constexpr int kWarpStages = (192 * 1024) / (kSuffixWarps * kStageBytes);
     static constexpr int kWarpRingBytes = kWarpStages * kStageBytes;
-    static constexpr int kNarrowBytes = kConsumerWarps * kWarpRingBytes;
-    static constexpr int kNarrowBars = kConsumerWarps * kWarpStages;
+    static constexpr int kNarrowBytes = kSuffixWarps * kWarpRingBytes;
+    static constexpr int kNarrowBars = kSuffixWarps * kWarpStages;
 
     // prefix pass: one ring + combine scratch [warp][16 rows][D/2 + 8] floats
     static constexpr int kHalf = D / 2;
@@ -92,6 +95,7 @@ struct Shape {
     static constexpr int kSmemBytes = kBodyBytes + kBars * 8 + 1024;   // + alignment slack
     static_assert(kRowBytes % 128 == 0, "token rows are whole 128-byte blocks");
     static_assert(kWarpStages >= 2, "suffix ring depth");
+    static_assert(kSuffixWarps <= kMaxSuffixWarps, "suffix-pass warps fit the item rings");
     static_assert(kWideStages >= 4, "prefix ring depth");
     static_assert(kSmemBytes <= kSmemBudget, "shared memory budget");
 
@@ -460,7 +464,7 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
     int fetch = 0;                   // 0: idle, 1: position claimed, 2: record requested
     // lane 0: the claimed queue position; a suffix CTA's warps own their first
     const int own_first = static_cast<int>(blockIdx.x) - a.num_wide_ctas;
-    int claimed = own_first >= 0 ? own_first * kConsumerWarps + warp : -1;
+    int claimed = own_first >= 0 ? own_first * S::kSuffixWarps + warp : -1;
     int nxt_id = -1;
     int32_t nxt_w = 0;               // lane i: word i of the next item's record
     int32_t cur_w = 0;               // lane i: word i of the current item's record
@@ -807,6 +811,7 @@ constexpr int kTcMmaWarp = 9;
 constexpr int kTcSchedulerWarp = 10;
 static_assert(kTcRingBytes <= Shape<128, KvBf16>::kBodyBytes, "tcgen05 ring fits the CTA's memory");
 static_assert(kTcSchedulerWarp < kThreads / 32, "every tcgen05 role has a warp");
+static_assert(kMaxSuffixWarps <= kThreads / 32, "every suffix-pass warp exists");
 
 // Metadata of one prefix item, staged by the scheduler warp.
 struct TcMeta {
@@ -1272,7 +1277,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t bars = dev::smem_addr(smem + S::kBodyBytes);
     __shared__ int abort_flag;
     __shared__ int id_slots[kIdSlots];                        // prefix-pass item ids
-    __shared__ WorkItem grab_items[kConsumerWarps][kGrabSlots];   // suffix-pass items per warp
+    __shared__ WorkItem grab_items[kMaxSuffixWarps][kGrabSlots];  // suffix-pass items per warp
     const bool wide = static_cast<int>(blockIdx.x) < a.num_wide_ctas;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -1335,7 +1340,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         __syncthreads();
     }
-    if (warp < kConsumerWarps)
+    if (warp < S::kSuffixWarps)
         suffix_warp<D, KV>(&tmap_k, &tmap_v, a, ring, bars, warp, lane, grab_items[warp]);
 }
 

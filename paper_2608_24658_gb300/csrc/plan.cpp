@@ -30,7 +30,8 @@ using parason::WorkItem;
 namespace {
 
 constexpr int kNarrowRows = 16;         // nodes with at most this many rows: suffix pass
-constexpr int kNarrowWarps = 8;         // autonomous warps per suffix-pass CTA
+// autonomous warps per suffix-pass CTA (the kernel's count for the KV format)
+int32_t narrow_warps(int32_t mode) { return mode == PARASON_FP8_E4M3_KV ? 12 : 8; }
 constexpr int kMinPiecePages = 8;       // suffix-pass pieces are at least this long
 constexpr int kMaxPiecePages = 128;     // and at most this long
 constexpr int kWideBlockPages = 4;      // prefix pieces are whole 64-token blocks
@@ -295,7 +296,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     // the kernel's CTAs own the first positions of each queue (one per
     // prefix CTA, one per warp of a suffix CTA); the counters start past them
     p->queue_start[0] = n_wide;
-    p->queue_start[1] = n_narrow_ctas * kNarrowWarps;
+    p->queue_start[1] = n_narrow_ctas * narrow_warps(mode);
 
     // Items: every run cut into pieces of at most `chunk` pages (the prefix
     // pass in whole 64-token blocks).  Each role's pieces form a queue,
@@ -338,7 +339,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         for (const Run &r : runs)
             if (!cut(r, kFp32ChunkPages, 1)) return PARASON_EUNSUPPORTED;
     } else {
-        const int64_t total_warps = static_cast<int64_t>(p->num_sms) * kNarrowWarps;
+        const int64_t total_warps = static_cast<int64_t>(p->num_sms) * narrow_warps(mode);
         const int64_t narrow_chunk = std::min<int64_t>(
             kMaxPiecePages,
             std::max<int64_t>(kMinPiecePages, narrow_pages / std::max<int64_t>(1, total_warps * 3)));
