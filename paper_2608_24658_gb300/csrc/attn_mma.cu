@@ -52,6 +52,7 @@ constexpr long long kDrainLimitNs = 1000000000LL;
 constexpr int kSmemBudget = 220 * 1024;                    // dynamic, one CTA per SM
 constexpr int kIdSlots = 8;      // prefix-pass item ids in flight from producer to consumers
 constexpr int kGrabSlots = 8;    // suffix-pass item ids a warp has pulled but not finished
+constexpr float kLazyRescaleLog2 = 8.f;   // mma.sync softmax: move the reference max past 2^8
 
 struct KvBf16 {
     static constexpr int kElemBytes = 2;
@@ -195,11 +196,28 @@ __device__ __forceinline__ void softmax_page(const float (&sc)[2][4], int valid,
     mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
     mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
     mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-    // token 0 of every page of an item is valid, so mx0/mx1 are finite
-    const float mn0 = fmaxf(st.m[0], mx0), mn1 = fmaxf(st.m[1], mx1);
-    const float al0 = dev::fast_exp2(st.m[0] - mn0), al1 = dev::fast_exp2(st.m[1] - mn1);
-    st.m[0] = mn0;
-    st.m[1] = mn1;
+    // token 0 of every page of an item is valid, so mx0/mx1 are finite.
+    // Lazy rescale: the reference max m (and with it o and l) moves only when
+    // some row's max grows by more than 2^8 (always at an item's first page,
+    // where m = -inf); otherwise P = 2^(x - m) stays below 2^8 and o, l keep
+    // accumulating against the old m, which the merge takes as it is.
+    const bool grow = mx0 > st.m[0] + kLazyRescaleLog2 || mx1 > st.m[1] + kLazyRescaleLog2;
+    if (__any_sync(0xffffffffu, grow)) {
+        const float mn0 = fmaxf(st.m[0], mx0), mn1 = fmaxf(st.m[1], mx1);
+        const float al0 = dev::fast_exp2(st.m[0] - mn0), al1 = dev::fast_exp2(st.m[1] - mn1);
+        st.m[0] = mn0;
+        st.m[1] = mn1;
+        st.l[0] *= al0;
+        st.l[1] *= al1;
+#pragma unroll
+        for (int dt = 0; dt < D / 8; ++dt) {
+            st.o[dt][0] *= al0;
+            st.o[dt][1] *= al0;
+            st.o[dt][2] *= al1;
+            st.o[dt][3] *= al1;
+        }
+    }
+    const float mn0 = st.m[0], mn1 = st.m[1];
     float p[2][4];
 #pragma unroll
     for (int nt = 0; nt < 2; ++nt) {
@@ -208,15 +226,8 @@ __device__ __forceinline__ void softmax_page(const float (&sc)[2][4], int valid,
         p[nt][2] = dev::fast_exp2(x[nt][2] - mn1);
         p[nt][3] = dev::fast_exp2(x[nt][3] - mn1);
     }
-    st.l[0] = st.l[0] * al0 + (p[0][0] + p[0][1] + p[1][0] + p[1][1]);
-    st.l[1] = st.l[1] * al1 + (p[0][2] + p[0][3] + p[1][2] + p[1][3]);
-#pragma unroll
-    for (int dt = 0; dt < D / 8; ++dt) {
-        st.o[dt][0] *= al0;
-        st.o[dt][1] *= al0;
-        st.o[dt][2] *= al1;
-        st.o[dt][3] *= al1;
-    }
+    st.l[0] += p[0][0] + p[0][1] + p[1][0] + p[1][1];
+    st.l[1] += p[0][2] + p[0][3] + p[1][2] + p[1][3];
     if constexpr (KV::kElemBytes == 2) {
         pa[0] = dev::pack_bf16(p[0][0], p[0][1]);
         pa[1] = dev::pack_bf16(p[0][2], p[0][3]);
