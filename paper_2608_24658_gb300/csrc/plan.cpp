@@ -38,7 +38,7 @@ constexpr int kWideBlockPages = 4;      // prefix pieces are whole 64-token bloc
 constexpr double kWideProvision = 1.15; // prefix CTAs relative to the cost model
 constexpr int kFp32ChunkPages = 32;
 constexpr double kWideGroupPageCost = 1.0;   // one 16-row group of one page, in suffix pages
-constexpr double kTcPageCost = 3.2;          // one page of a tcgen05 prefix tile (measured)
+constexpr double kTcPageCost = 2.4;          // one page of a tcgen05 prefix tile (tuned)
 constexpr int64_t kDefaultWaitNs = 2000000000LL;
 constexpr size_t kAlign = 256;
 
