@@ -129,10 +129,21 @@ __global__ void __launch_bounds__(kMergeThreads)
     for (int i0 = 0; e0 + w + W * i0 < e1; i0 += 32) {
         const int e = e0 + w + W * (i0 + lane);
         const bool valid = e < e1;
-        int slot = 0;
+        const int slot = valid ? (i0 == 0 ? first_slot : a.merge_ent[e] + r) : 0;
+        const int cnt = min(32, (e1 - (e0 + w) + W - 1) / W - i0);
+        // With few rows (W = 4: up to 8 entries a warp) the pass's first 8
+        // partial rows are requested together with the (m, l) of its entries,
+        // since they do not depend on the weights.  With many rows the extra
+        // registers cost more occupancy than the round trip they save.
+        constexpr int kEarly = W == 4 ? 8 : 0;
+        float v0[kEarly > 0 ? kEarly : 1][N];
+#pragma unroll
+        for (int k = 0; k < kEarly; ++k) {
+            const int si = __shfl_sync(0xffffffffu, slot, k);
+            if (k < cnt) load_f32<N>(a.part_o + static_cast<int64_t>(si) * D + lane * N, v0[k]);
+        }
         float m = -INFINITY, l = 0.f;
         if (valid) {
-            slot = i0 == 0 ? first_slot : a.merge_ent[e] + r;
             const float2 ml = a.part_ml[slot];
             m = ml.x;
             l = ml.y;
@@ -149,8 +160,14 @@ __global__ void __launch_bounds__(kMergeThreads)
         L = L * s_old + lw;
 #pragma unroll
         for (int i = 0; i < N; ++i) acc[i] *= s_old;
-        const int cnt = min(32, (e1 - (e0 + w) + W - 1) / W - i0);
-        for (int k0 = 0; k0 < cnt; k0 += 8) {
+#pragma unroll
+        for (int k = 0; k < kEarly; ++k) {
+            const float wk = __shfl_sync(0xffffffffu, wgt, k);
+            if (k < cnt)
+#pragma unroll
+                for (int c = 0; c < N; ++c) acc[c] += wk * v0[k][c];
+        }
+        for (int k0 = kEarly; k0 < cnt; k0 += 8) {
             float v[8][N];
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
