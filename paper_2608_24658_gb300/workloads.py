@@ -403,3 +403,71 @@ def host_subset(tree: ForkTree, sel: Sequence[int]) -> ForkTree:
                    num_physical_pages=len(phys), q=q, k_pages=k, v_pages=v,
                    k_scale=None if tree.k_scale is None else tree.k_scale.cpu(),
                    v_scale=None if tree.v_scale is None else tree.v_scale.cpu())
+
+
+# ----------------------------------------------------------------------------
+# reasoning traces (tag streams of the parallel-reasoning grammar, Fig. 4)
+# ----------------------------------------------------------------------------
+
+# tag codes of a trace symbol stream (text tokens are ids >= 0)
+TAG_THINK, TAG_THINK_END = -1, -2
+TAG_PARALLEL, TAG_PARALLEL_END = -3, -4
+TAG_OUTLINES, TAG_OUTLINES_END = -5, -6
+TAG_SUBTASK, TAG_SUBTASK_END = -7, -8
+TAG_TRIAL, TAG_TRIAL_END = -9, -10
+TAG_THREAD, TAG_THREAD_END = -11, -12
+
+
+def random_trace(seed: int, *, max_depth: int = 2, p_parallel: float = 0.5,
+                 text_len=(1, 24), entry_len=(1, 6), entries=(1, 4), body_items=(1, 3),
+                 p_mismatch: float = 0.1, p_empty_thread: float = 0.05) -> np.ndarray:
+    """A random trace in the grammar: bodies of text runs and parallel blocks
+    nested up to `max_depth`, outlines of 1..4 Subtask/Trial entries, usually
+    one thread per entry (sometimes one more or one fewer), occasionally an
+    empty thread body.  Text token ids are random non-negative ints."""
+    rng = np.random.default_rng(seed)
+    out = [TAG_THINK]
+
+    def text(lo_hi):
+        n = int(rng.integers(lo_hi[0], lo_hi[1] + 1))
+        out.extend(int(x) for x in rng.integers(0, 1 << 17, size=n))
+
+    def body(level, allow_empty):
+        if allow_empty and rng.random() < p_empty_thread:
+            return
+        for _ in range(int(rng.integers(body_items[0], body_items[1] + 1))):
+            if level < max_depth and rng.random() < p_parallel:
+                region(level)
+            else:
+                text(text_len)
+
+    def region(level):
+        out.extend([TAG_PARALLEL, TAG_OUTLINES])
+        k = int(rng.integers(entries[0], entries[1] + 1))
+        for _ in range(k):
+            sub = rng.random() < 0.5
+            out.append(TAG_SUBTASK if sub else TAG_TRIAL)
+            text(entry_len)
+            out.append(TAG_SUBTASK_END if sub else TAG_TRIAL_END)
+        out.append(TAG_OUTLINES_END)
+        nthreads = k
+        if rng.random() < p_mismatch:
+            nthreads = max(1, k + int(rng.choice([-1, 1])))
+        for _ in range(nthreads):
+            out.append(TAG_THREAD)
+            body(level + 1, True)
+            out.append(TAG_THREAD_END)
+        out.append(TAG_PARALLEL_END)
+
+    body(0, False)
+    out.append(TAG_THINK_END)
+    return np.asarray(out, dtype=np.int32)
+
+
+def paper_scale_trace(seed: int) -> np.ndarray:
+    """A trace of about the size the paper reports (tens of thousands of
+    generated tokens, token-level acceleration near 1.7-1.9; Tab. 4, Tab. 5):
+    one level of parallel blocks with 2-3 threads each."""
+    return random_trace(seed, max_depth=1, p_parallel=0.4, text_len=(250, 1200),
+                        entry_len=(10, 60), entries=(2, 3), body_items=(5, 10), p_mismatch=0.0,
+                        p_empty_thread=0.0)
