@@ -400,6 +400,53 @@ def kernel_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
+def run_trace(args):
+    """Host throughput of the tag-stream parser (grammar check, latency
+    metrics, fork tree of every top-level block) on paper-scale traces, the
+    oracle timed beside it.  Not part of the decode step."""
+    from paper_2608_24658_gb300 import api, build as lib_build, workloads
+    lib_build.build()
+    traces = [workloads.paper_scale_trace(seed) for seed in range(16)]
+    tokens = sum(len(t) for t in traces)
+
+    def one_pass():
+        for t in traces:
+            st = api.trace_stats(t)
+            for b in range(st["top_level_blocks"]):
+                api.trace_fork_tree(t, b)
+
+    for _ in range(args.warmup):
+        one_pass()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        one_pass()
+    el = time.perf_counter() - t0
+    value = tokens * args.steps / el
+    cpu = None
+    if not args.no_cpu_baseline:
+        from oracle import trace_oracle
+        t1 = time.perf_counter()
+        n = 0
+        for t in traces:
+            lst = t.tolist()
+            st = trace_oracle.stats(lst)
+            for b in range(st["parallel_blocks"]):
+                try:
+                    trace_oracle.fork_tree(lst, b)
+                except IndexError:
+                    break
+            n += len(t)
+        cpu = {"value": n / (time.perf_counter() - t1), "unit": "tokens/s", "cores": 1,
+               "kind": "oracle", "sample": f"{len(traces)} paper-scale traces, once"}
+    line = {"metric": "trace parse throughput", "value": value, "unit": "tokens/s", "n_gpus": 0,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
+            "higher_is_better": True, "data": "synthetic",
+            "config": {"workload": "16 paper-scale traces", "tokens_per_step": tokens},
+            "component": "trace", "cpu_baseline": cpu}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -410,9 +457,13 @@ def main(argv=None):
     ap.add_argument("--mode", choices=["bf16", "fp8", "fp32"], default="bf16")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--component", choices=["decode", "trace"], default="decode",
+                    help="decode: the attention step (default); trace: the tag-stream parser")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.component == "trace":
+        return run_trace(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_gpu(args)

@@ -300,6 +300,75 @@ parason_status parason_plan_read_timing(parason_plan plan, float *attn_ms, float
 /* Number of kernel launches one parason_attn_decode call of this plan makes. */
 int32_t parason_plan_launches_per_decode(parason_plan plan);
 
+/* ------------------------------------------------------------------------
+ * Reasoning traces: the tag stream of the parallel-reasoning grammar (Fig. 4)
+ *
+ *   S -> <think> B </think>        B -> T B | P B | (empty)
+ *   P -> <Parallel> O H </Parallel> O -> <Outlines> G </Outlines>
+ *   G -> E G | E                   E -> <Subtask> T </Subtask> | <Trial> T </Trial>
+ *   H -> W H | W                   W -> <Thread> B </Thread>
+ *   T -> one or more text tokens
+ *
+ * A trace is an array of int32 symbols: a text token is any id >= 0, a tag
+ * is one of the codes below (one generated token each).
+ * ------------------------------------------------------------------------ */
+enum {
+    PARASON_TAG_THINK = -1, PARASON_TAG_THINK_END = -2,
+    PARASON_TAG_PARALLEL = -3, PARASON_TAG_PARALLEL_END = -4,
+    PARASON_TAG_OUTLINES = -5, PARASON_TAG_OUTLINES_END = -6,
+    PARASON_TAG_SUBTASK = -7, PARASON_TAG_SUBTASK_END = -8,
+    PARASON_TAG_TRIAL = -9, PARASON_TAG_TRIAL_END = -10,
+    PARASON_TAG_THREAD = -11, PARASON_TAG_THREAD_END = -12
+};
+
+typedef struct {
+    int64_t total_tokens;     /* every symbol of the trace                          */
+    int64_t latency_tokens;   /* token length of the longest generation path
+                                 (Sec. 4): sequential tokens count one each, a
+                                 <Parallel> block counts its tags and outlines
+                                 plus its slowest thread                          */
+    int64_t subtask_tokens;   /* tokens whose innermost thread is a Subtask: thread
+                                 k of a block has the type of outline entry k     */
+    int64_t trial_tokens;     /* same for Trial (threads past the last entry are
+                                 untyped)                                         */
+    int32_t parallel_blocks;  /* <Parallel> blocks at any depth                     */
+    int32_t threads;          /* threads at any depth                              */
+    int32_t max_depth;        /* deepest nesting of blocks (0: none)               */
+    int32_t top_level_blocks; /* blocks directly in the <think> body               */
+    double acceleration;      /* total / latency (Tab. 4)                          */
+    double eta;               /* 1 - latency / total (Sec. 3.5)                    */
+} parason_trace_stats;
+
+/*
+ * Check a trace against the grammar and compute its token metrics (host
+ * only, no CUDA call).  `symbols` is host memory of n int32.  Returns
+ * PARASON_EINVAL for NULL pointers or a trace outside the grammar; then
+ * *error_pos (if not NULL) is the first symbol no derivation can accept (n if
+ * the trace ends early).  The grammar is LL(1), so that position is unique.
+ */
+parason_status parason_trace_analyze(const int32_t *symbols, int64_t n, parason_trace_stats *out,
+                                     int64_t *error_pos);
+
+/*
+ * Fork tree of top-level block `block` (0-based, in trace order), in the form
+ * parason_attn_plan takes: the decode state in which every innermost thread
+ * of the block runs, each at its full length in the trace.
+ *   node 0       every token before the block's first <Thread> (earlier
+ *                blocks are joined, so all of it is context);
+ *   thread node  its tokens up to the end of its first nested outlines block,
+ *                whose threads become its children -- or all its tokens, as
+ *                a branch, if it has no nested block.
+ * Nodes are in depth-first order (parent[i] < i); leaf_node lists the
+ * branches in that order.  parent and node_len hold `capacity` entries,
+ * leaf_node as many.  *num_nodes and *num_leaves are set whenever the trace
+ * parses; PARASON_EINVAL if it does not, if `block` is out of range or if
+ * capacity < *num_nodes (call again with a larger capacity).  Host only.
+ */
+parason_status parason_trace_fork_tree(const int32_t *symbols, int64_t n, int32_t block,
+                                       int32_t capacity, int32_t *parent, int32_t *node_len,
+                                       int32_t *leaf_node, int32_t *num_nodes,
+                                       int32_t *num_leaves);
+
 /* Library version, "major.minor.patch". */
 const char *parason_version(void);
 

@@ -42,6 +42,14 @@ class PlanInfo(ctypes.Structure):
                 ("num_narrow_items", ctypes.c_int32)]
 
 
+class TraceStats(ctypes.Structure):
+    _fields_ = [("total_tokens", ctypes.c_int64), ("latency_tokens", ctypes.c_int64),
+                ("subtask_tokens", ctypes.c_int64), ("trial_tokens", ctypes.c_int64),
+                ("parallel_blocks", ctypes.c_int32), ("threads", ctypes.c_int32),
+                ("max_depth", ctypes.c_int32), ("top_level_blocks", ctypes.c_int32),
+                ("acceleration", ctypes.c_double), ("eta", ctypes.c_double)]
+
+
 SIGNATURES = {
     "parason_attn_plan": (ctypes.c_int, [ctypes.POINTER(AttnConfig), _i32, _p, _p, _p, _p, _i32,
                                          _p, _i64, _p, _pp]),
@@ -50,6 +58,11 @@ SIGNATURES = {
     "parason_plan_workspace_bytes": (_sz, [_p]),
     "parason_attn_decode": (ctypes.c_int, [_p, _p, _p, _p, _p, _p, _p, _p, _p, _sz, _p]),
     "parason_attn_decode_no_alloc": (ctypes.c_int, [_p, _p, _p, _p, _p, _p, _p, _p, _p]),
+    "parason_trace_analyze": (ctypes.c_int, [_p, _i64, ctypes.POINTER(TraceStats),
+                                             ctypes.POINTER(ctypes.c_int64)]),
+    "parason_trace_fork_tree": (ctypes.c_int, [_p, _i64, _i32, _i32, _p, _p, _p,
+                                               ctypes.POINTER(ctypes.c_int32),
+                                               ctypes.POINTER(ctypes.c_int32)]),
     "parason_lse_merge": (ctypes.c_int, [_p, _p, _p, _p, _p, _p, _i64, _i32, _i32, _p]),
     "parason_plan_check": (ctypes.c_int, [_p, _p]),
     "parason_plan_destroy": (None, [_p]),

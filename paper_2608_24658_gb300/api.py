@@ -264,3 +264,53 @@ def version() -> str:
 
 
 __all__ = ["Plan", "lse_merge", "version", "ParasonError"]
+
+
+# ---------------------------------------------------------------------------
+# reasoning traces (tag streams of the parallel-reasoning grammar)
+# ---------------------------------------------------------------------------
+
+class TraceError(ParasonError):
+    """A trace outside the grammar; ``pos`` is the first symbol no derivation accepts."""
+
+    def __init__(self, pos: int):
+        super().__init__(_lib.EINVAL, f"trace outside the grammar at symbol {pos}")
+        self.pos = pos
+
+
+def _symbols(symbols) -> np.ndarray:
+    a = np.ascontiguousarray(np.asarray(symbols, dtype=np.int32))
+    if a.ndim != 1:
+        raise ValueError("a trace is a 1-D array of int32 symbols")
+    return a
+
+
+def trace_stats(symbols) -> dict:
+    """Token metrics of one trace (see parason_trace_analyze)."""
+    a = _symbols(symbols)
+    st = _lib.TraceStats()
+    err = ctypes.c_int64(-1)
+    rc = _lib.load().parason_trace_analyze(_ptr(a), a.size, ctypes.byref(st), ctypes.byref(err))
+    if rc == _lib.EINVAL and err.value >= 0:
+        raise TraceError(err.value)
+    check(rc, "parason_trace_analyze")
+    return {name: getattr(st, name) for name, _ in _lib.TraceStats._fields_}
+
+
+def trace_fork_tree(symbols, block: int = 0):
+    """(parent, node_len, leaf_node) of top-level block `block` (int32 arrays)."""
+    a = _symbols(symbols)
+    nn, nl = ctypes.c_int32(0), ctypes.c_int32(0)
+    lib = _lib.load()
+    cap = 64
+    while True:
+        parent = np.zeros(cap, np.int32)
+        node_len = np.zeros(cap, np.int32)
+        leaf = np.zeros(cap, np.int32)
+        rc = lib.parason_trace_fork_tree(_ptr(a), a.size, block, cap, _ptr(parent), _ptr(node_len),
+                                         _ptr(leaf), ctypes.byref(nn), ctypes.byref(nl))
+        if rc == _lib.EINVAL and nn.value > cap:
+            cap = nn.value
+            continue
+        check(rc, "parason_trace_fork_tree")
+        return parent[:nn.value].copy(), node_len[:nn.value].copy(), leaf[:nl.value].copy()
