@@ -447,6 +447,80 @@ def run_trace(args):
     return 0
 
 
+def run_append(args):
+    """One decode step's plan update (parason_plan_append: a token on every
+    branch) against building a new plan, on the Llama-3-shape workload with
+    room to grow; and the decode step before and after 64 appends."""
+    import torch
+    from paper_2608_24658_gb300 import build as lib_build
+    from paper_2608_24658_gb300.api import Plan
+    lib_build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    steps = 64          # within the room a plan leaves its branches
+    tree = W.make_config(args.config, args.mode, device=dev, extra_pages=4096)
+    pool = W.free_pages(tree)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+
+    def decode_us(plan, tree, n=50):
+        out = torch.empty_like(tree.q)
+        lse = torch.empty(tree.num_leaves, tree.num_q_heads, dtype=torch.float32, device=dev)
+        ws = plan.workspace(dev)
+        for _ in range(5):
+            plan.decode(tree.q, tree.k_pages, tree.v_pages, out=out, lse=lse, workspace=ws,
+                        k_scale=tree.k_scale, v_scale=tree.v_scale, stream=stream)
+        times = []
+        for _ in range(n):
+            flush.fill_(1.0)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            plan.decode(tree.q, tree.k_pages, tree.v_pages, out=out, lse=lse, workspace=ws,
+                        k_scale=tree.k_scale, v_scale=tree.v_scale, stream=stream)
+            b.record(stream)
+            b.synchronize()
+            times.append(a.elapsed_time(b) * 1e3)
+        plan.check(stream)
+        return float(np.median(times))
+
+    plan = Plan.for_tree(tree, stream=stream)
+    fresh_us = decode_us(plan, tree)
+    host_us, dev_us = [], []
+    for _ in range(steps):
+        tree, new_pages = W.grow_branches(tree, pool)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize(dev)
+        a.record(stream)
+        t0 = time.perf_counter()
+        plan.append(new_pages, stream=stream)
+        host_us.append((time.perf_counter() - t0) * 1e6)
+        b.record(stream)
+        b.synchronize()
+        dev_us.append(a.elapsed_time(b) * 1e3)
+    after_us = decode_us(plan, tree)
+    plan.close()
+    replan_us = []
+    for _ in range(10):
+        torch.cuda.synchronize(dev)
+        t0 = time.perf_counter()
+        p2 = Plan.for_tree(tree, stream=stream)
+        torch.cuda.synchronize(dev)
+        replan_us.append((time.perf_counter() - t0) * 1e6)
+        rebuilt_us = decode_us(p2, tree, n=20) if len(replan_us) == 10 else None
+        p2.close()
+    line = {"metric": "plan update per decode step", "value": float(np.median(host_us)),
+            "unit": "us (host)", "higher_is_better": False, "n_gpus": 1, "steps": steps,
+            "data": "synthetic", "component": "append",
+            "config": {"workload": tree.name, "branches": tree.num_leaves,
+                       "kv_heads": tree.num_kv_heads},
+            "append_device_us": float(np.median(dev_us)),
+            "rebuild_plan_us": float(np.median(replan_us)),
+            "decode_us_fresh_plan": fresh_us, "decode_us_after_appends": after_us,
+            "decode_us_rebuilt_after": rebuilt_us}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -457,13 +531,16 @@ def main(argv=None):
     ap.add_argument("--mode", choices=["bf16", "fp8", "fp32"], default="bf16")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--component", choices=["decode", "trace"], default="decode",
-                    help="decode: the attention step (default); trace: the tag-stream parser")
+    ap.add_argument("--component", choices=["decode", "trace", "append"], default="decode",
+                    help="decode: the attention step (default); trace: the tag-stream "
+                         "parser; append: the decode-loop plan update")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.component == "trace":
         return run_trace(args)
+    if args.component == "append":
+        return run_append(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_gpu(args)

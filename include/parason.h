@@ -53,7 +53,8 @@ typedef enum {
     PARASON_ENOMEM = 2,       /* host or device allocation failed (plan)  */
     PARASON_ECUDA = 3,        /* a CUDA runtime call failed               */
     PARASON_ETIMEOUT = 4,     /* a bounded device wait expired            */
-    PARASON_EUNSUPPORTED = 5  /* valid but not implemented (shape / mode) */
+    PARASON_EUNSUPPORTED = 5, /* valid but not implemented (shape / mode) */
+    PARASON_ENOSPACE = 6      /* the plan has no room for an update: build a new one */
 } parason_status;
 
 typedef enum {
@@ -196,6 +197,35 @@ parason_status parason_attn_decode_no_alloc(parason_plan plan, const void *q,
                                             void *out, float *lse, parason_stream_t stream);
 
 /*
+ * Decode-loop update: one generated token appended to every branch's own
+ * node (leaf_node[b] gains one token), without building a new plan.  The
+ * paper's engine runs every branch for one token per step (Sec. 3.4); this
+ * is the step between two parason_attn_decode calls, O(branches * H_kv).
+ *
+ *   new_pages  host int32 [num_leaves]: for a branch whose node length is a
+ *              multiple of 16 (the new token opens a page), the physical
+ *              page that takes it -- in range and owned by no node; entries
+ *              of the other branches are ignored (pass -1).  May be NULL when
+ *              no branch opens a page.
+ *
+ * The caller writes the new token's K and V into its slot (length % 16 of
+ * the node's last page) before the next decode.  On a plan built with
+ * parason_attn_plan the update is also made to the device copy, with one
+ * host-to-device copy and one small kernel on `stream`.  A plan's appends
+ * and decodes must be issued in order (one stream, or ordered streams).
+ *
+ * Returns PARASON_EINVAL for a missing, out-of-range or already used page;
+ * PARASON_ENOSPACE if some branch's node has no pages yet, or its last work
+ * item has no room left for another page: a plan leaves each branch room for
+ * half as many pages as its last item had (4 to 64 pages), beyond which the
+ * grown item would unbalance the decode; PARASON_EUNSUPPORTED in FP32 mode.  On any error
+ * nothing is changed.  Forking (new branches at an </Outlines>) needs a
+ * new plan.
+ */
+parason_status parason_plan_append(parason_plan plan, const int32_t *new_pages,
+                                   parason_stream_t stream);
+
+/*
  * Combine two attention results over disjoint key sets A and B (for example
  * two KV ranges of one branch, or a branch's context before and after a join)
  * into the result over A u B, row by row:
@@ -241,6 +271,7 @@ typedef struct {
     int32_t num_wide_ctas;      /* of which start on the prefix pass        */
     int32_t num_wide_items;     /* prefix-pass items (tiles x pieces)       */
     int32_t num_narrow_items;   /* suffix-pass items                        */
+    int64_t num_stream_rows;    /* entries of PARASON_TABLE_STREAM_ROWS     */
 } parason_plan_info;
 
 parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info);
@@ -262,6 +293,11 @@ parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info)
  *                            order the kernel's prefix CTAs pull them
  *   PARASON_TABLE_NARROW_QUEUE int32 [num_narrow_items]: suffix-pass items in
  *                            the order the kernel's warps pull them
+ *   PARASON_TABLE_ITEM_ROWS  int32 [num_items + 1]: start of each item's page
+ *                            rows in the stream (an item's rows are the first
+ *                            page-count entries from there)
+ *   PARASON_TABLE_STREAM_ROWS int32 [num_stream_rows]: the TMA row
+ *                            (page * H_kv + kv head) * 16 of every item page
  * Returns PARASON_EINVAL if `bytes` is smaller than the table.
  */
 enum {
@@ -270,7 +306,9 @@ enum {
     PARASON_TABLE_MERGE_PTR = 2,
     PARASON_TABLE_MERGE = 3,
     PARASON_TABLE_WIDE_QUEUE = 4,
-    PARASON_TABLE_NARROW_QUEUE = 5
+    PARASON_TABLE_NARROW_QUEUE = 5,
+    PARASON_TABLE_ITEM_ROWS = 6,
+    PARASON_TABLE_STREAM_ROWS = 7
 };
 parason_status parason_plan_export(parason_plan plan, int32_t table, void *dst, size_t bytes);
 

@@ -11,10 +11,10 @@ import os
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_build", "libparason.so")
 
-OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EUNSUPPORTED = range(6)
+OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EUNSUPPORTED, ENOSPACE = range(7)
 MODES = {"bf16": 0, "fp32": 1, "fp8": 2}
 (TABLE_ITEMS, TABLE_DFS_LEAVES, TABLE_MERGE_PTR, TABLE_MERGE, TABLE_WIDE_QUEUE,
- TABLE_NARROW_QUEUE) = range(6)
+ TABLE_NARROW_QUEUE, TABLE_ITEM_ROWS, TABLE_STREAM_ROWS) = range(8)
 DEBUG_SKIP_FIRST_LOAD = 1
 NO_ALLOC_SCRATCH_BYTES = 64 << 20   # PARASON_NO_ALLOC_SCRATCH_BYTES
 
@@ -39,7 +39,7 @@ class PlanInfo(ctypes.Structure):
                 ("path_tokens", ctypes.c_int64), ("num_sms", ctypes.c_int32),
                 ("on_device", ctypes.c_int32), ("num_ctas", ctypes.c_int32),
                 ("num_wide_ctas", ctypes.c_int32), ("num_wide_items", ctypes.c_int32),
-                ("num_narrow_items", ctypes.c_int32)]
+                ("num_narrow_items", ctypes.c_int32), ("num_stream_rows", ctypes.c_int64)]
 
 
 class TraceStats(ctypes.Structure):
@@ -58,6 +58,7 @@ SIGNATURES = {
     "parason_plan_workspace_bytes": (_sz, [_p]),
     "parason_attn_decode": (ctypes.c_int, [_p, _p, _p, _p, _p, _p, _p, _p, _p, _sz, _p]),
     "parason_attn_decode_no_alloc": (ctypes.c_int, [_p, _p, _p, _p, _p, _p, _p, _p, _p]),
+    "parason_plan_append": (ctypes.c_int, [_p, _p, _p]),
     "parason_trace_analyze": (ctypes.c_int, [_p, _i64, ctypes.POINTER(TraceStats),
                                              ctypes.POINTER(ctypes.c_int64)]),
     "parason_trace_fork_tree": (ctypes.c_int, [_p, _i64, _i32, _i32, _p, _p, _p,

@@ -74,6 +74,7 @@ class Plan:
         check(st, "parason_attn_plan")
         self._h = out
         self._ws = None
+        self.host_only = host_only
 
     @classmethod
     def for_tree(cls, tree, **kw) -> "Plan":
@@ -126,7 +127,9 @@ class Plan:
                  _lib.TABLE_MERGE_PTR: (inf["num_leaves"] * self.num_kv_heads + 1,),
                  _lib.TABLE_MERGE: (inf["num_merge_entries"],),
                  _lib.TABLE_WIDE_QUEUE: (inf["num_wide_items"],),
-                 _lib.TABLE_NARROW_QUEUE: (inf["num_narrow_items"],)}[table]
+                 _lib.TABLE_NARROW_QUEUE: (inf["num_narrow_items"],),
+                 _lib.TABLE_ITEM_ROWS: (inf["num_items"] + 1,),
+                 _lib.TABLE_STREAM_ROWS: (inf["num_stream_rows"],)}[table]
         buf = np.zeros(shape, dtype=np.int32)
         check(_lib.load().parason_plan_export(self.handle, table, _ptr(buf), buf.nbytes),
               "plan_export")
@@ -208,6 +211,18 @@ class Plan:
             _ptr(out), _ptr(lse), _stream_handle(stream))
         check(st, "parason_attn_decode_no_alloc")
         return out, lse
+
+    def append(self, new_pages=None, stream=None) -> None:
+        """One token appended to every branch's node (parason_plan_append).
+        ``new_pages``: int32 [num_leaves], the page for each branch whose
+        token opens one (-1 elsewhere), or None when no branch opens a page."""
+        a = None
+        if new_pages is not None:
+            a = np.ascontiguousarray(np.asarray(new_pages, dtype=np.int32))
+            if a.shape != (self.num_leaves,):
+                raise ValueError(f"new_pages must have shape ({self.num_leaves},)")
+        sh = None if self.host_only else _stream_handle(stream)
+        check(_lib.load().parason_plan_append(self.handle, _ptr(a), sh), "parason_plan_append")
 
     def decode_tree(self, tree, **kw):
         """``decode`` with the tensors of a ``workloads.ForkTree``."""

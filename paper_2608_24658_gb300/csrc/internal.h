@@ -115,6 +115,9 @@ cudaError_t launch_attn_fp32(const AttnArgs &a, const float *k_pages, const floa
                              int head_dim, cudaStream_t stream);
 cudaError_t launch_merge(const MergeArgs &a, int head_dim, int mode, bool programmatic,
                          cudaStream_t stream);
+// base[patches[i].x] = patches[i].y for i < n (plan updates)
+cudaError_t launch_scatter(int32_t *base, const int2 *patches, int32_t n, cudaStream_t stream);
+
 cudaError_t launch_lse_merge(const void *o_a, const float *lse_a, const void *o_b,
                              const float *lse_b, void *o_out, float *lse_out, int64_t rows,
                              int head_dim, int mode, cudaStream_t stream);

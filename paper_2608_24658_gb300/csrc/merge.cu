@@ -301,4 +301,17 @@ cudaError_t launch_lse_merge(const void *o_a, const float *lse_a, const void *o_
     return cudaGetLastError();
 }
 
+namespace {
+__global__ void scatter_kernel(int32_t *base, const int2 *patches, int32_t n) {
+    const int32_t i = static_cast<int32_t>(blockIdx.x * blockDim.x + threadIdx.x);
+    if (i < n) base[patches[i].x] = patches[i].y;
+}
+}  // namespace
+
+cudaError_t launch_scatter(int32_t *base, const int2 *patches, int32_t n, cudaStream_t stream) {
+    if (n <= 0) return cudaSuccess;
+    scatter_kernel<<<(n + 255) / 256, 256, 0, stream>>>(base, patches, n);
+    return cudaGetLastError();
+}
+
 }  // namespace parason

@@ -37,6 +37,10 @@ constexpr int kMaxPiecePages = 128;     // and at most this long
 constexpr int kWideBlockPages = 4;      // prefix pieces are whole 64-token blocks
 constexpr double kWideProvision = 1.15; // prefix CTAs relative to the cost model
 constexpr int kFp32ChunkPages = 32;
+// stream rows kept free after a branch's last item: half its pages, 4 to 64
+// (an item that grows further makes the launch's tail: build a new plan)
+constexpr int32_t kAppendSlackMin = 4, kAppendSlackMax = 64;
+constexpr int kPatchesPerTail = 6;      // words one append may change per tail item
 constexpr double kWideGroupPageCost = 1.0;   // one 16-row group of one page, in suffix pages
 constexpr double kTcPageCost = 2.4;          // one page of a tcgen05 prefix tile (tuned)
 constexpr int64_t kDefaultWaitNs = 2000000000LL;
@@ -86,6 +90,12 @@ struct parason_plan_s {
     std::vector<int32_t> item_rows;    // per item: start of its page rows
     std::vector<int32_t> stream_rows;  // TMA row of every page, item by item
     std::vector<int32_t> item_rec;     // kRecWords per item (suffix-warp record)
+
+    // decode-loop appends (parason_plan_append): each branch's own node
+    std::vector<int32_t> leaf_len;     // tokens in branch b's node
+    std::vector<int32_t> tail_ptr;     // CSR over branches into tail_items
+    std::vector<int32_t> tail_items;   // items that end at the node's last page
+    std::vector<uint8_t> page_used;    // physical pages some node owns
     int32_t num_ctas = 0;
     int32_t num_wide_ctas = 0;
     int64_t num_slots = 0;
@@ -102,6 +112,10 @@ struct parason_plan_s {
     int32_t *d_merge_ptr = nullptr;
     int32_t *d_merge_ent = nullptr;
     int32_t *d_item_rec = nullptr;
+    int2 *d_patch = nullptr;           // (word offset in the blob, value), tail_items * 6
+    std::vector<int2> patches;         // host side of the last append's patch list
+    size_t blob_words = 0;
+    size_t w_items = 0, w_rec = 0, w_strows = 0;   // word offsets of those arrays in the blob
     int32_t *d_item_rows = nullptr;
     int32_t *d_stream_rows = nullptr;
     int32_t *d_queue_next = nullptr;   // 2 counters, set back to queue_start by the merge kernel
@@ -305,6 +319,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     p->items.clear();
     int64_t slots = 0;
     std::vector<std::pair<int64_t, int32_t>> wide_q, narrow_q;   // (pages, item)
+    std::vector<std::pair<int32_t, int32_t>> tails;              // (branch, item)
     auto emit = [&](const Run &run, int64_t pg0, int64_t np) -> bool {
         WorkItem it;
         const int64_t P = run.pages;
@@ -323,6 +338,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         const int32_t id = static_cast<int32_t>(p->items.size());
         p->items.push_back(it);
         (run.wide ? wide_q : narrow_q).emplace_back(np, id);
+        if (pg0 + np == P && leaf_of_node[run.node] >= 0) tails.emplace_back(leaf_of_node[run.node], id);
         return true;
     };
     auto cut = [&](const Run &r, int64_t chunk, int64_t align) -> bool {
@@ -389,17 +405,42 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         // item ids in pull order: the prefix queue is items [0, W), the
         // suffix queue items [W, W + N), so a pull needs no queue lookup
         std::vector<WorkItem> sorted;
+        std::vector<int32_t> new_id(p->items.size(), -1);
         sorted.reserve(p->items.size());
-        for (int32_t id : p->wide_queue) sorted.push_back(p->items[id]);
-        for (int32_t id : p->narrow_queue) sorted.push_back(p->items[id]);
+        for (int32_t id : p->wide_queue) {
+            new_id[id] = static_cast<int32_t>(sorted.size());
+            sorted.push_back(p->items[id]);
+        }
+        for (int32_t id : p->narrow_queue) {
+            new_id[id] = static_cast<int32_t>(sorted.size());
+            sorted.push_back(p->items[id]);
+        }
         p->items.swap(sorted);
+        for (auto &t : tails) t.second = new_id[t.second];
         for (size_t k = 0; k < p->wide_queue.size(); ++k) p->wide_queue[k] = static_cast<int32_t>(k);
         for (size_t k = 0; k < p->narrow_queue.size(); ++k)
             p->narrow_queue[k] = static_cast<int32_t>(p->wide_queue.size() + k);
     }
 
+    // the items that end at each branch node's last page (appends grow them)
+    std::sort(tails.begin(), tails.end());
+    p->tail_ptr.assign(static_cast<size_t>(num_leaves) + 1, 0);
+    p->tail_items.clear();
+    std::vector<uint8_t> is_tail(p->items.size(), 0);
+    for (const auto &t : tails) {
+        p->tail_ptr[t.first + 1]++;
+        p->tail_items.push_back(t.second);
+        is_tail[t.second] = 1;
+    }
+    for (int32_t b = 0; b < num_leaves; ++b) p->tail_ptr[b + 1] += p->tail_ptr[b];
+    p->leaf_len.assign(static_cast<size_t>(num_leaves), 0);
+    for (int32_t b = 0; b < num_leaves; ++b) p->leaf_len[b] = node_len[leaf_node[b]];
+    p->page_used.assign(static_cast<size_t>(num_phys), 0);
+    for (int64_t i = 0; i < total_pages; ++i) p->page_used[page_ids[i]] = 1;
+
     // page streams: the TMA row (page * H_kv + kv head) * 16 of every page of
-    // every item, item by item
+    // every item, item by item; a tail item is followed by kAppendSlack free
+    // rows for the pages appends will add
     p->item_rows.assign(p->items.size() + 1, 0);
     p->stream_rows.clear();
     for (size_t i = 0; i < p->items.size(); ++i) {
@@ -407,6 +448,10 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         for (int32_t pg = 0; pg < it.num_pages; ++pg)
             p->stream_rows.push_back((page_ids[it.page_pos + pg] * H_kv + it.kv_head) *
                                      parason::kPageSize);
+        if (mode != PARASON_FP32 && is_tail[i])
+            p->stream_rows.insert(p->stream_rows.end(),
+                                  std::min(kAppendSlackMax, std::max(kAppendSlackMin, it.num_pages / 2)),
+                                  0);
         if (p->stream_rows.size() > static_cast<size_t>(INT32_MAX)) return PARASON_EUNSUPPORTED;
         p->item_rows[i + 1] = static_cast<int32_t>(p->stream_rows.size());
     }
@@ -462,11 +507,13 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     const size_t n_strows = (p->stream_rows.size() + 32) * sizeof(int32_t);
     const size_t n_qnext = 2 * sizeof(int32_t);
     const size_t n_err = parason::kErrWords * sizeof(int32_t);
-    constexpr int kArrays = 10;
+    const size_t n_patch = p->tail_items.size() * kPatchesPerTail * sizeof(int2);
+    constexpr int kArrays = 11;
     size_t off[kArrays], total = 0;
-    // the last two (queue counters, error record) are zero-filled, not copied
-    const size_t sizes[kArrays] = {n_items, n_pages,  n_dfs,   n_mptr,  n_ment,
-                                   n_rec,   n_irows,  n_strows, n_qnext, n_err};
+    // the queue counters and the error record are set separately; the patch
+    // buffer is written by parason_plan_append
+    const size_t sizes[kArrays] = {n_items, n_pages,  n_dfs,    n_mptr,  n_ment, n_rec,
+                                   n_irows, n_strows, n_qnext, n_err,   n_patch};
     for (int i = 0; i < kArrays; ++i) {
         off[i] = total;
         total = align_up(total + std::max<size_t>(sizes[i], 4), kAlign);
@@ -487,6 +534,11 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     p->d_stream_rows = reinterpret_cast<int32_t *>(base + off[7]);
     p->d_queue_next = reinterpret_cast<int32_t *>(base + off[8]);
     p->d_err = reinterpret_cast<int32_t *>(base + off[9]);
+    p->d_patch = reinterpret_cast<int2 *>(base + off[10]);
+    p->w_items = off[0] / sizeof(int32_t);
+    p->w_rec = off[5] / sizeof(int32_t);
+    p->w_strows = off[7] / sizeof(int32_t);
+    p->blob_words = total / sizeof(int32_t);
     const void *src[8] = {p->items.data(),     p->page_ids.data(),  p->dfs_leaf.data(),
                           p->merge_ptr.data(), p->merge_ent.data(), p->item_rec.data(),
                           p->item_rows.data(), p->stream_rows.data()};
@@ -811,6 +863,7 @@ const char *parason_status_string(parason_status s) {
     case PARASON_ECUDA: return "CUDA error";
     case PARASON_ETIMEOUT: return "device wait timed out";
     case PARASON_EUNSUPPORTED: return "unsupported";
+    case PARASON_ENOSPACE: return "no room in the plan: build a new one";
     }
     return "unknown status";
 }
@@ -830,6 +883,96 @@ parason_status parason_plan_get_info(parason_plan p, parason_plan_info *info) {
     info->num_wide_ctas = p->num_wide_ctas;
     info->num_wide_items = static_cast<int32_t>(p->wide_queue.size());
     info->num_narrow_items = static_cast<int32_t>(p->narrow_queue.size());
+    info->num_stream_rows = static_cast<int64_t>(p->stream_rows.size());
+    return PARASON_OK;
+}
+
+parason_status parason_plan_append(parason_plan p, const int32_t *new_pages,
+                                   parason_stream_t stream_) {
+    if (!p) return PARASON_EINVAL;
+    if (p->cfg.mode == PARASON_FP32) return PARASON_EUNSUPPORTED;
+    const int32_t L = p->num_leaves;
+    if (L == 0) return PARASON_OK;
+    if (p->on_device && p->blob_words > static_cast<size_t>(INT32_MAX)) return PARASON_EUNSUPPORTED;
+    const int32_t H_kv = p->cfg.num_kv_heads;
+    constexpr int32_t P16 = parason::kPageSize;
+
+    // check everything first: on any error nothing changes
+    std::vector<int32_t> claimed;
+    auto refuse = [&](parason_status st) {
+        for (int32_t pg : claimed) p->page_used[pg] = 0;
+        return st;
+    };
+    for (int32_t b = 0; b < L; ++b) {
+        if (p->tail_ptr[b] == p->tail_ptr[b + 1]) return refuse(PARASON_ENOSPACE);
+        if (p->leaf_len[b] == INT32_MAX) return refuse(PARASON_EUNSUPPORTED);
+        if (p->leaf_len[b] % P16 != 0) continue;
+        if (!new_pages) return refuse(PARASON_EINVAL);
+        const int32_t pg = new_pages[b];
+        if (pg < 0 || pg >= p->num_phys || p->page_used[pg]) return refuse(PARASON_EINVAL);
+        for (int32_t k = p->tail_ptr[b]; k < p->tail_ptr[b + 1]; ++k) {
+            const int32_t t = p->tail_items[k];
+            if (p->item_rows[t] + p->items[t].num_pages + 1 > p->item_rows[t + 1])
+                return refuse(PARASON_ENOSPACE);
+            if (p->items[t].num_pages == INT32_MAX) return refuse(PARASON_EUNSUPPORTED);
+            // a prefix-pass item stays within the prefix pass's page limit
+            if (t < static_cast<int32_t>(p->wide_queue.size()) &&
+                p->items[t].num_pages + 1 > kMaxPiecePages)
+                return refuse(PARASON_ENOSPACE);
+        }
+        p->page_used[pg] = 1;
+        claimed.push_back(pg);
+    }
+
+    // apply, host copy and patch list: (word offset in the device blob, value)
+    std::vector<int2> &patches = p->patches;
+    patches.clear();
+    for (int32_t b = 0; b < L; ++b) {
+        const bool opens_page = p->leaf_len[b] % P16 == 0;
+        for (int32_t k = p->tail_ptr[b]; k < p->tail_ptr[b + 1]; ++k) {
+            const int32_t t = p->tail_items[k];
+            WorkItem &it = p->items[t];
+            int32_t *rec = p->item_rec.data() + static_cast<size_t>(t) * parason::kRecWords;
+            const size_t w_item = p->w_items + static_cast<size_t>(t) * (sizeof(WorkItem) / 4);
+            const size_t w_rec = p->w_rec + static_cast<size_t>(t) * parason::kRecWords;
+            if (opens_page) {
+                const int32_t j = it.num_pages;                   // the new page's index
+                const int32_t row = (new_pages[b] * H_kv + it.kv_head) * P16;
+                it.num_pages += 1;
+                it.last_valid = 1;
+                p->stream_rows[p->item_rows[t] + j] = row;
+                patches.push_back(make_int2(static_cast<int32_t>(p->w_strows + p->item_rows[t] + j), row));
+                if (j < parason::kRecRows) {
+                    rec[parason::kRecRow0 + j] = row;
+                    patches.push_back(make_int2(static_cast<int32_t>(w_rec + parason::kRecRow0 + j), row));
+                }
+                rec[1] = it.num_pages;
+                patches.push_back(make_int2(static_cast<int32_t>(w_rec + 1), it.num_pages));
+                patches.push_back(make_int2(static_cast<int32_t>(w_item + 1), it.num_pages));
+            } else {
+                it.last_valid += 1;
+            }
+            rec[2] = it.last_valid;
+            patches.push_back(make_int2(static_cast<int32_t>(w_rec + 2), it.last_valid));
+            patches.push_back(make_int2(static_cast<int32_t>(w_item + 2), it.last_valid));
+        }
+        p->leaf_len[b] += 1;
+    }
+    p->unique_tokens += L;
+    p->path_tokens += L;
+    if (!p->on_device || patches.empty()) return PARASON_OK;
+
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev != p->device) return PARASON_ECUDA;
+    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+    // a pageable source is staged before the call returns, so the host list
+    // may be reused by the next append
+    if (cudaMemcpyAsync(p->d_patch, patches.data(), patches.size() * sizeof(int2),
+                        cudaMemcpyHostToDevice, stream) != cudaSuccess)
+        return PARASON_ECUDA;
+    if (parason::launch_scatter(static_cast<int32_t *>(p->d_blob), p->d_patch,
+                                static_cast<int32_t>(patches.size()), stream) != cudaSuccess)
+        return PARASON_ECUDA;
     return PARASON_OK;
 }
 
@@ -844,6 +987,8 @@ parason_status parason_plan_export(parason_plan p, int32_t table, void *dst, siz
     case PARASON_TABLE_MERGE: src = p->merge_ent.data(); n = p->merge_ent.size() * 4; break;
     case PARASON_TABLE_WIDE_QUEUE: src = p->wide_queue.data(); n = p->wide_queue.size() * 4; break;
     case PARASON_TABLE_NARROW_QUEUE: src = p->narrow_queue.data(); n = p->narrow_queue.size() * 4; break;
+    case PARASON_TABLE_ITEM_ROWS: src = p->item_rows.data(); n = p->item_rows.size() * 4; break;
+    case PARASON_TABLE_STREAM_ROWS: src = p->stream_rows.data(); n = p->stream_rows.size() * 4; break;
     default: return PARASON_EINVAL;
     }
     if (bytes < n || (n > 0 && !dst)) return PARASON_EINVAL;

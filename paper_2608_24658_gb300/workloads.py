@@ -471,3 +471,31 @@ def paper_scale_trace(seed: int) -> np.ndarray:
     return random_trace(seed, max_depth=1, p_parallel=0.4, text_len=(250, 1200),
                         entry_len=(10, 60), entries=(2, 3), body_items=(5, 10), p_mismatch=0.0,
                         p_empty_thread=0.0)
+
+
+def free_pages(tree: ForkTree) -> list:
+    """Physical pages no node owns, in index order."""
+    used = set(int(x) for x in tree.page_ids)
+    return [p for p in range(tree.num_physical_pages) if p not in used]
+
+
+def grow_branches(tree: ForkTree, pool: list):
+    """The tree after one generated token per branch: every branch node gains
+    one token; a branch whose node length is a multiple of 16 takes the next
+    page of `pool` (consumed in place).  Returns (tree, new_pages) with
+    new_pages[b] the page branch b took, or -1.  The token's K and V are the
+    values already in that slot of the pool."""
+    node_len = tree.node_len.copy()
+    pages = [list(tree.page_ids[tree.node_page_ptr[n]:tree.node_page_ptr[n + 1]])
+             for n in range(tree.num_nodes)]
+    new_pages = np.full(tree.num_leaves, -1, dtype=np.int32)
+    for b, n in enumerate(tree.leaf_node):
+        if node_len[n] % PAGE_SIZE == 0:
+            pg = pool.pop(0)
+            new_pages[b] = pg
+            pages[n].append(pg)
+        node_len[n] += 1
+    ptr = np.zeros(tree.num_nodes + 1, dtype=np.int32)
+    ptr[1:] = np.cumsum([len(p) for p in pages])
+    ids = np.asarray([x for p in pages for x in p], dtype=np.int32)
+    return replace(tree, node_len=node_len, node_page_ptr=ptr, page_ids=ids), new_pages
