@@ -54,6 +54,11 @@ class Oracle:
             i32, i32, i32, i32, i32, ctypes.c_double,
             i32, p, p, p, p, i32, p, p, p, p, p, p,
             i32, p, p, p, i32]
+        lib.parason_oracle_prefill.restype = ctypes.c_int
+        lib.parason_oracle_prefill.argtypes = [
+            i32, i32, i32, i32, i32, ctypes.c_double,
+            i32, p, p, p, p, i32, p, p, p, p, p, p,
+            i32, p, p, p, i32]
         lib.parason_oracle_lse_merge.restype = None
         lib.parason_oracle_lse_merge.argtypes = [p, p, p, p, p, p, ctypes.c_int64, i32]
         lib.parason_oracle_bf16_to_double.restype = ctypes.c_double
@@ -94,6 +99,31 @@ class Oracle:
             int(threads))
         if st != 0:
             raise ValueError(f"oracle decode failed with status {st}")
+        return out, lse
+
+    def prefill(self, *, num_q_heads, num_kv_heads, head_dim, mode, parent, node_len,
+                node_page_ptr, page_ids, chunk_node, q, k_pages, v_pages, k_scale=None,
+                v_scale=None, sm_scale=0.0, page_size=16, sel=None, threads=0, **_):
+        """Tree-masked prefill: (out [S, H_q, d], lse [S, H_q]) fp64 for queries ``sel``
+        (every token of every chunk node, chunk by chunk; all if None)."""
+        parent, node_len = _i32(parent), _i32(node_len)
+        node_page_ptr, page_ids, chunk_node = _i32(node_page_ptr), _i32(page_ids), _i32(chunk_node)
+        q, k_pages, v_pages = _cpu(q), _cpu(k_pages), _cpu(v_pages)
+        k_scale = None if k_scale is None else _cpu(k_scale).float().contiguous()
+        v_scale = None if v_scale is None else _cpu(v_scale).float().contiguous()
+        total = int(sum(int(node_len[c]) for c in chunk_node))
+        sel_arr = None if sel is None else _i32(sel)
+        n_sel = total if sel is None else len(sel_arr)
+        out = np.zeros((n_sel, num_q_heads, head_dim), dtype=np.float64)
+        lse = np.zeros((n_sel, num_q_heads), dtype=np.float64)
+        st = self.lib.parason_oracle_prefill(
+            num_q_heads, num_kv_heads, head_dim, page_size, MODES[mode], float(sm_scale),
+            len(parent), _ptr(parent), _ptr(node_len), _ptr(node_page_ptr), _ptr(page_ids),
+            len(chunk_node), _ptr(chunk_node), _ptr(q), _ptr(k_pages), _ptr(v_pages),
+            _ptr(k_scale), _ptr(v_scale), n_sel, _ptr(sel_arr), _ptr(out), _ptr(lse),
+            int(threads))
+        if st != 0:
+            raise ValueError(f"oracle prefill failed with status {st}")
         return out, lse
 
     def lse_merge(self, o_a, lse_a, o_b, lse_b):
@@ -137,6 +167,10 @@ def decode(**kw):
 
 def lse_merge(o_a, lse_a, o_b, lse_b):
     return default().lse_merge(o_a, lse_a, o_b, lse_b)
+
+
+def prefill(**kw):
+    return default().prefill(**kw)
 
 
 def bf16_to_double(bits: int) -> float:

@@ -254,6 +254,168 @@ int parason_oracle_decode(int32_t num_q_heads, int32_t num_kv_heads, int32_t hea
 }
 
 /*
+ * Tree-masked prefill (the join of a parallel block: the threads' text
+ * becomes context of the main trajectory, Fig. 1, Sec. 3.1; each new token
+ * attends causally).  Every token of every chunk node is a query:
+ * queries are numbered chunk by chunk (query k = token t of chunk c, with k =
+ * qbase_c + t), and query k attends to every token of every ancestor of
+ * chunk_node[c] (root first) and to tokens 0 .. t of chunk_node[c] itself.
+ *
+ * q [num_queries, H_q, d]; sel query indices to evaluate (NULL: all);
+ * out [num_sel, H_q, d] fp64; lse [num_sel, H_q] fp64 (natural log).
+ */
+int parason_oracle_prefill(int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                           int32_t page_size, int32_t mode, double sm_scale,
+                           int32_t num_nodes, const int32_t *parent,
+                           const int32_t *node_len, const int32_t *node_page_ptr,
+                           const int32_t *page_ids, int32_t num_chunks,
+                           const int32_t *chunk_node, const void *q,
+                           const void *k_pages, const void *v_pages,
+                           const float *k_scale, const float *v_scale,
+                           int32_t num_sel, const int32_t *sel, double *out,
+                           double *lse, int32_t num_threads)
+{
+    if (num_q_heads <= 0 || num_kv_heads <= 0 || num_q_heads % num_kv_heads != 0 ||
+        head_dim <= 0 || page_size <= 0 || num_nodes < 0 || num_chunks < 0)
+        return ORACLE_EINVAL;
+    if (mode != ORACLE_BF16 && mode != ORACLE_FP32 && mode != ORACLE_FP8_E4M3_KV)
+        return ORACLE_EINVAL;
+    if (mode == ORACLE_FP8_E4M3_KV && (!k_scale || !v_scale))
+        return ORACLE_EINVAL;
+    int64_t num_queries = 0;
+    for (int32_t c = 0; c < num_chunks; ++c) {
+        if (chunk_node[c] < 0 || chunk_node[c] >= num_nodes)
+            return ORACLE_EINVAL;
+        num_queries += node_len[chunk_node[c]];
+    }
+    if (!sel)
+        num_sel = (int32_t)num_queries;
+
+    const int group = num_q_heads / num_kv_heads;
+    const double scale = sm_scale > 0.0 ? sm_scale : 1.0 / sqrt((double)head_dim);
+    const int q_code = (mode == ORACLE_FP32) ? ORACLE_FP32 : ORACLE_BF16;
+    const int kv_code = mode;
+    int status = ORACLE_OK;
+
+#ifdef _OPENMP
+    if (num_threads > 0)
+        omp_set_num_threads(num_threads);
+#else
+    (void)num_threads;
+#endif
+
+#pragma omp parallel
+    {
+        int32_t *path = (int32_t *)malloc(sizeof(int32_t) * (size_t)(num_nodes > 0 ? num_nodes : 1));
+        double *qv = (double *)malloc(sizeof(double) * (size_t)head_dim);
+        double *acc = (double *)malloc(sizeof(double) * (size_t)head_dim);
+        double *scores = NULL;
+        int64_t scores_cap = 0;
+        if (!path || !qv || !acc) {
+#pragma omp atomic write
+            status = ORACLE_ENOMEM;
+        }
+
+#pragma omp for schedule(dynamic, 1)
+        for (int64_t task = 0; task < (int64_t)num_sel * num_q_heads; ++task) {
+            if (status != ORACLE_OK)
+                continue;
+            const int32_t si = (int32_t)(task / num_q_heads);
+            const int32_t h = (int32_t)(task % num_q_heads);
+            const int64_t k = sel ? sel[si] : si;
+            const int32_t kvh = h / group;
+            double *o = out + ((int64_t)si * num_q_heads + h) * head_dim;
+            double *lse_out = lse ? lse + (int64_t)si * num_q_heads + h : NULL;
+            if (k < 0 || k >= num_queries) {
+#pragma omp atomic write
+                status = ORACLE_EINVAL;
+                continue;
+            }
+            /* the query's chunk and token */
+            int32_t c = 0;
+            int64_t base = 0;
+            while (base + node_len[chunk_node[c]] <= k) {
+                base += node_len[chunk_node[c]];
+                ++c;
+            }
+            const int32_t own = chunk_node[c];
+            const int32_t t_q = (int32_t)(k - base);
+            const int plen = path_to_root(own, parent, num_nodes, path);
+            if (plen < 0) {
+#pragma omp atomic write
+                status = ORACLE_EINVAL;
+                continue;
+            }
+            /* visible tokens: all of every ancestor, tokens 0 .. t_q of own */
+            int64_t total = 0;
+            for (int i = 0; i < plen; ++i)
+                total += (path[i] == own) ? t_q + 1 : node_len[path[i]];
+
+            const double ks = (mode == ORACLE_FP8_E4M3_KV) ? (double)k_scale[kvh] : 1.0;
+            const double vs = (mode == ORACLE_FP8_E4M3_KV) ? (double)v_scale[kvh] : 1.0;
+            for (int dd = 0; dd < head_dim; ++dd)
+                qv[dd] = load_elem(q, (k * num_q_heads + h) * head_dim + dd, q_code, 1.0);
+            if (total > scores_cap) {
+                free(scores);
+                scores = (double *)malloc(sizeof(double) * (size_t)total);
+                scores_cap = scores ? total : 0;
+                if (!scores) {
+#pragma omp atomic write
+                    status = ORACLE_ENOMEM;
+                    continue;
+                }
+            }
+
+            /* pass 1: scores over the visible tokens, root first */
+            int64_t pos = 0;
+            double m = -INFINITY;
+            for (int i = 0; i < plen; ++i) {
+                const int32_t n = path[i];
+                const int32_t vis = (n == own) ? t_q + 1 : node_len[n];
+                for (int32_t t = 0; t < vis; ++t) {
+                    const int64_t page = page_ids[node_page_ptr[n] + t / page_size];
+                    const int64_t row = ((page * num_kv_heads + kvh) * page_size + t % page_size) * head_dim;
+                    double dot = 0.0;
+                    for (int dd = 0; dd < head_dim; ++dd)
+                        dot += qv[dd] * load_elem(k_pages, row + dd, kv_code, ks);
+                    const double s = scale * dot;
+                    scores[pos++] = s;
+                    if (s > m)
+                        m = s;
+                }
+            }
+
+            /* pass 2: l = sum exp(s - m), o = sum exp(s - m) v / l */
+            double l = 0.0;
+            for (int dd = 0; dd < head_dim; ++dd)
+                acc[dd] = 0.0;
+            pos = 0;
+            for (int i = 0; i < plen; ++i) {
+                const int32_t n = path[i];
+                const int32_t vis = (n == own) ? t_q + 1 : node_len[n];
+                for (int32_t t = 0; t < vis; ++t) {
+                    const int64_t page = page_ids[node_page_ptr[n] + t / page_size];
+                    const int64_t row = ((page * num_kv_heads + kvh) * page_size + t % page_size) * head_dim;
+                    const double p = exp(scores[pos++] - m);
+                    l += p;
+                    for (int dd = 0; dd < head_dim; ++dd)
+                        acc[dd] += p * load_elem(v_pages, row + dd, kv_code, vs);
+                }
+            }
+            for (int dd = 0; dd < head_dim; ++dd)
+                o[dd] = acc[dd] / l;
+            if (lse_out)
+                *lse_out = m + log(l);
+        }
+        free(scores);
+        free(acc);
+        free(qv);
+        free(path);
+    }
+    return status;
+}
+
+/*
  * Merge of two attention results over disjoint key sets A and B, each given
  * as its normalised output o and its log-sum-exp lse (natural log):
  *   w_A = exp(lse_A), w_B = exp(lse_B)

@@ -499,3 +499,23 @@ def grow_branches(tree: ForkTree, pool: list):
     ptr[1:] = np.cumsum([len(p) for p in pages])
     ids = np.asarray([x for p in pages for x in p], dtype=np.int32)
     return replace(tree, node_len=node_len, node_page_ptr=ptr, page_ids=ids), new_pages
+
+
+def build_prefill(name: str, parent, node_len, chunk_node, *, num_q_heads: int,
+                  num_kv_heads: int, head_dim: int, mode: str = "bf16", seed: int = 0,
+                  device="cpu", q_std: float = 1.0, **kw) -> ForkTree:
+    """A tree-masked prefill workload: the tree and KV of build_tree, with
+    every token of each chunk node (childless) a query.  leaf_node holds the
+    chunk nodes; q is [sum of chunk lengths, H_q, d], chunk by chunk."""
+    tree = build_tree(name, parent, node_len, chunk_node, num_q_heads=num_q_heads,
+                      num_kv_heads=num_kv_heads, head_dim=head_dim, mode=mode, seed=seed,
+                      device=device, q_std=q_std, **kw)
+    nq = int(sum(int(tree.node_len[c]) for c in tree.leaf_node))
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed + 7919)
+    q = torch.randn((nq, num_q_heads, head_dim), generator=gen, device=device,
+                    dtype=torch.float32) * q_std
+    q = q.to(torch.float32 if mode == "fp32" else torch.bfloat16)
+    meta = dict(tree.meta)
+    meta["prefill"] = True
+    return replace(tree, q=q, meta=meta)
