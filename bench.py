@@ -521,6 +521,100 @@ def run_append(args):
     return 0
 
 
+def run_prefill(args):
+    """Tree-masked prefill (parason_prefill_plan + parason_attn_decode): the
+    thread openings at </Outlines> and the join with the threads' KV reused,
+    on the Llama-3-8B attention shape.  Query tokens/s; the roofline is the
+    bf16 tensor peak over the attention FLOPs (4 d per visible key per q
+    head: Q K^T and P V); the oracle on sampled queries beside it."""
+    import torch
+    from paper_2608_24658_gb300 import build as lib_build
+    from paper_2608_24658_gb300.api import Plan
+    lib_build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+        peaks = json.load(f)
+    peak_tf, peak_kind = float(peaks["bf16_tflops"]), "measured (cuBLAS bf16 burst)"
+    kinds = [args.prefill] if args.prefill != "both" else sorted(W.PREFILL_CONFIGS)
+    for kind in kinds:
+        tree = W.PREFILL_CONFIGS[kind](device=dev)
+        plan = Plan.for_prefill(tree, stream=stream)
+        info = plan.info()
+        Q = info["num_leaves"]
+        flops = info["path_tokens"] * tree.num_q_heads * 4 * tree.head_dim
+        out = torch.empty_like(tree.q)
+        lse = torch.empty(Q, tree.num_q_heads, dtype=torch.float32, device=dev)
+        ws = plan.workspace(dev)
+
+        def step():
+            plan.decode(tree.q, tree.k_pages, tree.v_pages, out=out, lse=lse, workspace=ws,
+                        stream=stream)
+
+        for _ in range(args.warmup):
+            flush.fill_(1.0)
+            step()
+        plan.check(stream)
+        K = min(args.steps, 200)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(K)]
+        sampler = ClockSampler(0)
+        sampler.start()
+        time.sleep(0.3)
+        torch.cuda.synchronize(dev)
+        for i in range(K):
+            flush.fill_(float(i))
+            ev[i][0].record(stream)
+            step()
+            ev[i][1].record(stream)
+        torch.cuda.synchronize(dev)
+        clocks = sampler.stop()
+        plan.check(stream)
+        ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
+        plan.enable_timing(K)
+        for i in range(K):
+            flush.fill_(float(i))
+            step()
+        torch.cuda.synchronize(dev)
+        attn_ms, merge_ms = plan.read_timing(K)
+        plan.enable_timing(0)
+        attn_avg = float(np.mean(attn_ms))
+        achieved = flops / (attn_avg * 1e-3) / 1e12
+        cpu = None
+        if not args.no_cpu_baseline:
+            import oracle
+            host = tree.to("cpu")
+            kw = oracle.tree_kwargs(host)
+            kw["chunk_node"] = kw.pop("leaf_node")
+            done, t0 = 0, time.perf_counter()
+            while time.perf_counter() - t0 < args.cpu_seconds:
+                oracle.prefill(sel=[(done * 7919) % Q], **kw)
+                done += 1
+            el = time.perf_counter() - t0
+            cpu = {"value": done / el, "unit": "query tokens/s", "cores": oracle.num_threads(),
+                   "kind": "oracle", "sample": f"{done} of {Q} queries (all q heads), {el:.1f} s"}
+        line = {"metric": "tree-masked prefill throughput", "value": Q / (ms * 1e-3),
+                "unit": "query tokens/s", "n_gpus": 1, "steps": K, "warmup": args.warmup,
+                "ms_per_step": ms, "higher_is_better": True, "dtype": "bf16",
+                "data": "synthetic", "component": "prefill",
+                "config": {"workload": tree.name, "queries": Q, "kv_tokens": int(tree.node_len.sum()),
+                           "visible_keys": info["path_tokens"], "l2": "flushed between steps"},
+                "gpu_launches": K * plan.launches_per_decode(),
+                "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak_tf,
+                             "unit": "TFLOP/s", "frac": achieved / peak_tf, "traffic": None,
+                             "kernel": "attn_bf16_kernel", "peak_kind": peak_kind,
+                             "algorithmic_flops_per_launch": flops, "kernel_ms": attn_avg,
+                             "merge_ms": float(np.mean(merge_ms))},
+                "plan": {k: info[k] for k in ("num_items", "num_ctas", "num_slots",
+                                              "num_merge_entries")},
+                "cpu_baseline": cpu, "clocks": clocks}
+        print(json.dumps(line), flush=True)
+        plan.close()
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -531,9 +625,13 @@ def main(argv=None):
     ap.add_argument("--mode", choices=["bf16", "fp8", "fp32"], default="bf16")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--component", choices=["decode", "trace", "append"], default="decode",
+    ap.add_argument("--component", choices=["decode", "trace", "append", "prefill"],
+                    default="decode",
                     help="decode: the attention step (default); trace: the tag-stream "
-                         "parser; append: the decode-loop plan update")
+                         "parser; append: the decode-loop plan update; prefill: the "
+                         "tree-masked prefill")
+    ap.add_argument("--prefill", choices=["fork", "join", "both"], default="both",
+                    help="prefill workload (with --component prefill)")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -541,6 +639,8 @@ def main(argv=None):
         return run_trace(args)
     if args.component == "append":
         return run_append(args)
+    if args.component == "prefill":
+        return run_prefill(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_gpu(args)

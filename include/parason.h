@@ -127,6 +127,42 @@ parason_status parason_attn_plan_host(const parason_attn_config *cfg, int32_t nu
                                       int64_t num_physical_pages, int32_t num_sms,
                                       parason_plan *out);
 
+/*
+ * Tree-masked prefill (the join, Sec. 3.1 and Fig. 1: after a parallel block
+ * the threads' tokens become context of the main trajectory, and new text is
+ * prefilled against the fork tree): plan one attention pass in which every
+ * token of each chunk node is a query.
+ *
+ * Tree and pages as for parason_attn_plan; chunk_node[num_chunks] are
+ * distinct childless nodes whose tokens (K and V already written) are
+ * prefilled.  Queries are numbered chunk by chunk: query k = token t of
+ * chunk c with k = (sum of the lengths of chunks 0 .. c-1) + t.  Query k
+ * attends to every token of every ancestor of chunk_node[c] and to tokens
+ * 0 .. t of chunk_node[c] itself (causal within the chunk).
+ *
+ * The plan is run with parason_attn_decode: q [num_queries, H_q, head_dim],
+ * out the same shape, lse [num_queries, H_q]; parason_plan_info reports
+ * num_queries as num_leaves.  The causal tile is the tcgen05 prefix tile:
+ * PARASON_EUNSUPPORTED unless mode is PARASON_BF16 and head_dim is 128, and
+ * parason_plan_append on a prefill plan returns PARASON_EUNSUPPORTED.  Other
+ * errors, ownership and concurrency as parason_attn_plan.
+ */
+parason_status parason_prefill_plan(const parason_attn_config *cfg, int32_t num_nodes,
+                                    const int32_t *parent, const int32_t *node_len,
+                                    const int32_t *node_page_ptr, const int32_t *page_ids,
+                                    int32_t num_chunks, const int32_t *chunk_node,
+                                    int64_t num_physical_pages, parason_stream_t stream,
+                                    parason_plan *out);
+
+/* parason_prefill_plan without device memory or CUDA calls (inspection), as
+ * parason_attn_plan_host is to parason_attn_plan. */
+parason_status parason_prefill_plan_host(const parason_attn_config *cfg, int32_t num_nodes,
+                                         const int32_t *parent, const int32_t *node_len,
+                                         const int32_t *node_page_ptr, const int32_t *page_ids,
+                                         int32_t num_chunks, const int32_t *chunk_node,
+                                         int64_t num_physical_pages, int32_t num_sms,
+                                         parason_plan *out);
+
 /* Device workspace (bytes) that parason_attn_decode needs for this plan:
  * the split partial results (o, m, l) of every work item.  0 for NULL. */
 size_t parason_plan_workspace_bytes(parason_plan plan);
@@ -220,7 +256,7 @@ parason_status parason_attn_decode_no_alloc(parason_plan plan, const void *q,
  * half as many pages as its last item had (4 to 64 pages), beyond which the
  * grown item would unbalance the decode; PARASON_EUNSUPPORTED in FP32 mode.  On any error
  * nothing is changed.  Forking (new branches at an </Outlines>) needs a
- * new plan.
+ * new plan.  PARASON_EUNSUPPORTED on a prefill plan.
  */
 parason_status parason_plan_append(parason_plan plan, const int32_t *new_pages,
                                    parason_stream_t stream);
@@ -298,6 +334,10 @@ parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info)
  *                            page-count entries from there)
  *   PARASON_TABLE_STREAM_ROWS int32 [num_stream_rows]: the TMA row
  *                            (page * H_kv + kv head) * 16 of every item page
+ *   PARASON_TABLE_ITEM_KEY0  int32 [num_items] (prefill plans; empty for
+ *                            decode plans): for an item over its chunk's own
+ *                            node, the index in that node of its first key
+ *                            (the causal mask's origin), else -1
  * Returns PARASON_EINVAL if `bytes` is smaller than the table.
  */
 enum {
@@ -308,7 +348,8 @@ enum {
     PARASON_TABLE_WIDE_QUEUE = 4,
     PARASON_TABLE_NARROW_QUEUE = 5,
     PARASON_TABLE_ITEM_ROWS = 6,
-    PARASON_TABLE_STREAM_ROWS = 7
+    PARASON_TABLE_STREAM_ROWS = 7,
+    PARASON_TABLE_ITEM_KEY0 = 8
 };
 parason_status parason_plan_export(parason_plan plan, int32_t table, void *dst, size_t bytes);
 

@@ -44,13 +44,17 @@ class Plan:
     """Decode plan of one fork tree (C type ``parason_plan``).
 
     ``host_only=True`` builds the same work decomposition without touching
-    CUDA (for inspection on machines without a GPU).
+    CUDA (for inspection on machines without a GPU).  ``prefill=True`` plans a
+    tree-masked prefill instead (parason_prefill_plan): ``leaf_node`` then
+    lists the chunk nodes, and every token of every chunk is a query row of
+    ``q`` (chunk by chunk) in ``decode``.
     """
 
     def __init__(self, *, num_q_heads: int, num_kv_heads: int, head_dim: int, mode: str,
                  parent, node_len, node_page_ptr, page_ids, leaf_node,
                  num_physical_pages: int, sm_scale: float = 0.0, page_size: int = 16,
-                 stream=None, host_only: bool = False, num_sms: int = 152):
+                 stream=None, host_only: bool = False, num_sms: int = 152,
+                 prefill: bool = False):
         lib = _lib.load()
         self.mode = mode
         self.num_q_heads, self.num_kv_heads, self.head_dim = num_q_heads, num_kv_heads, head_dim
@@ -61,20 +65,24 @@ class Plan:
         parent, node_len = _i32(parent), _i32(node_len)
         node_page_ptr, page_ids, leaf_node = _i32(node_page_ptr), _i32(page_ids), _i32(leaf_node)
         out = ctypes.c_void_p()
+        kind = "prefill" if prefill else "attn"
         if host_only:
-            st = lib.parason_attn_plan_host(ctypes.byref(self._cfg), len(parent), _ptr(parent),
-                                            _ptr(node_len), _ptr(node_page_ptr), _ptr(page_ids),
-                                            len(leaf_node), _ptr(leaf_node),
-                                            self.num_physical_pages, num_sms, ctypes.byref(out))
+            fn = getattr(lib, f"parason_{kind}_plan_host")
+            st = fn(ctypes.byref(self._cfg), len(parent), _ptr(parent), _ptr(node_len),
+                    _ptr(node_page_ptr), _ptr(page_ids), len(leaf_node), _ptr(leaf_node),
+                    self.num_physical_pages, num_sms, ctypes.byref(out))
         else:
-            st = lib.parason_attn_plan(ctypes.byref(self._cfg), len(parent), _ptr(parent),
-                                       _ptr(node_len), _ptr(node_page_ptr), _ptr(page_ids),
-                                       len(leaf_node), _ptr(leaf_node), self.num_physical_pages,
-                                       _stream_handle(stream), ctypes.byref(out))
-        check(st, "parason_attn_plan")
+            fn = getattr(lib, f"parason_{kind}_plan")
+            st = fn(ctypes.byref(self._cfg), len(parent), _ptr(parent), _ptr(node_len),
+                    _ptr(node_page_ptr), _ptr(page_ids), len(leaf_node), _ptr(leaf_node),
+                    self.num_physical_pages, _stream_handle(stream), ctypes.byref(out))
+        check(st, f"parason_{kind}_plan")
         self._h = out
         self._ws = None
         self.host_only = host_only
+        self.prefill = prefill
+        if prefill:
+            self.num_leaves = int(self.info()["num_leaves"])     # queries
 
     @classmethod
     def for_tree(cls, tree, **kw) -> "Plan":
@@ -85,6 +93,12 @@ class Plan:
                    page_ids=tree.page_ids, leaf_node=tree.leaf_node,
                    num_physical_pages=tree.num_physical_pages, sm_scale=tree.sm_scale,
                    page_size=tree.page_size, **kw)
+
+    @classmethod
+    def for_prefill(cls, tree, **kw) -> "Plan":
+        """Prefill plan of a ``workloads.build_prefill`` workload (chunk nodes
+        in ``leaf_node``)."""
+        return cls.for_tree(tree, prefill=True, **kw)
 
     # ---------------------------------------------------------------- lifetime
     def close(self):
@@ -129,7 +143,8 @@ class Plan:
                  _lib.TABLE_WIDE_QUEUE: (inf["num_wide_items"],),
                  _lib.TABLE_NARROW_QUEUE: (inf["num_narrow_items"],),
                  _lib.TABLE_ITEM_ROWS: (inf["num_items"] + 1,),
-                 _lib.TABLE_STREAM_ROWS: (inf["num_stream_rows"],)}[table]
+                 _lib.TABLE_STREAM_ROWS: (inf["num_stream_rows"],),
+                 _lib.TABLE_ITEM_KEY0: (inf["num_items"] if self.prefill else 0,)}[table]
         buf = np.zeros(shape, dtype=np.int32)
         check(_lib.load().parason_plan_export(self.handle, table, _ptr(buf), buf.nbytes),
               "plan_export")

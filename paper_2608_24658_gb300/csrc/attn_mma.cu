@@ -828,7 +828,8 @@ static_assert(kMaxSuffixWarps <= kThreads / 32, "every suffix-pass warp exists")
 struct TcMeta {
     WorkItem it;
     int32_t id;                      // -1: the queue is empty
-    int32_t pad[3];
+    int32_t key0;                    // causal item: its first key's token index, else -1
+    int32_t pad[2];
     int32_t rows[kTcMetaPages];      // TMA row of each page
     int32_t leaves[kTcRows];         // branch of rows [g i, g i + g)
 };
@@ -915,7 +916,10 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                     }
                     id = -1;
                 } else {
-                    if (lane == 0) m.it = it;
+                    if (lane == 0) {
+                        m.it = it;
+                        m.key0 = a.item_key0 ? a.item_key0[id] : -1;
+                    }
                     const int32_t *src = a.stream_rows + a.item_rows[id];
                     for (int p = lane; p < it.num_pages; p += 32) m.rows[p] = src[p];
                     const int nbr = (it.nrows + a.group - 1) / a.group;
@@ -1091,11 +1095,16 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
             const int nb = tc_blocks(it.num_pages);
             const int tokens = (it.num_pages - 1) * kPageSize + it.last_valid;
             const uint32_t tO = lane_base + kTmemO + 128u * (k & 1);
+            // causal item (tree-masked prefill): the row's token, relative to
+            // the item's first key, is the last key it sees
+            const int key0 = meta[ms].key0;
+            const int t_rel = key0 < 0 ? (1 << 30) : (it.row0 + r) / a.group - key0;
             float m_use = -INFINITY, l = 0.f;
             bool ok = true;
             for (int i = 0; i < nb; ++i) {
                 const int b = blk + i;
                 const int valid = min(kTcBlockTokens, tokens - i * kTcBlockTokens);
+                const int seen = min(valid, t_rel - i * kTcBlockTokens + 1);   // keys the row sees
                 const uint32_t tS = lane_base + kTmemS + 64u * (b & 1);
                 if (!tc_warp_wait(bar(kBarSFull + (b & 1)), (b >> 1) & 1, limit, abort_flag, lane)) {
                     ok = false;
@@ -1110,7 +1119,7 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                 float mb = -INFINITY;
 #pragma unroll
                 for (int j = 0; j < 64; ++j) {
-                    x[j] = j < valid ? __uint_as_float(sr[j >> 5][j & 31]) * a.scale_log2 : -INFINITY;
+                    x[j] = j < seen ? __uint_as_float(sr[j >> 5][j & 31]) * a.scale_log2 : -INFINITY;
                     mb = fmaxf(mb, x[j]);
                 }
                 if (i == 0) {
@@ -1124,7 +1133,8 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                     }
                     tc::fence_after_sync();
                     const float m_new = fmaxf(m_use, mb);
-                    const float alpha = dev::fast_exp2(m_use - m_new);
+                    // (a row with no visible key yet keeps m = -inf and alpha 1)
+                    const float alpha = m_new == m_use ? 1.f : dev::fast_exp2(m_use - m_new);
 #pragma unroll
                     for (int c = 0; c < D / 32; ++c) {
                         uint32_t ov[32];
@@ -1139,11 +1149,13 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                     m_use = m_new;
                 }
                 // P = 2^(x - m) as bf16 pairs over the first 32 columns of S
+                // (0 for a row that has seen no key: every x is -inf)
+                const float m_ref = m_use == -INFINITY ? 0.f : m_use;
                 uint32_t pw[32];
 #pragma unroll
                 for (int c = 0; c < 32; ++c) {
-                    const float p0 = dev::fast_exp2(x[2 * c] - m_use);
-                    const float p1 = dev::fast_exp2(x[2 * c + 1] - m_use);
+                    const float p0 = dev::fast_exp2(x[2 * c] - m_ref);
+                    const float p1 = dev::fast_exp2(x[2 * c + 1] - m_ref);
                     l += p0 + p1;
                     pw[c] = dev::pack_bf16(p0, p1);
                 }

@@ -85,6 +85,9 @@ struct AttnArgs {
     int32_t num_wide_ctas;
     int32_t kv_rows;        // rows of the KV tensor maps (pages * H_kv * 16); a
                             // TMA box starting there is out of range: zeros
+    // tree-masked prefill: per item, the token index (in its node) of its
+    // first key when the item is causal, else -1; null for decode plans
+    const int32_t *item_key0;
 };
 
 struct MergeArgs {

@@ -101,6 +101,8 @@ struct parason_plan_s {
     int64_t num_slots = 0;
     int64_t unique_tokens = 0;
     int64_t path_tokens = 0;
+    bool prefill = false;              // a tree-masked prefill plan
+    std::vector<int32_t> item_key0;    // prefill: first key of a causal item, else -1
 
     // device side
     bool on_device = false;
@@ -112,7 +114,8 @@ struct parason_plan_s {
     int32_t *d_merge_ptr = nullptr;
     int32_t *d_merge_ent = nullptr;
     int32_t *d_item_rec = nullptr;
-    int2 *d_patch = nullptr;           // (word offset in the blob, value), tail_items * 6
+    int2 *d_patch = nullptr;
+    int32_t *d_item_key0 = nullptr;    // prefill plans only           // (word offset in the blob, value), tail_items * 6
     std::vector<int2> patches;         // host side of the last append's patch list
     size_t blob_words = 0;
     size_t w_items = 0, w_rec = 0, w_strows = 0;   // word offsets of those arrays in the blob
@@ -157,13 +160,19 @@ parason_status validate_config(const parason_attn_config *cfg) {
     return PARASON_OK;
 }
 
+// With `prefill`, leaf_node holds the chunk nodes of a tree-masked prefill:
+// every token of a chunk is a query (numbered chunk by chunk), attending to
+// every token of its node's ancestors and causally to its own node.
 parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int32_t num_nodes,
                           const int32_t *parent, const int32_t *node_len,
                           const int32_t *node_page_ptr, const int32_t *page_ids,
                           int32_t num_leaves, const int32_t *leaf_node,
-                          int64_t num_phys, int32_t num_sms) {
+                          int64_t num_phys, int32_t num_sms, bool prefill = false) {
     parason_status st = validate_config(cfg);
     if (st != PARASON_OK) return st;
+    // the prefill's causal mask is in the tcgen05 tile: bf16 at head_dim 128
+    if (prefill && (cfg->mode != PARASON_BF16 || cfg->head_dim != 128)) return PARASON_EUNSUPPORTED;
+    p->prefill = prefill;
     if (num_nodes < 0 || num_leaves < 0 || num_phys < 0) return PARASON_EINVAL;
     if (num_nodes > 0 && (!parent || !node_len || !node_page_ptr)) return PARASON_EINVAL;
     if (num_leaves > 0 && !leaf_node) return PARASON_EINVAL;
@@ -238,8 +247,18 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
             next_child[parent[i]] += cnt[i];
         }
     }
-    p->dfs_leaf.assign(num_leaves, -1);
-    for (int32_t b = 0; b < num_leaves; ++b) p->dfs_leaf[lo[leaf_node[b]]] = b;
+    // queries of a prefill: every token of every chunk, chunk by chunk
+    std::vector<int64_t> qbase(static_cast<size_t>(num_leaves) + 1, 0);
+    if (prefill) {
+        for (int32_t c = 0; c < num_leaves; ++c) qbase[c + 1] = qbase[c] + node_len[leaf_node[c]];
+        if (qbase[num_leaves] > INT32_MAX / 64) return PARASON_EUNSUPPORTED;
+        p->num_leaves = static_cast<int32_t>(qbase[num_leaves]);
+        p->dfs_leaf.resize(static_cast<size_t>(p->num_leaves));
+        for (int32_t k = 0; k < p->num_leaves; ++k) p->dfs_leaf[k] = k;
+    } else {
+        p->dfs_leaf.assign(num_leaves, -1);
+        for (int32_t b = 0; b < num_leaves; ++b) p->dfs_leaf[lo[leaf_node[b]]] = b;
+    }
 
     // ------------------------------------------------------------------
     // work decomposition
@@ -251,14 +270,65 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     const int32_t mode = cfg->mode;
     struct Run {
         int32_t node, head, row0, nrows;
-        int64_t pages;
+        int64_t pages;              // pages the run covers (from the node's first)
+        int64_t node_pages = 0;     // pages of the node
+        int64_t leaf_lo = 0;        // position of its first row's branch (query)
         double cost_per_page;
         bool wide;
+        bool causal = false;        // prefill: keys past the row's own token are masked
     };
     std::vector<Run> runs;
     int64_t narrow_pages = 0;
     double wide_cost = 0.0;
-    for (int32_t n = 0; n < num_nodes; ++n) {
+    if (prefill) {
+        // chunk c: rows (token t, q head r) = t * g + r of every kv head, in
+        // tiles; each tile reads every ancestor in full and its own node up
+        // to the tile's last token
+        for (int32_t c = 0; c < num_leaves; ++c) {
+            const int32_t n = leaf_node[c];
+            const int64_t C = node_len[n];
+            if (C == 0) continue;
+            const int64_t R = C * g;
+            const int32_t rt = tile_rows_for(static_cast<int32_t>(std::min<int64_t>(R, 1 << 20)), g, mode);
+            if (rt <= 0) return PARASON_EUNSUPPORTED;
+            std::vector<int32_t> path;
+            for (int32_t m = n; m >= 0; m = parent[m]) path.push_back(m);
+            std::reverse(path.begin(), path.end());
+            // (kv head, node, tile): the tiles of one ancestor read the same
+            // pages and sit next to each other for the piece interleaving
+            for (int32_t j = 0; j < H_kv; ++j)
+                for (int32_t m : path) {
+                    if (node_len[m] == 0) continue;
+                    for (int64_t r0 = 0; r0 < R; r0 += rt) {
+                        const int64_t nrows = std::min<int64_t>(rt, R - r0);
+                        const int64_t tb = (r0 + nrows) / g;         // tokens [r0 / g, tb)
+                        Run run;
+                        run.node = m;
+                        run.head = j;
+                        run.row0 = static_cast<int32_t>(r0);
+                        run.nrows = static_cast<int32_t>(nrows);
+                        run.node_pages = node_page_ptr[m + 1] - node_page_ptr[m];
+                        run.causal = m == n;
+                        run.pages = run.causal ? (tb + parason::kPageSize - 1) / parason::kPageSize
+                                               : run.node_pages;
+                        run.leaf_lo = qbase[c];
+                        run.wide = true;
+                        run.cost_per_page = wide_page_cost(run.nrows, true);
+                        wide_cost += run.cost_per_page * static_cast<double>(run.pages);
+                        runs.push_back(run);
+                    }
+                }
+        }
+        for (int32_t n = 0; n < num_nodes; ++n)
+            if (cnt[n] > 0) p->unique_tokens += node_len[n];
+        // keys a query sees: its ancestors and its own node up to itself
+        for (int32_t c = 0; c < num_leaves; ++c) {
+            const int64_t C = node_len[leaf_node[c]];
+            for (int32_t m = parent[leaf_node[c]]; m >= 0; m = parent[m]) p->path_tokens += C * node_len[m];
+            p->path_tokens += C * (C + 1) / 2;
+        }
+    }
+    for (int32_t n = 0; n < num_nodes && !prefill; ++n) {
         if (cnt[n] == 0 || node_len[n] == 0) continue;
         p->unique_tokens += node_len[n];
         const int64_t R = cnt[n] * g;
@@ -275,6 +345,8 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                 run.row0 = static_cast<int32_t>(r0);
                 run.nrows = static_cast<int32_t>(std::min<int64_t>(rt, R - r0));
                 run.pages = P;
+                run.node_pages = P;
+                run.leaf_lo = lo[n];
                 run.wide = wide;
                 run.cost_per_page =
                     wide ? wide_page_cost(run.nrows, mode == PARASON_BF16 && cfg->head_dim == 128)
@@ -296,7 +368,9 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     if (mode != PARASON_FP32) {
         const int32_t S = p->num_sms;
         const double narrow_cost = static_cast<double>(narrow_pages);
-        if (wide_cost > 0 && narrow_cost > 0) {
+        if (prefill) {
+            n_wide = S;
+        } else if (wide_cost > 0 && narrow_cost > 0) {
             n_wide = static_cast<int32_t>(
                 std::ceil(kWideProvision * S * wide_cost / (wide_cost + narrow_cost)));
             n_wide = std::min(std::max(n_wide, 1), std::max(S - 1, 1));
@@ -320,15 +394,16 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     int64_t slots = 0;
     std::vector<std::pair<int64_t, int32_t>> wide_q, narrow_q;   // (pages, item)
     std::vector<std::pair<int32_t, int32_t>> tails;              // (branch, item)
+    std::vector<int32_t> key0;                                   // per item (prefill)
     auto emit = [&](const Run &run, int64_t pg0, int64_t np) -> bool {
         WorkItem it;
-        const int64_t P = run.pages;
+        const int64_t P = run.node_pages;
         it.page_pos = node_page_ptr[run.node] + static_cast<int32_t>(pg0);
         it.num_pages = static_cast<int32_t>(np);
         it.last_valid = (pg0 + np == P)
                             ? node_len[run.node] - static_cast<int32_t>(P - 1) * parason::kPageSize
                             : parason::kPageSize;
-        it.leaf_lo = static_cast<int32_t>(lo[run.node]);
+        it.leaf_lo = static_cast<int32_t>(run.leaf_lo);
         it.row0 = run.row0;
         it.nrows = run.nrows;
         it.kv_head = run.head;
@@ -338,7 +413,9 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         const int32_t id = static_cast<int32_t>(p->items.size());
         p->items.push_back(it);
         (run.wide ? wide_q : narrow_q).emplace_back(np, id);
-        if (pg0 + np == P && leaf_of_node[run.node] >= 0) tails.emplace_back(leaf_of_node[run.node], id);
+        key0.push_back(run.causal ? static_cast<int32_t>(pg0 * parason::kPageSize) : -1);
+        if (!prefill && pg0 + np == P && leaf_of_node[run.node] >= 0)
+            tails.emplace_back(leaf_of_node[run.node], id);
         return true;
     };
     auto cut = [&](const Run &r, int64_t chunk, int64_t align) -> bool {
@@ -372,7 +449,9 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         // the first read of each page come from L2.
         for (size_t i = 0; i < runs.size();) {
             size_t j = i + 1;
-            while (j < runs.size() && runs[j].node == runs[i].node && runs[j].head == runs[i].head) ++j;
+            while (j < runs.size() && runs[j].node == runs[i].node && runs[j].head == runs[i].head &&
+                   runs[j].pages == runs[i].pages)
+                ++j;
             const Run &r = runs[i];
             const int64_t align = r.wide ? kWideBlockPages : 1;
             int64_t chunk = r.wide ? wide_chunk : narrow_chunk;
@@ -417,6 +496,9 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         }
         p->items.swap(sorted);
         for (auto &t : tails) t.second = new_id[t.second];
+        std::vector<int32_t> key0_sorted(key0.size());
+        for (size_t id = 0; id < key0.size(); ++id) key0_sorted[new_id[id]] = key0[id];
+        key0.swap(key0_sorted);
         for (size_t k = 0; k < p->wide_queue.size(); ++k) p->wide_queue[k] = static_cast<int32_t>(k);
         for (size_t k = 0; k < p->narrow_queue.size(); ++k)
             p->narrow_queue[k] = static_cast<int32_t>(p->wide_queue.size() + k);
@@ -467,25 +549,33 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
             rec[parason::kRecRow0 + j] = p->stream_rows[p->item_rows[i] + j];
     }
 
+    if (prefill) p->item_key0 = key0;
+    else p->item_key0.clear();
+
     // merge lists per (branch, kv head): the first of the branch's g partial
-    // slots in every item, on the branch's path, that covers its rows
-    std::vector<std::vector<int32_t>> ent(static_cast<size_t>(num_leaves) * H_kv);
-    for (const WorkItem &it : p->items) {
+    // slots in every item, on the branch's path, that covers its rows (in a
+    // prefill, not the chunk's own items whose keys all follow the token)
+    const int32_t L_rows = p->num_leaves;
+    std::vector<std::vector<int32_t>> ent(static_cast<size_t>(L_rows) * H_kv);
+    for (size_t ii = 0; ii < p->items.size(); ++ii) {
+        const WorkItem &it = p->items[ii];
+        const int32_t k0 = prefill ? key0[ii] : -1;
         const int32_t pos_lo = it.row0 / g, pos_hi = (it.row0 + it.nrows - 1) / g;
         for (int32_t pos = pos_lo; pos <= pos_hi; ++pos) {
+            if (k0 > pos) continue;
             const int32_t b = p->dfs_leaf[it.leaf_lo + pos];
             ent[static_cast<size_t>(b) * H_kv + it.kv_head].push_back(it.slot_base + pos * g -
                                                                        it.row0);
         }
     }
-    p->merge_ptr.assign(static_cast<size_t>(num_leaves) * H_kv + 1, 0);
+    p->merge_ptr.assign(static_cast<size_t>(L_rows) * H_kv + 1, 0);
     p->merge_ent.clear();
     for (size_t k = 0; k < ent.size(); ++k) {
         p->merge_ent.insert(p->merge_ent.end(), ent[k].begin(), ent[k].end());
         if (p->merge_ent.size() > static_cast<size_t>(INT32_MAX)) return PARASON_EUNSUPPORTED;
         p->merge_ptr[k + 1] = static_cast<int32_t>(p->merge_ent.size());
     }
-    for (int32_t b = 0; b < num_leaves; ++b)
+    for (int32_t b = 0; b < num_leaves && !prefill; ++b)
         for (int32_t n = leaf_node[b]; n >= 0; n = parent[n]) p->path_tokens += node_len[n];
     return PARASON_OK;
 }
@@ -508,12 +598,13 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     const size_t n_qnext = 2 * sizeof(int32_t);
     const size_t n_err = parason::kErrWords * sizeof(int32_t);
     const size_t n_patch = p->tail_items.size() * kPatchesPerTail * sizeof(int2);
-    constexpr int kArrays = 11;
+    const size_t n_key0 = p->item_key0.size() * sizeof(int32_t);
+    constexpr int kArrays = 12;
     size_t off[kArrays], total = 0;
     // the queue counters and the error record are set separately; the patch
     // buffer is written by parason_plan_append
-    const size_t sizes[kArrays] = {n_items, n_pages,  n_dfs,    n_mptr,  n_ment, n_rec,
-                                   n_irows, n_strows, n_qnext, n_err,   n_patch};
+    const size_t sizes[kArrays] = {n_items, n_pages,  n_dfs,   n_mptr, n_ment,  n_rec,
+                                   n_irows, n_strows, n_qnext, n_err,  n_patch, n_key0};
     for (int i = 0; i < kArrays; ++i) {
         off[i] = total;
         total = align_up(total + std::max<size_t>(sizes[i], 4), kAlign);
@@ -535,6 +626,7 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     p->d_queue_next = reinterpret_cast<int32_t *>(base + off[8]);
     p->d_err = reinterpret_cast<int32_t *>(base + off[9]);
     p->d_patch = reinterpret_cast<int2 *>(base + off[10]);
+    p->d_item_key0 = p->prefill ? reinterpret_cast<int32_t *>(base + off[11]) : nullptr;
     p->w_items = off[0] / sizeof(int32_t);
     p->w_rec = off[5] / sizeof(int32_t);
     p->w_strows = off[7] / sizeof(int32_t);
@@ -550,6 +642,9 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
             cudaSuccess)
             return PARASON_ECUDA;
     }
+    if (n_key0 > 0 && cudaMemcpyAsync(base + off[11], p->item_key0.data(), n_key0,
+                                      cudaMemcpyHostToDevice, stream) != cudaSuccess)
+        return PARASON_ECUDA;
     if (cudaMemsetAsync(p->d_err, 0, n_err, stream) != cudaSuccess) return PARASON_ECUDA;
     if (cudaMemcpyAsync(p->d_queue_next, p->queue_start, n_qnext, cudaMemcpyHostToDevice, stream) !=
         cudaSuccess)
@@ -616,16 +711,11 @@ void free_events(parason_plan_s *p) {
     p->timing_cap = p->timing_n = 0;
 }
 
-}  // namespace
-
-extern "C" {
-
-parason_status parason_attn_plan_host(const parason_attn_config *cfg, int32_t num_nodes,
-                                      const int32_t *parent, const int32_t *node_len,
-                                      const int32_t *node_page_ptr, const int32_t *page_ids,
-                                      int32_t num_leaves, const int32_t *leaf_node,
-                                      int64_t num_physical_pages, int32_t num_sms,
-                                      parason_plan *out) {
+parason_status plan_host(const parason_attn_config *cfg, int32_t num_nodes, const int32_t *parent,
+                         const int32_t *node_len, const int32_t *node_page_ptr,
+                         const int32_t *page_ids, int32_t num_leaves, const int32_t *leaf_node,
+                         int64_t num_physical_pages, int32_t num_sms, bool prefill,
+                         parason_plan *out) {
     if (!out) return PARASON_EINVAL;
     *out = nullptr;
     auto *p = new (std::nothrow) parason_plan_s();
@@ -633,7 +723,7 @@ parason_status parason_attn_plan_host(const parason_attn_config *cfg, int32_t nu
     parason_status st;
     try {
         st = build_host(p, cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves,
-                        leaf_node, num_physical_pages, num_sms);
+                        leaf_node, num_physical_pages, num_sms, prefill);
     } catch (const std::bad_alloc &) {
         st = PARASON_ENOMEM;
     }
@@ -645,12 +735,11 @@ parason_status parason_attn_plan_host(const parason_attn_config *cfg, int32_t nu
     return PARASON_OK;
 }
 
-parason_status parason_attn_plan(const parason_attn_config *cfg, int32_t num_nodes,
-                                 const int32_t *parent, const int32_t *node_len,
-                                 const int32_t *node_page_ptr, const int32_t *page_ids,
-                                 int32_t num_leaves, const int32_t *leaf_node,
-                                 int64_t num_physical_pages, parason_stream_t stream,
-                                 parason_plan *out) {
+parason_status plan_device(const parason_attn_config *cfg, int32_t num_nodes, const int32_t *parent,
+                           const int32_t *node_len, const int32_t *node_page_ptr,
+                           const int32_t *page_ids, int32_t num_leaves, const int32_t *leaf_node,
+                           int64_t num_physical_pages, bool prefill, parason_stream_t stream,
+                           parason_plan *out) {
     if (!out) return PARASON_EINVAL;
     *out = nullptr;
     // validate before touching CUDA, so malformed input is EINVAL everywhere
@@ -661,8 +750,8 @@ parason_status parason_attn_plan(const parason_attn_config *cfg, int32_t num_nod
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
         // still report malformed trees as EINVAL on machines without a GPU
         parason_plan probe = nullptr;
-        st = parason_attn_plan_host(cfg, num_nodes, parent, node_len, node_page_ptr, page_ids,
-                                    num_leaves, leaf_node, num_physical_pages, 152, &probe);
+        st = plan_host(cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves,
+                       leaf_node, num_physical_pages, 152, prefill, &probe);
         parason_plan_destroy(probe);
         cudaGetLastError();
         return st != PARASON_OK ? st : PARASON_ECUDA;
@@ -674,18 +763,10 @@ parason_status parason_attn_plan(const parason_attn_config *cfg, int32_t num_nod
         if (e != cudaSuccess) return PARASON_ECUDA;
         if (ctas_per_sm < 1) return PARASON_EUNSUPPORTED;
     }
-    auto *p = new (std::nothrow) parason_plan_s();
-    if (!p) return PARASON_ENOMEM;
-    try {
-        st = build_host(p, cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves,
-                        leaf_node, num_physical_pages, sms);
-    } catch (const std::bad_alloc &) {
-        st = PARASON_ENOMEM;
-    }
-    if (st != PARASON_OK) {
-        delete p;
-        return st;
-    }
+    parason_plan p = nullptr;
+    st = plan_host(cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves, leaf_node,
+                   num_physical_pages, sms, prefill, &p);
+    if (st != PARASON_OK) return st;
     st = upload(p, reinterpret_cast<cudaStream_t>(stream));
     if (st != PARASON_OK) {
         parason_plan_destroy(p);
@@ -693,6 +774,50 @@ parason_status parason_attn_plan(const parason_attn_config *cfg, int32_t num_nod
     }
     *out = p;
     return PARASON_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+parason_status parason_attn_plan_host(const parason_attn_config *cfg, int32_t num_nodes,
+                                      const int32_t *parent, const int32_t *node_len,
+                                      const int32_t *node_page_ptr, const int32_t *page_ids,
+                                      int32_t num_leaves, const int32_t *leaf_node,
+                                      int64_t num_physical_pages, int32_t num_sms,
+                                      parason_plan *out) {
+    return plan_host(cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves,
+                     leaf_node, num_physical_pages, num_sms, false, out);
+}
+
+parason_status parason_attn_plan(const parason_attn_config *cfg, int32_t num_nodes,
+                                 const int32_t *parent, const int32_t *node_len,
+                                 const int32_t *node_page_ptr, const int32_t *page_ids,
+                                 int32_t num_leaves, const int32_t *leaf_node,
+                                 int64_t num_physical_pages, parason_stream_t stream,
+                                 parason_plan *out) {
+    return plan_device(cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves,
+                       leaf_node, num_physical_pages, false, stream, out);
+}
+
+parason_status parason_prefill_plan_host(const parason_attn_config *cfg, int32_t num_nodes,
+                                         const int32_t *parent, const int32_t *node_len,
+                                         const int32_t *node_page_ptr, const int32_t *page_ids,
+                                         int32_t num_chunks, const int32_t *chunk_node,
+                                         int64_t num_physical_pages, int32_t num_sms,
+                                         parason_plan *out) {
+    return plan_host(cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_chunks,
+                     chunk_node, num_physical_pages, num_sms, true, out);
+}
+
+parason_status parason_prefill_plan(const parason_attn_config *cfg, int32_t num_nodes,
+                                    const int32_t *parent, const int32_t *node_len,
+                                    const int32_t *node_page_ptr, const int32_t *page_ids,
+                                    int32_t num_chunks, const int32_t *chunk_node,
+                                    int64_t num_physical_pages, parason_stream_t stream,
+                                    parason_plan *out) {
+    return plan_device(cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_chunks,
+                       chunk_node, num_physical_pages, true, stream, out);
 }
 
 size_t parason_plan_workspace_bytes(parason_plan p) {
@@ -762,6 +887,7 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
         a.num_ctas = p->num_ctas;
         a.num_wide_ctas = p->num_wide_ctas;
         a.kv_rows = static_cast<int32_t>(p->num_phys * p->cfg.num_kv_heads * parason::kPageSize);
+        a.item_key0 = p->d_item_key0;
         cudaError_t e;
         if (p->cfg.mode == PARASON_FP32) {
             e = parason::launch_attn_fp32(a, static_cast<const float *>(k_pages),
@@ -890,7 +1016,7 @@ parason_status parason_plan_get_info(parason_plan p, parason_plan_info *info) {
 parason_status parason_plan_append(parason_plan p, const int32_t *new_pages,
                                    parason_stream_t stream_) {
     if (!p) return PARASON_EINVAL;
-    if (p->cfg.mode == PARASON_FP32) return PARASON_EUNSUPPORTED;
+    if (p->cfg.mode == PARASON_FP32 || p->prefill) return PARASON_EUNSUPPORTED;
     const int32_t L = p->num_leaves;
     if (L == 0) return PARASON_OK;
     if (p->on_device && p->blob_words > static_cast<size_t>(INT32_MAX)) return PARASON_EUNSUPPORTED;
@@ -989,6 +1115,7 @@ parason_status parason_plan_export(parason_plan p, int32_t table, void *dst, siz
     case PARASON_TABLE_NARROW_QUEUE: src = p->narrow_queue.data(); n = p->narrow_queue.size() * 4; break;
     case PARASON_TABLE_ITEM_ROWS: src = p->item_rows.data(); n = p->item_rows.size() * 4; break;
     case PARASON_TABLE_STREAM_ROWS: src = p->stream_rows.data(); n = p->stream_rows.size() * 4; break;
+    case PARASON_TABLE_ITEM_KEY0: src = p->item_key0.data(); n = p->item_key0.size() * 4; break;
     default: return PARASON_EINVAL;
     }
     if (bytes < n || (n > 0 && !dst)) return PARASON_EINVAL;

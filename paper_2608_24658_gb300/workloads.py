@@ -519,3 +519,32 @@ def build_prefill(name: str, parent, node_len, chunk_node, *, num_q_heads: int,
     meta = dict(tree.meta)
     meta["prefill"] = True
     return replace(tree, q=q, meta=meta)
+
+
+def fork_prefill(mode="bf16", device="cpu", chunk=64, threads=16, **kw) -> ForkTree:
+    """Thread openings at </Outlines> on the Llama-3-8B shape (32 q / 8 kv, d
+    128): prefix 2048 and `threads` chunks of `chunk` tokens under it, each a
+    thread's first tokens prefilled against the shared prefix."""
+    rng = np.random.default_rng(6)
+    parent = [-1] + [0] * threads
+    lens = [2048] + [chunk] * threads
+    return build_prefill(f"fork_prefill_2048_{threads}x{chunk}", parent, lens,
+                         list(range(1, threads + 1)), num_q_heads=32, num_kv_heads=8,
+                         head_dim=128, mode=mode, rng=rng, q_std=1.0 / math.sqrt(128.0),
+                         device=device, **kw)
+
+
+def join_prefill(mode="bf16", device="cpu", chunk=1024, threads=16, **kw) -> ForkTree:
+    """The join with the threads' KV reused in place, on the Llama-3-8B shape:
+    a chain prefix 2048 -> `threads` thread nodes of U[512, 4096] tokens (the
+    trials of llama3_trials, concatenated in order) -> a `chunk`-token node
+    prefilled against all of it."""
+    rng = np.random.default_rng(1)
+    lens = [2048] + [_uniform(rng, 512, 4096) for _ in range(threads)] + [chunk]
+    parent = [-1] + list(range(len(lens) - 1))
+    return build_prefill(f"join_prefill_2048_{threads}threads_{chunk}", parent, lens,
+                         [len(lens) - 1], num_q_heads=32, num_kv_heads=8, head_dim=128,
+                         mode=mode, rng=rng, q_std=1.0 / math.sqrt(128.0), device=device, **kw)
+
+
+PREFILL_CONFIGS = {"fork": fork_prefill, "join": join_prefill}

@@ -1,0 +1,171 @@
+"""Tree-masked prefill plans (parason_prefill_plan_host), checked against the
+tree alone (CPU only): for every query (token t of chunk c) and q head, the
+partial slots its merge list names see, between them, every token of every
+ancestor of the chunk's node and tokens 0 .. t of the node itself, each
+exactly once; no slot is written twice; every key an item's row sees passes
+the causal rule; and the unsupported forms are refused."""
+import collections
+
+import numpy as np
+import pytest
+
+from paper_2608_24658_gb300 import _lib, build
+from paper_2608_24658_gb300 import workloads as W
+from paper_2608_24658_gb300.api import Plan, ParasonError
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    build.build()
+
+
+def ancestors(tree, n):
+    out = []
+    n = int(tree.parent[n])
+    while n >= 0:
+        out.append(n)
+        n = int(tree.parent[n])
+    return out
+
+
+def verify_prefill_plan(tree, plan):
+    g, H_kv = tree.group, tree.num_kv_heads
+    chunks = [int(c) for c in tree.leaf_node]
+    lens = [int(tree.node_len[c]) for c in chunks]
+    qbase = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    Q = int(qbase[-1])
+    info = plan.info()
+    assert info["num_leaves"] == Q
+    items = plan.export(_lib.TABLE_ITEMS)
+    key0 = plan.export(_lib.TABLE_ITEM_KEY0)
+    dfs = plan.export(_lib.TABLE_DFS_LEAVES)
+    mptr = plan.export(_lib.TABLE_MERGE_PTR)
+    ment = plan.export(_lib.TABLE_MERGE)
+    wq = plan.export(_lib.TABLE_WIDE_QUEUE)
+    nq = plan.export(_lib.TABLE_NARROW_QUEUE)
+    assert dfs.tolist() == list(range(Q))
+    assert len(key0) == len(items)
+    assert len(nq) == 0 and wq.tolist() == list(range(len(items)))    # all on the tcgen05 tile
+    owner = np.full(int(tree.node_page_ptr[-1]), -1, dtype=np.int64)
+    for n in range(tree.num_nodes):
+        owner[tree.node_page_ptr[n]:tree.node_page_ptr[n + 1]] = n
+
+    seen = {}                                        # slot -> list of (node, token)
+    for it, k0 in zip(items, key0):
+        page_pos, npg, last_valid, leaf_lo, row0, nrows, kvh, slot_base = (int(x) for x in it)
+        assert 1 <= nrows <= 128 and row0 % g == 0 and 0 <= kvh < H_kv and npg >= 1
+        n = int(owner[page_pos])
+        assert owner[page_pos + npg - 1] == n
+        first = page_pos - int(tree.node_page_ptr[n])
+        P = int(tree.node_page_ptr[n + 1] - tree.node_page_ptr[n])
+        ends = first + npg == P
+        assert last_valid == (int(tree.node_len[n]) - 16 * (P - 1) if ends else 16)
+        c = int(np.searchsorted(qbase, leaf_lo, side="right")) - 1
+        assert qbase[c] == leaf_lo, "an item's rows start at its chunk's first query"
+        own = n == chunks[c]
+        assert n in ancestors(tree, chunks[c]) or own
+        assert int(k0) == (16 * first if own else -1)
+        tokens = list(range(16 * first, 16 * (first + npg - 1) + last_valid))
+        for row in range(row0, row0 + nrows):
+            t = row // g
+            assert t < lens[c]
+            vis = [(n, x) for x in tokens if not own or x <= t]
+            slot = slot_base + row - row0
+            assert slot not in seen, "partial slot written twice"
+            seen[slot] = (int(leaf_lo) + t, kvh * g + row % g, vis)
+    assert sorted(seen) == list(range(info["num_slots"]))
+    assert mptr[0] == 0 and mptr[-1] == len(ment)
+    for c, n in enumerate(chunks):
+        want_anc = [(a, x) for a in ancestors(tree, n) for x in range(int(tree.node_len[a]))]
+        for t in range(lens[c]):
+            q = int(qbase[c]) + t
+            want = sorted(want_anc + [(n, x) for x in range(t + 1)])
+            for h in range(tree.num_q_heads):
+                j, r = divmod(h, g)
+                k = q * H_kv + j
+                got = []
+                for e in ment[mptr[k]:mptr[k + 1]]:
+                    qq, hh, vis = seen[int(e) + r]
+                    assert (qq, hh) == (q, h)
+                    assert vis, "a merged slot must see at least one key"
+                    got.extend(vis)
+                assert sorted(got) == want, (c, t, h)
+    # every written slot that sees a key is merged (no wasted tiles beyond the mask)
+    merged = {int(e) + r for e in ment for r in range(g)}
+    assert all(s in merged for s, (_, _, vis) in seen.items() if vis)
+    want_path = sum(lens[c] * sum(int(tree.node_len[a]) for a in ancestors(tree, n)) +
+                    lens[c] * (lens[c] + 1) // 2 for c, n in enumerate(chunks))
+    assert info["path_tokens"] == want_path
+    return info
+
+
+def prefill(name, parent, node_len, chunks, *, hq=8, hkv=2, **kw):
+    return W.build_prefill(name, parent, node_len, chunks, num_q_heads=hq, num_kv_heads=hkv,
+                           head_dim=128, values=False, **kw)
+
+
+CASES = {
+    # the join: a prefix, threads under it, the text after </Parallel> as chunks
+    "join": lambda: prefill("join", [-1, 0, 0, 0, 1], [300, 70, 33, 64, 41], [2, 3, 4]),
+    "root_chunk": lambda: prefill("root", [-1], [200], [0]),
+    "page_edges": lambda: prefill("edges", [-1, 0, 0, 0, 0, 0, 0],
+                                  [17, 1, 15, 16, 63, 64, 65], [1, 2, 3, 4, 5, 6]),
+    "g1": lambda: prefill("g1", [-1, 0, 1], [50, 90, 130], [2], hq=4, hkv=4),
+    "g16": lambda: prefill("g16", [-1, 0, 0], [77, 40, 9], [1, 2], hq=32, hkv=2),
+    "g6": lambda: prefill("g6", [-1, 0, 1, 1], [33, 21, 70, 5], [2, 3], hq=12, hkv=2),
+    "long_chunk": lambda: prefill("long", [-1, 0], [1000, 700], [1]),
+    "empty_ancestor": lambda: prefill("emptyanc", [-1, 0, 1], [0, 20, 35], [2]),
+    "empty_chunk": lambda: prefill("emptychunk", [-1, 0, 0], [40, 0, 19], [1, 2]),
+    "forest": lambda: prefill("forest", [-1, -1, 0, 1], [30, 45, 12, 80], [2, 3]),
+}
+
+
+@pytest.mark.parametrize("name", sorted(CASES))
+def test_prefill_plan_covers_keys_exactly(name):
+    tree = CASES[name]()
+    with Plan.for_prefill(tree, host_only=True) as plan:
+        verify_prefill_plan(tree, plan)
+
+
+def test_prefill_plan_sm_counts():
+    tree = CASES["join"]()
+    for sms in (1, 7, 152, 400):
+        with Plan.for_prefill(tree, host_only=True, num_sms=sms) as plan:
+            info = verify_prefill_plan(tree, plan)
+            assert info["num_ctas"] == info["num_wide_ctas"] == sms
+
+
+def test_prefill_plan_refusals():
+    tree = CASES["join"]()
+    for mode, d in (("fp32", 128), ("fp8", 128), ("bf16", 64)):
+        t = W.build_prefill("x", tree.parent, tree.node_len, tree.leaf_node, num_q_heads=8,
+                            num_kv_heads=2, head_dim=d, mode=mode, values=False)
+        with pytest.raises(ParasonError) as e:
+            Plan.for_prefill(t, host_only=True)
+        assert e.value.status == _lib.EUNSUPPORTED
+    # a chunk node with children, or named twice
+    for chunks in ([1, 2], [2, 2]):
+        t = W.build_tree("y", tree.parent, tree.node_len, [2, 3], num_q_heads=8, num_kv_heads=2,
+                         head_dim=128, values=False)
+        with pytest.raises(ParasonError) as e:
+            Plan(num_q_heads=8, num_kv_heads=2, head_dim=128, mode="bf16", parent=t.parent,
+                 node_len=t.node_len, node_page_ptr=t.node_page_ptr, page_ids=t.page_ids,
+                 leaf_node=chunks, num_physical_pages=t.num_physical_pages, host_only=True,
+                 prefill=True)
+        assert e.value.status == _lib.EINVAL
+    # appends are for decode plans
+    with Plan.for_prefill(tree, host_only=True) as plan:
+        with pytest.raises(ParasonError) as e:
+            plan.append(None)
+        assert e.value.status == _lib.EUNSUPPORTED
+
+
+def test_prefill_plan_deterministic():
+    tree = CASES["page_edges"]()
+    tabs = []
+    for _ in range(2):
+        with Plan.for_prefill(tree, host_only=True) as plan:
+            tabs.append([plan.export(t) for t in (_lib.TABLE_ITEMS, _lib.TABLE_ITEM_KEY0,
+                                                  _lib.TABLE_MERGE_PTR, _lib.TABLE_MERGE)])
+    for a, b in zip(*tabs):
+        assert np.array_equal(a, b)
