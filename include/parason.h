@@ -103,8 +103,10 @@ typedef struct parason_plan_s *parason_plan;
  * PARASON_EUNSUPPORTED for e4m3 KV with head_dim 64 (only 128 has a kernel).
  * PARASON_ENOMEM / PARASON_ECUDA if the metadata cannot be allocated or
  * copied.  On success *out owns host and device memory until
- * parason_plan_destroy.  The plan is immutable and may be used by any number
- * of decode calls, but calls that share a workspace must not overlap.
+ * parason_plan_destroy.  The plan may be used by any number of decode calls,
+ * one at a time: its device copy holds the work-queue positions that a
+ * call's kernels advance and rewind, so two calls on one plan must not
+ * overlap (issue them on one stream, or order their streams).
  */
 parason_status parason_attn_plan(const parason_attn_config *cfg, int32_t num_nodes,
                                  const int32_t *parent, const int32_t *node_len,
