@@ -145,7 +145,8 @@ parason_status parason_attn_plan_host(const parason_attn_config *cfg, int32_t nu
  * The plan is run with parason_attn_decode: q [num_queries, H_q, head_dim],
  * out the same shape, lse [num_queries, H_q]; parason_plan_info reports
  * num_queries as num_leaves.  The causal tile is the tcgen05 prefix tile:
- * PARASON_EUNSUPPORTED unless mode is PARASON_BF16 and head_dim is 128, and
+ * PARASON_EUNSUPPORTED unless head_dim is 128 and the mode is PARASON_BF16
+ * or PARASON_FP8_E4M3_KV (k_scale / v_scale as for decode), and
  * parason_plan_append on a prefill plan returns PARASON_EUNSUPPORTED.  Other
  * errors, ownership and concurrency as parason_attn_plan.
  */

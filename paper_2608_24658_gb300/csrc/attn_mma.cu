@@ -810,6 +810,14 @@ constexpr int kTcColBlockBytes = kTcBlockTokens * 128;        // 8 KB: 64 tokens
 constexpr int kTcKBytes = 2 * kTcColBlockBytes;               // d = 128: two column blocks
 constexpr int kTcStageBytes = 2 * kTcKBytes;                  // K + V
 constexpr int kTcRingBytes = kTcStages * kTcStageBytes;       // 192 KB
+// e4m3 KV: TMA stages the raw bytes (K and V of a block, 64 rows of 128 B
+// each: 16 KB) in kTcStages stages; the epilogue warps convert each block
+// to f16 (exactly) into kTcCvStages stages laid out like a bf16 stage.
+constexpr int kTcF8Bytes = kTcBlockTokens * 128;              // 8 KB: K (or V) of a block
+constexpr int kTcF8StageBytes = 2 * kTcF8Bytes;
+constexpr int kTcCvStages = 3;
+constexpr int kTcCvOffset = kTcStages * kTcF8StageBytes;      // 96 KB
+static_assert(kTcCvOffset + kTcCvStages * kTcStageBytes <= kTcRingBytes, "e4m3 rings fit");
 constexpr int kTcTmemCols = 512;
 constexpr uint32_t kTmemO = 0, kTmemS = 256, kTmemQ = 384;    // TMEM column bases
 constexpr float kTcRescaleLog2 = 8.f;                         // lazy rescale threshold
@@ -821,6 +829,7 @@ constexpr int kTcProducerWarp = 8;
 constexpr int kTcMmaWarp = 9;
 constexpr int kTcSchedulerWarp = 10;
 static_assert(kTcRingBytes <= Shape<128, KvBf16>::kBodyBytes, "tcgen05 ring fits the CTA's memory");
+static_assert(kTcRingBytes <= Shape<128, KvE4m3>::kBodyBytes, "tcgen05 ring fits the CTA's memory");
 static_assert(kTcSchedulerWarp < kThreads / 32, "every tcgen05 role has a warp");
 static_assert(kMaxSuffixWarps <= kThreads / 32, "every suffix-pass warp exists");
 
@@ -847,16 +856,49 @@ enum TcBar : int {
     kBarMetaFull = kBarOEmpty + 2,           // [kTcMeta] scheduler -> every role
     kBarMetaEmpty = kBarMetaFull + kTcMeta,  // [kTcMeta] epilogue (4 arrivals) -> scheduler
     kBarDrain = kBarMetaEmpty + kTcMeta,     // MMA commit -> MMA thread, before TMEM is freed
-    kTcBars
+    kBarCvFull,                              // [kTcCvStages] converters (4 arrivals) -> MMA
+    kBarCvEmpty = kBarCvFull + kTcCvStages,  // [kTcCvStages] MMA commit -> converters
+    kTcBars = kBarCvEmpty + kTcCvStages
 };
 
-__host__ __device__ constexpr int tc_bar_count(int i) {
+// arrivals each barrier waits for; with e4m3 KV the 4 converter warps free
+// the staging stages
+__host__ __device__ constexpr int tc_bar_count(int i, bool f8) {
     return (i == kBarPFull || i == kBarPFull + 1 || i == kBarQReady || i == kBarQReady + 1)
                ? kTcRows
                : ((i == kBarOEmpty || i == kBarOEmpty + 1 ||
-                   (i >= kBarMetaEmpty && i < kBarMetaEmpty + kTcMeta))
+                   (i >= kBarMetaEmpty && i < kBarMetaEmpty + kTcMeta) ||
+                   (f8 && i >= kBarKvEmpty && i < kBarKvEmpty + kTcStages))
                       ? 4
-                      : 1);
+                      : ((i >= kBarCvFull && i < kBarCvFull + kTcCvStages) ? kTcRows : 1));
+}
+
+// e4m3 -> f16 of one 64-token block by 128 threads (8 of its 1024 16-byte
+// chunks each): staged K and V rows of 128 bytes (128-byte swizzled) into two
+// 8 KB column blocks per operand (128-byte swizzled), the layout TMA gives a
+// bf16 block; rows from `valid` on become zeros.
+__device__ __forceinline__ void convert_block_e4m3(uint32_t src, uint32_t dst, int valid, int t) {
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+        const int idx = t + kTcRows * q;
+        const int op = idx >> 9;                 // 0: K, 1: V
+        const int r = (idx >> 3) & 63;           // token
+        const int c = idx & 7;                   // elements 16c .. 16c + 15
+        uint4 w = lds128(src + op * kTcF8Bytes + r * 128 + ((c ^ (r & 7)) << 4));
+        if (r >= valid) w = make_uint4(0u, 0u, 0u, 0u);
+        const uint32_t lo0 = e4m3x2_to_f16x2(w.x), lo1 = e4m3x2_to_f16x2(w.x >> 16);
+        const uint32_t lo2 = e4m3x2_to_f16x2(w.y), lo3 = e4m3x2_to_f16x2(w.y >> 16);
+        const uint32_t hi0 = e4m3x2_to_f16x2(w.z), hi1 = e4m3x2_to_f16x2(w.z >> 16);
+        const uint32_t hi2 = e4m3x2_to_f16x2(w.w), hi3 = e4m3x2_to_f16x2(w.w >> 16);
+        const int c2 = 2 * (c & 3);              // f16 chunk in column block c / 4
+        const uint32_t row = dst + op * kTcKBytes + (c >> 2) * kTcColBlockBytes + r * 128;
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(row + ((c2 ^ (r & 7)) << 4)),
+                     "r"(lo0), "r"(lo1), "r"(lo2), "r"(lo3)
+                     : "memory");
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(row + (((c2 + 1) ^ (r & 7)) << 4)),
+                     "r"(hi0), "r"(hi1), "r"(hi2), "r"(hi3)
+                     : "memory");
+    }
 }
 
 __device__ __forceinline__ bool tc_wait(uint32_t bar, uint32_t parity, long long limit,
@@ -883,14 +925,24 @@ __device__ __forceinline__ int tc_blocks(int num_pages) {
     return (num_pages + kTcBlockPages - 1) / kTcBlockPages;
 }
 
-template <int D>
+template <int D, class KV>
 __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
                               const AttnArgs &a, uint8_t *smem, uint32_t bars, uint32_t tmem,
                               int warp, int lane, volatile int *abort_flag, TcMeta *meta) {
     static_assert(D == 128, "the tcgen05 prefix tile is written for head_dim 128");
+    constexpr bool kF8 = KV::kElemBytes == 1;
     const uint32_t ring = dev::smem_addr(smem);
     auto bar = [&](int i) { return bars + 8u * static_cast<uint32_t>(i); };
     const long long limit = a.wait_limit_ns;
+    // the f16 (or bf16) K and V of block b, as the MMA reads them, and the
+    // barriers that hand them over
+    auto mma_stage = [&](int b) {
+        return kF8 ? ring + kTcCvOffset + (b % kTcCvStages) * kTcStageBytes
+                   : ring + (b % kTcStages) * kTcStageBytes;
+    };
+    auto mma_full = [&](int b) { return kF8 ? kBarCvFull + b % kTcCvStages : kBarKvFull + b % kTcStages; };
+    auto mma_full_parity = [&](int b) { return kF8 ? (b / kTcCvStages) & 1 : (b / kTcStages) & 1; };
+    auto mma_empty = [&](int b) { return kF8 ? kBarCvEmpty + b % kTcCvStages : kBarKvEmpty + b % kTcStages; };
 
     if (warp == kTcSchedulerWarp) {
         // ------------------------------------------------------------ scheduler
@@ -959,18 +1011,31 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                     break;
                 }
                 if (lane == 0 && !(skip_first && blk == 0)) {
-                    const uint32_t st = ring + s * kTcStageBytes;
                     const uint32_t fb = bar(kBarKvFull + s);
-                    dev::mbar_arrive_expect_tx(fb, kTcStageBytes);
+                    if constexpr (kF8) {
+                        // raw e4m3 rows: one 2 KB box per page of K and of V
+                        const uint32_t st = ring + s * kTcF8StageBytes;
+                        dev::mbar_arrive_expect_tx(fb, kTcF8StageBytes);
 #pragma unroll
-                    for (int j = 0; j < kTcBlockPages; ++j) {
-                        const int pg = bi * kTcBlockPages + j;
-                        const int row = pg < np ? m.rows[pg] : a.kv_rows;   // kv_rows: zero fill
+                        for (int j = 0; j < kTcBlockPages; ++j) {
+                            const int pg = bi * kTcBlockPages + j;
+                            const int row = pg < np ? m.rows[pg] : a.kv_rows;   // kv_rows: zero fill
+                            dev::tma_load_3d(st + j * kPageSize * 128, tmap_k, 0, 0, row, fb);
+                            dev::tma_load_3d(st + kTcF8Bytes + j * kPageSize * 128, tmap_v, 0, 0, row, fb);
+                        }
+                    } else {
+                        const uint32_t st = ring + s * kTcStageBytes;
+                        dev::mbar_arrive_expect_tx(fb, kTcStageBytes);
 #pragma unroll
-                        for (int cb = 0; cb < 2; ++cb) {
-                            const uint32_t off = cb * kTcColBlockBytes + j * kPageSize * 128;
-                            dev::tma_load_3d(st + off, tmap_k, 0, cb, row, fb);
-                            dev::tma_load_3d(st + kTcKBytes + off, tmap_v, 0, cb, row, fb);
+                        for (int j = 0; j < kTcBlockPages; ++j) {
+                            const int pg = bi * kTcBlockPages + j;
+                            const int row = pg < np ? m.rows[pg] : a.kv_rows;   // kv_rows: zero fill
+#pragma unroll
+                            for (int cb = 0; cb < 2; ++cb) {
+                                const uint32_t off = cb * kTcColBlockBytes + j * kPageSize * 128;
+                                dev::tma_load_3d(st + off, tmap_k, 0, cb, row, fb);
+                                dev::tma_load_3d(st + kTcKBytes + off, tmap_v, 0, cb, row, fb);
+                            }
                         }
                     }
                     last_issue[s] = blk;
@@ -986,14 +1051,16 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
     } else if (warp == kTcMmaWarp) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
-            constexpr uint32_t kIdS = tc::idesc_bf16_f32(kTcRows, kTcBlockTokens, false);
-            constexpr uint32_t kIdPV = tc::idesc_bf16_f32(kTcRows, D, true);
+            constexpr uint32_t kIdS = kF8 ? tc::idesc_f16_f32(kTcRows, kTcBlockTokens, false)
+                                          : tc::idesc_bf16_f32(kTcRows, kTcBlockTokens, false);
+            constexpr uint32_t kIdPV = kF8 ? tc::idesc_f16_f32(kTcRows, D, true)
+                                           : tc::idesc_bf16_f32(kTcRows, D, true);
             auto wait = [&](int i, int parity) {
                 return tc_wait(bar(i), static_cast<uint32_t>(parity & 1), limit, abort_flag);
             };
             // S(b) = Q(item k) K(b)^T into S buffer b & 1
             auto issue_s = [&](int b, int k) {
-                const uint32_t st = ring + (b % kTcStages) * kTcStageBytes;
+                const uint32_t st = mma_stage(b);
                 const uint32_t tS = tmem + kTmemS + 64u * (b & 1);
                 const uint32_t tQ = tmem + kTmemQ + 64u * (k & 1);
 #pragma unroll
@@ -1008,7 +1075,7 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
             bool have = ok && meta[0].id >= 0;
             int k = 0, b = 0, blk0 = 0, nb = have ? tc_blocks(meta[0].it.num_pages) : 0;
             if (have) {
-                ok = wait(kBarQReady, 0) && wait(kBarKvFull, 0);
+                ok = wait(kBarQReady, 0) && wait(mma_full(0), 0);
                 if (ok) {
                     tc::fence_after_sync();
                     issue_s(0, 0);
@@ -1019,7 +1086,7 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                 bool next = false;
                 int nb_next = 0;
                 if (!last) {
-                    if (!wait(kBarKvFull + (b + 1) % kTcStages, (b + 1) / kTcStages)) {
+                    if (!wait(mma_full(b + 1), mma_full_parity(b + 1))) {
                         ok = false;
                         break;
                     }
@@ -1036,7 +1103,7 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                         next = true;
                         nb_next = tc_blocks(meta[s1].it.num_pages);
                         if (!wait(kBarQReady + ((k + 1) & 1), (k + 1) >> 1) ||
-                            !wait(kBarKvFull + (b + 1) % kTcStages, (b + 1) / kTcStages)) {
+                            !wait(mma_full(b + 1), mma_full_parity(b + 1))) {
                             ok = false;
                             break;
                         }
@@ -1056,13 +1123,13 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                 tc::fence_after_sync();
                 const uint32_t tO = tmem + kTmemO + 128u * (k & 1);
                 const uint32_t tP = tmem + kTmemS + 64u * (b & 1);
-                const uint32_t vst = ring + (b % kTcStages) * kTcStageBytes + kTcKBytes;
+                const uint32_t vst = mma_stage(b) + kTcKBytes;
 #pragma unroll
                 for (int kk = 0; kk < kTcBlockTokens / 16; ++kk) {
                     const uint64_t bd = tc::smem_desc_sw128(vst + kk * 2048, kTcColBlockBytes, 1024);
                     tc::mma_bf16_tmem_a(tO, tP + 8u * kk, bd, kIdPV, b > blk0 || kk > 0);
                 }
-                tc::commit(bar(kBarKvEmpty + b % kTcStages));
+                tc::commit(bar(mma_empty(b)));
                 tc::commit(bar(kBarPvDone + (b & 1)));
                 if (last) {
                     tc::commit(bar(kBarOFull + (k & 1)));
@@ -1099,6 +1166,8 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
             // the item's first key, is the last key it sees
             const int key0 = meta[ms].key0;
             const int t_rel = key0 < 0 ? (1 << 30) : (it.row0 + r) / a.group - key0;
+            // e4m3 K: the kv head's scale goes into the logits
+            const float sl = kF8 ? a.scale_log2 * a.k_scale[it.kv_head] : a.scale_log2;
             float m_use = -INFINITY, l = 0.f;
             bool ok = true;
             for (int i = 0; i < nb; ++i) {
@@ -1119,7 +1188,7 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                 float mb = -INFINITY;
 #pragma unroll
                 for (int j = 0; j < 64; ++j) {
-                    x[j] = j < seen ? __uint_as_float(sr[j >> 5][j & 31]) * a.scale_log2 : -INFINITY;
+                    x[j] = j < seen ? __uint_as_float(sr[j >> 5][j & 31]) * sl : -INFINITY;
                     mb = fmaxf(mb, x[j]);
                 }
                 if (i == 0) {
@@ -1157,13 +1226,14 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                     const float p0 = dev::fast_exp2(x[2 * c] - m_ref);
                     const float p1 = dev::fast_exp2(x[2 * c + 1] - m_ref);
                     l += p0 + p1;
-                    pw[c] = dev::pack_bf16(p0, p1);
+                    pw[c] = kF8 ? dev::pack_f16(p0, p1) : dev::pack_bf16(p0, p1);
                 }
                 tc::st32(tS, pw);
                 tc::wait_st();
                 // V rows past the item's last token may hold anything (NaN
-                // included); P is 0 there but 0 * NaN is NaN, so zero them
-                if (valid < kTcBlockTokens) {
+                // included); P is 0 there but 0 * NaN is NaN, so zero them (the
+                // e4m3 converters write those rows as zeros)
+                if (!kF8 && valid < kTcBlockTokens) {
                     const uint32_t vst = ring + (b % kTcStages) * kTcStageBytes + kTcKBytes;
                     const int n16 = (kTcBlockTokens - valid) * 2 * 8;     // 16-byte chunks
                     for (int q = r; q < n16; q += kTcRows) {
@@ -1216,17 +1286,23 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                 for (int c = 0; c < 16; ++c) qv[c] = make_uint4(0u, 0u, 0u, 0u);
             }
         };
-        // ... then into TMEM Q buffer k & 1 (bf16 pairs, lane r)
+        // ... then into TMEM Q buffer k & 1 (bf16 pairs, or f16 pairs for
+        // the e4m3 tile, lane r)
         auto put_q = [&](int k, const uint4 (&qv)[16]) {
+            auto cv = [](uint32_t two) {
+                if constexpr (!kF8) return two;
+                const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162 *>(&two);
+                return dev::pack_f16(__low2float(b), __high2float(b));
+            };
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
                 uint32_t w[32];
 #pragma unroll
                 for (int c = 0; c < 8; ++c) {
-                    w[4 * c] = qv[8 * h + c].x;
-                    w[4 * c + 1] = qv[8 * h + c].y;
-                    w[4 * c + 2] = qv[8 * h + c].z;
-                    w[4 * c + 3] = qv[8 * h + c].w;
+                    w[4 * c] = cv(qv[8 * h + c].x);
+                    w[4 * c + 1] = cv(qv[8 * h + c].y);
+                    w[4 * c + 2] = cv(qv[8 * h + c].z);
+                    w[4 * c + 3] = cv(qv[8 * h + c].w);
                 }
                 tc::st32(lane_base + kTmemQ + 64u * (k & 1) + 32u * h, w);
             }
@@ -1234,6 +1310,94 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
             tc::fence_before_sync();
             dev::mbar_arrive(bar(kBarQReady + (k & 1)));
         };
+        if constexpr (kF8) {
+        // item j's O rows to its partials, times the kv head's V scale
+        auto store_o = [&](int j, const WorkItem &it) {
+            const float vs = a.v_scale[it.kv_head];
+            const uint32_t tO = lane_base + kTmemO + 128u * (j & 1);
+            float *dst = a.part_o + (static_cast<int64_t>(it.slot_base) + r) * D;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t ov[32];
+                tc::ld32(tO + 32 * c, ov);
+                tc::wait_ld();
+                if (r < it.nrows) {
+#pragma unroll
+                    for (int q = 0; q < 32; q += 4)
+                        *reinterpret_cast<float4 *>(dst + 32 * c + q) =
+                            make_float4(__uint_as_float(ov[q]) * vs, __uint_as_float(ov[q + 1]) * vs,
+                                        __uint_as_float(ov[q + 2]) * vs, __uint_as_float(ov[q + 3]) * vs);
+                }
+            }
+        };
+            // The converters take every block of every item in order.  An
+            // item's O is stored once the next item's first block is
+            // converted: the MMA issues that block's S before the item's last
+            // PV, so waiting for the O first could never end.
+            auto convert = [&](int gb, int valid) -> bool {
+                const int s = gb % kTcStages, c = gb % kTcCvStages;
+                if (!tc_warp_wait(bar(kBarKvFull + s), (gb / kTcStages) & 1, limit, abort_flag, lane))
+                    return false;
+                if (gb >= kTcCvStages &&
+                    !tc_warp_wait(bar(kBarCvEmpty + c), ((gb / kTcCvStages) - 1) & 1, limit, abort_flag,
+                                  lane))
+                    return false;
+                convert_block_e4m3(ring + s * kTcF8StageBytes, ring + kTcCvOffset + c * kTcStageBytes,
+                                   valid, r);
+                tc::fence_proxy_async_smem();
+                dev::mbar_arrive(bar(kBarCvFull + c));
+                __syncwarp();
+                if (lane == 0) dev::mbar_arrive(bar(kBarKvEmpty + s));
+                return true;
+            };
+            // store item j's O; load item j + 2's Q into the buffer j frees
+            auto finish = [&](int j, bool next_exists) -> bool {
+                const WorkItem it = meta[j % kTcMeta].it;
+                if (!tc_warp_wait(bar(kBarOFull + (j & 1)), (j >> 1) & 1, limit, abort_flag, lane))
+                    return false;
+                tc::fence_after_sync();
+                const bool has_j2 = next_exists && has_item(j + 2);
+                if (!ok) return false;
+                uint4 qv[16];
+                if (has_j2) fetch_q(j + 2, qv);
+                store_o(j, it);
+                if (has_j2) put_q(j + 2, qv);
+                tc::fence_before_sync();
+                __syncwarp();
+                if (lane == 0) {
+                    dev::mbar_arrive(bar(kBarOEmpty + (j & 1)));
+                    dev::mbar_arrive(bar(kBarMetaEmpty + j % kTcMeta));
+                }
+                return true;
+            };
+            if (has_item(0)) {
+                uint4 qv[16];
+                fetch_q(0, qv);
+                put_q(0, qv);
+                if (has_item(1)) {
+                    fetch_q(1, qv);
+                    put_q(1, qv);
+                }
+                for (int k = 0, gb = 0; ok; ++k) {
+                    const WorkItem it = meta[k % kTcMeta].it;
+                    const int nb = tc_blocks(it.num_pages);
+                    const int tokens = (it.num_pages - 1) * kPageSize + it.last_valid;
+                    for (int i = 0; i < nb && ok; ++i, ++gb) {
+                        ok = convert(gb, min(kTcBlockTokens, tokens - i * kTcBlockTokens));
+                        if (ok && i == 0 && k > 0) ok = finish(k - 1, true);
+                    }
+                    if (!ok) break;
+                    const bool more = has_item(k + 1);
+                    if (!ok) break;
+                    if (!more) {
+                        ok = finish(k, false);
+                        break;
+                    }
+                }
+            }
+            if (!ok && lane == 0) tc_fail(a, abort_flag, kSiteConsumerFull);
+            return;
+        }
         bool has_k = has_item(0), has_k1 = false;
         if (has_k) {
             uint4 qv[16];
@@ -1305,7 +1469,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     // the prefix pass of bf16 KV at head_dim 128 runs on tcgen05
-    constexpr bool kTcPrefix = (D == 128) && (KV::kElemBytes == 2);
+    constexpr bool kTcPrefix = D == 128;
     constexpr int kPrefixBars = kTcPrefix ? kTcBars : 2 * S::kWideStages + kIdSlots;
     static_assert(!kTcPrefix || kTcBars <= S::kBars, "barrier area holds the tcgen05 barriers");
     __shared__ TcMeta tc_meta[kTcPrefix ? kTcMeta : 1];
@@ -1316,7 +1480,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         abort_flag = 0;
         if (wide && kTcPrefix) {
-            for (int i = 0; i < kTcBars; ++i) dev::mbar_init(bars + 8 * i, tc_bar_count(i));
+            for (int i = 0; i < kTcBars; ++i)
+                dev::mbar_init(bars + 8 * i, tc_bar_count(i, KV::kElemBytes == 1));
         } else if (wide) {
             for (int s = 0; s < S::kWideStages; ++s) {
                 dev::mbar_init(bars + 8 * s, 1);
@@ -1341,7 +1506,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (wide) {
         if constexpr (kTcPrefix) {
             tc::fence_after_sync();
-            prefix_cta_tc<D>(&tmap_k, &tmap_v, a, smem, bars, tmem_base, warp, lane, &abort_flag,
+            prefix_cta_tc<D, KV>(&tmap_k, &tmap_v, a, smem, bars, tmem_base, warp, lane, &abort_flag,
                              tc_meta);
             tc::fence_before_sync();
             __syncthreads();

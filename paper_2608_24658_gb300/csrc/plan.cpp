@@ -170,8 +170,8 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                           int64_t num_phys, int32_t num_sms, bool prefill = false) {
     parason_status st = validate_config(cfg);
     if (st != PARASON_OK) return st;
-    // the prefill's causal mask is in the tcgen05 tile: bf16 at head_dim 128
-    if (prefill && (cfg->mode != PARASON_BF16 || cfg->head_dim != 128)) return PARASON_EUNSUPPORTED;
+    // the prefill's causal mask is in the tcgen05 tile: bf16 or e4m3 KV at head_dim 128
+    if (prefill && (cfg->mode == PARASON_FP32 || cfg->head_dim != 128)) return PARASON_EUNSUPPORTED;
     p->prefill = prefill;
     if (num_nodes < 0 || num_leaves < 0 || num_phys < 0) return PARASON_EINVAL;
     if (num_nodes > 0 && (!parent || !node_len || !node_page_ptr)) return PARASON_EINVAL;
@@ -349,7 +349,8 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                 run.leaf_lo = lo[n];
                 run.wide = wide;
                 run.cost_per_page =
-                    wide ? wide_page_cost(run.nrows, mode == PARASON_BF16 && cfg->head_dim == 128)
+                    // bf16 and e4m3 KV at head_dim 128 run the prefix on tcgen05
+                    wide ? wide_page_cost(run.nrows, cfg->head_dim == 128)
                          : 1.0;
                 if (wide)
                     wide_cost += run.cost_per_page * static_cast<double>(P);

@@ -23,6 +23,7 @@ def _built():
 
 
 def oracle_prefill(tree, sel=None):
+    """fp64 oracle on the host copy (e4m3 KV read with the tree's per-kv-head scales)."""
     host = tree.to("cpu")
     kw = oracle.tree_kwargs(host)
     kw["chunk_node"] = kw.pop("leaf_node")
@@ -37,9 +38,9 @@ def run(tree, sel=None, tag=""):
     return PT.compare(tree, out, lse, ref_o, ref_l, sel, tag or tree.name)
 
 
-def small(name, parent, node_len, chunks, *, hq=8, hkv=2, **kw):
+def small(name, parent, node_len, chunks, *, hq=8, hkv=2, mode="bf16", **kw):
     return W.build_prefill(name, parent, node_len, chunks, num_q_heads=hq, num_kv_heads=hkv,
-                           head_dim=128, mode="bf16", device="cuda",
+                           head_dim=128, mode=mode, device="cuda",
                            q_std=1.0 / np.sqrt(128.0) * 4, **kw)
 
 
@@ -56,6 +57,11 @@ CASES = {
     # V past each node's last token is NaN: the tile must not let it through
     "nan_tails": lambda: small("nantail", [-1, 0, 0], [45, 29, 50], [1, 2], seed=9,
                                tail_value=float("nan"), permute_pages=True, extra_pages=8),
+    # e4m3 KV (converted to f16 in the tile)
+    "fp8_join": lambda: small("join8", [-1, 0, 0, 0, 1], [300, 70, 33, 64, 41], [2, 3, 4], seed=10,
+                              mode="fp8"),
+    "fp8_g16": lambda: small("g16_8", [-1, 0, 0], [77, 40, 9], [1, 2], hq=32, hkv=2, seed=11,
+                             mode="fp8"),
 }
 
 
