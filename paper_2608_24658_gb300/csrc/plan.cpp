@@ -43,6 +43,8 @@ constexpr int32_t kAppendSlackMin = 4, kAppendSlackMax = 64;
 constexpr int kPatchesPerTail = 6;      // words one append may change per tail item
 constexpr double kWideGroupPageCost = 1.0;   // one 16-row group of one page, in suffix pages
 constexpr double kTcPageCost = 2.4;          // one page of a tcgen05 prefix tile (tuned)
+constexpr double kTcPageCostE4m3 = 4.8;      // the same with e4m3 KV, whose suffix pages
+                                             // take half the time (tuned)
 constexpr int64_t kDefaultWaitNs = 2000000000LL;
 constexpr size_t kAlign = 256;
 
@@ -53,10 +55,10 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // a prefix tile runs one 16-row MMA group of the page per warp, so a page of
 // a tile with G groups costs G suffix pages of warp time.
 //
-// The bf16 prefix tile at head_dim 128 runs on tcgen05: one 128-row MMA per
-// 64 tokens, so its pages cost about a suffix page each.
-double wide_page_cost(int32_t rows, bool tensor_core_tile) {
-    if (tensor_core_tile) return kTcPageCost;
+// The prefix tile at head_dim 128 runs on tcgen05: one 128-row MMA per 64
+// tokens, whatever the rows, at a cost measured against the suffix pass.
+double wide_page_cost(int32_t rows, bool tensor_core_tile, bool e4m3) {
+    if (tensor_core_tile) return e4m3 ? kTcPageCostE4m3 : kTcPageCost;
     const double groups = (rows + 15) / 16;
     return std::max(1.0, groups * kWideGroupPageCost);
 }
@@ -313,7 +315,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                                                : run.node_pages;
                         run.leaf_lo = qbase[c];
                         run.wide = true;
-                        run.cost_per_page = wide_page_cost(run.nrows, true);
+                        run.cost_per_page = wide_page_cost(run.nrows, true, mode == PARASON_FP8_E4M3_KV);
                         wide_cost += run.cost_per_page * static_cast<double>(run.pages);
                         runs.push_back(run);
                     }
@@ -350,7 +352,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                 run.wide = wide;
                 run.cost_per_page =
                     // bf16 and e4m3 KV at head_dim 128 run the prefix on tcgen05
-                    wide ? wide_page_cost(run.nrows, cfg->head_dim == 128)
+                    wide ? wide_page_cost(run.nrows, cfg->head_dim == 128, mode == PARASON_FP8_E4M3_KV)
                          : 1.0;
                 if (wide)
                     wide_cost += run.cost_per_page * static_cast<double>(P);
