@@ -336,6 +336,205 @@ __device__ __forceinline__ void page_step(uint32_t kbase, uint32_t vbase, int va
     }
 }
 
+// ---------------------------------------------------------------------------
+// Transposed page step for tiles of at most 8 rows (a suffix tile holds one
+// branch, g <= 8 q heads): S^T = K Q^T and O^T += V^T P^T, so that every
+// m16n8k16 MMA runs 16 tokens (or 16 output columns) against the 8 rows,
+// instead of 16 rows -- half of them padding -- against 8 tokens: half the
+// MMAs of page_step, and half its accumulators.
+//   S^T fragment: c0, c1 = token gid, rows 2tig and 2tig + 1; c2, c3 = token
+//   gid + 8.  O^T fragment of column tile dt: c0, c1 = column tcol(dt, gid),
+//   rows 2tig and 2tig + 1; c2, c3 = column tcol(dt, gid + 8).
+// The reduction index d of S^T may be permuted (the same way in K and Q); the
+// e4m3 path does so to read 4 bytes of K at a time, and picks its output
+// columns so that each lane's columns are one 16-byte chunk of V.
+// ---------------------------------------------------------------------------
+template <int D>
+struct WarpStateT {
+    float o[D / 16][4];
+    float m[2];        // rows 2tig, 2tig + 1 (equal in the 8 lanes of a tig)
+    float l[2];        // this lane's tokens; summed over the lanes at the end
+};
+
+template <int D>
+__device__ __forceinline__ void reset(WarpStateT<D> &st) {
+#pragma unroll
+    for (int dt = 0; dt < D / 16; ++dt) st.o[dt][0] = st.o[dt][1] = st.o[dt][2] = st.o[dt][3] = 0.f;
+    st.m[0] = st.m[1] = -INFINITY;
+    st.l[0] = st.l[1] = 0.f;
+}
+
+// output column of O^T row `r` (gid or gid + 8) of column tile dt
+template <class KV>
+__device__ __forceinline__ int tcol(int dt, int r) {
+    if constexpr (KV::kElemBytes == 2)
+        return dt * 16 + r;
+    else
+        return 16 * (r & 7) + 2 * dt + (r >> 3);
+}
+
+// Q^T fragments (B operand, d x 8 rows): row gid of the tile, d pairs of
+// k-step ks -- (16 ks + 2 tig, 16 ks + 8 + 2 tig) for bf16, (16 ks + 4 tig,
+// 16 ks + 4 tig + 2) widened to f16 for e4m3
+template <int D, class KV>
+__device__ __forceinline__ void load_q_fragments_t(const AttnArgs &a, const WorkItem &it, int lane,
+                                                   uint32_t (&qb)[D / 16][2]) {
+    const int gid = lane >> 2, tig = lane & 3;
+    const __nv_bfloat16 *qrow = nullptr;
+    if (gid < it.nrows) {
+        const int nr = it.row0 + gid;
+        const int leaf = a.dfs_leaf[it.leaf_lo + nr / a.group];
+        const int head = it.kv_head * a.group + nr % a.group;
+        qrow = static_cast<const __nv_bfloat16 *>(a.q) + (static_cast<int64_t>(leaf) * a.num_q_heads + head) * D;
+    }
+#pragma unroll
+    for (int ks = 0; ks < D / 16; ++ks) {
+        if constexpr (KV::kElemBytes == 2) {
+            qb[ks][0] = qrow ? *reinterpret_cast<const uint32_t *>(qrow + ks * 16 + 2 * tig) : 0u;
+            qb[ks][1] = qrow ? *reinterpret_cast<const uint32_t *>(qrow + ks * 16 + 8 + 2 * tig) : 0u;
+        } else {
+            uint2 u = make_uint2(0u, 0u);
+            if (qrow) u = *reinterpret_cast<const uint2 *>(qrow + ks * 16 + 4 * tig);
+            const __nv_bfloat162 p0 = *reinterpret_cast<const __nv_bfloat162 *>(&u.x);
+            const __nv_bfloat162 p1 = *reinterpret_cast<const __nv_bfloat162 *>(&u.y);
+            qb[ks][0] = dev::pack_f16(__low2float(p0), __high2float(p0));
+            qb[ks][1] = dev::pack_f16(__low2float(p1), __high2float(p1));
+        }
+    }
+}
+
+template <int D, class KV>
+__device__ __forceinline__ void page_step_t(uint32_t kbase, uint32_t vbase, int valid,
+                                            const uint32_t (&qb)[D / 16][2], WarpStateT<D> &st,
+                                            float scale_log2, int lane) {
+    using S = Shape<D, KV>;
+    const int gid = lane >> 2, tig = lane & 3;
+    const int mi = lane >> 3, r8 = lane & 7;
+
+    // S^T = K Q^T, two accumulators (first and second half of d)
+    float sc[4] = {0.f, 0.f, 0.f, 0.f}, sd[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int ks = 0; ks < D / 16; ++ks) {
+        float(&acc)[4] = ks < D / 32 ? sc : sd;
+        uint32_t ka[4];
+        if constexpr (KV::kElemBytes == 2) {
+            const int tok = r8 + ((mi & 1) << 3), dch = 2 * ks + (mi >> 1);
+            dev::ldsm_x4(kbase + (dch >> 3) * S::kSegBytes + dev::swz128(tok, dch & 7), ka[0], ka[1],
+                         ka[2], ka[3]);
+            dev::mma_bf16_16816(acc, ka, qb[ks][0], qb[ks][1]);
+        } else {
+            const uint32_t w0 = lds32(kbase + dev::swz128(gid, ks) + 4 * tig);
+            const uint32_t w1 = lds32(kbase + dev::swz128(gid + 8, ks) + 4 * tig);
+            ka[0] = e4m3x2_to_f16x2(w0);
+            ka[1] = e4m3x2_to_f16x2(w1);
+            ka[2] = e4m3x2_to_f16x2(w0 >> 16);
+            ka[3] = e4m3x2_to_f16x2(w1 >> 16);
+            dev::mma_f16_16816(acc, ka, qb[ks][0], qb[ks][1]);
+        }
+    }
+    float x[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const int tok = gid + ((e >> 1) << 3);
+        x[e] = tok < valid ? (sc[e] + sd[e]) * scale_log2 : -INFINITY;
+    }
+    // row maxima over the 16 tokens: the 8 lanes of a tig
+    float mx0 = fmaxf(x[0], x[2]), mx1 = fmaxf(x[1], x[3]);
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) {
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+    }
+    // (token 0 of every page of an item is valid: the maxima are finite)
+    const bool grow = mx0 > st.m[0] + kLazyRescaleLog2 || mx1 > st.m[1] + kLazyRescaleLog2;
+    if (__any_sync(0xffffffffu, grow)) {
+        const float mn0 = fmaxf(st.m[0], mx0), mn1 = fmaxf(st.m[1], mx1);
+        const float al0 = dev::fast_exp2(st.m[0] - mn0), al1 = dev::fast_exp2(st.m[1] - mn1);
+        st.m[0] = mn0;
+        st.m[1] = mn1;
+        st.l[0] *= al0;
+        st.l[1] *= al1;
+#pragma unroll
+        for (int dt = 0; dt < D / 16; ++dt) {
+            st.o[dt][0] *= al0;
+            st.o[dt][1] *= al1;
+            st.o[dt][2] *= al0;
+            st.o[dt][3] *= al1;
+        }
+    }
+    const float p0 = dev::fast_exp2(x[0] - st.m[0]), p1 = dev::fast_exp2(x[1] - st.m[1]);
+    const float p2 = dev::fast_exp2(x[2] - st.m[0]), p3 = dev::fast_exp2(x[3] - st.m[1]);
+    st.l[0] += p0 + p2;
+    st.l[1] += p1 + p3;
+    // P^T as the B operand (tokens x rows): transpose the two 8 x 8 halves
+    uint32_t pb0, pb1;
+    if constexpr (KV::kElemBytes == 2) {
+        pb0 = dev::movmatrix_trans(dev::pack_bf16(p0, p1));
+        pb1 = dev::movmatrix_trans(dev::pack_bf16(p2, p3));
+    } else {
+        pb0 = dev::movmatrix_trans(dev::pack_f16(p0, p1));
+        pb1 = dev::movmatrix_trans(dev::pack_f16(p2, p3));
+    }
+
+    // O^T += V^T P^T over the column tiles
+    if constexpr (KV::kElemBytes == 2) {
+        // slots past the node's length may hold anything (NaN included): V
+        // of those tokens is zeroed (this lane's A columns are tokens 2tig,
+        // 2tig + 1 and 2tig + 8, 2tig + 9)
+        uint32_t keep_lo = 0xffffffffu, keep_hi = 0xffffffffu;
+        if (valid < kPageSize) {
+            const int t0 = 2 * tig;
+            keep_lo = (t0 < valid ? 0x0000ffffu : 0u) | (t0 + 1 < valid ? 0xffff0000u : 0u);
+            keep_hi = (t0 + 8 < valid ? 0x0000ffffu : 0u) | (t0 + 9 < valid ? 0xffff0000u : 0u);
+        }
+        const int vtok = r8 + ((mi >> 1) << 3);
+#pragma unroll
+        for (int dt = 0; dt < D / 16; ++dt) {
+            const int dch = 2 * dt + (mi & 1);
+            uint32_t va[4];
+            dev::ldsm_x4_trans(vbase + (dch >> 3) * S::kSegBytes + dev::swz128(vtok, dch & 7), va[0],
+                               va[1], va[2], va[3]);
+            va[0] &= keep_lo;
+            va[1] &= keep_lo;
+            va[2] &= keep_hi;
+            va[3] &= keep_hi;
+            dev::mma_bf16_16816(st.o[dt], va, pb0, pb1);
+        }
+    } else {
+        static_assert(D == 128, "e4m3 KV path is written for head_dim 128");
+        // this lane's output columns are 16 gid .. 16 gid + 15: chunk gid of
+        // its four tokens 2tig, 2tig + 1, 2tig + 8, 2tig + 9
+        const int t0 = 2 * tig;
+        uint4 va = lds128(vbase + dev::swz128(t0, gid));
+        uint4 vb = lds128(vbase + dev::swz128(t0 + 1, gid));
+        uint4 vc = lds128(vbase + dev::swz128(t0 + 8, gid));
+        uint4 vd = lds128(vbase + dev::swz128(t0 + 9, gid));
+        if (valid < kPageSize) {
+            const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+            if (t0 >= valid) va = z;
+            if (t0 + 1 >= valid) vb = z;
+            if (t0 + 8 >= valid) vc = z;
+            if (t0 + 9 >= valid) vd = z;
+        }
+        const uint32_t wa[4] = {va.x, va.y, va.z, va.w}, wb[4] = {vb.x, vb.y, vb.z, vb.w};
+        const uint32_t wc[4] = {vc.x, vc.y, vc.z, vc.w}, wd[4] = {vd.x, vd.y, vd.z, vd.w};
+#pragma unroll
+        for (int dt = 0; dt < D / 16; ++dt) {
+            // columns 16 gid + 2 dt (+1): bytes b, b + 1 of word dt / 2
+            const uint32_t b = 2 * (dt & 1);
+            const uint32_t sel = b | ((4 + b) << 4) | ((b + 1) << 8) | ((5 + b) << 12);
+            const uint32_t lo = __byte_perm(wa[dt >> 1], wb[dt >> 1], sel);   // tokens 2tig, 2tig+1
+            const uint32_t hi = __byte_perm(wc[dt >> 1], wd[dt >> 1], sel);   // tokens 2tig+8, 2tig+9
+            uint32_t a4[4];
+            a4[0] = e4m3x2_to_f16x2(lo);         // column 16 gid + 2 dt
+            a4[1] = e4m3x2_to_f16x2(lo >> 16);   // column 16 gid + 2 dt + 1
+            a4[2] = e4m3x2_to_f16x2(hi);
+            a4[3] = e4m3x2_to_f16x2(hi >> 16);
+            dev::mma_f16_16816(st.o[dt], a4, pb0, pb1);
+        }
+    }
+}
+
 // Q fragments (A operand, row-major 16 x D) for tile rows rg*16 + {gid, gid+8}:
 // bf16 as stored, or widened to f16 with d permuted as the e4m3 QK^T wants.
 template <int D, class KV>
@@ -411,6 +610,37 @@ __device__ __forceinline__ void store_warp_partials(const AttnArgs &a, const Wor
             }
         }
         if (tig == 0) a.part_ml[slot] = make_float2(st.m[h], st.l[h]);
+    }
+}
+
+// The same for the transposed state: the lanes of a tig hold its two rows.
+template <int D, class KV>
+__device__ __forceinline__ void store_warp_partials_t(const AttnArgs &a, const WorkItem &it,
+                                                      WarpStateT<D> &st, int lane, float o_scale) {
+    const int gid = lane >> 2, tig = lane & 3;
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) {
+        st.l[0] += __shfl_xor_sync(0xffffffffu, st.l[0], o);
+        st.l[1] += __shfl_xor_sync(0xffffffffu, st.l[1], o);
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int r = 2 * tig + h;
+        if (r >= it.nrows) continue;
+        const int64_t slot = static_cast<int64_t>(it.slot_base) + r;
+        float *dst = a.part_o + slot * D;
+#pragma unroll
+        for (int dt = 0; dt < D / 16; ++dt) {
+            if constexpr (KV::kElemBytes == 2) {
+                dst[tcol<KV>(dt, gid)] = st.o[dt][h];
+                dst[tcol<KV>(dt, gid + 8)] = st.o[dt][2 + h];
+            } else {
+                // columns 16 gid + 2 dt and the next: one pair
+                *reinterpret_cast<float2 *>(dst + tcol<KV>(dt, gid)) =
+                    make_float2(st.o[dt][h] * o_scale, st.o[dt][2 + h] * o_scale);
+            }
+        }
+        if (gid == 0) a.part_ml[slot] = make_float2(st.m[h], st.l[h]);
     }
 }
 
@@ -542,6 +772,30 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
         __syncwarp();
         const WorkItem it = grab[k % kGrabSlots];
         const float2 scl = item_scales<KV>(a, it);
+        if (it.nrows <= 8) {
+            // one branch: the transposed step
+            uint32_t qb[D / 16][2];
+            load_q_fragments_t<D, KV>(a, it, lane, qb);
+            WarpStateT<D> st;
+            reset<D>(st);
+            for (int pg = 0; pg < it.num_pages; ++pg, ++consumed) {
+                const int s = consumed % NS;
+                if (!dev::mbar_wait_bounded(my_bar + s * 8, (consumed / NS) & 1, a.wait_limit_ns,
+                                            nullptr)) {
+                    ok = false;
+                    break;
+                }
+                const int valid = (pg == it.num_pages - 1) ? it.last_valid : kPageSize;
+                page_step_t<D, KV>(my_ring + s * S::kStageBytes,
+                                   my_ring + s * S::kStageBytes + S::kPageBytes, valid, qb, st, scl.x,
+                                   lane);
+                __syncwarp();
+                issue_next();
+            }
+            if (!ok) break;
+            store_warp_partials_t<D, KV>(a, it, st, lane, scl.y);
+            continue;
+        }
         uint32_t qa[D / 16][4];
         load_q_fragments<D, KV>(a, it, 0, lane, qa);
         WarpState<D> st;
