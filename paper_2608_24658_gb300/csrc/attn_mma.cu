@@ -1439,13 +1439,21 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                 tc::ld32(tS, sr[0]);
                 tc::ld32(tS + 32, sr[1]);
                 tc::wait_ld();
+                // raw scores; keys the row does not see (past the item's last
+                // token, or past the row's own token in a causal item) -inf
                 float x[64];
-                float mb = -INFINITY;
 #pragma unroll
-                for (int j = 0; j < 64; ++j) {
-                    x[j] = j < seen ? __uint_as_float(sr[j >> 5][j & 31]) * sl : -INFINITY;
-                    mb = fmaxf(mb, x[j]);
+                for (int j = 0; j < 64; ++j) x[j] = __uint_as_float(sr[j >> 5][j & 31]);
+                if (seen < kTcBlockTokens) {
+#pragma unroll
+                    for (int j = 0; j < 64; ++j) x[j] = j < seen ? x[j] : -INFINITY;
                 }
+                // the block's max in the log2 domain (sl > 0)
+                float mr = x[0];
+#pragma unroll
+                for (int j = 1; j + 1 < 64; j += 2) mr = dev::max3(mr, x[j], x[j + 1]);
+                mr = fmaxf(mr, x[63]);
+                const float mb = mr * sl;
                 if (i == 0) {
                     m_use = mb;
                 } else if (__any_sync(0xffffffffu, mb > m_use + kTcRescaleLog2)) {
@@ -1475,13 +1483,23 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                 // P = 2^(x - m) as bf16 pairs over the first 32 columns of S
                 // (0 for a row that has seen no key: every x is -inf)
                 const float m_ref = m_use == -INFINITY ? 0.f : m_use;
+                // 2^(x sl - m) with pairs of fp32 lanes: one packed FMA per
+                // two exponents, and two running sums
+                const unsigned long long slp = dev::f32x2(sl, sl), nmp = dev::f32x2(-m_ref, -m_ref);
+                unsigned long long lsum = dev::f32x2(0.f, 0.f);
                 uint32_t pw[32];
 #pragma unroll
                 for (int c = 0; c < 32; ++c) {
-                    const float p0 = dev::fast_exp2(x[2 * c] - m_ref);
-                    const float p1 = dev::fast_exp2(x[2 * c + 1] - m_ref);
-                    l += p0 + p1;
+                    float e0, e1;
+                    dev::f32x2_split(dev::fma_f32x2(dev::f32x2(x[2 * c], x[2 * c + 1]), slp, nmp), e0, e1);
+                    const float p0 = dev::fast_exp2(e0), p1 = dev::fast_exp2(e1);
+                    lsum = dev::add_f32x2(lsum, dev::f32x2(p0, p1));
                     pw[c] = kF8 ? dev::pack_f16(p0, p1) : dev::pack_bf16(p0, p1);
+                }
+                {
+                    float l0, l1;
+                    dev::f32x2_split(lsum, l0, l1);
+                    l += l0 + l1;
                 }
                 tc::st32(tS, pw);
                 tc::wait_st();
