@@ -1077,7 +1077,7 @@ constexpr int kTcTmemCols = 512;
 constexpr uint32_t kTmemO = 0, kTmemS = 256, kTmemQ = 384;    // TMEM column bases
 constexpr float kTcRescaleLog2 = 8.f;                         // lazy rescale threshold
 constexpr int kTcMeta = 4;                                    // item metadata slots
-constexpr int kTcMetaPages = 128;                             // pages of one item at most
+constexpr int kTcMetaPages = 512;                             // pages of one item at most
 constexpr int kTcSoftmaxWarps = 4;                            // warps 0-3
 constexpr int kTcEpilogueWarp = 4;                            // warps 4-7
 constexpr int kTcProducerWarp = 8;

@@ -34,6 +34,10 @@ constexpr int kNarrowRows = 16;         // nodes with at most this many rows: su
 int32_t narrow_warps(int32_t mode) { return mode == PARASON_FP8_E4M3_KV ? 12 : 8; }
 constexpr int kMinPiecePages = 8;       // suffix-pass pieces are at least this long
 constexpr int kMaxPiecePages = 128;     // and at most this long
+// Prefill pieces may be longer: the tile is compute-bound there, and every
+// piece costs a 64 KB partial (written, then read by the merge).  The
+// tcgen05 tile holds an item of up to 512 pages.
+constexpr int kMaxPrefillPiecePages = 512;
 constexpr int kWideBlockPages = 4;      // prefix pieces are whole 64-token blocks
 constexpr double kWideProvision = 1.15; // prefix CTAs relative to the cost model
 constexpr int kFp32ChunkPages = 32;
@@ -443,7 +447,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         for (const Run &r : runs)
             if (r.wide) wide_pages += r.pages;
         const int64_t wide_chunk = std::min<int64_t>(
-            kMaxPiecePages,
+            prefill ? kMaxPrefillPiecePages : kMaxPiecePages,
             std::max<int64_t>(kWideBlockPages,
                               wide_pages / std::max<int64_t>(1, static_cast<int64_t>(n_wide) * 3)));
         // The row tiles of one (node, kv head) read the same pages: their
