@@ -220,6 +220,99 @@ __global__ void __launch_bounds__(kMergeThreads)
     if (a.lse && lane == 0) a.lse[row] = empty ? -INFINITY : (M + log2f(L)) * kLn2;
 }
 
+// Many rows: one warp per (branch, kv head).  The kv head's G q heads share
+// its merge list (q head j G + r reads slot entry + r), so the warp reads the
+// list once and keeps the G rows' loads in flight together; per pass of up to
+// 32 entries, every row's weights come from warp reductions as above, then
+// the partial rows are requested 8 at a time over entries and heads.
+template <int D, int G>
+__global__ void __launch_bounds__(kMergeThreads)
+    tree_merge_group_kernel(const MergeArgs a, bool out_bf16) {
+    constexpr int N = Vec<D>::N;
+    constexpr int KB = G >= 8 ? 1 : 8 / G;          // entries per batch of loads
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t pair = static_cast<int64_t>(blockIdx.x) * (kMergeThreads / 32) + warp;
+    const bool active = pair < static_cast<int64_t>(a.num_leaves) * a.num_kv_heads;
+    // the merge lists are plan data: read them while the attention grid drains
+    const int e0 = active ? a.merge_ptr[pair] : 0, e1 = active ? a.merge_ptr[pair + 1] : 0;
+    const int first_slot = e0 + lane < e1 ? a.merge_ent[e0 + lane] : 0;
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    // the attention grid is complete: rewind its work queues for the next call
+    if (blockIdx.x == 0 && threadIdx.x == 0 && a.queue_next) {
+        a.queue_next[0] = a.queue_start[0];
+        a.queue_next[1] = a.queue_start[1];
+    }
+    if (!active) return;
+
+    float M[G], L[G], acc[G][N];
+#pragma unroll
+    for (int r = 0; r < G; ++r) {
+        M[r] = -INFINITY;
+        L[r] = 0.f;
+#pragma unroll
+        for (int c = 0; c < N; ++c) acc[r][c] = 0.f;
+    }
+    for (int i0 = 0; e0 + i0 < e1; i0 += 32) {
+        const int e = e0 + i0 + lane;
+        const bool valid = e < e1;
+        const int slot = valid ? (i0 == 0 ? first_slot : a.merge_ent[e]) : 0;
+        const int cnt = min(32, e1 - e0 - i0);
+        float wgt[G];
+#pragma unroll
+        for (int r = 0; r < G; ++r) {
+            float m = -INFINITY, l = 0.f;
+            if (valid) {
+                const float2 ml = a.part_ml[slot + r];
+                m = ml.x;
+                l = ml.y;
+            }
+            float mb = m;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) mb = fmaxf(mb, __shfl_xor_sync(0xffffffffu, mb, o));
+            const float Mn = fmaxf(M[r], mb);       // finite: the pass has a valid entry
+            const float s_old = exp2f(M[r] - Mn);
+            wgt[r] = valid ? exp2f(m - Mn) : 0.f;
+            float lw = l * wgt[r];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) lw += __shfl_xor_sync(0xffffffffu, lw, o);
+            L[r] = L[r] * s_old + lw;
+#pragma unroll
+            for (int c = 0; c < N; ++c) acc[r][c] *= s_old;
+            M[r] = Mn;
+        }
+        for (int k0 = 0; k0 < cnt; k0 += KB) {
+            float v[KB][G][N];
+#pragma unroll
+            for (int k = 0; k < KB; ++k) {
+                const int si = __shfl_sync(0xffffffffu, slot, (k0 + k) & 31);
+#pragma unroll
+                for (int r = 0; r < G; ++r)
+                    if (k0 + k < cnt)
+                        load_f32<N>(a.part_o + static_cast<int64_t>(si + r) * D + lane * N, v[k][r]);
+            }
+#pragma unroll
+            for (int k = 0; k < KB; ++k)
+#pragma unroll
+                for (int r = 0; r < G; ++r) {
+                    const float wk = __shfl_sync(0xffffffffu, wgt[r], (k0 + k) & 31);
+                    if (k0 + k < cnt)
+#pragma unroll
+                        for (int c = 0; c < N; ++c) acc[r][c] += wk * v[k][r][c];
+                }
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < G; ++r) {
+        const int64_t row = pair * G + r;            // b * H_q + j * G + r
+        const bool empty = !(L[r] > 0.f);
+        const float inv = empty ? 0.f : 1.f / L[r];
+#pragma unroll
+        for (int c = 0; c < N; ++c) acc[r][c] *= inv;
+        store_out<N>(a.out, row * D + lane * N, acc[r], out_bf16);
+        if (a.lse && lane == 0) a.lse[row] = empty ? -INFINITY : (M[r] + log2f(L[r])) * kLn2;
+    }
+}
+
 template <int D>
 __global__ void __launch_bounds__(kMergeThreads)
     lse_merge_kernel(const void *o_a, const float *lse_a, const void *o_b, const float *lse_b,
@@ -256,9 +349,15 @@ cudaError_t launch_merge(const MergeArgs &a, int head_dim, int mode, bool progra
                          cudaStream_t stream) {
     const int64_t rows = static_cast<int64_t>(a.num_leaves) * a.num_q_heads;
     if (rows == 0) return cudaSuccess;
-    // warps per row: as many as keep the grid near 4096 warps, at most 4
+    // warps per row: as many as keep the grid near 4096 warps, at most 4.
+    // With at least 4096 (branch, kv head) pairs and groups of 2 or 4, one
+    // warp per pair (measured: faster there; with groups of 8, or fewer
+    // pairs, too few warps are left to hide the loads' latency)
     const int W = rows * 4 <= 4096 ? 4 : (rows * 2 <= 4096 ? 2 : 1);
-    const int64_t blocks = (rows * W + kMergeThreads / 32 - 1) / (kMergeThreads / 32);
+    const int g = a.group;
+    const bool grouped = W < 4 && (g == 2 || g == 4) && rows / g >= 4096;
+    const int64_t warps = grouped ? rows / g : rows * W;
+    const int64_t blocks = (warps + kMergeThreads / 32 - 1) / (kMergeThreads / 32);
     if (blocks > 0x7fffffff) return cudaErrorInvalidValue;
     const bool bf16 = mode != PARASON_FP32;
     cudaLaunchConfig_t cfg = {};
@@ -271,6 +370,15 @@ cudaError_t launch_merge(const MergeArgs &a, int head_dim, int mode, bool progra
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = programmatic ? 1 : 0;
+    if (grouped) {
+        if (head_dim == 128)
+            return g == 2 ? cudaLaunchKernelEx(&cfg, tree_merge_group_kernel<128, 2>, a, bf16)
+                          : cudaLaunchKernelEx(&cfg, tree_merge_group_kernel<128, 4>, a, bf16);
+        if (head_dim == 64)
+            return g == 2 ? cudaLaunchKernelEx(&cfg, tree_merge_group_kernel<64, 2>, a, bf16)
+                          : cudaLaunchKernelEx(&cfg, tree_merge_group_kernel<64, 4>, a, bf16);
+        return cudaErrorNotSupported;
+    }
     if (head_dim == 128) {
         if (W == 4) return cudaLaunchKernelEx(&cfg, tree_merge_kernel<128, 4>, a, bf16);
         if (W == 2) return cudaLaunchKernelEx(&cfg, tree_merge_kernel<128, 2>, a, bf16);

@@ -65,6 +65,18 @@ def test_fixture_parity(name, mode):
     PT.run_and_compare(tree, tag=f"{name}/{mode}")
 
 
+@pytest.mark.parametrize("d", [64, 128])
+def test_many_branches_grouped_merge(d):
+    # 2048 branches x 2 kv heads: 4096 (branch, kv head) pairs with g = 2 take
+    # the merge kernel that serves every q head of a pair from one warp
+    rng = np.random.default_rng(12)
+    lens = [300] + [int(x) for x in rng.integers(1, 40, 2048)]
+    tree = W.build_tree("many", [-1] + [0] * 2048, lens, list(range(1, 2049)), num_q_heads=4,
+                        num_kv_heads=2, head_dim=d, mode="bf16", seed=12, device="cuda",
+                        tail_value=float("nan"))
+    PT.run_and_compare(PT.nan_fill_unused_pages(tree), tag=f"many_branches_d{d}")
+
+
 def test_empty_path_gives_zero_and_neg_inf():
     tree = W.build_tree("empty", [-1, 0, 0], [0, 0, 5], [1, 2], num_q_heads=4, num_kv_heads=2,
                         head_dim=64, seed=2, device="cuda")
