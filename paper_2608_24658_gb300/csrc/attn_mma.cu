@@ -1025,8 +1025,8 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
 
 
 // ---------------------------------------------------------------------------
-// prefix pass on tcgen05 (bf16 KV, head_dim 128): a tile of up to 128 stacked
-// rows against 64-token blocks (4 pages) of the node's pages
+// prefix pass on tcgen05 (bf16 or e4m3 KV, head_dim 128): a tile of up to 128
+// stacked rows against 64-token blocks (4 pages) of the node's pages
 //
 //   warp 10     scheduler: pulls items from the prefix queue and stages each
 //               one's metadata (the item, the TMA row of each page, the
@@ -1045,17 +1045,19 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
 //               tcgen05.commit releases ring stages and signals completion.
 //   warps 0-3   softmax: thread r owns row r (TMEM lane r); online softmax in
 //               the log2 domain with a lazy rescale of O (only when a row's
-//               max grows by more than 2^8); P (bf16) overwrites the first 32
-//               columns of its S buffer, the A operand of PV; writes the
-//               row's (m, l) at the end of an item
+//               max grows by more than 2^8); P (bf16, f16 with e4m3 KV)
+//               overwrites the first 32 columns of its S buffer, the A
+//               operand of PV; writes the row's (m, l) at the end of an item
 //   warps 4-7   epilogue: once an item's O is complete, stores its rows to the
 //               partials and loads the Q rows of the item two ahead into the
-//               TMEM Q buffer that item frees (Q of items 0 and 1 at start)
+//               TMEM Q buffer that item frees (Q of items 0 and 1 at start);
+//               with e4m3 KV they also convert every staged block to f16
 //
 // TMEM, 512 columns: O[2] at 0 and 128, S/P[2] at 256 and 320, Q[2] at 384
 // and 448.  Shared memory: the ring [6][K: 2 col blocks x 64 tokens x 128 B |
 // V: same], 128-byte swizzled (K-major descriptors for K, MN-major for V),
-// and the metadata slots.
+// and the metadata slots; with e4m3 KV the first half of the ring stages the
+// raw blocks (6 x 16 KB) and the second half holds 3 converted f16 blocks.
 // ---------------------------------------------------------------------------
 constexpr int kTcRows = 128;
 constexpr int kTcBlockPages = 4;
@@ -1741,7 +1743,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool wide = static_cast<int>(blockIdx.x) < a.num_wide_ctas;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-    // the prefix pass of bf16 KV at head_dim 128 runs on tcgen05
+    // the prefix pass at head_dim 128 (bf16 or e4m3 KV) runs on tcgen05
     constexpr bool kTcPrefix = D == 128;
     constexpr int kPrefixBars = kTcPrefix ? kTcBars : 2 * S::kWideStages + kIdSlots;
     static_assert(!kTcPrefix || kTcBars <= S::kBars, "barrier area holds the tcgen05 barriers");
