@@ -1267,32 +1267,33 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                     ok = false;
                     break;
                 }
-                if (lane == 0 && !(skip_first && blk == 0)) {
+                if (!(skip_first && blk == 0)) {
+                    // the block's boxes are issued by one lane each (one
+                    // thread issuing them all was the tile's bottleneck); the
+                    // expected bytes are registered first
                     const uint32_t fb = bar(kBarKvFull + s);
+                    if (lane == 0)
+                        dev::mbar_arrive_expect_tx(fb, kF8 ? kTcF8StageBytes : kTcStageBytes);
+                    __syncwarp();
                     if constexpr (kF8) {
-                        // raw e4m3 rows: one 2 KB box per page of K and of V
-                        const uint32_t st = ring + s * kTcF8StageBytes;
-                        dev::mbar_arrive_expect_tx(fb, kTcF8StageBytes);
-#pragma unroll
-                        for (int j = 0; j < kTcBlockPages; ++j) {
+                        // raw e4m3 rows: one 2 KB box per page of K (even lanes) and of V
+                        if (lane < 2 * kTcBlockPages) {
+                            const int j = lane >> 1;
                             const int pg = bi * kTcBlockPages + j;
                             const int row = pg < np ? m.rows[pg] : a.kv_rows;   // kv_rows: zero fill
-                            dev::tma_load_3d(st + j * kPageSize * 128, tmap_k, 0, 0, row, fb);
-                            dev::tma_load_3d(st + kTcF8Bytes + j * kPageSize * 128, tmap_v, 0, 0, row, fb);
+                            const uint32_t st = ring + s * kTcF8StageBytes + (lane & 1) * kTcF8Bytes;
+                            dev::tma_load_3d(st + j * kPageSize * 128, (lane & 1) ? tmap_v : tmap_k, 0, 0,
+                                             row, fb);
                         }
                     } else {
-                        const uint32_t st = ring + s * kTcStageBytes;
-                        dev::mbar_arrive_expect_tx(fb, kTcStageBytes);
-#pragma unroll
-                        for (int j = 0; j < kTcBlockPages; ++j) {
+                        // page j = lane / 4, column block (lane / 2) % 2, K (even lanes) or V
+                        if (lane < 4 * kTcBlockPages) {
+                            const int j = lane >> 2, cb = (lane >> 1) & 1;
                             const int pg = bi * kTcBlockPages + j;
                             const int row = pg < np ? m.rows[pg] : a.kv_rows;   // kv_rows: zero fill
-#pragma unroll
-                            for (int cb = 0; cb < 2; ++cb) {
-                                const uint32_t off = cb * kTcColBlockBytes + j * kPageSize * 128;
-                                dev::tma_load_3d(st + off, tmap_k, 0, cb, row, fb);
-                                dev::tma_load_3d(st + kTcKBytes + off, tmap_v, 0, cb, row, fb);
-                            }
+                            const uint32_t off = cb * kTcColBlockBytes + j * kPageSize * 128;
+                            const uint32_t st = ring + s * kTcStageBytes + (lane & 1) * kTcKBytes;
+                            dev::tma_load_3d(st + off, (lane & 1) ? tmap_v : tmap_k, 0, cb, row, fb);
                         }
                     }
                     last_issue[s] = blk;
