@@ -54,11 +54,22 @@ constexpr int kIdSlots = 8;      // prefix-pass item ids in flight from producer
 constexpr int kGrabSlots = 8;    // suffix-pass item ids a warp has pulled but not finished
 constexpr float kLazyRescaleLog2 = 8.f;   // mma.sync softmax: move the reference max past 2^8
 
+// KV formats, with the number of suffix-pass warps per CTA (each with a
+// private ring; the 192 KB of rings is split between them).  An e4m3 page
+// costs more issue per byte (widening to f16), so that pass runs more,
+// shallower warps; bf16 with few rows per tile (g <= 4) runs fewer, deeper
+// ones, whose extra pages in flight shorten the tail of the launch.
 struct KvBf16 {
     static constexpr int kElemBytes = 2;
+    static constexpr int kSuffixWarps = 8;
+};
+struct KvBf16Deep {
+    static constexpr int kElemBytes = 2;
+    static constexpr int kSuffixWarps = 6;
 };
 struct KvE4m3 {
     static constexpr int kElemBytes = 1;
+    static constexpr int kSuffixWarps = 12;
 };
 
 template <int D, class KV>
@@ -71,9 +82,8 @@ struct Shape {
     static constexpr int kSegBytes = kPageSize * 128;
     static constexpr int kStageBytes = 2 * kPageBytes;      // K and V of one page
 
-    // suffix pass: a private ring per warp.  An e4m3 page costs more issue
-    // per byte (widening to f16), so that pass runs more, shallower warps.
-    static constexpr int kSuffixWarps = KV::kElemBytes == 1 ? 12 : 8;
+    // suffix pass: a private ring per warp
+    static constexpr int kSuffixWarps = KV::kSuffixWarps;
     static constexpr int kWarpStages = (192 * 1024) / (kSuffixWarps * kStageBytes);
     static constexpr int kWarpRingBytes = kWarpStages * kStageBytes;
     static constexpr int kNarrowBytes = kSuffixWarps * kWarpRingBytes;
@@ -1086,6 +1096,7 @@ constexpr int kTcProducerWarp = 8;
 constexpr int kTcMmaWarp = 9;
 constexpr int kTcSchedulerWarp = 10;
 static_assert(kTcRingBytes <= Shape<128, KvBf16>::kBodyBytes, "tcgen05 ring fits the CTA's memory");
+static_assert(kTcRingBytes <= Shape<128, KvBf16Deep>::kBodyBytes, "tcgen05 ring fits the CTA's memory");
 static_assert(kTcRingBytes <= Shape<128, KvE4m3>::kBodyBytes, "tcgen05 ring fits the CTA's memory");
 static_assert(kTcSchedulerWarp < kThreads / 32, "every tcgen05 role has a warp");
 static_assert(kMaxSuffixWarps <= kThreads / 32, "every suffix-pass warp exists");
@@ -1854,7 +1865,11 @@ cudaError_t launch(const AttnArgs &a, const CUtensorMap &tk, const CUtensorMap &
 cudaError_t attn_mma_ctas_per_sm(int head_dim, int mode, int *ctas_per_sm) {
     if (mode == PARASON_FP8_E4M3_KV)
         return head_dim == 128 ? configure<128, KvE4m3>(ctas_per_sm) : cudaErrorNotSupported;
-    if (head_dim == 128) return configure<128, KvBf16>(ctas_per_sm);
+    if (head_dim == 128) {
+        const cudaError_t e = configure<128, KvBf16Deep>(nullptr);
+        if (e != cudaSuccess) return e;
+        return configure<128, KvBf16>(ctas_per_sm);
+    }
     if (head_dim == 64) return configure<64, KvBf16>(ctas_per_sm);
     return cudaErrorNotSupported;
 }
@@ -1862,7 +1877,9 @@ cudaError_t attn_mma_ctas_per_sm(int head_dim, int mode, int *ctas_per_sm) {
 cudaError_t launch_attn_bf16(const AttnArgs &a, const CUtensorMap &tk, const CUtensorMap &tv,
                              int head_dim, cudaStream_t stream) {
     if (a.num_items <= 0 || a.num_ctas <= 0) return cudaSuccess;
-    if (head_dim == 128) return launch<128, KvBf16>(a, tk, tv, stream);
+    if (head_dim == 128)
+        return a.suffix_warps == KvBf16Deep::kSuffixWarps ? launch<128, KvBf16Deep>(a, tk, tv, stream)
+                                                          : launch<128, KvBf16>(a, tk, tv, stream);
     if (head_dim == 64) return launch<64, KvBf16>(a, tk, tv, stream);
     return cudaErrorNotSupported;
 }

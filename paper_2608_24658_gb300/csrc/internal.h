@@ -88,6 +88,7 @@ struct AttnArgs {
     // tree-masked prefill: per item, the token index (in its node) of its
     // first key when the item is causal, else -1; null for decode plans
     const int32_t *item_key0;
+    int32_t suffix_warps;   // suffix-pass warps per CTA the plan was made for
 };
 
 struct MergeArgs {

@@ -31,7 +31,12 @@ namespace {
 
 constexpr int kNarrowRows = 16;         // nodes with at most this many rows: suffix pass
 // autonomous warps per suffix-pass CTA (the kernel's count for the KV format)
-int32_t narrow_warps(int32_t mode) { return mode == PARASON_FP8_E4M3_KV ? 12 : 8; }
+// (the kernel's count for the KV format: 6 deeper warps for bf16 at head_dim
+// 128 with g <= 4, where they are latency-bound)
+int32_t narrow_warps(int32_t mode, int32_t head_dim, int32_t g) {
+    if (mode == PARASON_FP8_E4M3_KV) return 12;
+    return (mode == PARASON_BF16 && head_dim == 128 && g <= 4) ? 6 : 8;
+}
 constexpr int kMinPiecePages = 8;       // suffix-pass pieces are at least this long
 constexpr int kMaxPiecePages = 128;     // and at most this long
 // Prefill pieces may be longer: the tile is compute-bound there, and every
@@ -104,6 +109,7 @@ struct parason_plan_s {
     std::vector<uint8_t> page_used;    // physical pages some node owns
     int32_t num_ctas = 0;
     int32_t num_wide_ctas = 0;
+    int32_t suffix_warps = 8;          // suffix-pass warps per CTA (kernel instantiation)
     int64_t num_slots = 0;
     int64_t unique_tokens = 0;
     int64_t path_tokens = 0;
@@ -391,7 +397,8 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     // the kernel's CTAs own the first positions of each queue (one per
     // prefix CTA, one per warp of a suffix CTA); the counters start past them
     p->queue_start[0] = n_wide;
-    p->queue_start[1] = n_narrow_ctas * narrow_warps(mode);
+    p->suffix_warps = narrow_warps(mode, cfg->head_dim, g);
+    p->queue_start[1] = n_narrow_ctas * p->suffix_warps;
 
     // Items: every run cut into pieces of at most `chunk` pages (the prefix
     // pass in whole 64-token blocks).  Each role's pieces form a queue,
@@ -439,7 +446,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         for (const Run &r : runs)
             if (!cut(r, kFp32ChunkPages, 1)) return PARASON_EUNSUPPORTED;
     } else {
-        const int64_t total_warps = static_cast<int64_t>(p->num_sms) * narrow_warps(mode);
+        const int64_t total_warps = static_cast<int64_t>(p->num_sms) * p->suffix_warps;
         const int64_t narrow_chunk = std::min<int64_t>(
             kMaxPiecePages,
             std::max<int64_t>(kMinPiecePages, narrow_pages / std::max<int64_t>(1, total_warps * 3)));
@@ -895,6 +902,7 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
         a.num_wide_ctas = p->num_wide_ctas;
         a.kv_rows = static_cast<int32_t>(p->num_phys * p->cfg.num_kv_heads * parason::kPageSize);
         a.item_key0 = p->d_item_key0;
+        a.suffix_warps = p->suffix_warps;
         cudaError_t e;
         if (p->cfg.mode == PARASON_FP32) {
             e = parason::launch_attn_fp32(a, static_cast<const float *>(k_pages),
