@@ -180,9 +180,13 @@ size_t parason_plan_workspace_bytes(parason_plan plan);
  *   v_pages  device, same layout and dtype as k_pages
  *   k_scale, v_scale  device fp32 [H_kv] in FP8 mode (k = e4m3 * k_scale),
  *            ignored otherwise (may be NULL)
- *   out      device, [num_leaves, H_q, head_dim], dtype of q
- *   lse      device fp32 [num_leaves, H_q] or NULL.  A branch whose whole
- *            path holds no token gets out = 0 and lse = -inf.
+ *   out      device, [num_leaves, H_q, head_dim], dtype of q, 16-byte
+ *            aligned; or page-locked host memory the device can address
+ *            (cudaHostAlloc / cudaHostRegister): the merge kernel then
+ *            writes the result straight to the host
+ *   lse      device (or such host memory) fp32 [num_leaves, H_q], or NULL.
+ *            A branch whose whole path holds no token gets out = 0 and
+ *            lse = -inf.
  *   workspace  device, at least parason_plan_workspace_bytes(plan) bytes,
  *            256-byte aligned; no contents are kept between calls.
  *

@@ -165,7 +165,9 @@ class Plan:
                out: Optional[torch.Tensor] = None, lse: Optional[torch.Tensor] = None,
                workspace: Optional[torch.Tensor] = None, k_scale=None, v_scale=None,
                stream=None, want_lse: bool = True):
-        """One decode step; returns (out, lse).  Asynchronous on ``stream``."""
+        """One decode step; returns (out, lse).  Asynchronous on ``stream``.
+        ``out`` and ``lse`` may be pinned host tensors: the merge kernel then
+        writes the result straight to host memory."""
         L, Hq, Hkv, d = self.num_leaves, self.num_q_heads, self.num_kv_heads, self.head_dim
         qd, kvd = _Q_DTYPES[self.mode], _KV_DTYPES[self.mode]
         if q.dtype != qd or tuple(q.shape) != (L, Hq, d) or not q.is_cuda or not q.is_contiguous():

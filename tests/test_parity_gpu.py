@@ -77,6 +77,18 @@ def test_many_branches_grouped_merge(d):
     PT.run_and_compare(PT.nan_fill_unused_pages(tree), tag=f"many_branches_d{d}")
 
 
+def test_result_written_to_pinned_host_memory():
+    # out and lse in page-locked host memory: the merge kernel stores there
+    tree = W.make_config(2, device="cuda")
+    with Plan.for_tree(tree) as plan:
+        ref_o, ref_l = plan.decode_tree(tree)
+        out_h = torch.empty(tuple(ref_o.shape), dtype=ref_o.dtype).pin_memory()
+        lse_h = torch.empty(tuple(ref_l.shape), dtype=ref_l.dtype).pin_memory()
+        plan.decode_tree(tree, out=out_h, lse=lse_h)
+        plan.check()
+    assert torch.equal(out_h, ref_o.cpu()) and torch.equal(lse_h, ref_l.cpu())
+
+
 def test_empty_path_gives_zero_and_neg_inf():
     tree = W.build_tree("empty", [-1, 0, 0], [0, 0, 5], [1, 2], num_q_heads=4, num_kv_heads=2,
                         head_dim=64, seed=2, device="cuda")
