@@ -174,7 +174,9 @@ size_t parason_plan_workspace_bytes(parason_plan plan);
  * One decode step: out[b, h, :] = softmax(s) V over branch b's root->leaf KV.
  * Asynchronous on `stream`; allocates nothing; capturable in a CUDA graph.
  *
- *   q        device, [num_leaves, H_q, head_dim], bf16 (fp32 in FP32 mode)
+ *   q        device, [num_leaves, H_q, head_dim], bf16 (fp32 in FP32 mode),
+ *            16-byte aligned; or page-locked host memory the device can
+ *            address (cudaHostAlloc / cudaHostRegister), read in place
  *   k_pages  device, [num_physical_pages, H_kv, 16, head_dim], bf16 / fp32 /
  *            e4m3 bytes by mode, 16-byte aligned
  *   v_pages  device, same layout and dtype as k_pages

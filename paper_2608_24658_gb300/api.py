@@ -166,24 +166,30 @@ class Plan:
                workspace: Optional[torch.Tensor] = None, k_scale=None, v_scale=None,
                stream=None, want_lse: bool = True):
         """One decode step; returns (out, lse).  Asynchronous on ``stream``.
-        ``out`` and ``lse`` may be pinned host tensors: the merge kernel then
-        writes the result straight to host memory."""
+        ``q``, ``out`` and ``lse`` may be pinned host tensors: the kernels
+        then read q from, and write the result to, host memory directly."""
         L, Hq, Hkv, d = self.num_leaves, self.num_q_heads, self.num_kv_heads, self.head_dim
         qd, kvd = _Q_DTYPES[self.mode], _KV_DTYPES[self.mode]
-        if q.dtype != qd or tuple(q.shape) != (L, Hq, d) or not q.is_cuda or not q.is_contiguous():
-            raise ValueError(f"q must be a contiguous cuda {qd} tensor of shape {(L, Hq, d)}")
+        if (q.dtype != qd or tuple(q.shape) != (L, Hq, d) or not q.is_contiguous()
+                or not (q.is_cuda or q.is_pinned())):
+            raise ValueError(f"q must be a contiguous cuda (or pinned host) {qd} tensor of "
+                             f"shape {(L, Hq, d)}")
+        dev = k_pages.device
         for name, t in (("k_pages", k_pages), ("v_pages", v_pages)):
             if (t.dtype != kvd or t.dim() != 4 or tuple(t.shape[1:]) != (Hkv, 16, d)
                     or t.shape[0] < self.num_physical_pages or not t.is_contiguous()
-                    or t.device != q.device):
-                raise ValueError(f"{name} must be a contiguous {kvd} tensor "
-                                 f"[>= {self.num_physical_pages}, {Hkv}, 16, {d}] on {q.device}")
+                    or not t.is_cuda or t.device != dev):
+                raise ValueError(f"{name} must be a contiguous cuda {kvd} tensor "
+                                 f"[>= {self.num_physical_pages}, {Hkv}, 16, {d}] on one device")
+        if q.is_cuda and q.device != dev:
+            raise ValueError(f"q must be on {dev}")
         if out is None:
-            out = torch.empty_like(q)
+            out = torch.empty_like(q) if q.is_cuda else torch.empty(q.shape, dtype=q.dtype).pin_memory()
         if lse is None and want_lse:
-            lse = torch.empty((L, Hq), dtype=torch.float32, device=q.device)
+            lse = (torch.empty((L, Hq), dtype=torch.float32, device=dev) if q.is_cuda else
+                   torch.empty((L, Hq), dtype=torch.float32).pin_memory())
         if workspace is None:
-            workspace = self.workspace(q.device)
+            workspace = self.workspace(dev)
         if self.mode == "fp8":
             if k_scale is None or v_scale is None:
                 raise ValueError("fp8 mode needs k_scale and v_scale")

@@ -77,16 +77,23 @@ def test_many_branches_grouped_merge(d):
     PT.run_and_compare(PT.nan_fill_unused_pages(tree), tag=f"many_branches_d{d}")
 
 
-def test_result_written_to_pinned_host_memory():
-    # out and lse in page-locked host memory: the merge kernel stores there
-    tree = W.make_config(2, device="cuda")
+@pytest.mark.parametrize("mode", ["bf16", "fp8"])
+def test_host_memory_q_and_result(mode):
+    # q, out and lse in page-locked host memory: the kernels read and store
+    # there directly; bit-identical to device buffers
+    tree = W.make_config(2, mode=mode, device="cuda")
     with Plan.for_tree(tree) as plan:
         ref_o, ref_l = plan.decode_tree(tree)
         out_h = torch.empty(tuple(ref_o.shape), dtype=ref_o.dtype).pin_memory()
         lse_h = torch.empty(tuple(ref_l.shape), dtype=ref_l.dtype).pin_memory()
         plan.decode_tree(tree, out=out_h, lse=lse_h)
         plan.check()
-    assert torch.equal(out_h, ref_o.cpu()) and torch.equal(lse_h, ref_l.cpu())
+        assert torch.equal(out_h, ref_o.cpu()) and torch.equal(lse_h, ref_l.cpu())
+        q_h = tree.q.cpu().pin_memory()
+        o2, l2 = plan.decode(q_h, tree.k_pages, tree.v_pages, k_scale=tree.k_scale,
+                             v_scale=tree.v_scale)
+        plan.check()
+        assert o2.is_pinned() and torch.equal(o2, ref_o.cpu()) and torch.equal(l2, ref_l.cpu())
 
 
 def test_empty_path_gives_zero_and_neg_inf():
