@@ -1046,12 +1046,12 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
 //   warp 8      producer: TMA of K and V, one block per ring stage; pages past
 //               the item's end are loaded from an out-of-range row, which
 //               TMA fills with zeros
-//   warp 9      MMA issuer (one thread): S = Q K^T (M 128, N 64, K 128) into
-//               one of two TMEM buffers, then O += P V (M 128, N 128, K 64)
-//               into the item's TMEM accumulator (two, alternating by item).
+//   warp 9      S issuer (one thread): S = Q K^T (M 128, N 64, K 128) into
+//               one of two TMEM buffers, once PV of the block two back has
+//               freed it; runs ahead across item boundaries
+//   warp 11     PV issuer (one thread): O += P V (M 128, N 128, K 64) into
+//               the item's TMEM accumulator (two, alternating by item).
 //               A (Q or P) comes from TMEM, B (K or V) from shared memory.
-//               Blocks form one stream across items: S of a block is issued
-//               before PV of the block before it, item boundaries included.
 //               tcgen05.commit releases ring stages and signals completion.
 //   warps 0-3   softmax: thread r owns row r (TMEM lane r); online softmax in
 //               the log2 domain with a lazy rescale of O (only when a row's
@@ -1072,6 +1072,7 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
 constexpr int kTcRows = 128;
 constexpr int kTcBlockPages = 4;
 constexpr int kTcBlockTokens = kTcBlockPages * kPageSize;    // 64
+static_assert(kTcRunPages == kTcBlockPages, "a run box holds one block's pages");
 constexpr int kTcStages = 6;
 constexpr int kTcColBlockBytes = kTcBlockTokens * 128;        // 8 KB: 64 tokens x 128 B
 constexpr int kTcKBytes = 2 * kTcColBlockBytes;               // d = 128: two column blocks
@@ -1095,10 +1096,12 @@ constexpr int kTcEpilogueWarp = 4;                            // warps 4-7
 constexpr int kTcProducerWarp = 8;
 constexpr int kTcMmaWarp = 9;
 constexpr int kTcSchedulerWarp = 10;
+constexpr int kTcPvWarp = 11;
 static_assert(kTcRingBytes <= Shape<128, KvBf16>::kBodyBytes, "tcgen05 ring fits the CTA's memory");
 static_assert(kTcRingBytes <= Shape<128, KvBf16Deep>::kBodyBytes, "tcgen05 ring fits the CTA's memory");
 static_assert(kTcRingBytes <= Shape<128, KvE4m3>::kBodyBytes, "tcgen05 ring fits the CTA's memory");
-static_assert(kTcSchedulerWarp < kThreads / 32, "every tcgen05 role has a warp");
+static_assert(kTcSchedulerWarp < kThreads / 32 && kTcPvWarp < kThreads / 32,
+              "every tcgen05 role has a warp");
 static_assert(kMaxSuffixWarps <= kThreads / 32, "every suffix-pass warp exists");
 
 // Metadata of one prefix item, staged by the scheduler warp.
@@ -1123,7 +1126,7 @@ enum TcBar : int {
     kBarOEmpty = kBarOFull + 2,              // [2] epilogue (4 arrivals) -> MMA
     kBarMetaFull = kBarOEmpty + 2,           // [kTcMeta] scheduler -> every role
     kBarMetaEmpty = kBarMetaFull + kTcMeta,  // [kTcMeta] epilogue (4 arrivals) -> scheduler
-    kBarDrain = kBarMetaEmpty + kTcMeta,     // MMA commit -> MMA thread, before TMEM is freed
+    kBarDrain = kBarMetaEmpty + kTcMeta,     // both issuers' commits -> issuers, before TMEM is freed
     kBarCvFull,                              // [kTcCvStages] converters (4 arrivals) -> MMA
     kBarCvEmpty = kBarCvFull + kTcCvStages,  // [kTcCvStages] MMA commit -> converters
     kTcBars = kBarCvEmpty + kTcCvStages
@@ -1138,7 +1141,9 @@ __host__ __device__ constexpr int tc_bar_count(int i, bool f8) {
                    (i >= kBarMetaEmpty && i < kBarMetaEmpty + kTcMeta) ||
                    (f8 && i >= kBarKvEmpty && i < kBarKvEmpty + kTcStages))
                       ? 4
-                      : ((i >= kBarCvFull && i < kBarCvFull + kTcCvStages) ? kTcRows : 1));
+                      : ((i >= kBarCvFull && i < kBarCvFull + kTcCvStages)
+                             ? kTcRows
+                             : (i == kBarDrain ? 2 : 1)));
 }
 
 // e4m3 -> f16 of one 64-token block by 128 threads (8 of its 1024 16-byte
@@ -1194,23 +1199,14 @@ __device__ __forceinline__ int tc_blocks(int num_pages) {
 }
 
 template <int D, class KV>
-__device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
-                              const AttnArgs &a, uint8_t *smem, uint32_t bars, uint32_t tmem,
-                              int warp, int lane, volatile int *abort_flag, TcMeta *meta) {
+__device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *smem, uint32_t bars,
+                              uint32_t tmem, int warp, int lane, volatile int *abort_flag,
+                              TcMeta *meta) {
     static_assert(D == 128, "the tcgen05 prefix tile is written for head_dim 128");
     constexpr bool kF8 = KV::kElemBytes == 1;
     const uint32_t ring = dev::smem_addr(smem);
     auto bar = [&](int i) { return bars + 8u * static_cast<uint32_t>(i); };
     const long long limit = a.wait_limit_ns;
-    // the f16 (or bf16) K and V of block b, as the MMA reads them, and the
-    // barriers that hand them over
-    auto mma_stage = [&](int b) {
-        return kF8 ? ring + kTcCvOffset + (b % kTcCvStages) * kTcStageBytes
-                   : ring + (b % kTcStages) * kTcStageBytes;
-    };
-    auto mma_full = [&](int b) { return kF8 ? kBarCvFull + b % kTcCvStages : kBarKvFull + b % kTcStages; };
-    auto mma_full_parity = [&](int b) { return kF8 ? (b / kTcCvStages) & 1 : (b / kTcStages) & 1; };
-    auto mma_empty = [&](int b) { return kF8 ? kBarCvEmpty + b % kTcCvStages : kBarKvEmpty + b % kTcStages; };
 
     if (warp == kTcSchedulerWarp) {
         // ------------------------------------------------------------ scheduler
@@ -1259,6 +1255,9 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
         // Llama-3-shape step 42.9 -> 41.4 us, the long-prefix one -1 us, the
         // join prefill +1%; no gain with e4m3 KV, which keeps the default)
         const uint64_t last_pol = dev::l2_evict_last_policy();
+        // e4m3 blocks keep the default L2 policy (the per-page boxes use no hint)
+        const uint64_t f8_pol = dev::l2_evict_normal_policy();
+        const int kv_page_rows = a.num_kv_heads * kPageSize;   // TMA rows between consecutive pages
         int last_issue[kTcStages];
         for (int s = 0; s < kTcStages; ++s) last_issue[s] = -1;
         int blk = 0;
@@ -1290,15 +1289,39 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                     if (lane == 0)
                         dev::mbar_arrive_expect_tx(fb, kF8 ? kTcF8StageBytes : kTcStageBytes);
                     __syncwarp();
-                    if constexpr (kF8) {
+                    // the TMA unit takes about 90 cycles a box, so a block of
+                    // pages that are consecutive in the pool (the common case)
+                    // goes in one box per column block of K and of V
+                    const int pg0 = bi * kTcBlockPages;
+                    bool run = pg0 + kTcBlockPages <= np;
+                    const int row0 = m.rows[pg0 < np ? pg0 : 0];
+#pragma unroll
+                    for (int j = 1; j < kTcBlockPages; ++j)
+                        run = run && m.rows[pg0 + j] == row0 + j * kv_page_rows;
+                    if (run) {
+                        const int page = row0 / kv_page_rows;
+                        if constexpr (kF8) {
+                            if (lane < 2)
+                                dev::tma_load_5d_hint(ring + s * kTcF8StageBytes + lane * kTcF8Bytes,
+                                                      lane ? &maps->v_run : &maps->k_run, 0, 0, 0,
+                                                      m.it.kv_head, page, fb, f8_pol);
+                        } else {
+                            // lane: K (even) or V, column block lane / 2
+                            if (lane < 4)
+                                dev::tma_load_5d_hint(ring + s * kTcStageBytes + (lane & 1) * kTcKBytes +
+                                                          (lane >> 1) * kTcColBlockBytes,
+                                                      (lane & 1) ? &maps->v_run : &maps->k_run, 0,
+                                                      lane >> 1, 0, m.it.kv_head, page, fb, last_pol);
+                        }
+                    } else if constexpr (kF8) {
                         // raw e4m3 rows: one 2 KB box per page of K (even lanes) and of V
                         if (lane < 2 * kTcBlockPages) {
                             const int j = lane >> 1;
                             const int pg = bi * kTcBlockPages + j;
                             const int row = pg < np ? m.rows[pg] : a.kv_rows;   // kv_rows: zero fill
                             const uint32_t st = ring + s * kTcF8StageBytes + (lane & 1) * kTcF8Bytes;
-                            dev::tma_load_3d(st + j * kPageSize * 128, (lane & 1) ? tmap_v : tmap_k, 0, 0,
-                                             row, fb);
+                            dev::tma_load_3d(st + j * kPageSize * 128, (lane & 1) ? &maps->v : &maps->k,
+                                             0, 0, row, fb);
                         }
                     } else {
                         // page j = lane / 4, column block (lane / 2) % 2, K (even lanes) or V
@@ -1308,8 +1331,8 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                             const int row = pg < np ? m.rows[pg] : a.kv_rows;   // kv_rows: zero fill
                             const uint32_t off = cb * kTcColBlockBytes + j * kPageSize * 128;
                             const uint32_t st = ring + s * kTcStageBytes + (lane & 1) * kTcKBytes;
-                            dev::tma_load_3d_hint(st + off, (lane & 1) ? tmap_v : tmap_k, 0, cb, row, fb,
-                                                  last_pol);
+                            dev::tma_load_3d_hint(st + off, (lane & 1) ? &maps->v : &maps->k, 0, cb,
+                                                  row, fb, last_pol);
                         }
                     }
                     last_issue[s] = blk;
@@ -1322,100 +1345,96 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
                 if (last_issue[s] >= 0)
                     dev::mbar_wait_bounded(bar(kBarKvFull + s), (last_issue[s] / kTcStages) & 1,
                                            kDrainLimitNs, nullptr);
-    } else if (warp == kTcMmaWarp) {
-        // ------------------------------------------------------------ MMA issuer
+    } else if (warp == kTcMmaWarp || warp == kTcPvWarp) {
+        // ------------------------------------------------------------ MMA issuers
         if (lane == 0) {
+            // Two threads issue, so that neither product waits behind the other's
+            // issue (an MMA takes about 45 cycles to issue; twelve per block on
+            // one thread held the tile back).  Warp 9 issues S = Q K^T of every
+            // block, warp 11 O += P V.  S(b) overwrites the buffer of P(b - 2),
+            // so it waits for PV(b - 2) to complete.
             constexpr uint32_t kIdS = kF8 ? tc::idesc_f16_f32(kTcRows, kTcBlockTokens, false)
                                           : tc::idesc_bf16_f32(kTcRows, kTcBlockTokens, false);
             constexpr uint32_t kIdPV = kF8 ? tc::idesc_f16_f32(kTcRows, D, true)
                                            : tc::idesc_bf16_f32(kTcRows, D, true);
+            constexpr int kMmaStages = kF8 ? kTcCvStages : kTcStages;
             auto wait = [&](int i, int parity) {
                 return tc_wait(bar(i), static_cast<uint32_t>(parity & 1), limit, abort_flag);
             };
-            // S(b) = Q(item k) K(b)^T into S buffer b & 1
-            auto issue_s = [&](int b, int k) {
-                const uint32_t st = mma_stage(b);
-                const uint32_t tS = tmem + kTmemS + 64u * (b & 1);
-                const uint32_t tQ = tmem + kTmemQ + 64u * (k & 1);
-#pragma unroll
-                for (int ks = 0; ks < D / 16; ++ks) {
-                    const uint32_t cb = ks >> 2, kk = ks & 3;
-                    const uint64_t bd = tc::smem_desc_sw128(st + cb * kTcColBlockBytes + kk * 32, 16, 1024);
-                    tc::mma_bf16_tmem_a(tS, tQ + 8u * ks, bd, kIdS, ks > 0);
+            // descriptors of stage 0; a stage, a column block or a K step moves
+            // the start address field (address / 16) by a constant
+            const uint32_t mma_ring = kF8 ? ring + kTcCvOffset : ring;
+            const uint64_t desc_k = tc::smem_desc_sw128(mma_ring, 16, 1024);
+            const uint64_t desc_v = tc::smem_desc_sw128(mma_ring + kTcKBytes, kTcColBlockBytes, 1024);
+            constexpr uint32_t kStageStep = kTcStageBytes >> 4;
+            bool ok = true;
+            int b = 0;                       // block of the CTA's stream
+            int st = 0, ph = 0;              // its stage and the stage's phase parity
+            for (int k = 0; ok; ++k) {
+                const int ms = k % kTcMeta;
+                if (!wait(kBarMetaFull + ms, k / kTcMeta)) {
+                    ok = false;
+                    break;
                 }
-                tc::commit(bar(kBarSFull + (b & 1)));
-            };
-            bool ok = wait(kBarMetaFull, 0);
-            bool have = ok && meta[0].id >= 0;
-            int k = 0, b = 0, blk0 = 0, nb = have ? tc_blocks(meta[0].it.num_pages) : 0;
-            if (have) {
-                ok = wait(kBarQReady, 0) && wait(mma_full(0), 0);
-                if (ok) {
-                    tc::fence_after_sync();
-                    issue_s(0, 0);
-                }
-            }
-            while (have && ok) {
-                const bool last = b == blk0 + nb - 1;
-                bool next = false;
-                int nb_next = 0;
-                if (!last) {
-                    if (!wait(mma_full(b + 1), mma_full_parity(b + 1))) {
+                if (meta[ms].id < 0) break;
+                const int nb = tc_blocks(meta[ms].it.num_pages);
+                if (warp == kTcMmaWarp) {
+                    // S of the item's blocks, with its Q (buffer k & 1)
+                    if (!wait(kBarQReady + (k & 1), k >> 1)) {
                         ok = false;
                         break;
                     }
-                    tc::fence_after_sync();
-                    issue_s(b + 1, k);
-                } else {
-                    // first S of the next item before the last PV of this one
-                    const int s1 = (k + 1) % kTcMeta;
-                    if (!wait(kBarMetaFull + s1, (k + 1) / kTcMeta)) {
-                        ok = false;
-                        break;
-                    }
-                    if (meta[s1].id >= 0) {
-                        next = true;
-                        nb_next = tc_blocks(meta[s1].it.num_pages);
-                        if (!wait(kBarQReady + ((k + 1) & 1), (k + 1) >> 1) ||
-                            !wait(mma_full(b + 1), mma_full_parity(b + 1))) {
+                    const uint32_t tQ = tmem + kTmemQ + 64u * (k & 1);
+                    for (int i = 0; i < nb; ++i, ++b) {
+                        if (!wait((kF8 ? kBarCvFull : kBarKvFull) + st, ph) ||
+                            (b >= 2 && !wait(kBarPvDone + (b & 1), (b - 2) >> 1))) {
                             ok = false;
                             break;
                         }
                         tc::fence_after_sync();
-                        issue_s(b + 1, k + 1);
+                        const uint32_t tS = tmem + kTmemS + 64u * (b & 1);
+                        const uint64_t kd = desc_k + static_cast<uint64_t>(st * kStageStep);
+#pragma unroll
+                        for (int ks = 0; ks < D / 16; ++ks) {
+                            constexpr uint32_t kCb = kTcColBlockBytes;
+                            const uint32_t off = ((ks >> 2) * kCb + (ks & 3) * 32) >> 4;
+                            tc::mma_bf16_tmem_a(tS, tQ + 8u * ks, kd + off, kIdS, ks > 0);
+                        }
+                        tc::commit(bar(kBarSFull + (b & 1)));
+                        if (++st == kMmaStages) {
+                            st = 0;
+                            ph ^= 1;
+                        }
+                    }
+                } else {
+                    // PV of the item's blocks into O (buffer k & 1)
+                    const uint32_t tO = tmem + kTmemO + 128u * (k & 1);
+                    for (int i = 0; i < nb; ++i, ++b) {
+                        if (!wait(kBarPFull + (b & 1), b >> 1) ||
+                            // the O buffer was last used by item k - 2: its epilogue must be done
+                            (i == 0 && k >= 2 && !wait(kBarOEmpty + (k & 1), (k >> 1) - 1))) {
+                            ok = false;
+                            break;
+                        }
+                        tc::fence_after_sync();
+                        const uint32_t tP = tmem + kTmemS + 64u * (b & 1);
+                        const uint64_t vd = desc_v + static_cast<uint64_t>(st * kStageStep);
+#pragma unroll
+                        for (int kk = 0; kk < kTcBlockTokens / 16; ++kk)
+                            tc::mma_bf16_tmem_a(tO, tP + 8u * kk,
+                                                vd + static_cast<uint32_t>((kk * 2048) >> 4), kIdPV,
+                                                i > 0 || kk > 0);
+                        // S(b) completed before P(b) was written: both products
+                        // of the stage are done when these arrive
+                        tc::commit(bar((kF8 ? kBarCvEmpty : kBarKvEmpty) + st));
+                        tc::commit(bar(kBarPvDone + (b & 1)));
+                        if (i == nb - 1) tc::commit(bar(kBarOFull + (k & 1)));
+                        if (++st == kMmaStages) st = 0;
                     }
                 }
-                if (!wait(kBarPFull + (b & 1), b >> 1)) {
-                    ok = false;
-                    break;
-                }
-                // the item's O buffer was last used by item k - 2: its epilogue must be done
-                if (b == blk0 && k >= 2 && !wait(kBarOEmpty + (k & 1), (k >> 1) - 1)) {
-                    ok = false;
-                    break;
-                }
-                tc::fence_after_sync();
-                const uint32_t tO = tmem + kTmemO + 128u * (k & 1);
-                const uint32_t tP = tmem + kTmemS + 64u * (b & 1);
-                const uint32_t vst = mma_stage(b) + kTcKBytes;
-#pragma unroll
-                for (int kk = 0; kk < kTcBlockTokens / 16; ++kk) {
-                    const uint64_t bd = tc::smem_desc_sw128(vst + kk * 2048, kTcColBlockBytes, 1024);
-                    tc::mma_bf16_tmem_a(tO, tP + 8u * kk, bd, kIdPV, b > blk0 || kk > 0);
-                }
-                tc::commit(bar(mma_empty(b)));
-                tc::commit(bar(kBarPvDone + (b & 1)));
-                if (last) {
-                    tc::commit(bar(kBarOFull + (k & 1)));
-                    if (!next) break;
-                    blk0 += nb;
-                    nb = nb_next;
-                    ++k;
-                }
-                ++b;
             }
             if (!ok) tc_fail(a, abort_flag, kSiteConsumerFull);
-            // every MMA must finish before TMEM is freed
+            // every MMA of both issuers must finish before TMEM is freed
             tc::commit(bar(kBarDrain));
             dev::mbar_wait_bounded(bar(kBarDrain), 0, kDrainLimitNs, nullptr);
         }
@@ -1746,8 +1765,7 @@ __device__ void prefix_cta_tc(const CUtensorMap *tmap_k, const CUtensorMap *tmap
 // on one sub-partition of 16K registers).
 template <int D, class KV>
 __global__ void __launch_bounds__(kThreads, 1)
-    attn_kernel(const __grid_constant__ CUtensorMap tmap_k,
-                const __grid_constant__ CUtensorMap tmap_v, const AttnArgs a) {
+    attn_kernel(const __grid_constant__ KvMaps maps, const AttnArgs a) {
     using S = Shape<D, KV>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
@@ -1784,8 +1802,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             init_suffix_barriers();
         }
         dev::fence_mbar_init();
-        dev::prefetch_tensormap(&tmap_k);
-        dev::prefetch_tensormap(&tmap_v);
+        dev::prefetch_tensormap(&maps.k);
+        dev::prefetch_tensormap(&maps.v);
     }
     if constexpr (kTcPrefix) {
         if (wide && warp == kTcMmaWarp) tc::alloc<kTcTmemCols>(dev::smem_addr(&tmem_base));
@@ -1798,14 +1816,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (wide) {
         if constexpr (kTcPrefix) {
             tc::fence_after_sync();
-            prefix_cta_tc<D, KV>(&tmap_k, &tmap_v, a, smem, bars, tmem_base, warp, lane, &abort_flag,
+            prefix_cta_tc<D, KV>(&maps, a, smem, bars, tmem_base, warp, lane, &abort_flag,
                              tc_meta);
             tc::fence_before_sync();
             __syncthreads();
             tc::fence_after_sync();
             if (warp == kTcMmaWarp) tc::dealloc<kTcTmemCols>(tmem_base);
         } else {
-            prefix_cta<D, KV>(&tmap_k, &tmap_v, a, smem, ring, bars, warp, lane, &abort_flag,
+            prefix_cta<D, KV>(&maps.k, &maps.v, a, smem, ring, bars, warp, lane, &abort_flag,
                               id_slots);
         }
         // the prefix queue is empty: this CTA joins the suffix queue with the
@@ -1821,7 +1839,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncthreads();
     }
     if (warp < S::kSuffixWarps)
-        suffix_warp<D, KV>(&tmap_k, &tmap_v, a, ring, bars, warp, lane, grab_items[warp]);
+        suffix_warp<D, KV>(&maps.k, &maps.v, a, ring, bars, warp, lane, grab_items[warp]);
 }
 
 // Shared memory and carveout are set once per device; reports the number of
@@ -1851,12 +1869,11 @@ cudaError_t configure(int *ctas_per_sm) {
 }
 
 template <int D, class KV>
-cudaError_t launch(const AttnArgs &a, const CUtensorMap &tk, const CUtensorMap &tv,
-                   cudaStream_t stream) {
+cudaError_t launch(const AttnArgs &a, const KvMaps &maps, cudaStream_t stream) {
     using S = Shape<D, KV>;
     cudaError_t e = configure<D, KV>(nullptr);
     if (e != cudaSuccess) return e;
-    attn_kernel<D, KV><<<a.num_ctas, kThreads, S::kSmemBytes, stream>>>(tk, tv, a);
+    attn_kernel<D, KV><<<a.num_ctas, kThreads, S::kSmemBytes, stream>>>(maps, a);
     return cudaGetLastError();
 }
 
@@ -1874,20 +1891,20 @@ cudaError_t attn_mma_ctas_per_sm(int head_dim, int mode, int *ctas_per_sm) {
     return cudaErrorNotSupported;
 }
 
-cudaError_t launch_attn_bf16(const AttnArgs &a, const CUtensorMap &tk, const CUtensorMap &tv,
-                             int head_dim, cudaStream_t stream) {
+cudaError_t launch_attn_bf16(const AttnArgs &a, const KvMaps &maps, int head_dim,
+                             cudaStream_t stream) {
     if (a.num_items <= 0 || a.num_ctas <= 0) return cudaSuccess;
     if (head_dim == 128)
-        return a.suffix_warps == KvBf16Deep::kSuffixWarps ? launch<128, KvBf16Deep>(a, tk, tv, stream)
-                                                          : launch<128, KvBf16>(a, tk, tv, stream);
-    if (head_dim == 64) return launch<64, KvBf16>(a, tk, tv, stream);
+        return a.suffix_warps == KvBf16Deep::kSuffixWarps ? launch<128, KvBf16Deep>(a, maps, stream)
+                                                          : launch<128, KvBf16>(a, maps, stream);
+    if (head_dim == 64) return launch<64, KvBf16>(a, maps, stream);
     return cudaErrorNotSupported;
 }
 
-cudaError_t launch_attn_fp8(const AttnArgs &a, const CUtensorMap &tk, const CUtensorMap &tv,
-                            int head_dim, cudaStream_t stream) {
+cudaError_t launch_attn_fp8(const AttnArgs &a, const KvMaps &maps, int head_dim,
+                            cudaStream_t stream) {
     if (a.num_items <= 0 || a.num_ctas <= 0) return cudaSuccess;
-    if (head_dim == 128) return launch<128, KvE4m3>(a, tk, tv, stream);
+    if (head_dim == 128) return launch<128, KvE4m3>(a, maps, stream);
     return cudaErrorNotSupported;
 }
 

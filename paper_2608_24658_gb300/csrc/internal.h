@@ -110,11 +110,20 @@ struct MergeArgs {
 // attributes); cudaErrorNotSupported for a shape it has no kernel for.
 cudaError_t attn_mma_ctas_per_sm(int head_dim, int mode, int *ctas_per_sm);
 
+// TMA views of the K and V pools.  k / v: one box is one 128-byte column
+// block of one page of one kv head (16 rows).  k_run / v_run: one box is the
+// same column block of kTcRunPages consecutive pages of one kv head, for
+// blocks whose pages are consecutive in the pool.
+constexpr int kTcRunPages = 4;
+struct KvMaps {
+    CUtensorMap k, v, k_run, v_run;
+};
+
 // Kernel launchers; each returns the launch's cudaError_t.
-cudaError_t launch_attn_bf16(const AttnArgs &a, const CUtensorMap &tmap_k,
-                             const CUtensorMap &tmap_v, int head_dim, cudaStream_t stream);
-cudaError_t launch_attn_fp8(const AttnArgs &a, const CUtensorMap &tmap_k,
-                            const CUtensorMap &tmap_v, int head_dim, cudaStream_t stream);
+cudaError_t launch_attn_bf16(const AttnArgs &a, const KvMaps &maps, int head_dim,
+                             cudaStream_t stream);
+cudaError_t launch_attn_fp8(const AttnArgs &a, const KvMaps &maps, int head_dim,
+                            cudaStream_t stream);
 cudaError_t launch_attn_fp32(const AttnArgs &a, const float *k_pages, const float *v_pages,
                              int head_dim, cudaStream_t stream);
 cudaError_t launch_merge(const MergeArgs &a, int head_dim, int mode, bool programmatic,

@@ -143,8 +143,7 @@ struct parason_plan_s {
     std::mutex tm_mutex;
     const void *tm_k_ptr = nullptr;
     const void *tm_v_ptr = nullptr;
-    CUtensorMap tm_k{};
-    CUtensorMap tm_v{};
+    parason::KvMaps tm{};
 
     // timing
     int32_t timing_cap = 0;
@@ -712,6 +711,38 @@ parason_status encode_kv_map(CUtensorMap *map, const void *pages, int64_t num_ph
     return r == CUDA_SUCCESS ? PARASON_OK : PARASON_ECUDA;
 }
 
+// The same pool as a 5-D view: dim0 = 128 bytes of one segment, dim1 =
+// segment, dim2 = slot in the page (16), dim3 = kv head, dim4 = page.  One
+// box {seg, 1, 16, 1, kTcRunPages} is one 128-byte column block of
+// kTcRunPages consecutive pages of one kv head: 16 kTcRunPages rows of 128
+// bytes, laid out as the per-page boxes of those pages would be.
+parason_status encode_kv_run_map(CUtensorMap *map, const void *pages, int64_t num_phys,
+                                 int32_t H_kv, int32_t head_dim, int32_t mode) {
+    auto fn = encode_fn();
+    if (!fn) return PARASON_ECUDA;
+    const int esize = (mode == PARASON_FP8_E4M3_KV) ? 1 : 2;
+    const CUtensorMapDataType dt =
+        (mode == PARASON_FP8_E4M3_KV) ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    const int row_bytes = head_dim * esize;
+    if (row_bytes % 128 != 0) return PARASON_EUNSUPPORTED;
+    const int nseg = row_bytes / 128;
+    const int seg_elems = 128 / esize;
+    const cuuint64_t page_head_bytes = static_cast<cuuint64_t>(parason::kPageSize) * row_bytes;
+    cuuint64_t dims[5] = {static_cast<cuuint64_t>(seg_elems), static_cast<cuuint64_t>(nseg),
+                          static_cast<cuuint64_t>(parason::kPageSize), static_cast<cuuint64_t>(H_kv),
+                          static_cast<cuuint64_t>(num_phys)};
+    cuuint64_t strides[4] = {128, static_cast<cuuint64_t>(row_bytes), page_head_bytes,
+                             page_head_bytes * static_cast<cuuint64_t>(H_kv)};
+    cuuint32_t box[5] = {static_cast<cuuint32_t>(seg_elems), 1u,
+                         static_cast<cuuint32_t>(parason::kPageSize), 1u,
+                         static_cast<cuuint32_t>(parason::kTcRunPages)};
+    cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    CUresult r = fn(map, dt, 5, const_cast<void *>(pages), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? PARASON_OK : PARASON_ECUDA;
+}
+
 parason_status record_event(parason_plan_s *p, int which, cudaStream_t stream) {
     if (p->timing_cap <= 0 || p->timing_n >= p->timing_cap) return PARASON_OK;
     cudaEvent_t ev = p->events[3 * p->timing_n + which];
@@ -908,24 +939,30 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
             e = parason::launch_attn_fp32(a, static_cast<const float *>(k_pages),
                                           static_cast<const float *>(v_pages), d, stream);
         } else {
-            CUtensorMap tk, tv;
+            parason::KvMaps maps;
             {
                 std::lock_guard<std::mutex> lock(p->tm_mutex);
+                const int32_t H = p->cfg.num_kv_heads, mode = p->cfg.mode;
                 if (p->tm_k_ptr != k_pages) {
-                    st = encode_kv_map(&p->tm_k, k_pages, p->num_phys, p->cfg.num_kv_heads, d, p->cfg.mode);
+                    p->tm_k_ptr = nullptr;
+                    st = encode_kv_map(&p->tm.k, k_pages, p->num_phys, H, d, mode);
+                    if (st == PARASON_OK)
+                        st = encode_kv_run_map(&p->tm.k_run, k_pages, p->num_phys, H, d, mode);
                     if (st != PARASON_OK) return st;
                     p->tm_k_ptr = k_pages;
                 }
                 if (p->tm_v_ptr != v_pages) {
-                    st = encode_kv_map(&p->tm_v, v_pages, p->num_phys, p->cfg.num_kv_heads, d, p->cfg.mode);
+                    p->tm_v_ptr = nullptr;
+                    st = encode_kv_map(&p->tm.v, v_pages, p->num_phys, H, d, mode);
+                    if (st == PARASON_OK)
+                        st = encode_kv_run_map(&p->tm.v_run, v_pages, p->num_phys, H, d, mode);
                     if (st != PARASON_OK) return st;
                     p->tm_v_ptr = v_pages;
                 }
-                tk = p->tm_k;
-                tv = p->tm_v;
+                maps = p->tm;
             }
-            e = (p->cfg.mode == PARASON_BF16) ? parason::launch_attn_bf16(a, tk, tv, d, stream)
-                                              : parason::launch_attn_fp8(a, tk, tv, d, stream);
+            e = (p->cfg.mode == PARASON_BF16) ? parason::launch_attn_bf16(a, maps, d, stream)
+                                              : parason::launch_attn_fp8(a, maps, d, stream);
         }
         if (e == cudaErrorNotSupported) return PARASON_EUNSUPPORTED;
         if (e != cudaSuccess) return PARASON_ECUDA;
