@@ -1149,20 +1149,30 @@ __host__ __device__ constexpr int tc_bar_count(int i, bool f8) {
 // e4m3 -> f16 of one 64-token block by 128 threads (8 of its 1024 16-byte
 // chunks each): staged K and V rows of 128 bytes (128-byte swizzled) into two
 // 8 KB column blocks per operand (128-byte swizzled), the layout TMA gives a
-// bf16 block; rows from `valid` on become zeros.
+// bf16 block; rows from `valid` on become zeros.  The thread's 8 chunks are
+// loaded before any is stored, so that their latencies overlap (a load may
+// not pass an earlier shared store).
 __device__ __forceinline__ void convert_block_e4m3(uint32_t src, uint32_t dst, int valid, int t) {
+    uint4 w[8];
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
         const int idx = t + kTcRows * q;
         const int op = idx >> 9;                 // 0: K, 1: V
         const int r = (idx >> 3) & 63;           // token
         const int c = idx & 7;                   // elements 16c .. 16c + 15
-        uint4 w = lds128(src + op * kTcF8Bytes + r * 128 + ((c ^ (r & 7)) << 4));
-        if (r >= valid) w = make_uint4(0u, 0u, 0u, 0u);
-        const uint32_t lo0 = e4m3x2_to_f16x2(w.x), lo1 = e4m3x2_to_f16x2(w.x >> 16);
-        const uint32_t lo2 = e4m3x2_to_f16x2(w.y), lo3 = e4m3x2_to_f16x2(w.y >> 16);
-        const uint32_t hi0 = e4m3x2_to_f16x2(w.z), hi1 = e4m3x2_to_f16x2(w.z >> 16);
-        const uint32_t hi2 = e4m3x2_to_f16x2(w.w), hi3 = e4m3x2_to_f16x2(w.w >> 16);
+        w[q] = lds128(src + op * kTcF8Bytes + r * 128 + ((c ^ (r & 7)) << 4));
+    }
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+        const int idx = t + kTcRows * q;
+        const int op = idx >> 9;
+        const int r = (idx >> 3) & 63;
+        const int c = idx & 7;
+        if (r >= valid) w[q] = make_uint4(0u, 0u, 0u, 0u);
+        const uint32_t lo0 = e4m3x2_to_f16x2(w[q].x), lo1 = e4m3x2_to_f16x2(w[q].x >> 16);
+        const uint32_t lo2 = e4m3x2_to_f16x2(w[q].y), lo3 = e4m3x2_to_f16x2(w[q].y >> 16);
+        const uint32_t hi0 = e4m3x2_to_f16x2(w[q].z), hi1 = e4m3x2_to_f16x2(w[q].z >> 16);
+        const uint32_t hi2 = e4m3x2_to_f16x2(w[q].w), hi3 = e4m3x2_to_f16x2(w[q].w >> 16);
         const int c2 = 2 * (c & 3);              // f16 chunk in column block c / 4
         const uint32_t row = dst + op * kTcKBytes + (c >> 2) * kTcColBlockBytes + r * 128;
         asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(row + ((c2 ^ (r & 7)) << 4)),
@@ -1643,8 +1653,11 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
         };
             // The converters take every block of every item in order.  An
             // item's O is stored once the next item's first block is
-            // converted: the MMA issues that block's S before the item's last
-            // PV, so waiting for the O first could never end.
+            // converted (the S issuer needs that block before the item's
+            // last PV can follow, so waiting for the O first could never
+            // end), and its second block too where there is one, so that the
+            // wait for the O is short (long-prefix step with e4m3 KV: 668 ->
+            // 655 us).
             auto convert = [&](int gb, int valid) -> bool {
                 const int s = gb % kTcStages, c = gb % kTcCvStages;
                 if (!tc_warp_wait(bar(kBarKvFull + s), (gb / kTcStages) & 1, limit, abort_flag, lane))
@@ -1695,7 +1708,7 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
                     const int tokens = (it.num_pages - 1) * kPageSize + it.last_valid;
                     for (int i = 0; i < nb && ok; ++i, ++gb) {
                         ok = convert(gb, min(kTcBlockTokens, tokens - i * kTcBlockTokens));
-                        if (ok && i == 0 && k > 0) ok = finish(k - 1, true);
+                        if (ok && k > 0 && i == min(1, nb - 1)) ok = finish(k - 1, true);
                     }
                     if (!ok) break;
                     const bool more = has_item(k + 1);
