@@ -44,9 +44,10 @@ namespace {
 constexpr int kConsumerWarps = 8;                          // prefix pass on mma.sync
 constexpr int kConsumerThreads = kConsumerWarps * 32;
 constexpr int kMaxSuffixWarps = 12;                        // suffix pass: warps per CTA, at most
-// 12 warps: the suffix pass runs 8 autonomous warps; the prefix pass on
-// tcgen05 uses 11 (softmax 4, epilogue 4, producer, MMA issuer, scheduler),
-// the one on mma.sync 9 (8 consumers and a producer)
+// 12 warps: the suffix pass runs 6, 8 or 12 autonomous warps (by KV type);
+// the prefix pass on tcgen05 uses all 12 (softmax 4, epilogue 4, producer,
+// S issuer, scheduler, PV issuer), the one on mma.sync 9 (8 consumers and a
+// producer)
 constexpr int kThreads = 12 * 32;
 constexpr long long kDrainLimitNs = 1000000000LL;
 constexpr int kSmemBudget = 220 * 1024;                    // dynamic, one CTA per SM
@@ -1043,9 +1044,11 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
 //               branch of each group of g rows) in one of kTcMeta shared
 //               slots, so that no other role waits on a dependent chain of
 //               global loads when it moves to the next item
-//   warp 8      producer: TMA of K and V, one block per ring stage; pages past
-//               the item's end are loaded from an out-of-range row, which
-//               TMA fills with zeros
+//   warp 8      producer: TMA of K and V, one block per ring stage: one box
+//               per column block of K and of V when the block's 4 pages are
+//               consecutive in the pool (the 5-D run maps), else one per
+//               page and column block; pages past the item's end are loaded
+//               from an out-of-range row, which TMA fills with zeros
 //   warp 9      S issuer (one thread): S = Q K^T (M 128, N 64, K 128) into
 //               one of two TMEM buffers, once PV of the block two back has
 //               freed it; runs ahead across item boundaries
