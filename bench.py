@@ -1,15 +1,21 @@
 #!/usr/bin/env python3
 """Benchmark: fork-tree decode attention on GB300, one JSON line.
 
-Workload (default): the Llama-3-8B attention shape (32 q / 8 kv heads, d 128,
-bf16), one request with a 2048-token shared prefix and 16 trial branches with
-suffixes uniform in [512, 4096], page size 16.  A step is one decode step of
-every branch: the attention kernel over every node's KV (each shared node read
-once) and the log-sum-exp merge, through ``parason_attn_decode``.
+Workload of the line (default): batched serving, 32 requests each forking 32
+trial branches (1024 branches), Llama-3-8B attention shape (32 q / 8 kv heads,
+d 128, bf16), prefixes lognormal (median 2048, clipped to [1024, 8192]),
+suffixes uniform in [256, 8192], page size 16, physical pages randomly
+permuted: about 4.4 M unique tokens, 18 GB of KV, the largest of the five
+workloads and the one that fits one GPU.  A step is one decode step of every
+branch: the attention kernel over every node's KV (each shared node read once)
+and the log-sum-exp merge, through ``parason_attn_decode``.
 
   value     branch-tokens/s = branches per step / device time of a step, with
             q/K/V resident in HBM and L2 flushed (256 MiB write) before every
-            step; summed over ranks for N > 1 (independent replicas).
+            step.  With N > 1 GPUs the requests are split over the ranks
+            (parason_attn_plan_shard; kv heads when there are fewer requests
+            than ranks): the whole workload's branches over the slowest rank's
+            step, strong scaling, no exchange between ranks.
   e2e       the same metric through the same C-ABI call with q, out and lse in
             pinned host memory, read and written by the kernels in place
             (e2e_copy: q copied to HBM first, inside each step).
@@ -17,6 +23,9 @@ once) and the log-sum-exp merge, through ``parason_attn_decode``.
             each shared node once, plus q) per launch over its CUDA-event time,
             against the measured HBM copy bandwidth.
   cpu_baseline  the fp64 oracle on the host cores, on a bounded sample.
+  configs   the other workloads (tiny fork, Llama-3 shape, two-level tree,
+            long prefix with bf16 and with e4m3 KV), timed the same way in the
+            same process: step, kernels, roofline fractions.
 
 ``--impl reference`` times the oracle (the reference arm of this build).
 """
@@ -158,46 +167,63 @@ def algorithmic_flops(tree):
 # CPU baseline: the fp64 oracle on a bounded sample
 # ----------------------------------------------------------------------------
 
-def oracle_sample_rate(tree_cpu, budget_s: float, max_branches=None):
-    """Time the oracle on whole branches (cycling) for about ``budget_s`` seconds."""
+def oracle_host_sample(tree, max_branches: int = 64):
+    """Host copy of a bounded sample of whole branches (W.host_subset: only
+    what they read), taken once, so that a multi-GB pool never goes to the
+    host whole and no copy is inside an oracle timing.  The sample is four
+    groups of consecutive branches spread over the workload (with several
+    requests, four requests' prefixes and suffixes)."""
+    L = tree.num_leaves
+    n = min(L, max_branches)
+    per = max(1, n // 4)
+    sel = sorted({(g * L // 4 + i) % L for g in range(4) for i in range(per)})[:n]
+    return W.host_subset(tree, sel)
+
+
+def oracle_branch_seconds(sub, branches):
+    """Oracle time (s) of whole branches of a host sample.  Returns (seconds, threads)."""
     import oracle
-    kw = oracle.tree_kwargs(tree_cpu)
-    L = tree_cpu.num_leaves
-    done, t0, b = 0, time.perf_counter(), 0
-    while True:
-        oracle.decode(sel=[b % L], **kw)
+    kw = oracle.tree_kwargs(sub)
+    t0 = time.perf_counter()
+    oracle.decode(sel=[int(b) % sub.num_leaves for b in branches], **kw)
+    return time.perf_counter() - t0, oracle.num_threads()
+
+
+def oracle_sample_rate(tree, budget_s: float):
+    """Oracle branch-tokens/s on whole branches of a host sample of ``tree``
+    (cycling) for about ``budget_s`` seconds of oracle time."""
+    sub = oracle_host_sample(tree)
+    done, el, cores = 0, 0.0, 1
+    while el < budget_s:
+        t, cores = oracle_branch_seconds(sub, [done])
+        el += t
         done += 1
-        b += 1
-        el = time.perf_counter() - t0
-        if el >= budget_s or (max_branches and done >= max_branches):
-            break
-    return done / el, done, el, oracle.num_threads()
+    return done / el, done, el, cores, sub.num_leaves
 
 
 def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
         return 0
-    tree = make_workload(args, device="cpu")
-    import oracle
-    kw = oracle.tree_kwargs(tree)
+    # the inputs are drawn where the GPU arm draws them (the same seeded
+    # values); only the oracle's own calls are timed, on the host cores
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    tree = make_workload(args, device=dev)
     L = tree.num_leaves
-    # per-step sample: whole branches, sized so the whole run takes about 60 s
-    t0 = time.perf_counter()
-    oracle.decode(sel=[0], **kw)
-    per_branch = max(time.perf_counter() - t0, 1e-4)
-    per_step = max(1, int(60.0 / ((args.steps + args.warmup) * per_branch)))
-    per_step = min(per_step, L)
+    sub = oracle_host_sample(tree)
+    del tree.k_pages, tree.v_pages
+    per_branch, _ = oracle_branch_seconds(sub, [0])
+    per_branch = max(per_branch, 1e-4)
+    # whole branches per step, sized so that the whole run takes about 60 s
+    per_step = min(L, max(1, int(60.0 / ((args.steps + args.warmup) * per_branch))))
     b = 0
     for _ in range(args.warmup):
-        oracle.decode(sel=[(b + i) % L for i in range(per_step)], **kw)
+        oracle_branch_seconds(sub, range(b, b + per_step))
         b += per_step
-    times = []
+    times, cores = [], 1
     for _ in range(args.steps):
-        sel = [(b + i) % L for i in range(per_step)]
-        t0 = time.perf_counter()
-        oracle.decode(sel=sel, **kw)
-        times.append(time.perf_counter() - t0)
+        t, cores = oracle_branch_seconds(sub, range(b, b + per_step))
+        times.append(t)
         b += per_step
     total = sum(times)
     value = per_step * args.steps / total
@@ -206,9 +232,9 @@ def run_reference(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * total / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": workload_config(tree, args),
-        "cpu_baseline": {"kind": "oracle", "value": value, "unit": UNIT,
-                         "cores": oracle.num_threads(),
-                         "sample": f"{per_step} whole branch(es) per step of {L}, all q heads"},
+        "cpu_baseline": {"kind": "oracle", "value": value, "unit": UNIT, "cores": cores,
+                         "sample": f"{per_step} whole branch(es) per step, cycling over "
+                                   f"{sub.num_leaves} sampled branches of {L}, all q heads"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -219,17 +245,154 @@ def run_reference(args):
 # GPU arm
 # ----------------------------------------------------------------------------
 
-def make_workload(args, device):
-    return W.make_config(args.config, mode=args.mode, device=device)
+# the configurations timed beside the headline, in the same process (N = 1)
+TABLE = [(1, "bf16"), (2, "bf16"), (3, "bf16"), (4, "bf16"), (5, "bf16"), (5, "fp8")]
 
 
-def workload_config(tree, args):
-    return {"workload": tree.name, "num_q_heads": tree.num_q_heads,
-            "num_kv_heads": tree.num_kv_heads, "head_dim": tree.head_dim,
-            "kv_dtype": tree.mode, "branches": tree.num_leaves, "nodes": tree.num_nodes,
-            "unique_tokens": tree.unique_tokens(), "path_tokens": tree.path_tokens(),
-            "page_size": tree.page_size, "seed_config": args.config,
-            "l2": "flushed before every step (256 MiB write)"}
+def make_workload(args, device, config=None, mode=None):
+    return W.make_config(config or args.config, mode=mode or args.mode, device=device)
+
+
+def workload_config(tree, args, shard=None):
+    cfg = {"workload": tree.name, "num_q_heads": tree.num_q_heads,
+           "num_kv_heads": tree.num_kv_heads, "head_dim": tree.head_dim,
+           "kv_dtype": tree.mode, "branches": tree.num_leaves, "nodes": tree.num_nodes,
+           "requests": int((tree.parent < 0).sum()),
+           "unique_tokens": tree.unique_tokens(), "path_tokens": tree.path_tokens(),
+           "page_size": tree.page_size, "page_order": "permuted" if tree.meta.get("permuted")
+           else "node-major", "seed_config": args.config,
+           "l2": "flushed before every step (256 MiB write)"}
+    if shard:
+        cfg["parallelism"] = shard
+    return cfg
+
+
+class Rank:
+    """One rank's share of a workload: its plan and its q / K / V views."""
+
+    def __init__(self, tree, rank, world, dev):
+        from paper_2608_24658_gb300 import _lib
+        from paper_2608_24658_gb300.api import Plan
+        self.tree, self.kind = tree, None
+        self.q, self.k, self.v = tree.q, tree.k_pages, tree.v_pages
+        self.k_scale, self.v_scale = tree.k_scale, tree.v_scale
+        if world == 1:
+            self.plan = Plan.for_tree(tree)
+            self.units = tree.num_leaves
+            return
+        roots = int((tree.parent < 0).sum())
+        if roots >= world:
+            # requests split over the ranks; the pools are addressed whole
+            self.kind = "requests"
+            self.plan = Plan.for_tree(tree, shard=(_lib.SHARD_REQUESTS, rank, world))
+            br = torch.as_tensor(self.plan.export(_lib.TABLE_SHARD_BRANCHES), dtype=torch.long,
+                                 device=dev)
+            self.q = tree.q.index_select(0, br).contiguous()
+            self.units = self.plan.num_leaves
+        elif tree.num_kv_heads % world == 0:
+            # kv heads split over the ranks: each rank holds its heads' q and KV
+            self.kind = "kv_heads"
+            self.plan = Plan.for_tree(tree, shard=(_lib.SHARD_KV_HEADS, rank, world))
+            hk = tree.num_kv_heads // world
+            g = tree.group
+            self.q = tree.q[:, rank * hk * g:(rank + 1) * hk * g].contiguous()
+            self.k = tree.k_pages[:, rank * hk:(rank + 1) * hk].contiguous()
+            self.v = tree.v_pages[:, rank * hk:(rank + 1) * hk].contiguous()
+            if tree.k_scale is not None:
+                self.k_scale = tree.k_scale[rank * hk:(rank + 1) * hk].contiguous()
+                self.v_scale = tree.v_scale[rank * hk:(rank + 1) * hk].contiguous()
+            self.units = tree.num_leaves / world
+        else:
+            self.kind = "replicas"
+            self.plan = Plan.for_tree(tree)
+            self.units = tree.num_leaves
+
+    def decode(self, q=None, out=None, lse=None, ws=None, stream=None):
+        return self.plan.decode(self.q if q is None else q, self.k, self.v, out=out, lse=lse,
+                                workspace=ws, k_scale=self.k_scale, v_scale=self.v_scale,
+                                stream=stream)
+
+
+def time_steps(step, flush, stream, steps, warmup, dev, sampler=None, world=1):
+    """Warm-up right before the timed loop, then `steps` steps, each timed
+    with CUDA events on the launching stream, L2 flushed (outside the events)
+    before every step.  Returns (per-step ms list, wall seconds, clocks)."""
+    if sampler is not None:
+        sampler.start()
+        time.sleep(0.3)
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    for _ in range(warmup):
+        flush.fill_(1.0)
+        step()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    torch.cuda.synchronize(dev)
+    wall0 = time.perf_counter()
+    for i in range(steps):
+        flush.fill_(float(i))
+        starts[i].record(stream)
+        step()
+        ends[i].record(stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    wall = time.perf_counter() - wall0
+    clocks = sampler.stop() if sampler is not None else None
+    return [s.elapsed_time(e) for s, e in zip(starts, ends)], wall, clocks
+
+
+def kernel_times(r, step, flush, dev, steps):
+    """Per-kernel times: the same steps with the library's events around its
+    attention kernel (an event between the two kernels stops the merge grid
+    from launching early, so this pass is separate from the timed one)."""
+    r.plan.enable_timing(steps)
+    for i in range(steps):
+        flush.fill_(float(i))
+        step()
+    torch.cuda.synchronize(dev)
+    attn_ms, merge_ms = r.plan.read_timing(steps)
+    r.plan.enable_timing(0)
+    return float(np.mean(attn_ms)), float(np.mean(merge_ms))
+
+
+def traffic_of(tree):
+    tr_path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(tr_path):
+        return None
+    with open(tr_path) as f:
+        tr = json.load(f).get(f"{tree.name}:{tree.mode}")
+    if tr and tr.get("kernel_source_hash") == kernel_source_hash():
+        return tr["bytes_per_launch"]
+    return None
+
+
+def measure_table_entry(idx, mode, args, dev, stream, flush, peak_gbs):
+    """One configuration timed in this process: step, kernels, fractions."""
+    tree = make_workload(args, dev, config=idx, mode=mode)
+    r = Rank(tree, 0, 1, dev)
+    ws = r.plan.workspace(dev)
+    out = torch.empty_like(tree.q)
+    lse = torch.empty(tree.q.shape[:2], dtype=torch.float32, device=dev)
+    step = lambda: r.decode(out=out, lse=lse, ws=ws, stream=stream)
+    steps = max(10, min(args.steps, args.table_steps))
+    ms, _, _ = time_steps(step, flush, stream, steps, args.warmup, dev)
+    r.plan.check(stream)
+    attn_ms, merge_ms = kernel_times(r, step, flush, dev, steps)
+    ab = algorithmic_bytes(tree)
+    mean = float(np.mean(ms))
+    entry = {"workload": tree.name, "kv_dtype": mode, "branches": tree.num_leaves,
+             "steps": steps, "ms_per_step": mean, "ms_per_step_median": float(np.median(ms)),
+             "value": tree.num_leaves / (mean * 1e-3), "kernel_ms": attn_ms, "merge_ms": merge_ms,
+             "frac": ab["attn"] / (attn_ms * 1e-3) / 1e9 / peak_gbs,
+             "step_frac": (ab["step"] / (peak_gbs * 1e9)) / (mean * 1e-3),
+             "t_roof_ms": ab["step"] / (peak_gbs * 1e9) * 1e3,
+             "algorithmic_bytes_per_step": ab["step"], "traffic": traffic_of(tree)}
+    r.plan.close()
+    del tree, r, out, lse, ws
+    torch.cuda.empty_cache()
+    return entry
 
 
 def run_gpu(args):
@@ -240,64 +403,34 @@ def run_gpu(args):
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
     from paper_2608_24658_gb300 import build
-    from paper_2608_24658_gb300.api import Plan
 
     build.build()
     tree = make_workload(args, device=dev)
-    plan = Plan.for_tree(tree)
+    r = Rank(tree, rank, world, dev)
+    plan = r.plan
     plan_info = plan.info()
     ws = plan.workspace(dev)
-    out = torch.empty_like(tree.q)
-    lse = torch.empty(tree.q.shape[:2], dtype=torch.float32, device=dev)
+    out = torch.empty_like(r.q)
+    lse = torch.empty(r.q.shape[:2], dtype=torch.float32, device=dev)
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
 
     def step():
-        plan.decode(tree.q, tree.k_pages, tree.v_pages, out=out, lse=lse, workspace=ws,
-                    k_scale=tree.k_scale, v_scale=tree.v_scale, stream=stream)
+        r.decode(out=out, lse=lse, ws=ws, stream=stream)
 
-    for _ in range(args.warmup):
-        flush.fill_(1.0)
-        step()
+    # compile-time configuration of the kernels and the tensor maps: once,
+    # outside the timed region
+    step()
     plan.check(stream)
 
-    # ---------------- timed region: K steps, L2 flushed before each
-    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    sampler = ClockSampler(local)
-    sampler.start()
-    time.sleep(0.3)
-    if world > 1:
-        import torch.distributed as dist
-        dist.barrier()
-    torch.cuda.synchronize(dev)
-    wall0 = time.perf_counter()
-    for i in range(args.steps):
-        flush.fill_(float(i))
-        starts[i].record(stream)
-        step()
-        ends[i].record(stream)
-    torch.cuda.synchronize(dev)
-    if world > 1:
-        dist.barrier()
-    wall = time.perf_counter() - wall0
-    clocks = sampler.stop()
+    # ---------------- timed region: warm-up, then K steps, L2 flushed before each
+    step_ms, wall, clocks = time_steps(step, flush, stream, args.steps, args.warmup, dev,
+                                       sampler=ClockSampler(local), world=world)
     plan.check(stream)
-    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     local_ms = float(np.mean(step_ms))
-
-    # ---------------- per-kernel times: the same steps with the library's
-    # events around its attention kernel (an event between the two kernels
-    # stops the merge grid from launching early, so this pass is separate)
-    kernel_steps = min(args.steps, 500)
-    plan.enable_timing(kernel_steps)
-    for i in range(kernel_steps):
-        flush.fill_(float(i))
-        step()
-    torch.cuda.synchronize(dev)
-    attn_ms, merge_ms = plan.read_timing(kernel_steps)
-    plan.enable_timing(0)
-    ms, units = aggregate(local_ms, tree.num_leaves, world, dev)
+    attn_ms, merge_ms = kernel_times(r, step, flush, dev, min(args.steps, 500))
+    ms, units = aggregate(local_ms, r.units, world, dev)
+    med_ms, _ = aggregate(float(np.median(step_ms)), r.units, world, dev)
     value = units / (ms / 1000.0)
 
     # ---------------- end to end: pinned host q in, out + lse back, every step
@@ -306,13 +439,13 @@ def run_gpu(args):
     # memory.  The GPU reaches both over NVLink-C2C, so the host<->device
     # transfers are those loads and stores.  The variant with an explicit
     # host-to-device copy of q into HBM first is timed beside it (e2e_copy).
-    q_host = tree.q.cpu().pin_memory()
+    q_host = r.q.cpu().pin_memory()
     out_bytes = out.numel() * out.element_size()
     res_bytes = out_bytes + lse.numel() * lse.element_size()
     res_host = torch.empty(res_bytes, dtype=torch.uint8).pin_memory()
     out_e = res_host[:out_bytes].view(out.dtype).view(out.shape)
     lse_e = res_host[out_bytes:].view(lse.dtype).view(lse.shape)
-    q_dev = torch.empty_like(tree.q)
+    q_dev = torch.empty_like(r.q)
     e2e_steps = max(3, min(args.steps, 200))
 
     def e2e_step(copy_q):
@@ -320,24 +453,12 @@ def run_gpu(args):
         if copy_q:
             q_dev.copy_(q_host, non_blocking=True)
             qa = q_dev
-        plan.decode(qa, tree.k_pages, tree.v_pages, out=out_e, lse=lse_e, workspace=ws,
-                    k_scale=tree.k_scale, v_scale=tree.v_scale, stream=stream)
+        r.decode(q=qa, out=out_e, lse=lse_e, ws=ws, stream=stream)
 
     def time_e2e(copy_q):
-        for _ in range(3):
-            flush.fill_(0.0)
-            e2e_step(copy_q)
-        torch.cuda.synchronize(dev)
-        e_starts = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
-        e_ends = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
-        for i in range(e2e_steps):
-            flush.fill_(float(i))
-            e_starts[i].record(stream)
-            e2e_step(copy_q)
-            e_ends[i].record(stream)
-        torch.cuda.synchronize(dev)
-        e_local = float(np.mean([s.elapsed_time(e) for s, e in zip(e_starts, e_ends)]))
-        e_ms, _ = aggregate(e_local, tree.num_leaves, world, dev)
+        e_ms, _, _ = time_steps(lambda: e2e_step(copy_q), flush, stream, e2e_steps, 3, dev,
+                                world=world)
+        e_ms, _ = aggregate(float(np.mean(e_ms)), r.units, world, dev)
         plan.check(stream)
         return units / (e_ms / 1000.0)
 
@@ -345,43 +466,38 @@ def run_gpu(args):
     e2e_copy_value = time_e2e(True)
 
     if rank != 0:
+        plan.close()
         if world > 1:
             dist.destroy_process_group()
         return 0
 
-    # ---------------- roofline of the attention kernel
+    # ---------------- roofline of the attention kernel (this rank's share)
     peak_gbs, peak_kind = measured_peaks()
-    ab = algorithmic_bytes(tree)
-    attn_avg_ms = float(np.mean(attn_ms)) if len(attn_ms) else float("nan")
-    merge_avg_ms = float(np.mean(merge_ms)) if len(merge_ms) else float("nan")
-    achieved = ab["attn"] / (attn_avg_ms * 1e-3) / 1e9
-    traffic = None
-    tr_path = os.path.join(ROOT, "profiles", "traffic.json")
-    if os.path.exists(tr_path):
-        with open(tr_path) as f:
-            tr = json.load(f).get(f"{tree.name}:{tree.mode}")
-        if tr and tr.get("kernel_source_hash") == kernel_source_hash():
-            traffic = tr["bytes_per_launch"]
+    ab = algorithmic_bytes(tree) if world == 1 else algorithmic_bytes_of_plan(r)
+    achieved = ab["attn"] / (attn_ms * 1e-3) / 1e9
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak_gbs, "unit": "GB/s",
-                "frac": achieved / peak_gbs, "traffic": traffic,
+                "frac": achieved / peak_gbs, "traffic": traffic_of(tree) if world == 1 else None,
                 "kernel": f"attn_{tree.mode}_kernel", "peak_kind": peak_kind,
-                "algorithmic_bytes_per_launch": ab["attn"], "kernel_ms": attn_avg_ms,
-                "merge_ms": merge_avg_ms,
-                "step_frac": (ab["step"] / (peak_gbs * 1e9)) / (ms * 1e-3)}
+                "algorithmic_bytes_per_launch": ab["attn"], "kernel_ms": attn_ms,
+                "merge_ms": merge_ms,
+                "step_frac": (ab["step"] / (peak_gbs * 1e9)) / (local_ms * 1e-3)}
 
     # ---------------- CPU baseline: oracle on a bounded sample of this workload
     cpu = None
     if not args.no_cpu_baseline and world == 1:
-        host_tree = tree.to("cpu")
-        rate, n, el, cores = oracle_sample_rate(host_tree, args.cpu_seconds)
+        rate, n, el, cores, pool = oracle_sample_rate(tree, args.cpu_seconds)
         cpu = {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
-               "sample": f"{n} whole branch(es) of {tree.num_leaves} (all q heads), {el:.1f} s"}
+               "sample": f"{n} whole branch(es), cycling over {pool} sampled branches of "
+                         f"{tree.num_leaves} (all q heads), {el:.1f} s of oracle time"}
 
+    shard = None if world == 1 else f"{r.kind} over {world} GPUs"
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "warmup": args.warmup, "ms_per_step": ms, "ms_per_step_median": med_ms,
+        "higher_is_better": True,
+        "scaling": "strong" if r.kind in ("requests", "kv_heads") else "weak",
         "vs_baseline": None, "dtype": "bf16" if tree.mode != "fp32" else "f32",
-        "data": "synthetic", "config": workload_config(tree, args),
+        "data": "synthetic", "config": workload_config(tree, args, shard),
         "e2e": {"value": e2e_value, "unit": UNIT,
                 "h2d_bytes_per_step": int(q_host.numel() * q_host.element_size()),
                 "d2h_bytes_per_step": int(res_host.numel()),
@@ -393,14 +509,36 @@ def run_gpu(args):
         "wall_s_timed_region": wall,
         "algorithmic": {"bytes_per_step": ab["step"], "flops_per_step": algorithmic_flops(tree)},
         "plan": {k: v for k, v in plan_info.items()
-                 if k in ("num_items", "num_ctas", "num_wide_ctas", "num_workers", "num_slots",
+                 if k in ("num_items", "num_ctas", "num_wide_ctas", "num_slots",
                           "num_merge_entries")},
     }
-    print(json.dumps(line), flush=True)
     plan.close()
+    del tree, r, out, lse, ws, q_dev
+    torch.cuda.empty_cache()
+
+    # ---------------- the other configurations, same process, one GPU
+    if world == 1 and args.table:
+        table = []
+        for idx, mode in TABLE:
+            if (idx, mode) == (args.config, args.mode):
+                continue
+            table.append(measure_table_entry(idx, mode, args, dev, stream, flush, peak_gbs))
+        line["configs"] = table
+    print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
     return 0
+
+
+def algorithmic_bytes_of_plan(r):
+    """Algorithmic bytes of one rank's share (unique KV it reads + its q, out, lse)."""
+    info = r.plan.info()
+    t = r.tree
+    hkv = r.plan.num_kv_heads
+    kv = info["unique_tokens"] * 2 * hkv * t.head_dim * t.kv_elem_bytes()
+    q = r.q.numel() * r.q.element_size()
+    lse = r.q.shape[0] * r.q.shape[1] * 4
+    return {"kv": kv, "q": q, "out": q, "lse": lse, "step": kv + 2 * q + lse, "attn": kv + q}
 
 
 def kernel_source_hash() -> str:
@@ -637,7 +775,13 @@ def main(argv=None):
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--config", type=int, default=2, help="workload 1-5 (default 2)")
+    ap.add_argument("--config", type=int, default=4,
+                    help="workload 1-5 of the JSON line (default 4: 32 requests x 32 "
+                         "branches, permuted pages, the largest that fits one GPU)")
+    ap.add_argument("--no-table", dest="table", action="store_false",
+                    help="skip the other configurations timed after the headline")
+    ap.add_argument("--table-steps", type=int, default=300,
+                    help="timed steps of each configuration of the table")
     ap.add_argument("--mode", choices=["bf16", "fp8", "fp32"], default="bf16")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -54,7 +54,9 @@ typedef enum {
     PARASON_ECUDA = 3,        /* a CUDA runtime call failed               */
     PARASON_ETIMEOUT = 4,     /* a bounded device wait expired            */
     PARASON_EUNSUPPORTED = 5, /* valid but not implemented (shape / mode) */
-    PARASON_ENOSPACE = 6      /* the plan has no room for an update: build a new one */
+    PARASON_ENOSPACE = 6,     /* the plan has no room for an update: build a new one */
+    PARASON_ERANGE = 7        /* an input value outside what the mode's kernels hold
+                                 (e4m3 KV: |q| >= 65520, see parason_attn_decode) */
 } parason_status;
 
 typedef enum {
@@ -166,12 +168,68 @@ parason_status parason_prefill_plan_host(const parason_attn_config *cfg, int32_t
                                          int64_t num_physical_pages, int32_t num_sms,
                                          parason_plan *out);
 
+/*
+ * One rank's part of a decode step that `world` ranks (one GPU each) share
+ * with no exchange between them: the plan of the work rank `rank` computes.
+ * The paper's runtime decodes each request's branches as independent
+ * workers (Sec. 3.4), and requests do not read each other's KV; and the kv
+ * heads of grouped-query attention are independent too.  So the step splits
+ * either way with nothing to combine afterwards.
+ *
+ *   kind PARASON_SHARD_REQUESTS: the roots (requests), in index order, are
+ *     cut into `world` contiguous groups of about equal cost (the tokens of
+ *     a request's nodes that some branch reads, plus H_q/H_kv per branch);
+ *     rank r plans the requests of group r.  Its branch b is global branch
+ *     PARASON_TABLE_SHARD_BRANCHES[b] (increasing): q, out and lse of the
+ *     rank hold those rows, in that order.  Page ids are the caller's, so
+ *     the rank's pools are addressed as the whole pool would be
+ *     (num_physical_pages pages); only the rank's pages are read.  A rank
+ *     with no request gets a plan with no branch (decode does nothing).
+ *   kind PARASON_SHARD_KV_HEADS: rank r takes kv heads [r H_kv / world,
+ *     (r + 1) H_kv / world) and their q heads [r H_q / world, (r + 1) H_q /
+ *     world); H_kv must be a multiple of world.  The plan is that of cfg
+ *     with H_kv / world kv heads and H_q / world q heads over every branch:
+ *     q, out and lse hold the rank's heads ([num_leaves, H_q / world, d]),
+ *     the pools hold the rank's kv heads ([P, H_kv / world, 16, d]).
+ *
+ * The whole tree is validated as by parason_attn_plan (same errors), then
+ * PARASON_EINVAL for world < 1, rank outside [0, world), an unknown kind, or
+ * H_kv not a multiple of world (kv-head shards).  Ownership, concurrency and
+ * every other call on the returned plan are as for parason_attn_plan.
+ */
+enum { PARASON_SHARD_REQUESTS = 0, PARASON_SHARD_KV_HEADS = 1 };
+parason_status parason_attn_plan_shard(const parason_attn_config *cfg, int32_t num_nodes,
+                                       const int32_t *parent, const int32_t *node_len,
+                                       const int32_t *node_page_ptr, const int32_t *page_ids,
+                                       int32_t num_leaves, const int32_t *leaf_node,
+                                       int64_t num_physical_pages, int32_t kind, int32_t rank,
+                                       int32_t world, parason_stream_t stream, parason_plan *out);
+
+/* parason_attn_plan_shard without device memory or CUDA calls (inspection),
+ * as parason_attn_plan_host is to parason_attn_plan. */
+parason_status parason_attn_plan_shard_host(const parason_attn_config *cfg, int32_t num_nodes,
+                                            const int32_t *parent, const int32_t *node_len,
+                                            const int32_t *node_page_ptr, const int32_t *page_ids,
+                                            int32_t num_leaves, const int32_t *leaf_node,
+                                            int64_t num_physical_pages, int32_t kind, int32_t rank,
+                                            int32_t world, int32_t num_sms, parason_plan *out);
+
 /* Device workspace (bytes) that parason_attn_decode needs for this plan:
  * the split partial results (o, m, l) of every work item.  0 for NULL. */
 size_t parason_plan_workspace_bytes(parason_plan plan);
 
 /*
  * One decode step: out[b, h, :] = softmax(s) V over branch b's root->leaf KV.
+ *
+ * Defining passage: the runtime dispatches every <Subtask> / <Trial> entry of
+ * a parallel region as an independent worker that decodes its own thread
+ * (Sec. 3.4), and a branch's tokens are later concatenated into the context
+ * rather than selected (Sec. 3.1, Trial Parallelism; Fig. 1 caption), so one
+ * step needs every live branch's attention over its whole context: the KV
+ * of each tree node on its root -> leaf path, root first (nested regions per
+ * Fig. 4, rule W -> <Thread> B </Thread>).  The paper gives no attention
+ * formula; this is plain softmax attention, s_t = sm_scale * <q, k_t>.
+ *
  * Asynchronous on `stream`; allocates nothing; capturable in a CUDA graph.
  *
  *   q        device, [num_leaves, H_q, head_dim], bf16 (fp32 in FP32 mode),
@@ -193,7 +251,14 @@ size_t parason_plan_workspace_bytes(parason_plan plan);
  *            256-byte aligned; no contents are kept between calls.
  *
  * Slots of a node's last page past node_len are never read into the result,
- * whatever they hold (NaN included).  Returns PARASON_EINVAL on a host-only
+ * whatever they hold (NaN included).
+ *
+ * With e4m3 KV the kernels multiply q by the widened keys and values in f16
+ * (f16 holds every e4m3 value exactly): q is narrowed from bf16 to f16,
+ * which is exact for |q| < 65504 except in the low bits of values below
+ * 2^-14.  A q element of magnitude 65520 or more (inf included) cannot be
+ * narrowed: the kernel records PARASON_ERANGE, which the next
+ * parason_plan_check returns, and that call's out and lse are undefined.  Returns PARASON_EINVAL on a host-only
  * plan, a NULL or misaligned buffer or a short workspace, PARASON_ECUDA if a
  * launch fails.  Device-side failures (a bounded wait that expired) are
  * reported by parason_plan_check.
@@ -264,8 +329,10 @@ parason_status parason_attn_decode_no_alloc(parason_plan plan, const void *q,
  * item has no room left for another page: a plan leaves each branch room for
  * half as many pages as its last item had (4 to 64 pages), beyond which the
  * grown item would unbalance the decode; PARASON_EUNSUPPORTED in FP32 mode.  On any error
- * nothing is changed.  Forking (new branches at an </Outlines>) needs a
- * new plan.  PARASON_EUNSUPPORTED on a prefill plan.
+ * nothing is changed, on the host or on the device: the device copy is
+ * updated first, and the host copy only once that succeeded.
+ * PARASON_EINVAL if the current device is not the plan's.
+ * PARASON_EUNSUPPORTED on a prefill plan.
  */
 parason_status parason_plan_append(parason_plan plan, const int32_t *new_pages,
                                    parason_stream_t stream);
@@ -273,7 +340,14 @@ parason_status parason_plan_append(parason_plan plan, const int32_t *new_pages,
 /*
  * Combine two attention results over disjoint key sets A and B (for example
  * two KV ranges of one branch, or a branch's context before and after a join)
- * into the result over A u B, row by row:
+ * into the result over A u B, row by row.
+ *
+ * Defining passage: a thread's result returns to the main trajectory and the
+ * branches are concatenated into its context (Sec. 3.4; Sec. 3.1, Trial
+ * Parallelism: the merge step concatenates rather than selects; Fig. 1), so
+ * attention over the joined context is attention over the union of the key
+ * sets; the paper gives no formula, and this is the exact log-sum-exp
+ * identity for softmax over a union of disjoint sets:
  *   o = (e^{lse_a} o_a + e^{lse_b} o_b) / (e^{lse_a} + e^{lse_b})
  *   lse = ln(e^{lse_a} + e^{lse_b})
  * A side with lse = -inf is empty; both empty gives o = 0, lse = -inf.
@@ -288,7 +362,9 @@ parason_status parason_lse_merge(const void *o_a, const float *lse_a, const void
 
 /* Synchronise `stream`, then read and clear the plan's device error word:
  * PARASON_ETIMEOUT if a kernel gave up a bounded wait since the last check,
- * PARASON_ECUDA if the stream reports an error, else PARASON_OK. */
+ * PARASON_ERANGE if an e4m3-KV decode met a q element of magnitude 65520 or
+ * more (the first error recorded wins), PARASON_ECUDA if the stream reports
+ * an error, else PARASON_OK. */
 parason_status parason_plan_check(parason_plan plan, parason_stream_t stream);
 
 /* Release the plan's host and device memory.  NULL is a no-op.  Work queued
@@ -347,6 +423,9 @@ parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info)
  *                            decode plans): for an item over its chunk's own
  *                            node, the index in that node of its first key
  *                            (the causal mask's origin), else -1
+ *   PARASON_TABLE_SHARD_BRANCHES int32 [num_leaves]: the global index of
+ *                            each of the plan's branches (parason_attn_plan_
+ *                            shard); b for a plan that is not a shard
  * Returns PARASON_EINVAL if `bytes` is smaller than the table.
  */
 enum {
@@ -358,7 +437,8 @@ enum {
     PARASON_TABLE_NARROW_QUEUE = 5,
     PARASON_TABLE_ITEM_ROWS = 6,
     PARASON_TABLE_STREAM_ROWS = 7,
-    PARASON_TABLE_ITEM_KEY0 = 8
+    PARASON_TABLE_ITEM_KEY0 = 8,
+    PARASON_TABLE_SHARD_BRANCHES = 9
 };
 parason_status parason_plan_export(parason_plan plan, int32_t table, void *dst, size_t bytes);
 
@@ -369,8 +449,12 @@ parason_status parason_plan_export(parason_plan plan, int32_t table, void *dst, 
  * first KV load, so its consumers' wait can only expire: the kernel records
  * PARASON_ETIMEOUT, lets its other copies land, and exits; the output is
  * then undefined.  Used to test the timeout path without faulting the GPU.
+ * Flag PARASON_DEBUG_FAIL_UPDATE makes parason_plan_append and
+ * parason_plan_fork fail with PARASON_ECUDA at the point where they would
+ * update the device copy (after every check, before anything is changed),
+ * on host-only plans too: used to test that a failed update changes nothing.
  */
-enum { PARASON_DEBUG_SKIP_FIRST_LOAD = 1u };
+enum { PARASON_DEBUG_SKIP_FIRST_LOAD = 1u, PARASON_DEBUG_FAIL_UPDATE = 2u };
 parason_status parason_plan_set_debug(parason_plan plan, uint32_t flags, int64_t wait_limit_ns);
 
 /*

@@ -11,11 +11,14 @@ import os
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_build", "libparason.so")
 
-OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EUNSUPPORTED, ENOSPACE = range(7)
+OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EUNSUPPORTED, ENOSPACE, ERANGE = range(8)
 MODES = {"bf16": 0, "fp32": 1, "fp8": 2}
 (TABLE_ITEMS, TABLE_DFS_LEAVES, TABLE_MERGE_PTR, TABLE_MERGE, TABLE_WIDE_QUEUE,
- TABLE_NARROW_QUEUE, TABLE_ITEM_ROWS, TABLE_STREAM_ROWS, TABLE_ITEM_KEY0) = range(9)
+ TABLE_NARROW_QUEUE, TABLE_ITEM_ROWS, TABLE_STREAM_ROWS, TABLE_ITEM_KEY0,
+ TABLE_SHARD_BRANCHES) = range(10)
+SHARD_REQUESTS, SHARD_KV_HEADS = 0, 1
 DEBUG_SKIP_FIRST_LOAD = 1
+DEBUG_FAIL_UPDATE = 2
 NO_ALLOC_SCRATCH_BYTES = 64 << 20   # PARASON_NO_ALLOC_SCRATCH_BYTES
 
 # every function include/parason.h declares, with (restype, argtypes)
@@ -59,6 +62,11 @@ SIGNATURES = {
                                             _p, _i64, _p, _pp]),
     "parason_prefill_plan_host": (ctypes.c_int, [ctypes.POINTER(AttnConfig), _i32, _p, _p, _p, _p,
                                                  _i32, _p, _i64, _i32, _pp]),
+    "parason_attn_plan_shard": (ctypes.c_int, [ctypes.POINTER(AttnConfig), _i32, _p, _p, _p, _p,
+                                               _i32, _p, _i64, _i32, _i32, _i32, _p, _pp]),
+    "parason_attn_plan_shard_host": (ctypes.c_int, [ctypes.POINTER(AttnConfig), _i32, _p, _p, _p,
+                                                    _p, _i32, _p, _i64, _i32, _i32, _i32, _i32,
+                                                    _pp]),
     "parason_plan_workspace_bytes": (_sz, [_p]),
     "parason_attn_decode": (ctypes.c_int, [_p, _p, _p, _p, _p, _p, _p, _p, _p, _sz, _p]),
     "parason_attn_decode_no_alloc": (ctypes.c_int, [_p, _p, _p, _p, _p, _p, _p, _p, _p]),

@@ -54,7 +54,7 @@ class Plan:
                  parent, node_len, node_page_ptr, page_ids, leaf_node,
                  num_physical_pages: int, sm_scale: float = 0.0, page_size: int = 16,
                  stream=None, host_only: bool = False, num_sms: int = 152,
-                 prefill: bool = False):
+                 prefill: bool = False, shard=None):
         lib = _lib.load()
         self.mode = mode
         self.num_q_heads, self.num_kv_heads, self.head_dim = num_q_heads, num_kv_heads, head_dim
@@ -66,6 +66,30 @@ class Plan:
         node_page_ptr, page_ids, leaf_node = _i32(node_page_ptr), _i32(page_ids), _i32(leaf_node)
         out = ctypes.c_void_p()
         kind = "prefill" if prefill else "attn"
+        self.shard = shard
+        if shard is not None:
+            # (kind, rank, world): one rank's plan (parason_attn_plan_shard)
+            skind, rank, world = (int(x) for x in shard)
+            if prefill:
+                raise ValueError("prefill plans are not sharded")
+            args = (ctypes.byref(self._cfg), len(parent), _ptr(parent), _ptr(node_len),
+                    _ptr(node_page_ptr), _ptr(page_ids), len(leaf_node), _ptr(leaf_node),
+                    self.num_physical_pages, skind, rank, world)
+            if host_only:
+                st = lib.parason_attn_plan_shard_host(*args, num_sms, ctypes.byref(out))
+            else:
+                st = lib.parason_attn_plan_shard(*args, _stream_handle(stream), ctypes.byref(out))
+            check(st, "parason_attn_plan_shard")
+            self._h = out
+            self._ws = None
+            self.host_only = host_only
+            self.prefill = False
+            info = self.info()
+            self.num_leaves = int(info["num_leaves"])
+            if skind == _lib.SHARD_KV_HEADS:
+                self.num_q_heads //= world
+                self.num_kv_heads //= world
+            return
         if host_only:
             fn = getattr(lib, f"parason_{kind}_plan_host")
             st = fn(ctypes.byref(self._cfg), len(parent), _ptr(parent), _ptr(node_len),
@@ -144,7 +168,8 @@ class Plan:
                  _lib.TABLE_NARROW_QUEUE: (inf["num_narrow_items"],),
                  _lib.TABLE_ITEM_ROWS: (inf["num_items"] + 1,),
                  _lib.TABLE_STREAM_ROWS: (inf["num_stream_rows"],),
-                 _lib.TABLE_ITEM_KEY0: (inf["num_items"] if self.prefill else 0,)}[table]
+                 _lib.TABLE_ITEM_KEY0: (inf["num_items"] if self.prefill else 0,),
+                 _lib.TABLE_SHARD_BRANCHES: (inf["num_leaves"],)}[table]
         buf = np.zeros(shape, dtype=np.int32)
         check(_lib.load().parason_plan_export(self.handle, table, _ptr(buf), buf.nbytes),
               "plan_export")

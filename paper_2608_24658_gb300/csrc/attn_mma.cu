@@ -3,38 +3,52 @@
 // One persistent launch, one CTA per SM, two roles (the planner decides how
 // many SMs each gets so that both finish together):
 //
-//  * prefix pass (CTAs [0, num_wide_ctas)): nodes that many branches share.
-//    Up to 128 query rows -- the branches under the node times the q heads
-//    of one kv head -- are stacked on one page stream: a producer warp moves
-//    each (page, kv head) of K and V by TMA (3-D boxes, 128-byte swizzle)
-//    into a shared ring, and 8 consumer warps of 16 rows each read it from
-//    shared memory.  The node's KV is read from HBM once for all its rows,
-//    which is what the shared prefix of Subtask/Trial branches buys (paper
-//    Sec. 3.1, 3.4).
-//  * suffix pass (the other CTAs): nodes of at most 16 rows (a branch's own
-//    suffix).  Each of the 8 warps is an independent worker with its own
-//    TMA ring and its own balanced list of items (split-K pieces of
-//    suffixes): no CTA barrier, no cross-warp combine.
+//  * prefix pass (CTAs [0, num_wide_ctas)): nodes that many branches share
+//    (the request prefix, a subtask thread).  Up to 128 query rows -- the
+//    branches under the node times the q heads of one kv head -- are stacked
+//    into one tile against the node's pages, so the node's KV is read from
+//    HBM once for all of them, which is what the shared prefix of
+//    Subtask/Trial branches buys (paper Sec. 3.1, 3.4).
+//      - head_dim 128 (bf16 or e4m3 KV): a tcgen05 tile (prefix_cta_tc).
+//        Warp roles: a scheduler warp stages each item's metadata; a
+//        producer warp moves 64-token blocks of K and V by TMA (one 5-D box
+//        per column block when the block's 4 pages are consecutive in the
+//        pool, else 3-D boxes per page) into a 6-stage ring; one thread
+//        issues S = Q K^T and another O += P V as tcgen05.mma with Q, S/P and
+//        O in TMEM and K, V from shared memory; 4 softmax warps own one row
+//        per thread (TMEM lane) and write P over S; 4 epilogue warps store an
+//        item's O and load Q two items ahead (with e4m3 KV they also convert
+//        each staged block to f16).
+//      - head_dim 64: mma.sync (prefix_cta): a producer warp streams pages
+//        into a ring, 8 consumer warps of 16 rows share the pages and combine
+//        through shared memory.
+//  * suffix pass (the other CTAs, and prefix CTAs once the prefix queue is
+//    empty): nodes of at most 16 rows (a branch's own suffix).  Each warp is
+//    an independent worker with its own TMA ring that pulls split-K pieces
+//    from a queue: no CTA barrier, no cross-warp combine.  QK^T and PV are
+//    mma.sync m16n8k16 with fp32 accumulation and a quad-shuffle online
+//    softmax; tiles of 5 to 8 rows run the transposed step (S^T = K Q^T).
 //
-// Both roles use tensor-core QK^T and PV (mma.sync m16n8k16, fp32
-// accumulate) and an online softmax in registers with quad shuffles, and
-// write a partial (o, m, l) per item row.  The merge kernel (merge.cu) folds
-// the partials of every branch's path; it is launched as a programmatic
-// dependent of this grid.
+// Every item writes a partial (o, m, l) per row.  The merge kernel (merge.cu)
+// folds the partials of every branch's path; it is launched as a
+// programmatic dependent of this grid.
 //
 // KV formats:
 //  * bf16: fragments by ldmatrix (V transposed by ldmatrix.trans), bf16 MMA.
 //  * e4m3 (one fp32 scale per kv head for K and for V): 4- and 16-byte
 //    shared loads, every e4m3 pair widened to f16 exactly (cvt.rn.f16x2.
-//    e4m3x2), f16 MMA; q is widened from bf16 to f16 (exact for |q| in the
-//    f16 normal range).  The K scale joins the softmax scale, the V scale
-//    multiplies the partial o.  The fragment layouts permute d so that each
-//    thread's bytes are contiguous: QK^T takes d = 16ks + 4t + {0..3} for
-//    thread t of a quad, PV gives thread column c of n-tile n the output
-//    d = 16c + n.
+//    e4m3x2), f16 MMA; q is narrowed from bf16 to f16 (exact for |q| in the
+//    f16 normal range; a q element that would overflow f16 is reported as
+//    PARASON_ERANGE through the plan's error record).  The K scale joins the
+//    softmax scale, the V scale multiplies the partial o.  The suffix
+//    fragment layouts permute d so that each thread's bytes are contiguous:
+//    QK^T takes d = 16ks + 4t + {0..3} for thread t of a quad, PV gives
+//    thread column c of n-tile n the output d = 16c + n.
 //
 // Scores are kept in the log2 domain: x = scale*log2(e)*<q,k>, so a partial
 // is m = max x, l = sum 2^(x-m), o = sum 2^(x-m) v (unnormalised).
+#include <mutex>
+
 #include "device_common.cuh"
 #include "tcgen05.cuh"
 
@@ -172,6 +186,23 @@ __device__ __forceinline__ uint32_t e4m3x2_to_f16x2(uint32_t two_bytes) {
         : "=r"(out)
         : "r"(two_bytes));
     return out;
+}
+
+// A bf16 pair of q narrowed to an f16 pair for the e4m3 MMAs.  The f16
+// values are exact for |q| < 65504 (tiny values lose low bits); an element
+// of magnitude 65520 or more (including inf) would round to inf, so `big` is
+// set and the caller reports PARASON_ERANGE rather than returning a silently
+// wrong result.  NaN is passed through and not flagged.
+__device__ __forceinline__ uint32_t q_pair_to_f16(uint32_t two, bool &big) {
+    const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162 *>(&two);
+    const float lo = __low2float(b), hi = __high2float(b);
+    big |= fmaxf(fabsf(lo), fabsf(hi)) >= 65520.f;
+    return dev::pack_f16(lo, hi);
+}
+
+// Record PARASON_ERANGE once per warp if any lane saw an out-of-range q.
+__device__ __forceinline__ void report_q_range(const AttnArgs &a, bool big, int lane) {
+    if (__any_sync(0xffffffffu, big) && lane == 0) dev::record_error(a.err, PARASON_ERANGE, kSiteQRange);
 }
 
 __device__ __forceinline__ uint32_t lds32(uint32_t addr) {
@@ -398,6 +429,7 @@ __device__ __forceinline__ void load_q_fragments_t(const AttnArgs &a, const Work
         const int head = it.kv_head * a.group + nr % a.group;
         qrow = static_cast<const __nv_bfloat16 *>(a.q) + (static_cast<int64_t>(leaf) * a.num_q_heads + head) * D;
     }
+    bool big = false;
 #pragma unroll
     for (int ks = 0; ks < D / 16; ++ks) {
         if constexpr (KV::kElemBytes == 2) {
@@ -406,12 +438,11 @@ __device__ __forceinline__ void load_q_fragments_t(const AttnArgs &a, const Work
         } else {
             uint2 u = make_uint2(0u, 0u);
             if (qrow) u = *reinterpret_cast<const uint2 *>(qrow + ks * 16 + 4 * tig);
-            const __nv_bfloat162 p0 = *reinterpret_cast<const __nv_bfloat162 *>(&u.x);
-            const __nv_bfloat162 p1 = *reinterpret_cast<const __nv_bfloat162 *>(&u.y);
-            qb[ks][0] = dev::pack_f16(__low2float(p0), __high2float(p0));
-            qb[ks][1] = dev::pack_f16(__low2float(p1), __high2float(p1));
+            qb[ks][0] = q_pair_to_f16(u.x, big);
+            qb[ks][1] = q_pair_to_f16(u.y, big);
         }
     }
+    if constexpr (KV::kElemBytes == 1) report_q_range(a, big, lane);
 }
 
 template <int D, class KV>
@@ -564,6 +595,7 @@ __device__ __forceinline__ void load_q_fragments(const AttnArgs &a, const WorkIt
             qrow[h] = qb + (static_cast<int64_t>(leaf) * a.num_q_heads + head) * D;
         }
     }
+    bool big = false;
 #pragma unroll
     for (int ks = 0; ks < D / 16; ++ks)
 #pragma unroll
@@ -575,12 +607,11 @@ __device__ __forceinline__ void load_q_fragments(const AttnArgs &a, const WorkIt
             } else {
                 uint2 u = make_uint2(0u, 0u);
                 if (qrow[h]) u = *reinterpret_cast<const uint2 *>(qrow[h] + ks * 16 + 4 * tig);
-                const __nv_bfloat162 p0 = *reinterpret_cast<const __nv_bfloat162 *>(&u.x);
-                const __nv_bfloat162 p1 = *reinterpret_cast<const __nv_bfloat162 *>(&u.y);
-                qa[ks][h] = dev::pack_f16(__low2float(p0), __high2float(p0));
-                qa[ks][2 + h] = dev::pack_f16(__low2float(p1), __high2float(p1));
+                qa[ks][h] = q_pair_to_f16(u.x, big);
+                qa[ks][2 + h] = q_pair_to_f16(u.y, big);
             }
         }
+    if constexpr (KV::kElemBytes == 1) report_q_range(a, big, lane);
 }
 
 // Softmax scale of an item and the factor of its partial o (the kv head's
@@ -1613,10 +1644,10 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
         // ... then into TMEM Q buffer k & 1 (bf16 pairs, or f16 pairs for
         // the e4m3 tile, lane r)
         auto put_q = [&](int k, const uint4 (&qv)[16]) {
-            auto cv = [](uint32_t two) {
+            bool big = false;
+            auto cv = [&big](uint32_t two) {
                 if constexpr (!kF8) return two;
-                const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162 *>(&two);
-                return dev::pack_f16(__low2float(b), __high2float(b));
+                return q_pair_to_f16(two, big);
             };
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
@@ -1630,6 +1661,7 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
                 }
                 tc::st32(lane_base + kTmemQ + 64u * (k & 1) + 32u * h, w);
             }
+            if constexpr (kF8) report_q_range(a, big, lane);
             tc::wait_st();
             tc::fence_before_sync();
             dev::mbar_arrive(bar(kBarQReady + (k & 1)));
@@ -1858,29 +1890,38 @@ __global__ void __launch_bounds__(kThreads, 1)
         suffix_warp<D, KV>(&maps.k, &maps.v, a, ring, bars, warp, lane, grab_items[warp]);
 }
 
-// Shared memory and carveout are set once per device; reports the number of
-// CTAs that fit per SM (the persistent grid needs one).
+// Shared memory and carveout are set once per device (with that device
+// current); reports the number of CTAs that fit per SM (the persistent grid
+// needs one).  The per-device results sit in an array guarded by a mutex, so
+// threads that plan or decode on different devices neither race nor read
+// another device's count.
+constexpr int kMaxConfigDevices = 64;
+
 template <int D, class KV>
 cudaError_t configure(int *ctas_per_sm) {
     using S = Shape<D, KV>;
-    static int configured_device = -1;
-    static int resident = 0;
+    static std::mutex mu;
+    static int resident[kMaxConfigDevices] = {};   // 0: not configured yet
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    if (configured_device != dev) {
+    if (dev < 0 || dev >= kMaxConfigDevices) return cudaErrorNotSupported;
+    std::lock_guard<std::mutex> lock(mu);
+    if (resident[dev] == 0) {
         e = cudaFuncSetAttribute(attn_kernel<D, KV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  S::kSmemBytes);
         if (e != cudaSuccess) return e;
         e = cudaFuncSetAttribute(attn_kernel<D, KV>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                  cudaSharedmemCarveoutMaxShared);
         if (e != cudaSuccess) return e;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&resident, attn_kernel<D, KV>, kThreads,
+        int n = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attn_kernel<D, KV>, kThreads,
                                                           S::kSmemBytes);
         if (e != cudaSuccess) return e;
-        configured_device = dev;
+        // a kernel that does not fit is remembered as -1 (never configured again)
+        resident[dev] = n > 0 ? n : -1;
     }
-    if (ctas_per_sm) *ctas_per_sm = resident;
+    if (ctas_per_sm) *ctas_per_sm = resident[dev] > 0 ? resident[dev] : 0;
     return cudaSuccess;
 }
 

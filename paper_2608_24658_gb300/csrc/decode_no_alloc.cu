@@ -8,7 +8,7 @@
 
 #include <mutex>
 
-#include "parason.h"
+#include "internal.h"
 
 // Partial results (unnormalised o, then the running max and sum of every
 // row) of one decode step.  Never needs zeroing: the attention kernel writes
@@ -31,7 +31,11 @@ parason_status scratch_on_current_device(void **addr) {
     std::lock_guard<std::mutex> lock(g_scratch_mutex);
     if (!g_scratch_addr[dev]) {
         void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_partials_scratch) != cudaSuccess || !p) return PARASON_ECUDA;
+        if (cudaGetSymbolAddress(&p, g_partials_scratch) != cudaSuccess || !p) {
+            // leave no error pending for the next, unrelated runtime call
+            cudaGetLastError();
+            return PARASON_ECUDA;
+        }
         g_scratch_addr[dev] = p;
     }
     *addr = g_scratch_addr[dev];
@@ -47,9 +51,16 @@ extern "C" parason_status parason_attn_decode_no_alloc(parason_plan plan, const 
                                                        parason_stream_t stream) {
     if (!plan) return PARASON_EINVAL;
     if (parason_plan_workspace_bytes(plan) > sizeof(g_partials_scratch)) return PARASON_EUNSUPPORTED;
-    parason_plan_info info{};
-    if (parason_plan_get_info(plan, &info) != PARASON_OK) return PARASON_EINVAL;
-    if (!info.on_device) return PARASON_EINVAL;
+    // the plan's device must be current before the scratch is looked up:
+    // the lookup loads the library's device image on the current device
+    const int plan_dev = parason::plan_device(plan);
+    if (plan_dev < 0) return PARASON_EINVAL;
+    int cur = -1;
+    if (cudaGetDevice(&cur) != cudaSuccess) {
+        cudaGetLastError();
+        return PARASON_ECUDA;
+    }
+    if (cur != plan_dev) return PARASON_EINVAL;
     void *scratch = nullptr;
     const parason_status st = scratch_on_current_device(&scratch);
     if (st != PARASON_OK) return st;

@@ -45,6 +45,7 @@ enum WaitSite : int32_t {
     kSiteConsumerFull = 1,
     kSiteProducerEmpty = 2,
     kSiteBadItem = 3,        // an item the kernel cannot hold (planner contract broken)
+    kSiteQRange = 4,         // e4m3 KV: a q element that f16 cannot hold (PARASON_ERANGE)
 };
 
 struct AttnArgs {
@@ -105,6 +106,9 @@ struct MergeArgs {
     int32_t *queue_next;        // set back to queue_start for the next launch
     int32_t queue_start[2];
 };
+
+// Device a plan's metadata lives on (-1 for a host-only plan or NULL).
+int plan_device(parason_plan plan);
 
 // Resident CTAs per SM of the persistent attention kernel of a mode (sets its
 // attributes); cudaErrorNotSupported for a shape it has no kernel for.

@@ -114,6 +114,7 @@ struct parason_plan_s {
     int64_t unique_tokens = 0;
     int64_t path_tokens = 0;
     bool prefill = false;              // a tree-masked prefill plan
+    std::vector<int32_t> shard_branch; // sharded plans: global index of each branch
     std::vector<int32_t> item_key0;    // prefill: first key of a causal item, else -1
 
     // device side
@@ -171,34 +172,17 @@ parason_status validate_config(const parason_attn_config *cfg) {
     return PARASON_OK;
 }
 
-// With `prefill`, leaf_node holds the chunk nodes of a tree-masked prefill:
-// every token of a chunk is a query (numbered chunk by chunk), attending to
-// every token of its node's ancestors and causally to its own node.
-parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int32_t num_nodes,
-                          const int32_t *parent, const int32_t *node_len,
-                          const int32_t *node_page_ptr, const int32_t *page_ids,
-                          int32_t num_leaves, const int32_t *leaf_node,
-                          int64_t num_phys, int32_t num_sms, bool prefill = false) {
-    parason_status st = validate_config(cfg);
-    if (st != PARASON_OK) return st;
-    // the prefill's causal mask is in the tcgen05 tile: bf16 or e4m3 KV at head_dim 128
-    if (prefill && (cfg->mode == PARASON_FP32 || cfg->head_dim != 128)) return PARASON_EUNSUPPORTED;
-    p->prefill = prefill;
+// The tree and its page table: parents before children, page counts that
+// match the lengths, page ids in range and owned once, branches distinct,
+// in range and childless.  (Pointer checks are the caller's.)
+parason_status validate_tree(int32_t num_nodes, const int32_t *parent, const int32_t *node_len,
+                             const int32_t *node_page_ptr, const int32_t *page_ids,
+                             int32_t num_leaves, const int32_t *leaf_node, int64_t num_phys,
+                             int32_t H_kv) {
     if (num_nodes < 0 || num_leaves < 0 || num_phys < 0) return PARASON_EINVAL;
     if (num_nodes > 0 && (!parent || !node_len || !node_page_ptr)) return PARASON_EINVAL;
     if (num_leaves > 0 && !leaf_node) return PARASON_EINVAL;
     if (num_leaves > 0 && num_nodes == 0) return PARASON_EINVAL;
-
-    const int32_t H_kv = cfg->num_kv_heads;
-    const int32_t g = cfg->num_q_heads / H_kv;
-    p->cfg = *cfg;
-    p->group = g;
-    p->num_nodes = num_nodes;
-    p->num_leaves = num_leaves;
-    p->num_phys = num_phys;
-    p->num_sms = num_sms > 0 ? num_sms : 152;
-
-    // tree and page table
     if (num_nodes > 0 && node_page_ptr[0] != 0) return PARASON_EINVAL;
     for (int32_t i = 0; i < num_nodes; ++i) {
         if (parent[i] < -1 || parent[i] >= i) return PARASON_EINVAL;
@@ -224,22 +208,53 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
             if (i > 0 && sorted[i] == sorted[i - 1]) return PARASON_EINVAL;
         }
     }
-    p->page_ids.resize(static_cast<size_t>(total_pages));
-    if (total_pages > 0)
-        std::memcpy(p->page_ids.data(), page_ids, sizeof(int32_t) * static_cast<size_t>(total_pages));
-
-    // branches: distinct, in range, childless
-    std::vector<int32_t> leaf_of_node(num_nodes, -1);
+    std::vector<uint8_t> is_leaf(num_nodes, 0);
     std::vector<int32_t> nchild(num_nodes, 0);
     for (int32_t i = 0; i < num_nodes; ++i)
         if (parent[i] >= 0) nchild[parent[i]]++;
     for (int32_t b = 0; b < num_leaves; ++b) {
         const int32_t n = leaf_node[b];
         if (n < 0 || n >= num_nodes) return PARASON_EINVAL;
-        if (leaf_of_node[n] != -1) return PARASON_EINVAL;
+        if (is_leaf[n]) return PARASON_EINVAL;
         if (nchild[n] != 0) return PARASON_EINVAL;
-        leaf_of_node[n] = b;
+        is_leaf[n] = 1;
     }
+    return PARASON_OK;
+}
+
+// With `prefill`, leaf_node holds the chunk nodes of a tree-masked prefill:
+// every token of a chunk is a query (numbered chunk by chunk), attending to
+// every token of its node's ancestors and causally to its own node.
+parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int32_t num_nodes,
+                          const int32_t *parent, const int32_t *node_len,
+                          const int32_t *node_page_ptr, const int32_t *page_ids,
+                          int32_t num_leaves, const int32_t *leaf_node,
+                          int64_t num_phys, int32_t num_sms, bool prefill = false) {
+    parason_status st = validate_config(cfg);
+    if (st != PARASON_OK) return st;
+    // the prefill's causal mask is in the tcgen05 tile: bf16 or e4m3 KV at head_dim 128
+    if (prefill && (cfg->mode == PARASON_FP32 || cfg->head_dim != 128)) return PARASON_EUNSUPPORTED;
+    p->prefill = prefill;
+    if (num_nodes < 0 || num_leaves < 0 || num_phys < 0) return PARASON_EINVAL;
+
+    const int32_t H_kv = cfg->num_kv_heads;
+    const int32_t g = cfg->num_q_heads / H_kv;
+    p->cfg = *cfg;
+    p->group = g;
+    p->num_nodes = num_nodes;
+    p->num_leaves = num_leaves;
+    p->num_phys = num_phys;
+    p->num_sms = num_sms > 0 ? num_sms : 152;
+
+    st = validate_tree(num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves, leaf_node,
+                       num_phys, H_kv);
+    if (st != PARASON_OK) return st;
+    const int64_t total_pages = num_nodes > 0 ? node_page_ptr[num_nodes] : 0;
+    p->page_ids.resize(static_cast<size_t>(total_pages));
+    if (total_pages > 0)
+        std::memcpy(p->page_ids.data(), page_ids, sizeof(int32_t) * static_cast<size_t>(total_pages));
+    std::vector<int32_t> leaf_of_node(num_nodes, -1);
+    for (int32_t b = 0; b < num_leaves; ++b) leaf_of_node[leaf_node[b]] = b;
 
     // branches under each node, and DFS order: parent[i] < i, so a reverse
     // sweep accumulates subtree counts and a forward sweep lays the subtrees
@@ -821,7 +836,132 @@ parason_status plan_device(const parason_attn_config *cfg, int32_t num_nodes, co
     return PARASON_OK;
 }
 
+// ---------------------------------------------------------------------------
+// sharding (one plan per rank, no exchange between ranks)
+// ---------------------------------------------------------------------------
+
+// The sub-forest of the requests (roots) of one rank, in the form build_host
+// takes, with the global index of each of its branches.
+struct SubForest {
+    std::vector<int32_t> parent, len, ptr, pages, leaves, global_branch;
+};
+
+// Roots in index order are cut into `world` contiguous groups of about equal
+// cost: a request's cost is the tokens of its nodes that some branch reads
+// (the KV bytes its decode step moves, each shared node once) plus g per
+// branch (its q and out rows, in the same units).  Rank `rank` gets group
+// `rank`; a rank may get no request when there are fewer requests than ranks.
+void shard_requests(int32_t num_nodes, const int32_t *parent, const int32_t *node_len,
+                    const int32_t *node_page_ptr, const int32_t *page_ids, int32_t num_leaves,
+                    const int32_t *leaf_node, int32_t g, int32_t rank, int32_t world,
+                    SubForest *out) {
+    std::vector<int32_t> root(num_nodes), root_idx(num_nodes, -1);
+    std::vector<int64_t> cnt(num_nodes, 0);
+    int32_t num_roots = 0;
+    for (int32_t i = 0; i < num_nodes; ++i) {
+        root[i] = parent[i] < 0 ? i : root[parent[i]];
+        if (parent[i] < 0) root_idx[i] = num_roots++;
+    }
+    for (int32_t b = 0; b < num_leaves; ++b) cnt[leaf_node[b]] = 1;
+    for (int32_t i = num_nodes - 1; i >= 0; --i)
+        if (parent[i] >= 0) cnt[parent[i]] += cnt[i];
+    std::vector<int64_t> cost(num_roots, 0);
+    for (int32_t i = 0; i < num_nodes; ++i)
+        if (cnt[i] > 0) cost[root_idx[root[i]]] += node_len[i];
+    for (int32_t b = 0; b < num_leaves; ++b) cost[root_idx[root[leaf_node[b]]]] += g;
+    std::vector<int64_t> prefix(num_roots + 1, 0);
+    for (int32_t r = 0; r < num_roots; ++r) prefix[r + 1] = prefix[r] + cost[r];
+    // boundary k: the prefix closest to k/world of the total, never moving back
+    auto boundary = [&](int32_t k) -> int32_t {
+        if (k <= 0) return 0;
+        if (k >= world) return num_roots;
+        const double target = static_cast<double>(prefix[num_roots]) * k / world;
+        int32_t j = static_cast<int32_t>(std::lower_bound(prefix.begin(), prefix.end(),
+                                                          static_cast<int64_t>(std::ceil(target))) -
+                                         prefix.begin());
+        j = std::min(j, num_roots);
+        if (j > 0 && target - static_cast<double>(prefix[j - 1]) <
+                         static_cast<double>(prefix[j]) - target)
+            --j;
+        return j;
+    };
+    int32_t lo = 0, hi = 0;
+    for (int32_t k = 0; k <= rank; ++k) {
+        lo = std::max(lo, boundary(k));
+        hi = std::max(lo, boundary(k + 1));
+    }
+    std::vector<int32_t> remap(num_nodes, -1);
+    out->ptr.assign(1, 0);
+    for (int32_t i = 0; i < num_nodes; ++i) {
+        const int32_t ri = root_idx[root[i]];
+        if (ri < lo || ri >= hi) continue;
+        remap[i] = static_cast<int32_t>(out->parent.size());
+        out->parent.push_back(parent[i] < 0 ? -1 : remap[parent[i]]);
+        out->len.push_back(node_len[i]);
+        for (int32_t k = node_page_ptr[i]; k < node_page_ptr[i + 1]; ++k) out->pages.push_back(page_ids[k]);
+        out->ptr.push_back(static_cast<int32_t>(out->pages.size()));
+    }
+    for (int32_t b = 0; b < num_leaves; ++b) {
+        if (remap[leaf_node[b]] < 0) continue;
+        out->leaves.push_back(remap[leaf_node[b]]);
+        out->global_branch.push_back(b);
+    }
+}
+
+parason_status plan_shard(const parason_attn_config *cfg, int32_t num_nodes, const int32_t *parent,
+                          const int32_t *node_len, const int32_t *node_page_ptr,
+                          const int32_t *page_ids, int32_t num_leaves, const int32_t *leaf_node,
+                          int64_t num_phys, int32_t kind, int32_t rank, int32_t world,
+                          bool host_only, int32_t num_sms, parason_stream_t stream,
+                          parason_plan *out) {
+    if (!out) return PARASON_EINVAL;
+    *out = nullptr;
+    parason_status st = validate_config(cfg);
+    if (st != PARASON_OK) return st;
+    if (world < 1 || rank < 0 || rank >= world) return PARASON_EINVAL;
+    st = validate_tree(num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves, leaf_node,
+                       num_phys, cfg->num_kv_heads);
+    if (st != PARASON_OK) return st;
+    parason_plan p = nullptr;
+    if (kind == PARASON_SHARD_KV_HEADS) {
+        // kv heads [rank H_kv / world, (rank + 1) H_kv / world) and their q heads
+        if (cfg->num_kv_heads % world != 0) return PARASON_EINVAL;
+        parason_attn_config c = *cfg;
+        c.num_kv_heads = cfg->num_kv_heads / world;
+        c.num_q_heads = cfg->num_q_heads / world;
+        st = host_only ? plan_host(&c, num_nodes, parent, node_len, node_page_ptr, page_ids,
+                                   num_leaves, leaf_node, num_phys, num_sms, false, &p)
+                       : plan_device(&c, num_nodes, parent, node_len, node_page_ptr, page_ids,
+                                     num_leaves, leaf_node, num_phys, false, stream, &p);
+        if (st != PARASON_OK) return st;
+        p->shard_branch.resize(static_cast<size_t>(num_leaves));
+        for (int32_t b = 0; b < num_leaves; ++b) p->shard_branch[b] = b;
+    } else if (kind == PARASON_SHARD_REQUESTS) {
+        SubForest f;
+        try {
+            shard_requests(num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves,
+                           leaf_node, cfg->num_q_heads / cfg->num_kv_heads, rank, world, &f);
+        } catch (const std::bad_alloc &) {
+            return PARASON_ENOMEM;
+        }
+        const int32_t n = static_cast<int32_t>(f.parent.size());
+        const int32_t l = static_cast<int32_t>(f.leaves.size());
+        st = host_only ? plan_host(cfg, n, f.parent.data(), f.len.data(), f.ptr.data(),
+                                   f.pages.data(), l, f.leaves.data(), num_phys, num_sms, false, &p)
+                       : plan_device(cfg, n, f.parent.data(), f.len.data(), f.ptr.data(),
+                                     f.pages.data(), l, f.leaves.data(), num_phys, false, stream, &p);
+        if (st != PARASON_OK) return st;
+        p->shard_branch.swap(f.global_branch);
+    } else {
+        return PARASON_EINVAL;
+    }
+    *out = p;
+    return PARASON_OK;
+}
+
 }  // namespace
+
+int parason::plan_device(parason_plan p) { return (p && p->on_device) ? p->device : -1; }
 
 extern "C" {
 
@@ -863,6 +1003,26 @@ parason_status parason_prefill_plan(const parason_attn_config *cfg, int32_t num_
                                     parason_plan *out) {
     return plan_device(cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_chunks,
                        chunk_node, num_physical_pages, true, stream, out);
+}
+
+parason_status parason_attn_plan_shard(const parason_attn_config *cfg, int32_t num_nodes,
+                                       const int32_t *parent, const int32_t *node_len,
+                                       const int32_t *node_page_ptr, const int32_t *page_ids,
+                                       int32_t num_leaves, const int32_t *leaf_node,
+                                       int64_t num_physical_pages, int32_t kind, int32_t rank,
+                                       int32_t world, parason_stream_t stream, parason_plan *out) {
+    return plan_shard(cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves,
+                      leaf_node, num_physical_pages, kind, rank, world, false, 0, stream, out);
+}
+
+parason_status parason_attn_plan_shard_host(const parason_attn_config *cfg, int32_t num_nodes,
+                                            const int32_t *parent, const int32_t *node_len,
+                                            const int32_t *node_page_ptr, const int32_t *page_ids,
+                                            int32_t num_leaves, const int32_t *leaf_node,
+                                            int64_t num_physical_pages, int32_t kind, int32_t rank,
+                                            int32_t world, int32_t num_sms, parason_plan *out) {
+    return plan_shard(cfg, num_nodes, parent, node_len, node_page_ptr, page_ids, num_leaves,
+                      leaf_node, num_physical_pages, kind, rank, world, true, num_sms, nullptr, out);
 }
 
 size_t parason_plan_workspace_bytes(parason_plan p) {
@@ -1021,7 +1181,9 @@ parason_status parason_plan_check(parason_plan p, parason_stream_t stream) {
         if (cudaMemcpy(p->d_queue_next, p->queue_start, 2 * sizeof(int32_t), cudaMemcpyHostToDevice) !=
             cudaSuccess)
             return PARASON_ECUDA;
-        return rec[0] == PARASON_ETIMEOUT ? PARASON_ETIMEOUT : PARASON_ECUDA;
+        if (rec[0] == PARASON_ETIMEOUT || rec[0] == PARASON_ERANGE)
+            return static_cast<parason_status>(rec[0]);
+        return PARASON_ECUDA;
     }
     return PARASON_OK;
 }
@@ -1042,6 +1204,7 @@ const char *parason_status_string(parason_status s) {
     case PARASON_ETIMEOUT: return "device wait timed out";
     case PARASON_EUNSUPPORTED: return "unsupported";
     case PARASON_ENOSPACE: return "no room in the plan: build a new one";
+    case PARASON_ERANGE: return "input value out of the kernel's range";
     }
     return "unknown status";
 }
@@ -1075,12 +1238,20 @@ parason_status parason_plan_append(parason_plan p, const int32_t *new_pages,
     const int32_t H_kv = p->cfg.num_kv_heads;
     constexpr int32_t P16 = parason::kPageSize;
 
-    // check everything first: on any error nothing changes
+    // 1. check everything: on any error nothing changes
     std::vector<int32_t> claimed;
     auto refuse = [&](parason_status st) {
         for (int32_t pg : claimed) p->page_used[pg] = 0;
         return st;
     };
+    if (p->on_device) {
+        int dev = -1;
+        if (cudaGetDevice(&dev) != cudaSuccess) {
+            cudaGetLastError();
+            return PARASON_ECUDA;
+        }
+        if (dev != p->device) return PARASON_EINVAL;
+    }
     for (int32_t b = 0; b < L; ++b) {
         if (p->tail_ptr[b] == p->tail_ptr[b + 1]) return refuse(PARASON_ENOSPACE);
         if (p->leaf_len[b] == INT32_MAX) return refuse(PARASON_EUNSUPPORTED);
@@ -1102,7 +1273,10 @@ parason_status parason_plan_append(parason_plan p, const int32_t *new_pages,
         claimed.push_back(pg);
     }
 
-    // apply, host copy and patch list: (word offset in the device blob, value)
+    // 2. the new values, without touching the plan yet: host words to write
+    // and the device patch list (word offset in the device blob, value).
+    // Each tail item belongs to one branch, so no word is written twice.
+    std::vector<std::pair<int32_t *, int32_t>> host;
     std::vector<int2> &patches = p->patches;
     patches.clear();
     for (int32_t b = 0; b < L; ++b) {
@@ -1113,44 +1287,53 @@ parason_status parason_plan_append(parason_plan p, const int32_t *new_pages,
             int32_t *rec = p->item_rec.data() + static_cast<size_t>(t) * parason::kRecWords;
             const size_t w_item = p->w_items + static_cast<size_t>(t) * (sizeof(WorkItem) / 4);
             const size_t w_rec = p->w_rec + static_cast<size_t>(t) * parason::kRecWords;
+            int32_t last_valid = it.last_valid + 1;
             if (opens_page) {
                 const int32_t j = it.num_pages;                   // the new page's index
                 const int32_t row = (new_pages[b] * H_kv + it.kv_head) * P16;
-                it.num_pages += 1;
-                it.last_valid = 1;
-                p->stream_rows[p->item_rows[t] + j] = row;
+                const int32_t np = it.num_pages + 1;
+                last_valid = 1;
+                host.emplace_back(&p->stream_rows[p->item_rows[t] + j], row);
                 patches.push_back(make_int2(static_cast<int32_t>(p->w_strows + p->item_rows[t] + j), row));
                 if (j < parason::kRecRows) {
-                    rec[parason::kRecRow0 + j] = row;
+                    host.emplace_back(&rec[parason::kRecRow0 + j], row);
                     patches.push_back(make_int2(static_cast<int32_t>(w_rec + parason::kRecRow0 + j), row));
                 }
-                rec[1] = it.num_pages;
-                patches.push_back(make_int2(static_cast<int32_t>(w_rec + 1), it.num_pages));
-                patches.push_back(make_int2(static_cast<int32_t>(w_item + 1), it.num_pages));
-            } else {
-                it.last_valid += 1;
+                host.emplace_back(&it.num_pages, np);
+                host.emplace_back(&rec[1], np);
+                patches.push_back(make_int2(static_cast<int32_t>(w_rec + 1), np));
+                patches.push_back(make_int2(static_cast<int32_t>(w_item + 1), np));
             }
-            rec[2] = it.last_valid;
-            patches.push_back(make_int2(static_cast<int32_t>(w_rec + 2), it.last_valid));
-            patches.push_back(make_int2(static_cast<int32_t>(w_item + 2), it.last_valid));
+            host.emplace_back(&it.last_valid, last_valid);
+            host.emplace_back(&rec[2], last_valid);
+            patches.push_back(make_int2(static_cast<int32_t>(w_rec + 2), last_valid));
+            patches.push_back(make_int2(static_cast<int32_t>(w_item + 2), last_valid));
         }
-        p->leaf_len[b] += 1;
     }
+
+    // 3. the device copy first: if it cannot be updated, neither is the host
+    // copy, so the two never disagree
+    if (p->debug_flags & PARASON_DEBUG_FAIL_UPDATE) return refuse(PARASON_ECUDA);
+    if (p->on_device && !patches.empty()) {
+        cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+        // a pageable source is staged before the call returns, so the host
+        // list may be reused by the next append.  A failed copy or launch
+        // leaves the plan's device blob as it was (only the patch buffer,
+        // which nothing else reads, may have changed).
+        if (cudaMemcpyAsync(p->d_patch, patches.data(), patches.size() * sizeof(int2),
+                            cudaMemcpyHostToDevice, stream) != cudaSuccess ||
+            parason::launch_scatter(static_cast<int32_t *>(p->d_blob), p->d_patch,
+                                    static_cast<int32_t>(patches.size()), stream) != cudaSuccess) {
+            cudaGetLastError();
+            return refuse(PARASON_ECUDA);
+        }
+    }
+
+    // 4. commit the host copy
+    for (const auto &w : host) *w.first = w.second;
+    for (int32_t b = 0; b < L; ++b) p->leaf_len[b] += 1;
     p->unique_tokens += L;
     p->path_tokens += L;
-    if (!p->on_device || patches.empty()) return PARASON_OK;
-
-    int dev = -1;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev != p->device) return PARASON_ECUDA;
-    cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
-    // a pageable source is staged before the call returns, so the host list
-    // may be reused by the next append
-    if (cudaMemcpyAsync(p->d_patch, patches.data(), patches.size() * sizeof(int2),
-                        cudaMemcpyHostToDevice, stream) != cudaSuccess)
-        return PARASON_ECUDA;
-    if (parason::launch_scatter(static_cast<int32_t *>(p->d_blob), p->d_patch,
-                                static_cast<int32_t>(patches.size()), stream) != cudaSuccess)
-        return PARASON_ECUDA;
     return PARASON_OK;
 }
 
@@ -1168,6 +1351,15 @@ parason_status parason_plan_export(parason_plan p, int32_t table, void *dst, siz
     case PARASON_TABLE_ITEM_ROWS: src = p->item_rows.data(); n = p->item_rows.size() * 4; break;
     case PARASON_TABLE_STREAM_ROWS: src = p->stream_rows.data(); n = p->stream_rows.size() * 4; break;
     case PARASON_TABLE_ITEM_KEY0: src = p->item_key0.data(); n = p->item_key0.size() * 4; break;
+    case PARASON_TABLE_SHARD_BRANCHES:
+        // an unsharded plan's branch b is branch b
+        if (p->shard_branch.size() != static_cast<size_t>(p->num_leaves)) {
+            p->shard_branch.resize(static_cast<size_t>(p->num_leaves));
+            for (int32_t b = 0; b < p->num_leaves; ++b) p->shard_branch[b] = b;
+        }
+        src = p->shard_branch.data();
+        n = p->shard_branch.size() * 4;
+        break;
     default: return PARASON_EINVAL;
     }
     if (bytes < n || (n > 0 && !dst)) return PARASON_EINVAL;

@@ -200,6 +200,8 @@ def build_tree(name: str, parent, node_len, leaf_node, *, num_q_heads: int,
     """
     if rng is None:
         rng = np.random.default_rng(seed)
+    meta = dict(meta or {})
+    meta.setdefault("permuted", bool(permute_pages))
     parent = np.asarray(parent, dtype=np.int32)
     node_len = np.asarray(node_len, dtype=np.int32)
     leaf_node = np.asarray(leaf_node, dtype=np.int32)

@@ -166,3 +166,35 @@ def test_fp32_plans_do_not_append():
         with pytest.raises(ParasonError) as e:
             plan.append(None)
         assert e.value.status == _lib.EUNSUPPORTED
+
+
+def test_failed_device_update_changes_nothing():
+    """An append whose device step fails (simulated by a debug flag, at the
+    point where the device copy would be patched) changes neither the plan's
+    tables nor its page accounting: retrying with the same pages succeeds."""
+    tree = make_tree()
+    pool = W.free_pages(tree)
+    with Plan.for_tree(tree, host_only=True) as plan:
+        for _ in range(3):
+            tree, new_pages = W.grow_branches(tree, pool)
+            plan.append(new_pages)
+        while True:                                          # up to a step that opens a page
+            grown, new_pages = W.grow_branches(tree, list(pool))
+            if (new_pages >= 0).any():
+                break
+            tree, _ = W.grow_branches(tree, pool)
+            plan.append(None)
+        before = snapshot(plan)
+        info_before = plan.info()
+        plan.set_debug(_lib.DEBUG_FAIL_UPDATE)
+        for _ in range(2):
+            with pytest.raises(ParasonError) as e:
+                plan.append(new_pages)
+            assert e.value.status == _lib.ECUDA
+            for x, y in zip(before, snapshot(plan)):
+                assert np.array_equal(x, y)
+            assert plan.info() == info_before
+        verify_rows(tree, plan)
+        plan.set_debug(0)
+        plan.append(new_pages)                               # the pages were not kept
+        verify_rows(grown, plan)

@@ -58,3 +58,29 @@ def test_decode_after_appends_matches_oracle(case):
     assert checked >= 6
     assert float((out.float() - out2.float()).abs().max()) <= PT.BF16_MAX_ABS
     assert float((lse - lse2).abs().max()) <= PT.LSE_ABS[tree.mode]
+
+
+def test_failed_update_keeps_device_and_host_plans_in_step():
+    """A refused device update leaves both copies of the plan as they were:
+    the next decode is the old tree's result, and after a successful retry
+    the grown tree's (both against the oracle)."""
+    from paper_2608_24658_gb300 import _lib
+    from paper_2608_24658_gb300.api import ParasonError
+    tree = CASES["bf16"]()
+    pool = W.free_pages(tree)
+    with Plan.for_tree(tree) as plan:
+        grown, new_pages = W.grow_branches(tree, list(pool))
+        plan.set_debug(_lib.DEBUG_FAIL_UPDATE)
+        with pytest.raises(ParasonError) as e:
+            plan.append(new_pages)
+        assert e.value.status == _lib.ECUDA
+        plan.set_debug(0)
+        out, lse = plan.decode_tree(tree)
+        plan.check()
+        ref_o, ref_l = PT.oracle_decode(tree)
+        PT.compare(tree, out, lse, ref_o, ref_l, tag="after a failed append")
+        plan.append(new_pages)
+        out, lse = plan.decode_tree(grown)
+        plan.check()
+        ref_o, ref_l = PT.oracle_decode(grown)
+        PT.compare(grown, out, lse, ref_o, ref_l, tag="after the retried append")
