@@ -603,8 +603,10 @@ def run_trace(args):
 
 def run_append(args):
     """One decode step's plan update (parason_plan_append: a token on every
-    branch) against building a new plan, on the Llama-3-shape workload with
-    room to grow; and the decode step before and after 64 appends."""
+    branch) against building a new plan, on the workload (with room to
+    grow); the decode step before and after 64 appends; and a fork of one
+    branch into four threads (parason_plan_fork) against building a plan for
+    the forked tree, with the decode step after each."""
     import torch
     from paper_2608_24658_gb300 import build as lib_build
     from paper_2608_24658_gb300.api import Plan
@@ -662,6 +664,27 @@ def run_append(args):
         replan_us.append((time.perf_counter() - t0) * 1e6)
         rebuilt_us = decode_us(p2, tree, n=20) if len(replan_us) == 10 else None
         p2.close()
+    # a fork: a branch opens four threads (one token each) at </Outlines>;
+    # against building a plan for the forked tree
+    fork_host, fork_dev, after_fork, fresh_fork = [], [], [], []
+    for r in range(10):
+        fpool = list(W.free_pages(tree))
+        forked, pages = W.fork_branch(tree, r % tree.num_leaves, [1, 1, 1, 1], fpool)
+        pf = Plan.for_tree(tree, stream=stream)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize(dev)
+        a.record(stream)
+        t0 = time.perf_counter()
+        pf.fork(r % tree.num_leaves, [1, 1, 1, 1], pages, stream=stream)
+        fork_host.append((time.perf_counter() - t0) * 1e6)
+        b.record(stream)
+        b.synchronize()
+        fork_dev.append(a.elapsed_time(b) * 1e3)
+        if r == 0:
+            after_fork.append(decode_us(pf, forked))
+            with Plan.for_tree(forked, stream=stream) as pn:
+                fresh_fork.append(decode_us(pn, forked))
+        pf.close()
     line = {"metric": "plan update per decode step", "value": float(np.median(host_us)),
             "unit": "us (host)", "higher_is_better": False, "n_gpus": 1, "steps": steps,
             "data": "synthetic", "component": "append",
@@ -670,7 +693,10 @@ def run_append(args):
             "append_device_us": float(np.median(dev_us)),
             "rebuild_plan_us": float(np.median(replan_us)),
             "decode_us_fresh_plan": fresh_us, "decode_us_after_appends": after_us,
-            "decode_us_rebuilt_after": rebuilt_us}
+            "decode_us_rebuilt_after": rebuilt_us,
+            "fork_4_threads_us_host": float(np.median(fork_host)),
+            "fork_4_threads_us_device": float(np.median(fork_dev)),
+            "decode_us_after_fork": after_fork[0], "decode_us_fresh_plan_of_forked_tree": fresh_fork[0]}
     print(json.dumps(line), flush=True)
     return 0
 

@@ -338,6 +338,51 @@ parason_status parason_plan_append(parason_plan plan, const int32_t *new_pages,
                                    parason_stream_t stream);
 
 /*
+ * Decode-loop update at a fork: branch `branch` reaches the end of an
+ * <Outlines> block and its k = num_children threads start (Sec. 3.4: the
+ * runtime dispatches each <Subtask> / <Trial> entry as an independent worker;
+ * Fig. 4, rule W -> <Thread> B </Thread>: a thread may itself open a nested
+ * region).  The branch's node stops being a branch node and gets k child
+ * nodes; the plan is patched without being rebuilt.
+ *
+ *   child_len       host int32 [k]: tokens already held by each child (>= 0;
+ *                   with 0 the child has no page, and appends to it need a
+ *                   new plan)
+ *   child_page_ptr  host int32 [k + 1]: CSR into child_pages; child c owns
+ *                   ceil(child_len[c] / 16) pages
+ *   child_pages     host int32: fresh physical pages (in range, owned by no
+ *                   node); the caller has written their K and V
+ *
+ * Numbering: the children become nodes num_nodes .. num_nodes + k - 1 in
+ * order, under the branch's node.  Child 0 is branch `branch` (row `branch`
+ * of q, out, lse); child c >= 1 is the new branch num_leaves + c - 1.  So q,
+ * out and lse of the next decode have num_leaves + k - 1 rows
+ * (parason_plan_get_info reports the new count).
+ *
+ * The new branches' rows of every node on the branch's path, and every
+ * child's own rows, become suffix-pass work items appended to the plan:
+ * O(k * H_kv * (pages on the path) / piece) items, merge entries and page
+ * rows, copied to the device with a few host-to-device copies and one small
+ * kernel on `stream` (from pageable memory, so the call may wait for work
+ * already queued on `stream`).  The ancestors' pages are then read once more
+ * for the new branches than a new plan would read them: build a new plan
+ * when convenient.  parason_plan_workspace_bytes grows by the new partial
+ * rows: the next decode needs a workspace of the new size.
+ *
+ * Returns PARASON_EINVAL for a branch out of range, k < 1, a negative
+ * length, a page count that is not ceil(len / 16), a page out of range, used
+ * or repeated, a NULL array, or a current device that is not the plan's;
+ * PARASON_EUNSUPPORTED in FP32 mode, on a prefill plan, or with more than 16
+ * q heads per kv head; PARASON_ENOSPACE if the room the plan keeps for
+ * forks (about as much again as it held when built) is used up -- build a
+ * new plan then.  On any error nothing is changed, on the host or the
+ * device.  Forks and appends of a plan are issued in order with its decodes.
+ */
+parason_status parason_plan_fork(parason_plan plan, int32_t branch, int32_t num_children,
+                                 const int32_t *child_len, const int32_t *child_page_ptr,
+                                 const int32_t *child_pages, parason_stream_t stream);
+
+/*
  * Combine two attention results over disjoint key sets A and B (for example
  * two KV ranges of one branch, or a branch's context before and after a join)
  * into the result over A u B, row by row.
@@ -405,8 +450,10 @@ parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info)
  *                            order), first node row, row count, kv head,
  *                            partial slot of the item's first row
  *   PARASON_TABLE_DFS_LEAVES int32 [num_leaves]: branches in DFS order
- *   PARASON_TABLE_MERGE_PTR  int32 [num_leaves * H_kv + 1]: CSR into the
- *                            entries, per (branch, kv head)
+ *   PARASON_TABLE_MERGE_RANGES int32 [num_leaves * H_kv][2]: per (branch,
+ *                            kv head), the begin and end of its entries in
+ *                            PARASON_TABLE_MERGE (a fork moves a branch's
+ *                            list to the end, so lists need not be in order)
  *   PARASON_TABLE_MERGE      int32 [num_merge_entries]: partial slot of the
  *                            branch's first q head of the kv head; q head
  *                            j*g + r reads slot entry + r
@@ -431,7 +478,7 @@ parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info)
 enum {
     PARASON_TABLE_ITEMS = 0,
     PARASON_TABLE_DFS_LEAVES = 1,
-    PARASON_TABLE_MERGE_PTR = 2,
+    PARASON_TABLE_MERGE_RANGES = 2,
     PARASON_TABLE_MERGE = 3,
     PARASON_TABLE_WIDE_QUEUE = 4,
     PARASON_TABLE_NARROW_QUEUE = 5,

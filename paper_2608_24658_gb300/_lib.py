@@ -13,7 +13,7 @@ LIB_PATH = os.path.join(_HERE, "_build", "libparason.so")
 
 OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EUNSUPPORTED, ENOSPACE, ERANGE = range(8)
 MODES = {"bf16": 0, "fp32": 1, "fp8": 2}
-(TABLE_ITEMS, TABLE_DFS_LEAVES, TABLE_MERGE_PTR, TABLE_MERGE, TABLE_WIDE_QUEUE,
+(TABLE_ITEMS, TABLE_DFS_LEAVES, TABLE_MERGE_RANGES, TABLE_MERGE, TABLE_WIDE_QUEUE,
  TABLE_NARROW_QUEUE, TABLE_ITEM_ROWS, TABLE_STREAM_ROWS, TABLE_ITEM_KEY0,
  TABLE_SHARD_BRANCHES) = range(10)
 SHARD_REQUESTS, SHARD_KV_HEADS = 0, 1
@@ -71,6 +71,7 @@ SIGNATURES = {
     "parason_attn_decode": (ctypes.c_int, [_p, _p, _p, _p, _p, _p, _p, _p, _p, _sz, _p]),
     "parason_attn_decode_no_alloc": (ctypes.c_int, [_p, _p, _p, _p, _p, _p, _p, _p, _p]),
     "parason_plan_append": (ctypes.c_int, [_p, _p, _p]),
+    "parason_plan_fork": (ctypes.c_int, [_p, _i32, _i32, _p, _p, _p, _p]),
     "parason_trace_analyze": (ctypes.c_int, [_p, _i64, ctypes.POINTER(TraceStats),
                                              ctypes.POINTER(ctypes.c_int64)]),
     "parason_trace_fork_tree": (ctypes.c_int, [_p, _i64, _i32, _i32, _p, _p, _p,

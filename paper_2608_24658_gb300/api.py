@@ -162,7 +162,7 @@ class Plan:
         inf = self.info()
         shape = {_lib.TABLE_ITEMS: (inf["num_items"], 8),
                  _lib.TABLE_DFS_LEAVES: (inf["num_leaves"],),
-                 _lib.TABLE_MERGE_PTR: (inf["num_leaves"] * self.num_kv_heads + 1,),
+                 _lib.TABLE_MERGE_RANGES: (inf["num_leaves"] * self.num_kv_heads, 2),
                  _lib.TABLE_MERGE: (inf["num_merge_entries"],),
                  _lib.TABLE_WIDE_QUEUE: (inf["num_wide_items"],),
                  _lib.TABLE_NARROW_QUEUE: (inf["num_narrow_items"],),
@@ -271,6 +271,23 @@ class Plan:
                 raise ValueError(f"new_pages must have shape ({self.num_leaves},)")
         sh = None if self.host_only else _stream_handle(stream)
         check(_lib.load().parason_plan_append(self.handle, _ptr(a), sh), "parason_plan_append")
+
+    def fork(self, branch: int, child_len, child_pages, stream=None) -> list:
+        """Branch ``branch`` forks into len(child_len) threads
+        (parason_plan_fork).  ``child_pages``: one list of fresh physical
+        pages per child, ceil(len / 16) each.  Returns the branch index of
+        every child: child 0 keeps ``branch``, the others are appended."""
+        lens = np.ascontiguousarray(np.asarray(child_len, dtype=np.int32))
+        ptr = np.zeros(len(lens) + 1, dtype=np.int32)
+        ptr[1:] = np.cumsum([len(pg) for pg in child_pages]) if len(child_pages) else []
+        flat = np.ascontiguousarray(np.asarray([x for pg in child_pages for x in pg] or [0],
+                                               dtype=np.int32))
+        sh = None if self.host_only else _stream_handle(stream)
+        L = self.num_leaves
+        check(_lib.load().parason_plan_fork(self.handle, int(branch), len(lens), _ptr(lens),
+                                            _ptr(ptr), _ptr(flat), sh), "parason_plan_fork")
+        self.num_leaves = int(self.info()["num_leaves"])
+        return [int(branch)] + list(range(L, L + len(lens) - 1))
 
     def decode_tree(self, tree, **kw):
         """``decode`` with the tensors of a ``workloads.ForkTree``."""

@@ -93,7 +93,7 @@ struct AttnArgs {
 };
 
 struct MergeArgs {
-    const int32_t *merge_ptr;   // [num_leaves * H_kv + 1]
+    const int2 *merge_rng;      // [num_leaves * H_kv]: [begin, end) in merge_ent
     const int32_t *merge_ent;   // first partial slot of the branch's rows
     const float *part_o;
     const float2 *part_ml;

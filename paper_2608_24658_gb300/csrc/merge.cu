@@ -111,7 +111,8 @@ __global__ void __launch_bounds__(kMergeThreads)
     const int j = h / a.group, r = h % a.group;
     const int64_t pair = static_cast<int64_t>(b) * a.num_kv_heads + j;
     // the merge lists are plan data: read them while the attention grid drains
-    const int e0 = active ? a.merge_ptr[pair] : 0, e1 = active ? a.merge_ptr[pair + 1] : 0;
+    const int2 rg = active ? a.merge_rng[pair] : make_int2(0, 0);
+    const int e0 = rg.x, e1 = rg.y;
     const int first_e = e0 + w + W * lane;
     const int first_slot = first_e < e1 ? a.merge_ent[first_e] + r : 0;
     asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -234,7 +235,8 @@ __global__ void __launch_bounds__(kMergeThreads)
     const int64_t pair = static_cast<int64_t>(blockIdx.x) * (kMergeThreads / 32) + warp;
     const bool active = pair < static_cast<int64_t>(a.num_leaves) * a.num_kv_heads;
     // the merge lists are plan data: read them while the attention grid drains
-    const int e0 = active ? a.merge_ptr[pair] : 0, e1 = active ? a.merge_ptr[pair + 1] : 0;
+    const int2 rg = active ? a.merge_rng[pair] : make_int2(0, 0);
+    const int e0 = rg.x, e1 = rg.y;
     const int first_slot = e0 + lane < e1 ? a.merge_ent[e0 + lane] : 0;
     asm volatile("griddepcontrol.wait;" ::: "memory");
     // the attention grid is complete: rewind its work queues for the next call

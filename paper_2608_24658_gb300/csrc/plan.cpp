@@ -94,7 +94,7 @@ struct parason_plan_s {
     std::vector<WorkItem> items;
     std::vector<int32_t> page_ids;
     std::vector<int32_t> dfs_leaf;
-    std::vector<int32_t> merge_ptr;
+    std::vector<int2> merge_rng;       // per (branch, kv head): [begin, end) of its entries
     std::vector<int32_t> merge_ent;   // first partial slot of the branch's rows
     std::vector<int32_t> wide_queue;   // prefix-pass items, in pull order
     std::vector<int32_t> narrow_queue; // suffix-pass items, in pull order
@@ -102,11 +102,17 @@ struct parason_plan_s {
     std::vector<int32_t> stream_rows;  // TMA row of every page, item by item
     std::vector<int32_t> item_rec;     // kRecWords per item (suffix-warp record)
 
-    // decode-loop appends (parason_plan_append): each branch's own node
-    std::vector<int32_t> leaf_len;     // tokens in branch b's node
-    std::vector<int32_t> tail_ptr;     // CSR over branches into tail_items
-    std::vector<int32_t> tail_items;   // items that end at the node's last page
-    std::vector<uint8_t> page_used;    // physical pages some node owns
+    // the tree as it stands: appends grow branch nodes, forks add nodes and
+    // branches (parason_plan_append / parason_plan_fork)
+    std::vector<int32_t> tree_parent, tree_len, leaf_node;
+    std::vector<std::vector<int32_t>> node_pages;   // physical pages of each node
+    std::vector<int32_t> node_page_pos;             // each node's first position in page_ids
+    std::vector<int32_t> dfs_pos;                   // branch -> its position in dfs_leaf
+    std::vector<std::vector<int32_t>> tails;        // per branch: items ending at its node's last page
+    std::vector<uint8_t> page_used;                 // physical pages some node owns
+    int64_t narrow_chunk = kMinPiecePages;          // suffix piece length of the plan
+    // room the device copy keeps for forks (a fork past it is PARASON_ENOSPACE)
+    size_t cap_items = 0, cap_rows = 0, cap_leaves = 0, cap_ent = 0, cap_patch = 0;
     int32_t num_ctas = 0;
     int32_t num_wide_ctas = 0;
     int32_t suffix_warps = 8;          // suffix-pass warps per CTA (kernel instantiation)
@@ -124,14 +130,15 @@ struct parason_plan_s {
     WorkItem *d_items = nullptr;
     int32_t *d_page_ids = nullptr;
     int32_t *d_dfs_leaf = nullptr;
-    int32_t *d_merge_ptr = nullptr;
+    int2 *d_merge_rng = nullptr;
     int32_t *d_merge_ent = nullptr;
     int32_t *d_item_rec = nullptr;
     int2 *d_patch = nullptr;
-    int32_t *d_item_key0 = nullptr;    // prefill plans only           // (word offset in the blob, value), tail_items * 6
+    int32_t *d_item_key0 = nullptr;    // prefill plans only
     std::vector<int2> patches;         // host side of the last append's patch list
     size_t blob_words = 0;
-    size_t w_items = 0, w_rec = 0, w_strows = 0;   // word offsets of those arrays in the blob
+    // word offsets of arrays in the blob (patch targets)
+    size_t w_items = 0, w_rec = 0, w_strows = 0, w_mrng = 0, w_qnext = 0;
     int32_t *d_item_rows = nullptr;
     int32_t *d_stream_rows = nullptr;
     int32_t *d_queue_next = nullptr;   // 2 counters, set back to queue_start by the merge kernel
@@ -464,6 +471,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         const int64_t narrow_chunk = std::min<int64_t>(
             kMaxPiecePages,
             std::max<int64_t>(kMinPiecePages, narrow_pages / std::max<int64_t>(1, total_warps * 3)));
+        p->narrow_chunk = narrow_chunk;
         int64_t wide_pages = 0;
         for (const Run &r : runs)
             if (r.wide) wide_pages += r.pages;
@@ -534,19 +542,24 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
 
     // the items that end at each branch node's last page (appends grow them)
     std::sort(tails.begin(), tails.end());
-    p->tail_ptr.assign(static_cast<size_t>(num_leaves) + 1, 0);
-    p->tail_items.clear();
+    p->tails.assign(static_cast<size_t>(num_leaves), {});
     std::vector<uint8_t> is_tail(p->items.size(), 0);
     for (const auto &t : tails) {
-        p->tail_ptr[t.first + 1]++;
-        p->tail_items.push_back(t.second);
+        p->tails[t.first].push_back(t.second);
         is_tail[t.second] = 1;
     }
-    for (int32_t b = 0; b < num_leaves; ++b) p->tail_ptr[b + 1] += p->tail_ptr[b];
-    p->leaf_len.assign(static_cast<size_t>(num_leaves), 0);
-    for (int32_t b = 0; b < num_leaves; ++b) p->leaf_len[b] = node_len[leaf_node[b]];
     p->page_used.assign(static_cast<size_t>(num_phys), 0);
     for (int64_t i = 0; i < total_pages; ++i) p->page_used[page_ids[i]] = 1;
+    // the tree, for appends and forks
+    p->tree_parent.assign(parent, parent + num_nodes);
+    p->tree_len.assign(node_len, node_len + num_nodes);
+    p->leaf_node.assign(leaf_node, leaf_node + num_leaves);
+    p->node_page_pos.assign(node_page_ptr, node_page_ptr + num_nodes);
+    p->node_pages.assign(static_cast<size_t>(num_nodes), {});
+    for (int32_t n = 0; n < num_nodes; ++n)
+        p->node_pages[n].assign(page_ids + node_page_ptr[n], page_ids + node_page_ptr[n + 1]);
+    p->dfs_pos.assign(static_cast<size_t>(p->num_leaves), 0);
+    for (size_t k = 0; k < p->dfs_leaf.size(); ++k) p->dfs_pos[p->dfs_leaf[k]] = static_cast<int32_t>(k);
 
     // page streams: the TMA row (page * H_kv + kv head) * 16 of every page of
     // every item, item by item; a tail item is followed by kAppendSlack free
@@ -596,15 +609,26 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                                                                        it.row0);
         }
     }
-    p->merge_ptr.assign(static_cast<size_t>(L_rows) * H_kv + 1, 0);
+    p->merge_rng.assign(static_cast<size_t>(L_rows) * H_kv, make_int2(0, 0));
     p->merge_ent.clear();
     for (size_t k = 0; k < ent.size(); ++k) {
+        const int32_t e0 = static_cast<int32_t>(p->merge_ent.size());
         p->merge_ent.insert(p->merge_ent.end(), ent[k].begin(), ent[k].end());
         if (p->merge_ent.size() > static_cast<size_t>(INT32_MAX)) return PARASON_EUNSUPPORTED;
-        p->merge_ptr[k + 1] = static_cast<int32_t>(p->merge_ent.size());
+        p->merge_rng[k] = make_int2(e0, static_cast<int32_t>(p->merge_ent.size()));
     }
     for (int32_t b = 0; b < num_leaves && !prefill; ++b)
         for (int32_t n = leaf_node[b]; n >= 0; n = parent[n]) p->path_tokens += node_len[n];
+
+    // room for forks: about as much again as the plan holds, with floors
+    // that let a small plan take a few forks
+    p->cap_items = p->items.size() + std::max<size_t>(4096, p->items.size());
+    p->cap_rows = p->stream_rows.size() + std::max<size_t>(65536, p->stream_rows.size());
+    p->cap_leaves = static_cast<size_t>(p->num_leaves) + std::max<size_t>(64, p->num_leaves);
+    p->cap_ent = p->merge_ent.size() + std::max<size_t>(16384, p->merge_ent.size());
+    // an append patches 6 words per tail item (at most H_kv per branch); a
+    // fork one branch's merge ranges and the queue counters
+    p->cap_patch = p->cap_leaves * H_kv * kPatchesPerTail + 2 * static_cast<size_t>(H_kv) + 2;
     return PARASON_OK;
 }
 
@@ -614,24 +638,26 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
 
 parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     if (cudaGetDevice(&p->device) != cudaSuccess) return PARASON_ECUDA;
-    const size_t n_items = p->items.size() * sizeof(WorkItem);
+    const int32_t H = p->cfg.num_kv_heads;
+    // the arrays forks grow are allocated at their capacity
+    const size_t n_items = p->cap_items * sizeof(WorkItem);
     const size_t n_pages = p->page_ids.size() * sizeof(int32_t);
-    const size_t n_dfs = p->dfs_leaf.size() * sizeof(int32_t);
-    const size_t n_mptr = p->merge_ptr.size() * sizeof(int32_t);
-    const size_t n_ment = p->merge_ent.size() * sizeof(int32_t);
-    const size_t n_rec = p->item_rec.size() * sizeof(int32_t);
-    const size_t n_irows = p->item_rows.size() * sizeof(int32_t);
+    const size_t n_dfs = p->cap_leaves * sizeof(int32_t);
+    const size_t n_mrng = p->cap_leaves * H * sizeof(int2);
+    const size_t n_ment = p->cap_ent * sizeof(int32_t);
+    const size_t n_rec = p->cap_items * parason::kRecWords * sizeof(int32_t);
+    const size_t n_irows = (p->cap_items + 1) * sizeof(int32_t);
     // page rows are read 32 entries past their end by whole warps: pad
-    const size_t n_strows = (p->stream_rows.size() + 32) * sizeof(int32_t);
+    const size_t n_strows = (p->cap_rows + 32) * sizeof(int32_t);
     const size_t n_qnext = 2 * sizeof(int32_t);
     const size_t n_err = parason::kErrWords * sizeof(int32_t);
-    const size_t n_patch = p->tail_items.size() * kPatchesPerTail * sizeof(int2);
+    const size_t n_patch = p->cap_patch * sizeof(int2);
     const size_t n_key0 = p->item_key0.size() * sizeof(int32_t);
     constexpr int kArrays = 12;
     size_t off[kArrays], total = 0;
     // the queue counters and the error record are set separately; the patch
-    // buffer is written by parason_plan_append
-    const size_t sizes[kArrays] = {n_items, n_pages,  n_dfs,   n_mptr, n_ment,  n_rec,
+    // buffer is written by parason_plan_append and parason_plan_fork
+    const size_t sizes[kArrays] = {n_items, n_pages,  n_dfs,   n_mrng, n_ment,  n_rec,
                                    n_irows, n_strows, n_qnext, n_err,  n_patch, n_key0};
     for (int i = 0; i < kArrays; ++i) {
         off[i] = total;
@@ -646,7 +672,7 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     p->d_items = reinterpret_cast<WorkItem *>(base + off[0]);
     p->d_page_ids = reinterpret_cast<int32_t *>(base + off[1]);
     p->d_dfs_leaf = reinterpret_cast<int32_t *>(base + off[2]);
-    p->d_merge_ptr = reinterpret_cast<int32_t *>(base + off[3]);
+    p->d_merge_rng = reinterpret_cast<int2 *>(base + off[3]);
     p->d_merge_ent = reinterpret_cast<int32_t *>(base + off[4]);
     p->d_item_rec = reinterpret_cast<int32_t *>(base + off[5]);
     p->d_item_rows = reinterpret_cast<int32_t *>(base + off[6]);
@@ -656,13 +682,18 @@ parason_status upload(parason_plan_s *p, cudaStream_t stream) {
     p->d_patch = reinterpret_cast<int2 *>(base + off[10]);
     p->d_item_key0 = p->prefill ? reinterpret_cast<int32_t *>(base + off[11]) : nullptr;
     p->w_items = off[0] / sizeof(int32_t);
+    p->w_mrng = off[3] / sizeof(int32_t);
     p->w_rec = off[5] / sizeof(int32_t);
     p->w_strows = off[7] / sizeof(int32_t);
+    p->w_qnext = off[8] / sizeof(int32_t);
     p->blob_words = total / sizeof(int32_t);
     const void *src[8] = {p->items.data(),     p->page_ids.data(),  p->dfs_leaf.data(),
-                          p->merge_ptr.data(), p->merge_ent.data(), p->item_rec.data(),
+                          p->merge_rng.data(), p->merge_ent.data(), p->item_rec.data(),
                           p->item_rows.data(), p->stream_rows.data()};
-    const size_t copy[8] = {n_items, n_pages, n_dfs, n_mptr, n_ment, n_rec, n_irows,
+    const size_t copy[8] = {p->items.size() * sizeof(WorkItem), n_pages,
+                            p->dfs_leaf.size() * sizeof(int32_t), p->merge_rng.size() * sizeof(int2),
+                            p->merge_ent.size() * sizeof(int32_t), p->item_rec.size() * sizeof(int32_t),
+                            p->item_rows.size() * sizeof(int32_t),
                             p->stream_rows.size() * sizeof(int32_t)};
     for (int i = 0; i < 8; ++i) {
         if (copy[i] == 0) continue;
@@ -1130,7 +1161,7 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
     st = record_event(p, 1, stream);
     if (st != PARASON_OK) return st;
     parason::MergeArgs m{};
-    m.merge_ptr = p->d_merge_ptr;
+    m.merge_rng = p->d_merge_rng;
     m.merge_ent = p->d_merge_ent;
     m.part_o = part_o;
     m.part_ml = part_ml;
@@ -1253,14 +1284,14 @@ parason_status parason_plan_append(parason_plan p, const int32_t *new_pages,
         if (dev != p->device) return PARASON_EINVAL;
     }
     for (int32_t b = 0; b < L; ++b) {
-        if (p->tail_ptr[b] == p->tail_ptr[b + 1]) return refuse(PARASON_ENOSPACE);
-        if (p->leaf_len[b] == INT32_MAX) return refuse(PARASON_EUNSUPPORTED);
-        if (p->leaf_len[b] % P16 != 0) continue;
+        const int32_t len = p->tree_len[p->leaf_node[b]];
+        if (p->tails[b].empty()) return refuse(PARASON_ENOSPACE);
+        if (len == INT32_MAX) return refuse(PARASON_EUNSUPPORTED);
+        if (len % P16 != 0) continue;
         if (!new_pages) return refuse(PARASON_EINVAL);
         const int32_t pg = new_pages[b];
         if (pg < 0 || pg >= p->num_phys || p->page_used[pg]) return refuse(PARASON_EINVAL);
-        for (int32_t k = p->tail_ptr[b]; k < p->tail_ptr[b + 1]; ++k) {
-            const int32_t t = p->tail_items[k];
+        for (const int32_t t : p->tails[b]) {
             if (p->item_rows[t] + p->items[t].num_pages + 1 > p->item_rows[t + 1])
                 return refuse(PARASON_ENOSPACE);
             if (p->items[t].num_pages == INT32_MAX) return refuse(PARASON_EUNSUPPORTED);
@@ -1280,9 +1311,8 @@ parason_status parason_plan_append(parason_plan p, const int32_t *new_pages,
     std::vector<int2> &patches = p->patches;
     patches.clear();
     for (int32_t b = 0; b < L; ++b) {
-        const bool opens_page = p->leaf_len[b] % P16 == 0;
-        for (int32_t k = p->tail_ptr[b]; k < p->tail_ptr[b + 1]; ++k) {
-            const int32_t t = p->tail_items[k];
+        const bool opens_page = p->tree_len[p->leaf_node[b]] % P16 == 0;
+        for (const int32_t t : p->tails[b]) {
             WorkItem &it = p->items[t];
             int32_t *rec = p->item_rec.data() + static_cast<size_t>(t) * parason::kRecWords;
             const size_t w_item = p->w_items + static_cast<size_t>(t) * (sizeof(WorkItem) / 4);
@@ -1331,9 +1361,269 @@ parason_status parason_plan_append(parason_plan p, const int32_t *new_pages,
 
     // 4. commit the host copy
     for (const auto &w : host) *w.first = w.second;
-    for (int32_t b = 0; b < L; ++b) p->leaf_len[b] += 1;
+    for (int32_t b = 0; b < L; ++b) {
+        const int32_t n = p->leaf_node[b];
+        if (p->tree_len[n] % P16 == 0) p->node_pages[n].push_back(new_pages[b]);
+        p->tree_len[n] += 1;
+    }
     p->unique_tokens += L;
     p->path_tokens += L;
+    return PARASON_OK;
+}
+
+parason_status parason_plan_fork(parason_plan p, int32_t branch, int32_t num_children,
+                                 const int32_t *child_len, const int32_t *child_page_ptr,
+                                 const int32_t *child_pages, parason_stream_t stream_) {
+    if (!p) return PARASON_EINVAL;
+    if (p->cfg.mode == PARASON_FP32 || p->prefill) return PARASON_EUNSUPPORTED;
+    const int32_t L = p->num_leaves;
+    const int32_t H = p->cfg.num_kv_heads, g = p->group;
+    constexpr int32_t P16 = parason::kPageSize;
+    if (branch < 0 || branch >= L || num_children < 1 || !child_len || !child_page_ptr)
+        return PARASON_EINVAL;
+    if (num_children > INT32_MAX - L || num_children > INT32_MAX - p->num_nodes) return PARASON_EINVAL;
+    // a new branch's rows of every node on its path go to suffix-pass tiles
+    if (g > kNarrowRows) return PARASON_EUNSUPPORTED;
+    if (p->on_device && p->blob_words > static_cast<size_t>(INT32_MAX)) return PARASON_EUNSUPPORTED;
+
+    // 1. check the children: lengths, page counts, fresh distinct pages
+    if (child_page_ptr[0] != 0) return PARASON_EINVAL;
+    for (int32_t c = 0; c < num_children; ++c) {
+        if (child_len[c] < 0) return PARASON_EINVAL;
+        const int64_t want = (static_cast<int64_t>(child_len[c]) + P16 - 1) / P16;
+        if (static_cast<int64_t>(child_page_ptr[c + 1]) - child_page_ptr[c] != want)
+            return PARASON_EINVAL;
+    }
+    const int32_t n_child_pages = child_page_ptr[num_children];
+    if (n_child_pages > 0 && !child_pages) return PARASON_EINVAL;
+    std::vector<int32_t> claimed;
+    auto refuse = [&](parason_status st) {
+        for (int32_t pg : claimed) p->page_used[pg] = 0;
+        return st;
+    };
+    for (int32_t k = 0; k < n_child_pages; ++k) {
+        const int32_t pg = child_pages[k];
+        if (pg < 0 || pg >= p->num_phys || p->page_used[pg]) return refuse(PARASON_EINVAL);
+        p->page_used[pg] = 1;
+        claimed.push_back(pg);
+    }
+    if (p->on_device) {
+        int dev = -1;
+        if (cudaGetDevice(&dev) != cudaSuccess) {
+            cudaGetLastError();
+            return refuse(PARASON_ECUDA);
+        }
+        if (dev != p->device) return refuse(PARASON_EINVAL);
+    }
+
+    // 2. the new work, without touching the plan: branches L .. L + E - 1
+    // are children 1 .. E (child 0 keeps index `branch`); node N0 + c is
+    // child c, under the branch's node nb, which stops being a branch node
+    const int32_t E = num_children - 1;
+    const int32_t nb = p->leaf_node[branch];
+    const int32_t N0 = p->num_nodes;
+    const int32_t D0 = static_cast<int32_t>(p->dfs_leaf.size());   // new branches' DFS positions
+    std::vector<int32_t> path;
+    for (int32_t m = nb; m >= 0; m = p->tree_parent[m]) path.push_back(m);
+    std::reverse(path.begin(), path.end());
+    int64_t path_tok = 0;
+    for (int32_t m : path) path_tok += p->tree_len[m];
+
+    std::vector<WorkItem> items;
+    std::vector<int32_t> rec, irows, rows;          // records, item row starts, page rows
+    std::vector<std::vector<int32_t>> tails(num_children);
+    // merge entries per (child, kv head); child 0 starts from the branch's list
+    std::vector<std::vector<int32_t>> ent(static_cast<size_t>(num_children) * H);
+    for (int32_t j = 0; j < H; ++j) {
+        const int2 r = p->merge_rng[static_cast<size_t>(branch) * H + j];
+        ent[j].assign(p->merge_ent.begin() + r.x, p->merge_ent.begin() + r.y);
+    }
+    int64_t slots = p->num_slots;
+    const size_t item0 = p->items.size(), row0 = p->stream_rows.size();
+    const int32_t page_pos0 = static_cast<int32_t>(p->page_ids.size());
+    bool overflow = false;
+    // one suffix-pass item: `np` pages of `pages` from `pg`, rows of DFS
+    // positions [leaf_lo, leaf_lo + nrows / g) of kv head j
+    auto add_item = [&](const std::vector<int32_t> &pages, int32_t node_len, int32_t page_pos,
+                        int32_t pg, int32_t np, int32_t leaf_lo, int32_t nrows, int32_t j,
+                        bool tail) -> int32_t {
+        const int32_t P = static_cast<int32_t>(pages.size());
+        WorkItem it;
+        it.page_pos = page_pos + pg;
+        it.num_pages = np;
+        it.last_valid = pg + np == P ? node_len - (P - 1) * P16 : P16;
+        it.leaf_lo = leaf_lo;
+        it.row0 = 0;
+        it.nrows = nrows;
+        it.kv_head = j;
+        if (slots + nrows > INT32_MAX) overflow = true;
+        it.slot_base = static_cast<int32_t>(slots);
+        slots += nrows;
+        const int32_t start = static_cast<int32_t>(row0 + rows.size());
+        irows.push_back(start);
+        for (int32_t k = 0; k < np; ++k) rows.push_back((pages[pg + k] * H + j) * P16);
+        if (tail) rows.insert(rows.end(), std::min(kAppendSlackMax, std::max(kAppendSlackMin, np / 2)), 0);
+        const size_t r0 = rec.size();
+        rec.resize(r0 + parason::kRecWords, 0);
+        std::memcpy(&rec[r0], &it, sizeof(WorkItem));
+        rec[r0 + parason::kRecRowsOff] = start;
+        for (int32_t k = 0; k < std::min(np, parason::kRecRows); ++k)
+            rec[r0 + parason::kRecRow0 + k] = (pages[pg + k] * H + j) * P16;
+        items.push_back(it);
+        return static_cast<int32_t>(item0 + items.size() - 1);
+    };
+    // equal pieces of at most the plan's suffix piece length
+    auto pieces = [&](int32_t P, auto &&fn) {
+        const int64_t chunk = std::max<int64_t>(1, p->narrow_chunk);
+        const int64_t n = (P + chunk - 1) / chunk;
+        const int32_t per = static_cast<int32_t>((P + n - 1) / std::max<int64_t>(1, n));
+        for (int32_t pg = 0; pg < P; pg += per) fn(pg, std::min(per, P - pg));
+    };
+    // (a) the new branches on every node of the path, in tiles of whole
+    // branches of at most 16 rows
+    const int32_t bpt = kNarrowRows / g;
+    for (int32_t m : path) {
+        const int32_t P = static_cast<int32_t>(p->node_pages[m].size());
+        if (p->tree_len[m] == 0 || P == 0) continue;
+        for (int32_t j = 0; j < H; ++j)
+            for (int32_t t0 = 0; t0 < E; t0 += bpt) {
+                const int32_t nbr = std::min(bpt, E - t0);
+                pieces(P, [&](int32_t pg, int32_t np) {
+                    const int32_t id = add_item(p->node_pages[m], p->tree_len[m], p->node_page_pos[m],
+                                                pg, np, D0 + t0, nbr * g, j, false);
+                    for (int32_t i = 0; i < nbr; ++i)
+                        ent[static_cast<size_t>(1 + t0 + i) * H + j].push_back(items[id - item0].slot_base +
+                                                                              i * g);
+                });
+            }
+    }
+    // (b) every child's own node: one tile of its g rows per kv head; the
+    // last piece is the branch's tail, followed by room for appends
+    std::vector<std::vector<int32_t>> cpages(num_children);
+    int32_t cpos = page_pos0;
+    std::vector<int32_t> cpage_pos(num_children);
+    for (int32_t c = 0; c < num_children; ++c) {
+        cpages[c].assign(child_pages + child_page_ptr[c], child_pages + child_page_ptr[c + 1]);
+        cpage_pos[c] = cpos;
+        cpos += static_cast<int32_t>(cpages[c].size());
+        const int32_t P = static_cast<int32_t>(cpages[c].size());
+        if (P == 0) continue;
+        const int32_t pos = c == 0 ? p->dfs_pos[branch] : D0 + c - 1;
+        for (int32_t j = 0; j < H; ++j)
+            pieces(P, [&](int32_t pg, int32_t np) {
+                const bool tail = pg + np == P;
+                const int32_t id = add_item(cpages[c], child_len[c], cpage_pos[c], pg, np, pos, g, j, tail);
+                ent[static_cast<size_t>(c) * H + j].push_back(items[id - item0].slot_base);
+                if (tail) tails[c].push_back(id);
+            });
+    }
+    // merge lists, appended: the branch's moved list, then the new branches'
+    std::vector<int32_t> ents;
+    std::vector<int2> rng(static_cast<size_t>(num_children) * H);
+    const size_t ent0 = p->merge_ent.size();
+    for (size_t k = 0; k < ent.size(); ++k) {
+        const int32_t e0 = static_cast<int32_t>(ent0 + ents.size());
+        ents.insert(ents.end(), ent[k].begin(), ent[k].end());
+        rng[k] = make_int2(e0, static_cast<int32_t>(ent0 + ents.size()));
+    }
+    // room in the device copy (the host copy keeps to it too)
+    if (overflow || p->items.size() + items.size() > p->cap_items ||
+        row0 + rows.size() > p->cap_rows || static_cast<size_t>(L) + E > p->cap_leaves ||
+        ent0 + ents.size() > p->cap_ent || ent0 + ents.size() > static_cast<size_t>(INT32_MAX) ||
+        row0 + rows.size() > static_cast<size_t>(INT32_MAX) ||
+        (static_cast<size_t>(L) + E) * H * kPatchesPerTail + 2 * static_cast<size_t>(H) + 2 > p->cap_patch)
+        return refuse(PARASON_ENOSPACE);
+    std::vector<int32_t> dfs_new(static_cast<size_t>(E));
+    for (int32_t i = 0; i < E; ++i) dfs_new[i] = L + i;
+    // a plan that had no attention work has no grid yet: the new items get
+    // one of suffix CTAs, whose warps own the first queue positions
+    const bool new_grid = p->num_ctas == 0 && !items.empty();
+    const int32_t queue_start1 = new_grid ? p->num_sms * p->suffix_warps : p->queue_start[1];
+
+    // 3. the device copy: the appended regions lie past what the kernels
+    // read until the host counts grow, and one scatter then moves the
+    // branch's merge ranges -- so a failure leaves the device plan as it was
+    if (p->debug_flags & PARASON_DEBUG_FAIL_UPDATE) return refuse(PARASON_ECUDA);
+    if (p->on_device) {
+        cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+        std::vector<int2> &patches = p->patches;
+        patches.clear();
+        for (int32_t j = 0; j < H; ++j) {
+            const size_t w = p->w_mrng + 2 * (static_cast<size_t>(branch) * H + j);
+            patches.push_back(make_int2(static_cast<int32_t>(w), rng[j].x));
+            patches.push_back(make_int2(static_cast<int32_t>(w + 1), rng[j].y));
+        }
+        if (new_grid) patches.push_back(make_int2(static_cast<int32_t>(p->w_qnext + 1), queue_start1));
+        struct Copy {
+            void *dst;
+            const void *src;
+            size_t bytes;
+        };
+        const Copy copies[] = {
+            {p->d_items + item0, items.data(), items.size() * sizeof(WorkItem)},
+            {p->d_item_rec + item0 * parason::kRecWords, rec.data(), rec.size() * sizeof(int32_t)},
+            // starts of the new items, and the end of the last one
+            {p->d_item_rows + item0, irows.data(), irows.size() * sizeof(int32_t)},
+            {p->d_stream_rows + row0, rows.data(), rows.size() * sizeof(int32_t)},
+            {p->d_dfs_leaf + D0, dfs_new.data(), dfs_new.size() * sizeof(int32_t)},
+            {p->d_merge_ent + ent0, ents.data(), ents.size() * sizeof(int32_t)},
+            {p->d_merge_rng + static_cast<size_t>(L) * H, rng.data() + H,
+             static_cast<size_t>(E) * H * sizeof(int2)},
+        };
+        const int32_t rows_end = static_cast<int32_t>(row0 + rows.size());
+        bool ok = true;
+        for (const Copy &c : copies)
+            if (c.bytes && cudaMemcpyAsync(c.dst, c.src, c.bytes, cudaMemcpyHostToDevice, stream) !=
+                               cudaSuccess)
+                ok = false;
+        if (ok && cudaMemcpyAsync(p->d_item_rows + item0 + irows.size(), &rows_end, sizeof(int32_t),
+                                  cudaMemcpyHostToDevice, stream) != cudaSuccess)
+            ok = false;
+        if (ok && (cudaMemcpyAsync(p->d_patch, patches.data(), patches.size() * sizeof(int2),
+                                   cudaMemcpyHostToDevice, stream) != cudaSuccess ||
+                   parason::launch_scatter(static_cast<int32_t *>(p->d_blob), p->d_patch,
+                                           static_cast<int32_t>(patches.size()), stream) != cudaSuccess))
+            ok = false;
+        if (!ok) {
+            cudaGetLastError();
+            return refuse(PARASON_ECUDA);
+        }
+    }
+
+    // 4. commit the host copy
+    p->items.insert(p->items.end(), items.begin(), items.end());
+    p->item_rec.insert(p->item_rec.end(), rec.begin(), rec.end());
+    p->item_rows.pop_back();                         // the old end is the first new start
+    p->item_rows.insert(p->item_rows.end(), irows.begin(), irows.end());
+    p->item_rows.push_back(static_cast<int32_t>(row0 + rows.size()));
+    p->stream_rows.insert(p->stream_rows.end(), rows.begin(), rows.end());
+    for (size_t i = item0; i < p->items.size(); ++i) p->narrow_queue.push_back(static_cast<int32_t>(i));
+    p->merge_ent.insert(p->merge_ent.end(), ents.begin(), ents.end());
+    for (int32_t j = 0; j < H; ++j) p->merge_rng[static_cast<size_t>(branch) * H + j] = rng[j];
+    p->merge_rng.insert(p->merge_rng.end(), rng.begin() + H, rng.end());
+    p->dfs_leaf.insert(p->dfs_leaf.end(), dfs_new.begin(), dfs_new.end());
+    for (int32_t i = 0; i < E; ++i) p->dfs_pos.push_back(D0 + i);
+    p->num_slots = slots;
+    for (int32_t c = 0; c < num_children; ++c) {
+        p->tree_parent.push_back(nb);
+        p->tree_len.push_back(child_len[c]);
+        p->node_pages.push_back(cpages[c]);
+        p->node_page_pos.push_back(cpage_pos[c]);
+        p->page_ids.insert(p->page_ids.end(), cpages[c].begin(), cpages[c].end());
+        p->unique_tokens += child_len[c];
+        p->path_tokens += child_len[c] + (c > 0 ? path_tok : 0);
+    }
+    p->tails[branch] = tails[0];
+    for (int32_t c = 1; c < num_children; ++c) p->tails.push_back(tails[c]);
+    p->leaf_node[branch] = N0;
+    for (int32_t c = 1; c < num_children; ++c) p->leaf_node.push_back(N0 + c);
+    p->num_nodes += num_children;
+    p->num_leaves += E;
+    if (new_grid) {
+        p->num_ctas = p->num_sms;
+        p->num_wide_ctas = 0;
+        p->queue_start[1] = queue_start1;
+    }
     return PARASON_OK;
 }
 
@@ -1344,7 +1634,7 @@ parason_status parason_plan_export(parason_plan p, int32_t table, void *dst, siz
     switch (table) {
     case PARASON_TABLE_ITEMS: src = p->items.data(); n = p->items.size() * sizeof(WorkItem); break;
     case PARASON_TABLE_DFS_LEAVES: src = p->dfs_leaf.data(); n = p->dfs_leaf.size() * 4; break;
-    case PARASON_TABLE_MERGE_PTR: src = p->merge_ptr.data(); n = p->merge_ptr.size() * 4; break;
+    case PARASON_TABLE_MERGE_RANGES: src = p->merge_rng.data(); n = p->merge_rng.size() * 8; break;
     case PARASON_TABLE_MERGE: src = p->merge_ent.data(); n = p->merge_ent.size() * 4; break;
     case PARASON_TABLE_WIDE_QUEUE: src = p->wide_queue.data(); n = p->wide_queue.size() * 4; break;
     case PARASON_TABLE_NARROW_QUEUE: src = p->narrow_queue.data(); n = p->narrow_queue.size() * 4; break;

@@ -202,6 +202,7 @@ def build_tree(name: str, parent, node_len, leaf_node, *, num_q_heads: int,
         rng = np.random.default_rng(seed)
     meta = dict(meta or {})
     meta.setdefault("permuted", bool(permute_pages))
+    meta.setdefault("q_std", float(q_std))
     parent = np.asarray(parent, dtype=np.int32)
     node_len = np.asarray(node_len, dtype=np.int32)
     leaf_node = np.asarray(leaf_node, dtype=np.int32)
@@ -501,6 +502,41 @@ def grow_branches(tree: ForkTree, pool: list):
     ptr[1:] = np.cumsum([len(p) for p in pages])
     ids = np.asarray([x for p in pages for x in p], dtype=np.int32)
     return replace(tree, node_len=node_len, node_page_ptr=ptr, page_ids=ids), new_pages
+
+
+def fork_branch(tree: ForkTree, b: int, child_lens: Sequence[int], pool: list, seed: int = 0):
+    """The tree after branch b forks into len(child_lens) threads (its node
+    gets one child node per thread, appended in order).  Child 0 is branch
+    b; child c >= 1 is the new branch num_leaves + c - 1, with a fresh query
+    row drawn from ``seed``.  Each child takes ceil(len / 16) pages of `pool`
+    (consumed in place); their K and V are the values already in the pool.
+    Returns (tree, child_pages) with child_pages[c] the pages of child c."""
+    k = len(child_lens)
+    nb = int(tree.leaf_node[b])
+    n0 = tree.num_nodes
+    child_pages = []
+    for ln in child_lens:
+        child_pages.append([pool.pop(0) for _ in range((int(ln) + PAGE_SIZE - 1) // PAGE_SIZE)])
+    parent = np.concatenate([tree.parent, np.full(k, nb, dtype=np.int32)]).astype(np.int32)
+    node_len = np.concatenate([tree.node_len, np.asarray(child_lens, dtype=np.int32)]).astype(np.int32)
+    counts = [len(p) for p in child_pages]
+    ptr = np.concatenate([tree.node_page_ptr,
+                          tree.node_page_ptr[-1] + np.cumsum(counts, dtype=np.int64)]).astype(np.int32)
+    page_ids = np.concatenate([tree.page_ids,
+                               np.asarray([x for p in child_pages for x in p], dtype=np.int32)])
+    leaf_node = tree.leaf_node.copy()
+    leaf_node[b] = n0
+    leaf_node = np.concatenate([leaf_node, np.arange(n0 + 1, n0 + k, dtype=np.int32)])
+    q = tree.q
+    if k > 1 and q.numel():
+        gen = torch.Generator(device=q.device)
+        gen.manual_seed(int(seed) + 104729)
+        extra = torch.randn((k - 1,) + tuple(q.shape[1:]), generator=gen, device=q.device,
+                            dtype=torch.float32) * float(tree.meta.get("q_std", 1.0))
+        q = torch.cat([q, extra.to(q.dtype)], dim=0)
+    return replace(tree, parent=parent, node_len=node_len, node_page_ptr=ptr,
+                   page_ids=page_ids.astype(np.int32), leaf_node=leaf_node.astype(np.int32),
+                   q=q), child_pages
 
 
 def build_prefill(name: str, parent, node_len, chunk_node, *, num_q_heads: int,

@@ -39,7 +39,7 @@ def verify_plan(tree, plan):
     info = plan.info()
     items = plan.export(_lib.TABLE_ITEMS)
     dfs = plan.export(_lib.TABLE_DFS_LEAVES)
-    mptr = plan.export(_lib.TABLE_MERGE_PTR)
+    mrng = plan.export(_lib.TABLE_MERGE_RANGES)
     ment = plan.export(_lib.TABLE_MERGE)
     assert sorted(dfs.tolist()) == list(range(tree.num_leaves))
     owner = node_of_page_pos(tree)
@@ -85,12 +85,13 @@ def verify_plan(tree, plan):
     # nothing computed for nodes no branch reads
     assert all(k[0] in under and tree.node_len[k[0]] > 0 for k in coverage)
     # merge lists per (branch, kv head): exactly the slots written for each q head
-    assert mptr[0] == 0 and mptr[-1] == len(ment)
+    # a fresh plan lays the lists out in (branch, kv head) order, end to end
+    assert mrng[0, 0] == 0 and mrng[-1, 1] == len(ment) and (mrng[1:, 0] == mrng[:-1, 1]).all()
     for b in range(tree.num_leaves):
         for h in range(tree.num_q_heads):
             j, r = divmod(h, g)
             k = b * H_kv + j
-            got = sorted(int(e) + r for e in ment[mptr[k]:mptr[k + 1]])
+            got = sorted(int(e) + r for e in ment[mrng[k, 0]:mrng[k, 1]])
             assert got == sorted(slots_of[(b, h)]), (b, h)
     assert info["unique_tokens"] == tree.unique_tokens()
     assert info["path_tokens"] == tree.path_tokens()

@@ -39,7 +39,7 @@ def verify_prefill_plan(tree, plan):
     items = plan.export(_lib.TABLE_ITEMS)
     key0 = plan.export(_lib.TABLE_ITEM_KEY0)
     dfs = plan.export(_lib.TABLE_DFS_LEAVES)
-    mptr = plan.export(_lib.TABLE_MERGE_PTR)
+    mrng = plan.export(_lib.TABLE_MERGE_RANGES)
     ment = plan.export(_lib.TABLE_MERGE)
     wq = plan.export(_lib.TABLE_WIDE_QUEUE)
     nq = plan.export(_lib.TABLE_NARROW_QUEUE)
@@ -74,7 +74,8 @@ def verify_prefill_plan(tree, plan):
             assert slot not in seen, "partial slot written twice"
             seen[slot] = (int(leaf_lo) + t, kvh * g + row % g, vis)
     assert sorted(seen) == list(range(info["num_slots"]))
-    assert mptr[0] == 0 and mptr[-1] == len(ment)
+    # a fresh plan lays the lists out in (branch, kv head) order, end to end
+    assert mrng[0, 0] == 0 and mrng[-1, 1] == len(ment) and (mrng[1:, 0] == mrng[:-1, 1]).all()
     for c, n in enumerate(chunks):
         want_anc = [(a, x) for a in ancestors(tree, n) for x in range(int(tree.node_len[a]))]
         for t in range(lens[c]):
@@ -84,7 +85,7 @@ def verify_prefill_plan(tree, plan):
                 j, r = divmod(h, g)
                 k = q * H_kv + j
                 got = []
-                for e in ment[mptr[k]:mptr[k + 1]]:
+                for e in ment[mrng[k, 0]:mrng[k, 1]]:
                     qq, hh, vis = seen[int(e) + r]
                     assert (qq, hh) == (q, h)
                     assert vis, "a merged slot must see at least one key"
@@ -166,6 +167,6 @@ def test_prefill_plan_deterministic():
     for _ in range(2):
         with Plan.for_prefill(tree, host_only=True) as plan:
             tabs.append([plan.export(t) for t in (_lib.TABLE_ITEMS, _lib.TABLE_ITEM_KEY0,
-                                                  _lib.TABLE_MERGE_PTR, _lib.TABLE_MERGE)])
+                                                  _lib.TABLE_MERGE_RANGES, _lib.TABLE_MERGE)])
     for a, b in zip(*tabs):
         assert np.array_equal(a, b)

@@ -6,7 +6,6 @@ counts, and no (branch, kv head) is computed by two ranks.  The decode step
 needs no exchange between ranks (Sec. 3.4: branches are independent workers,
 requests do not share KV; grouped kv heads are independent), so matching
 coverage is the whole correctness condition of the split."""
-import collections
 import os
 import socket
 import sys
@@ -18,6 +17,7 @@ import torch.multiprocessing as mp
 from paper_2608_24658_gb300 import _lib, build
 from paper_2608_24658_gb300 import workloads as W
 from paper_2608_24658_gb300.api import Plan, ParasonError
+from tests.plan_cover import coverage, definition
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
@@ -25,51 +25,6 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 @pytest.fixture(scope="module", autouse=True)
 def _built():
     build.build()
-
-
-def coverage(plan, head0=0):
-    """{(global branch, global kv head): sorted ((physical page, valid tokens), ...)}
-    read from the plan's merge lists, items and page streams."""
-    H = plan.num_kv_heads
-    items = plan.export(_lib.TABLE_ITEMS)
-    irows = plan.export(_lib.TABLE_ITEM_ROWS)
-    srows = plan.export(_lib.TABLE_STREAM_ROWS)
-    mptr = plan.export(_lib.TABLE_MERGE_PTR)
-    ment = plan.export(_lib.TABLE_MERGE)
-    glob = plan.export(_lib.TABLE_SHARD_BRANCHES)
-    owner = {}
-    for i, it in enumerate(items):
-        for s in range(int(it[7]), int(it[7]) + int(it[5])):
-            owner[s] = i
-    out = {}
-    for b in range(plan.num_leaves):
-        for j in range(H):
-            cov = []
-            for e in ment[mptr[b * H + j]:mptr[b * H + j + 1]]:
-                i = owner[int(e)]
-                npg, last_valid = int(items[i][1]), int(items[i][2])
-                r = srows[irows[i]:irows[i] + npg].astype(np.int64) // 16
-                assert ((r % H) == j).all()
-                for k, pg in enumerate(r // H):
-                    cov.append((int(pg), last_valid if k == npg - 1 else 16))
-            out[(int(glob[b]), head0 + j)] = tuple(sorted(cov))
-    return out
-
-
-def definition(tree):
-    """What each (branch, kv head) must attend to: every page of every node on
-    its path with its valid tokens (empty nodes hold no page)."""
-    out = {}
-    for b in range(tree.num_leaves):
-        cov = []
-        for n in tree.path(b):
-            ln = int(tree.node_len[n])
-            pages = tree.page_ids[tree.node_page_ptr[n]:tree.node_page_ptr[n + 1]]
-            for k, pg in enumerate(pages):
-                cov.append((int(pg), ln - 16 * k if k == len(pages) - 1 else 16))
-        for j in range(tree.num_kv_heads):
-            out[(b, j)] = tuple(sorted(cov))
-    return out
 
 
 def shard_tree():
