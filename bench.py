@@ -250,6 +250,8 @@ TABLE = [(1, "bf16"), (2, "bf16"), (3, "bf16"), (4, "bf16"), (5, "bf16"), (5, "f
 
 
 def make_workload(args, device, config=None, mode=None):
+    if config is None and getattr(args, "workload", None):
+        return W.EXTRA[args.workload](mode=mode or args.mode, device=device)
     return W.make_config(config or args.config, mode=mode or args.mode, device=device)
 
 
@@ -804,6 +806,10 @@ def main(argv=None):
     ap.add_argument("--config", type=int, default=4,
                     help="workload 1-5 of the JSON line (default 4: 32 requests x 32 "
                          "branches, permuted pages, the largest that fits one GPU)")
+    ap.add_argument("--workload", choices=sorted(W.EXTRA), default=None,
+                    help="a measurement workload instead of --config (for profiling: "
+                         "batched_4req = the batched workload with 4 requests; "
+                         "prefix_only = the 32k prefix under 128 one-token branches)")
     ap.add_argument("--no-table", dest="table", action="store_false",
                     help="skip the other configurations timed after the headline")
     ap.add_argument("--table-steps", type=int, default=300,

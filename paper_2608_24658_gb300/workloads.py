@@ -318,8 +318,26 @@ def long_reasoning(mode="bf16", device="cpu", branches=128, **kw) -> ForkTree:
                       head_dim=128, mode=mode, rng=rng, device=device, **kw)
 
 
+def long_prefix_only(mode="bf16", device="cpu", branches=128, **kw) -> ForkTree:
+    """The long-reasoning prefix (32768 tokens, 64 q / 8 kv heads, d 128)
+    under `branches` branches of one token each: nearly all of the step is
+    the stacked prefix tile (1024 rows per kv head), for measuring it alone."""
+    rng = np.random.default_rng(4)
+    lens = [32768] + [1] * branches
+    parent = [-1] + [0] * branches
+    return build_tree(f"prefix_only_32768_{branches}x1", parent, lens,
+                      list(range(1, branches + 1)), num_q_heads=64, num_kv_heads=8,
+                      head_dim=128, mode=mode, rng=rng, device=device, **kw)
+
+
 CONFIGS = {1: tiny_fork, 2: llama3_trials, 3: subtask_trial_tree, 4: batched_serving,
            5: long_reasoning}
+
+# measurement workloads beside the five: a scaled-down batched workload (for
+# counter captures that must stay small) and the prefix tile alone
+EXTRA = {"batched_4req": lambda mode="bf16", device="cpu", **kw: batched_serving(
+             mode=mode, device=device, requests=4, **kw),
+         "prefix_only": long_prefix_only}
 
 
 def make_config(idx: int, mode: Optional[str] = None, device="cpu", **kw) -> ForkTree:
