@@ -745,9 +745,13 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
     int pulled = 0, iss_pg = 0, iss_np = 0, issued = 0;
     bool iss_done = false;
     int fetch = 0;                   // 0: idle, 1: position claimed, 2: record requested
-    // lane 0: the claimed queue position; a suffix CTA's warps own their first
+    // lane 0: the claimed queue position.  Warp w of suffix CTA c owns
+    // position w * Nc + c (Nc suffix CTAs): consecutive positions, often
+    // neighbouring pieces of one run, start on different SMs instead of all
+    // on one (same-box A/B: the Llama-3-shape step 40.1 -> 39.7 us, the
+    // other workloads level)
     const int own_first = static_cast<int>(blockIdx.x) - a.num_wide_ctas;
-    int claimed = own_first >= 0 ? own_first * S::kSuffixWarps + warp : -1;
+    int claimed = own_first >= 0 ? warp * (a.num_ctas - a.num_wide_ctas) + own_first : -1;
     int nxt_id = -1;
     int32_t nxt_w = 0;               // lane i: word i of the next item's record
     int32_t cur_w = 0;               // lane i: word i of the current item's record

@@ -71,9 +71,10 @@ struct AttnArgs {
     // pull prefix-pass items and then suffix-pass items; every warp of the
     // other CTAs pulls suffix-pass items.  queue_next[0] / [1] are the next
     // positions to claim.  The first claims need no atomic: position c of
-    // the prefix queue belongs to prefix CTA c, position 8 (c - W) + w of the
-    // suffix queue to warp w of suffix CTA c, so the counters start past
-    // them (queue_start; the merge kernel sets them back).
+    // the prefix queue belongs to prefix CTA c, position w Nc + (c - W) of
+    // the suffix queue to warp w of suffix CTA c (Nc = num_ctas - W suffix
+    // CTAs), so the counters start past them (queue_start; the merge kernel
+    // sets them back).
     const int32_t *item_rec;        // kRecWords per item, items in pull order
     int32_t num_wide_items;
     int32_t num_narrow_items;
