@@ -39,11 +39,21 @@ int32_t narrow_warps(int32_t mode, int32_t head_dim, int32_t g) {
 }
 constexpr int kMinPiecePages = 8;       // suffix-pass pieces are at least this long
 constexpr int kMaxPiecePages = 128;     // and at most this long
-// Prefill pieces may be longer: the tile is compute-bound there, and every
-// piece costs a 64 KB partial (written, then read by the merge).  The
-// tcgen05 tile holds an item of up to 512 pages.
-constexpr int kMaxPrefillPiecePages = 512;
+// The tcgen05 tile holds an item of up to 512 pages (its metadata slot).
+constexpr int kMaxTileItemPages = 512;
 constexpr int kWideBlockPages = 4;      // prefix pieces are whole 64-token blocks
+// Prefix pieces: about one prefix CTA's share of the prefix work each, at
+// most what the tile's metadata holds.  Every piece writes 64 KB of partial
+// rows (128 rows) that the merge reads back and costs the tile an item
+// change; the prefix CTAs join the suffix queue when theirs is empty, which
+// evens out their uneven shares.  Same-box A/B against a third of a share
+// and at most 128 pages: two-level step 81.8 -> 78.7 us, Llama-3 shape
+// 39.8 -> 39.2 us, long prefix 854.5 -> 843 us (e4m3 KV 655.4 -> 600.2
+// us), batched 2460 -> 2447 us.
+constexpr int64_t kWidePiecesPerCta = 1;
+// suffix pieces: about this many per warp of the launch (at least
+// kMinPiecePages and at most kMaxPiecePages pages)
+constexpr int64_t kNarrowPiecesPerWarp = 3;
 constexpr double kWideProvision = 1.15; // prefix CTAs relative to the cost model
 constexpr int kFp32ChunkPages = 32;
 // stream rows kept free after a branch's last item: half its pages, 4 to 64
@@ -470,15 +480,17 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         const int64_t total_warps = static_cast<int64_t>(p->num_sms) * p->suffix_warps;
         const int64_t narrow_chunk = std::min<int64_t>(
             kMaxPiecePages,
-            std::max<int64_t>(kMinPiecePages, narrow_pages / std::max<int64_t>(1, total_warps * 3)));
+            std::max<int64_t>(kMinPiecePages,
+                              narrow_pages / std::max<int64_t>(1, total_warps * kNarrowPiecesPerWarp)));
         p->narrow_chunk = narrow_chunk;
         int64_t wide_pages = 0;
         for (const Run &r : runs)
             if (r.wide) wide_pages += r.pages;
         const int64_t wide_chunk = std::min<int64_t>(
-            prefill ? kMaxPrefillPiecePages : kMaxPiecePages,
+            kMaxTileItemPages,
             std::max<int64_t>(kWideBlockPages,
-                              wide_pages / std::max<int64_t>(1, static_cast<int64_t>(n_wide) * 3)));
+                              wide_pages / std::max<int64_t>(1, static_cast<int64_t>(n_wide) *
+                                                                    kWidePiecesPerCta)));
         // The row tiles of one (node, kv head) read the same pages: their
         // pieces are emitted piece by piece across the tiles, so that the
         // queue hands out the copies of one page range together and all but
@@ -1295,9 +1307,9 @@ parason_status parason_plan_append(parason_plan p, const int32_t *new_pages,
             if (p->item_rows[t] + p->items[t].num_pages + 1 > p->item_rows[t + 1])
                 return refuse(PARASON_ENOSPACE);
             if (p->items[t].num_pages == INT32_MAX) return refuse(PARASON_EUNSUPPORTED);
-            // a prefix-pass item stays within the prefix pass's page limit
+            // a prefix-pass item stays within what the tile's metadata holds
             if (t < static_cast<int32_t>(p->wide_queue.size()) &&
-                p->items[t].num_pages + 1 > kMaxPiecePages)
+                p->items[t].num_pages + 1 > kMaxTileItemPages)
                 return refuse(PARASON_ENOSPACE);
         }
         p->page_used[pg] = 1;
