@@ -52,8 +52,10 @@ constexpr int kWideBlockPages = 4;      // prefix pieces are whole 64-token bloc
 // us), batched 2460 -> 2447 us.
 constexpr int64_t kWidePiecesPerCta = 1;
 // suffix pieces: about this many per warp of the launch (at least
-// kMinPiecePages and at most kMaxPiecePages pages)
-constexpr int64_t kNarrowPiecesPerWarp = 3;
+// kMinPiecePages and at most kMaxPiecePages pages).  Same-box A/B against
+// 3: two-level step 79.7 -> 78.8 us, the Llama-3 shape level (its pieces
+// stay at the 8-page floor); 2 made the Llama-3-shape step 2 us slower.
+constexpr double kNarrowPiecesPerWarp = 2.5;
 constexpr double kWideProvision = 1.15; // prefix CTAs relative to the cost model
 constexpr int kFp32ChunkPages = 32;
 // stream rows kept free after a branch's last item: half its pages, 4 to 64
@@ -481,7 +483,8 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         const int64_t narrow_chunk = std::min<int64_t>(
             kMaxPiecePages,
             std::max<int64_t>(kMinPiecePages,
-                              narrow_pages / std::max<int64_t>(1, total_warps * kNarrowPiecesPerWarp)));
+                              static_cast<int64_t>(static_cast<double>(narrow_pages) /
+                                                   (kNarrowPiecesPerWarp * std::max<int64_t>(1, total_warps)))));
         p->narrow_chunk = narrow_chunk;
         int64_t wide_pages = 0;
         for (const Run &r : runs)

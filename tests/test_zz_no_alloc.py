@@ -16,7 +16,7 @@ from paper_2608_24658_gb300.api import Plan, ParasonError
 def test_plan_over_scratch_limit_is_rejected_first():
     """No device work: the size check comes before any other."""
     build.build()
-    big = W.make_config(5, values=False)                    # 128 branches x 36 K tokens
+    big = W.batched_serving(requests=64, values=False)     # 2048 branches
     with Plan.for_tree(big, host_only=True) as p:
         assert p.workspace_bytes > _lib.NO_ALLOC_SCRATCH_BYTES
         st = _lib.load().parason_attn_decode_no_alloc(p.handle, *([None] * 8))
