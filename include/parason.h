@@ -438,6 +438,12 @@ typedef struct {
     int32_t num_wide_items;     /* prefix-pass items (tiles x pieces)       */
     int32_t num_narrow_items;   /* suffix-pass items                        */
     int64_t num_stream_rows;    /* entries of PARASON_TABLE_STREAM_ROWS     */
+    int32_t tile_pairs;         /* 1: the prefix queue holds pairs of row
+                                   tiles of one piece (bf16 KV, head_dim
+                                   128): entries 2k and 2k + 1 are pulled
+                                   together, and the second has no rows
+                                   (row count 0) when the piece's tile
+                                   count is odd                              */
 } parason_plan_info;
 
 parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info);
@@ -458,7 +464,8 @@ parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info)
  *                            branch's first q head of the kv head; q head
  *                            j*g + r reads slot entry + r
  *   PARASON_TABLE_WIDE_QUEUE int32 [num_wide_items]: prefix-pass items in the
- *                            order the kernel's prefix CTAs pull them
+ *                            order the kernel's prefix CTAs pull them (two
+ *                            at a time when tile_pairs is set)
  *   PARASON_TABLE_NARROW_QUEUE int32 [num_narrow_items]: suffix-pass items in
  *                            the order the kernel's warps pull them
  *   PARASON_TABLE_ITEM_ROWS  int32 [num_items + 1]: start of each item's page

@@ -42,7 +42,8 @@ class PlanInfo(ctypes.Structure):
                 ("path_tokens", ctypes.c_int64), ("num_sms", ctypes.c_int32),
                 ("on_device", ctypes.c_int32), ("num_ctas", ctypes.c_int32),
                 ("num_wide_ctas", ctypes.c_int32), ("num_wide_items", ctypes.c_int32),
-                ("num_narrow_items", ctypes.c_int32), ("num_stream_rows", ctypes.c_int64)]
+                ("num_narrow_items", ctypes.c_int32), ("num_stream_rows", ctypes.c_int64),
+                ("tile_pairs", ctypes.c_int32)]
 
 
 class TraceStats(ctypes.Structure):

@@ -1147,9 +1147,12 @@ struct TcMeta {
     WorkItem it;
     int32_t id;                      // -1: the queue is empty
     int32_t key0;                    // causal item: its first key's token index, else -1
-    int32_t pad[2];
+    int32_t key0B;                   // pair mode: the same for the second tile
+    int32_t pad;
+    WorkItem itB;                    // pair mode: the second tile (no rows: none)
     int32_t rows[kTcMetaPages];      // TMA row of each page
     int32_t leaves[kTcRows];         // branch of rows [g i, g i + g)
+    int32_t leavesB[kTcRows];        // pair mode: the same for the second tile
 };
 
 // barrier slots (8 bytes each) in the CTA's barrier area
@@ -1813,6 +1816,512 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
     }
 }
 
+// ---------------------------------------------------------------------------
+// prefix pass on tcgen05, pair mode (bf16 KV, head_dim 128): two 128-row
+// tiles of one piece -- consecutive row tiles of one node and kv head, over
+// the same pages -- against every staged 64-token block, so that each block
+// is staged once for 256 rows.  The prefix queue holds pairs: position k is
+// items 2k (tile A) and 2k + 1 (tile B, no rows when the piece has one
+// tile).
+//
+//   warp 10     scheduler: pulls pairs and stages their metadata
+//   warp 8      producer: TMA of each block of the pair's pages, once, into
+//               a 4-stage ring
+//   warp 9      S issuer (one thread): S_t = Q_t K^T for t = A, B of a block,
+//               A and B from shared memory
+//   warp 11     PV issuer (one thread): O_t += P_t V; the stage goes back to
+//               the producer after the block's last PV
+//   warps 0-3   tile A: softmax (thread r owns row r, TMEM lane r), the next
+//               pair's Q rows into shared memory, then the row's (m, l) and O
+//   warps 4-7   tile B: the same for the second tile
+//
+// TMEM, 512 columns: O_A, O_B at 0 and 128; S/P of tile A at 256 and 320, of
+// tile B at 384 and 448 (each tile alternates its two buffers by block, as
+// the single-tile pass does).  Shared memory: the ring [4][K | V] as in the
+// single-tile pass, then Q_A and Q_B, 32 KB each, in the layout TMA gives a
+// K block (two 16 KB column blocks of 128 rows x 128 bytes, 128-byte
+// swizzle).  Every wait is bounded, as in the single-tile pass.
+// ---------------------------------------------------------------------------
+constexpr int kTpStages = 4;
+constexpr int kTpQOffset = kTpStages * kTcStageBytes;         // 128 KB
+constexpr int kTpQColBlockBytes = kTcRows * 128;              // 16 KB
+constexpr int kTpQBytes = 2 * kTpQColBlockBytes;              // 32 KB: d = 128
+static_assert(kTpQOffset + 2 * kTpQBytes <= kTcRingBytes, "pair-mode ring and Q fit");
+
+enum TcPairBar : int {
+    kPbKvFull = 0,                            // [stages] producer -> S issuer (TMA bytes)
+    kPbKvEmpty = kPbKvFull + kTpStages,       // [stages] PV issuer commit -> producer
+    kPbSFull = kPbKvEmpty + kTpStages,        // [2 tiles x 2] S issuer commit -> tile warps
+    kPbPFull = kPbSFull + 4,                  // [2 x 2] tile warps (128 arrivals) -> PV issuer
+    kPbPvDone = kPbPFull + 4,                 // [2 x 2] PV commit -> S issuer, tile warps (rescale)
+    kPbQReady = kPbPvDone + 4,                // [2] tile warps (128 arrivals) -> S issuer
+    kPbOFull = kPbQReady + 2,                 // [2] PV commit -> tile warps
+    kPbOEmpty = kPbOFull + 2,                 // [2] tile warps (4 arrivals) -> PV issuer
+    kPbMetaFull = kPbOEmpty + 2,              // [kTcMeta] scheduler -> every role
+    kPbMetaEmpty = kPbMetaFull + kTcMeta,     // [kTcMeta] the 8 tile warps -> scheduler
+    kPbDrain = kPbMetaEmpty + kTcMeta,        // both issuers' commits -> issuers
+    kTcPairBars
+};
+
+__host__ __device__ constexpr int tc_pair_bar_count(int i) {
+    return ((i >= kPbPFull && i < kPbPFull + 4) || (i >= kPbQReady && i < kPbQReady + 2))
+               ? kTcRows
+               : ((i >= kPbOEmpty && i < kPbOEmpty + 2)
+                      ? 4
+                      : ((i >= kPbMetaEmpty && i < kPbMetaEmpty + kTcMeta) ? 8
+                                                                          : (i == kPbDrain ? 2 : 1)));
+}
+
+// Queue position k of the prefix queue in pair mode: item 2k (-1: empty).
+__device__ __forceinline__ int pair_item(const AttnArgs &a, int k) {
+    return 2 * k + 1 < a.num_wide_items ? 2 * k : -1;
+}
+
+template <int D>
+__device__ void prefix_cta_tc_pair(const KvMaps *maps, const AttnArgs &a, uint8_t *smem, uint32_t bars,
+                                   uint32_t tmem, int warp, int lane, volatile int *abort_flag,
+                                   TcMeta *meta) {
+    static_assert(D == 128, "the tcgen05 prefix tile is written for head_dim 128");
+    const uint32_t ring = dev::smem_addr(smem);
+    auto bar = [&](int i) { return bars + 8u * static_cast<uint32_t>(i); };
+    const long long limit = a.wait_limit_ns;
+
+    if (warp == kTcSchedulerWarp) {
+        // ------------------------------------------------------------ scheduler
+        for (int k = 0;; ++k) {
+            const int s = k % kTcMeta;
+            if (k >= kTcMeta &&
+                !tc_warp_wait(bar(kPbMetaEmpty + s), ((k / kTcMeta) - 1) & 1, limit, abort_flag, lane)) {
+                if (lane == 0) tc_fail(a, abort_flag, kSiteProducerEmpty);
+                break;
+            }
+            // a prefix CTA owns pair blockIdx.x of the prefix queue
+            int id = -1;
+            if (!*abort_flag) {
+                if (k == 0) {
+                    id = pair_item(a, static_cast<int>(blockIdx.x));
+                } else {
+                    int pos = 0;
+                    if (lane == 0) pos = atomicAdd(a.queue_next, 1);
+                    id = pair_item(a, __shfl_sync(0xffffffffu, pos, 0));
+                }
+            }
+            TcMeta &m = meta[s];
+            if (id >= 0) {
+                const WorkItem it = a.items[id], itB = a.items[id + 1];
+                bool bad = it.num_pages <= 0 || it.num_pages > kTcMetaPages || it.nrows <= 0 ||
+                           it.nrows > kTcRows || it.row0 % a.group != 0;
+                if (itB.nrows != 0)
+                    bad = bad || itB.nrows < 0 || itB.nrows > kTcRows || itB.row0 % a.group != 0 ||
+                          itB.num_pages != it.num_pages || itB.page_pos != it.page_pos ||
+                          itB.last_valid != it.last_valid || itB.kv_head != it.kv_head;
+                if (bad) {
+                    if (lane == 0 && !*abort_flag) {
+                        *abort_flag = 1;
+                        dev::record_error(a.err, PARASON_EINVAL, kSiteBadItem);
+                    }
+                    id = -1;
+                } else {
+                    if (lane == 0) {
+                        m.it = it;
+                        m.itB = itB;
+                        m.key0 = a.item_key0 ? a.item_key0[id] : -1;
+                        m.key0B = a.item_key0 ? a.item_key0[id + 1] : -1;
+                    }
+                    const int32_t *src = a.stream_rows + a.item_rows[id];
+                    for (int p = lane; p < it.num_pages; p += 32) m.rows[p] = src[p];
+                    const int nbr = (it.nrows + a.group - 1) / a.group;
+                    const int32_t *lv = a.dfs_leaf + it.leaf_lo + it.row0 / a.group;
+                    for (int i = lane; i < nbr; i += 32) m.leaves[i] = lv[i];
+                    if (itB.nrows > 0) {
+                        const int nbrB = (itB.nrows + a.group - 1) / a.group;
+                        const int32_t *lvB = a.dfs_leaf + itB.leaf_lo + itB.row0 / a.group;
+                        for (int i = lane; i < nbrB; i += 32) m.leavesB[i] = lvB[i];
+                    }
+                }
+            }
+            if (lane == 0) m.id = id;
+            __syncwarp();
+            if (lane == 0) dev::mbar_arrive(bar(kPbMetaFull + s));
+            if (id < 0) break;
+        }
+    } else if (warp == kTcProducerWarp) {
+        // ------------------------------------------------------------ producer
+        const bool skip_first = a.debug_flags & PARASON_DEBUG_SKIP_FIRST_LOAD;
+        const uint64_t last_pol = dev::l2_evict_last_policy();
+        const int kv_page_rows = a.num_kv_heads * kPageSize;
+        int last_issue[kTpStages];
+        for (int s = 0; s < kTpStages; ++s) last_issue[s] = -1;
+        int blk = 0;
+        bool ok = true;
+        for (int k = 0; ok; ++k) {
+            const int ms = k % kTcMeta;
+            if (!tc_warp_wait(bar(kPbMetaFull + ms), (k / kTcMeta) & 1, limit, abort_flag, lane)) {
+                if (lane == 0) tc_fail(a, abort_flag, kSiteProducerEmpty);
+                break;
+            }
+            const TcMeta &m = meta[ms];
+            if (m.id < 0) break;
+            const int np = m.it.num_pages;
+            const int nb = tc_blocks(np);
+            for (int bi = 0; bi < nb; ++bi, ++blk) {
+                const int s = blk % kTpStages;
+                if (blk >= kTpStages &&
+                    !tc_warp_wait(bar(kPbKvEmpty + s), ((blk / kTpStages) - 1) & 1, limit, abort_flag,
+                                  lane)) {
+                    if (lane == 0) tc_fail(a, abort_flag, kSiteProducerEmpty);
+                    ok = false;
+                    break;
+                }
+                if (!(skip_first && blk == 0)) {
+                    const uint32_t fb = bar(kPbKvFull + s);
+                    if (lane == 0) dev::mbar_arrive_expect_tx(fb, kTcStageBytes);
+                    __syncwarp();
+                    const int pg0 = bi * kTcBlockPages;
+                    bool run = pg0 + kTcBlockPages <= np;
+                    const int row0 = m.rows[pg0 < np ? pg0 : 0];
+#pragma unroll
+                    for (int j = 1; j < kTcBlockPages; ++j)
+                        run = run && m.rows[pg0 + j] == row0 + j * kv_page_rows;
+                    if (run) {
+                        const int page = row0 / kv_page_rows;
+                        // lane: K (even) or V, column block lane / 2
+                        if (lane < 4)
+                            dev::tma_load_5d_hint(ring + s * kTcStageBytes + (lane & 1) * kTcKBytes +
+                                                      (lane >> 1) * kTcColBlockBytes,
+                                                  (lane & 1) ? &maps->v_run : &maps->k_run, 0, lane >> 1,
+                                                  0, m.it.kv_head, page, fb, last_pol);
+                    } else if (lane < 4 * kTcBlockPages) {
+                        // page j = lane / 4, column block (lane / 2) % 2, K (even lanes) or V
+                        const int j = lane >> 2, cb = (lane >> 1) & 1;
+                        const int pg = bi * kTcBlockPages + j;
+                        const int row = pg < np ? m.rows[pg] : a.kv_rows;   // kv_rows: zero fill
+                        const uint32_t off = cb * kTcColBlockBytes + j * kPageSize * 128;
+                        const uint32_t st = ring + s * kTcStageBytes + (lane & 1) * kTcKBytes;
+                        dev::tma_load_3d_hint(st + off, (lane & 1) ? &maps->v : &maps->k, 0, cb, row, fb,
+                                              last_pol);
+                    }
+                    last_issue[s] = blk;
+                }
+            }
+        }
+        // every copy this CTA issued must land before its shared memory is reused
+        if (lane == 0)
+            for (int s = 0; s < kTpStages; ++s)
+                if (last_issue[s] >= 0)
+                    dev::mbar_wait_bounded(bar(kPbKvFull + s), (last_issue[s] / kTpStages) & 1,
+                                           kDrainLimitNs, nullptr);
+    } else if (warp == kTcMmaWarp || warp == kTcPvWarp) {
+        // ------------------------------------------------------------ MMA issuers
+        if (lane == 0) {
+            constexpr uint32_t kIdS = tc::idesc_bf16_f32(kTcRows, kTcBlockTokens, false);
+            constexpr uint32_t kIdPV = tc::idesc_bf16_f32(kTcRows, D, true);
+            auto wait = [&](int i, int parity) {
+                return tc_wait(bar(i), static_cast<uint32_t>(parity & 1), limit, abort_flag);
+            };
+            const uint64_t desc_k = tc::smem_desc_sw128(ring, 16, 1024);
+            const uint64_t desc_v = tc::smem_desc_sw128(ring + kTcKBytes, kTcColBlockBytes, 1024);
+            const uint64_t desc_q[2] = {tc::smem_desc_sw128(ring + kTpQOffset, 16, 1024),
+                                        tc::smem_desc_sw128(ring + kTpQOffset + kTpQBytes, 16, 1024)};
+            constexpr uint32_t kStageStep = kTcStageBytes >> 4;
+            bool ok = true;
+            int st = 0, ph = 0;              // stage of the block and the stage's phase parity
+            int u[2] = {0, 0};               // blocks of each tile so far
+            int j[2] = {0, 0};               // pairs in which each tile had rows
+            for (int k = 0; ok; ++k) {
+                const int ms = k % kTcMeta;
+                if (!wait(kPbMetaFull + ms, k / kTcMeta)) {
+                    ok = false;
+                    break;
+                }
+                if (meta[ms].id < 0) break;
+                const bool on[2] = {true, meta[ms].itB.nrows > 0};
+                const int nb = tc_blocks(meta[ms].it.num_pages);
+                if (warp == kTcMmaWarp) {
+                    for (int t = 0; t < 2 && ok; ++t)
+                        if (on[t] && !wait(kPbQReady + t, j[t])) ok = false;
+                    if (ok) tc::fence_after_sync();
+                    for (int i = 0; i < nb && ok; ++i) {
+                        if (!wait(kPbKvFull + st, ph)) {
+                            ok = false;
+                            break;
+                        }
+                        const uint64_t kd = desc_k + static_cast<uint64_t>(st * kStageStep);
+                        for (int t = 0; t < 2; ++t) {
+                            if (!on[t]) continue;
+                            const int buf = u[t] & 1;
+                            // the buffer holds the tile's P of two blocks back until its PV is done
+                            if (u[t] >= 2 && !wait(kPbPvDone + 2 * t + buf, (u[t] - 2) >> 1)) {
+                                ok = false;
+                                break;
+                            }
+                            tc::fence_after_sync();
+                            const uint32_t tS = tmem + kTmemS + 128u * t + 64u * buf;
+#pragma unroll
+                            for (int ks = 0; ks < D / 16; ++ks) {
+                                const uint32_t koff = ((ks >> 2) * kTcColBlockBytes + (ks & 3) * 32) >> 4;
+                                const uint32_t qoff = ((ks >> 2) * kTpQColBlockBytes + (ks & 3) * 32) >> 4;
+                                tc::mma_bf16(tS, desc_q[t] + qoff, kd + koff, kIdS, ks > 0);
+                            }
+                            tc::commit(bar(kPbSFull + 2 * t + buf));
+                            ++u[t];
+                        }
+                        if (++st == kTpStages) {
+                            st = 0;
+                            ph ^= 1;
+                        }
+                    }
+                } else {
+                    for (int i = 0; i < nb && ok; ++i) {
+                        const uint64_t vd = desc_v + static_cast<uint64_t>(st * kStageStep);
+                        for (int t = 0; t < 2; ++t) {
+                            if (!on[t]) continue;
+                            const int buf = u[t] & 1;
+                            if (!wait(kPbPFull + 2 * t + buf, u[t] >> 1) ||
+                                // the tile's O was last used by its previous pair: stored?
+                                (i == 0 && j[t] > 0 && !wait(kPbOEmpty + t, j[t] - 1))) {
+                                ok = false;
+                                break;
+                            }
+                            tc::fence_after_sync();
+                            const uint32_t tO = tmem + kTmemO + 128u * t;
+                            const uint32_t tP = tmem + kTmemS + 128u * t + 64u * buf;
+#pragma unroll
+                            for (int kk = 0; kk < kTcBlockTokens / 16; ++kk)
+                                tc::mma_bf16_tmem_a(tO, tP + 8u * kk,
+                                                    vd + static_cast<uint32_t>((kk * 2048) >> 4), kIdPV,
+                                                    i > 0 || kk > 0);
+                            tc::commit(bar(kPbPvDone + 2 * t + buf));
+                            if (i == nb - 1) tc::commit(bar(kPbOFull + t));
+                            ++u[t];
+                        }
+                        if (!ok) break;
+                        // both tiles' products of the stage are done when this arrives
+                        // (each S completed before its P was written)
+                        tc::commit(bar(kPbKvEmpty + st));
+                        if (++st == kTpStages) st = 0;
+                    }
+                }
+                for (int t = 0; t < 2; ++t)
+                    if (on[t]) ++j[t];
+            }
+            if (!ok) tc_fail(a, abort_flag, kSiteConsumerFull);
+            // every MMA of both issuers must finish before TMEM is freed
+            tc::commit(bar(kPbDrain));
+            dev::mbar_wait_bounded(bar(kPbDrain), 0, kDrainLimitNs, nullptr);
+        }
+        __syncwarp();
+    } else if (warp < 8) {
+        // ------------------------------------------------------------ tile warps
+        const int t = warp >> 2;                         // tile A (warps 0-3) or B (4-7)
+        const int quarter = warp & 3;                    // its TMEM lanes
+        const int r = quarter * 32 + lane;               // tile row == TMEM lane
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+        const uint32_t tO = lane_base + kTmemO + 128u * t;
+        const uint32_t q_smem = ring + kTpQOffset + t * kTpQBytes;
+        bool ok = true;
+        int u = 0, jp = 0;                               // this tile's blocks and pairs so far
+        auto tile_of = [&](const TcMeta &m) -> const WorkItem & { return t == 0 ? m.it : m.itB; };
+        // Q rows of the tile in pair k into the tile's Q buffer in shared
+        // memory (row r: 16 chunks of 16 bytes, 128-byte swizzle) by
+        // asynchronous copies (zeros past the tile's rows) ...
+        auto issue_q = [&](int k) {
+            const TcMeta &m = meta[k % kTcMeta];
+            const WorkItem &it = tile_of(m);
+            const bool live = r < it.nrows;
+            const int leaf = live ? (t == 0 ? m.leaves : m.leavesB)[r / a.group] : 0;
+            const int head = live ? it.kv_head * a.group + r % a.group : 0;
+            const char *src = reinterpret_cast<const char *>(
+                static_cast<const __nv_bfloat16 *>(a.q) +
+                (static_cast<int64_t>(leaf) * a.num_q_heads + head) * D);
+            const uint32_t bytes = live ? 16u : 0u;
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+                const uint32_t dst = q_smem + (c >> 3) * kTpQColBlockBytes + r * 128 +
+                                     (((c & 7) ^ (r & 7)) << 4);
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst),
+                             "l"(src + 16 * c), "r"(bytes)
+                             : "memory");
+            }
+        };
+        // ... that are waited for, made visible to the tensor cores and
+        // announced to the S issuer later
+        auto publish_q = [&]() {
+            asm volatile("cp.async.wait_all;" ::: "memory");
+            tc::fence_proxy_async_smem();
+            dev::mbar_arrive(bar(kPbQReady + t));
+        };
+        // wait for slot k; true if it holds a pair
+        auto has_pair = [&](int k) {
+            if (!tc_warp_wait(bar(kPbMetaFull + k % kTcMeta), (k / kTcMeta) & 1, limit, abort_flag, lane)) {
+                ok = false;
+                return false;
+            }
+            return meta[k % kTcMeta].id >= 0;
+        };
+        auto on_in = [&](int k) { return t == 0 || meta[k % kTcMeta].itB.nrows > 0; };
+        bool have = has_pair(0);
+        if (have && on_in(0)) {
+            issue_q(0);
+            publish_q();
+        }
+        for (int k = 0; ok && have; ++k) {
+            const TcMeta &m = meta[k % kTcMeta];
+            const bool on = on_in(k);
+            bool more = false, loaded_next = false;
+            if (on) {
+                const WorkItem it = tile_of(m);
+                const int nb = tc_blocks(it.num_pages);
+                const int tokens = (it.num_pages - 1) * kPageSize + it.last_valid;
+                const int key0 = t == 0 ? m.key0 : m.key0B;
+                const int t_rel = key0 < 0 ? (1 << 30) : (it.row0 + r) / a.group - key0;
+                float m_use = -INFINITY, l = 0.f;
+                for (int i = 0; i < nb; ++i) {
+                    const int buf = u & 1;
+                    const uint32_t tS = lane_base + kTmemS + 128u * t + 64u * buf;
+                    const int valid = min(kTcBlockTokens, tokens - i * kTcBlockTokens);
+                    const int seen = min(valid, t_rel - i * kTcBlockTokens + 1);
+                    if (!tc_warp_wait(bar(kPbSFull + 2 * t + buf), (u >> 1) & 1, limit, abort_flag, lane)) {
+                        ok = false;
+                        break;
+                    }
+                    tc::fence_after_sync();
+                    uint32_t sr[2][32];
+                    tc::ld32(tS, sr[0]);
+                    tc::ld32(tS + 32, sr[1]);
+                    tc::wait_ld();
+                    // the tile's last S of the pair is done: its Q buffer takes the
+                    // next pair's rows while this block's softmax runs
+                    if (i == nb - 1) {
+                        more = has_pair(k + 1);
+                        if (!ok) break;
+                        if (more && on_in(k + 1)) {
+                            issue_q(k + 1);
+                            loaded_next = true;
+                        }
+                    }
+                    float x[64];
+#pragma unroll
+                    for (int q = 0; q < 64; ++q) x[q] = __uint_as_float(sr[q >> 5][q & 31]);
+                    if (seen < kTcBlockTokens) {
+#pragma unroll
+                        for (int q = 0; q < 64; ++q) x[q] = q < seen ? x[q] : -INFINITY;
+                    }
+                    float mr = x[0];
+#pragma unroll
+                    for (int q = 1; q + 1 < 64; q += 2) mr = dev::max3(mr, x[q], x[q + 1]);
+                    mr = fmaxf(mr, x[63]);
+                    const float sl = a.scale_log2;
+                    const float mb = mr * sl;
+                    if (i == 0) {
+                        m_use = mb;
+                    } else if (__any_sync(0xffffffffu, mb > m_use + kTcRescaleLog2)) {
+                        // O must hold the tile's previous PV before it is rescaled
+                        if (!tc_warp_wait(bar(kPbPvDone + 2 * t + ((u - 1) & 1)), ((u - 1) >> 1) & 1, limit,
+                                          abort_flag, lane)) {
+                            ok = false;
+                            break;
+                        }
+                        tc::fence_after_sync();
+                        const float m_new = fmaxf(m_use, mb);
+                        const float alpha = m_new == m_use ? 1.f : dev::fast_exp2(m_use - m_new);
+#pragma unroll
+                        for (int c = 0; c < D / 32; ++c) {
+                            uint32_t ov[32];
+                            tc::ld32(tO + 32 * c, ov);
+                            tc::wait_ld();
+#pragma unroll
+                            for (int q = 0; q < 32; ++q)
+                                ov[q] = __float_as_uint(__uint_as_float(ov[q]) * alpha);
+                            tc::st32(tO + 32 * c, ov);
+                        }
+                        tc::wait_st();
+                        l *= alpha;
+                        m_use = m_new;
+                    }
+                    const float m_ref = m_use == -INFINITY ? 0.f : m_use;
+                    const unsigned long long slp = dev::f32x2(sl, sl), nmp = dev::f32x2(-m_ref, -m_ref);
+                    unsigned long long lsum = dev::f32x2(0.f, 0.f);
+                    uint32_t pw[32];
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) {
+                        float e0, e1;
+                        dev::f32x2_split(dev::fma_f32x2(dev::f32x2(x[2 * c], x[2 * c + 1]), slp, nmp), e0, e1);
+                        const float p0 = dev::fast_exp2(e0), p1 = dev::fast_exp2(e1);
+                        lsum = dev::add_f32x2(lsum, dev::f32x2(p0, p1));
+                        pw[c] = dev::pack_bf16(p0, p1);
+                    }
+                    {
+                        float l0, l1;
+                        dev::f32x2_split(lsum, l0, l1);
+                        l += l0 + l1;
+                    }
+                    tc::st32(tS, pw);
+                    tc::wait_st();
+                    // V rows past the item's last token may hold anything (NaN
+                    // included); P is 0 there but 0 * NaN is NaN, so tile A zeroes
+                    // them before its PV -- tile B's PV of the block is issued after
+                    if (t == 0 && valid < kTcBlockTokens) {
+                        const int stage = u % kTpStages;   // tile A has a block of every stage
+                        const uint32_t vst = ring + stage * kTcStageBytes + kTcKBytes;
+                        const int n16 = (kTcBlockTokens - valid) * 2 * 8;
+                        for (int q = r; q < n16; q += kTcRows) {
+                            const int tt = valid + q / 16, cb = (q / 8) & 1, c = q & 7;
+                            asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
+                                             vst + cb * kTcColBlockBytes + tt * 128 + (c << 4)),
+                                         "r"(0u)
+                                         : "memory");
+                        }
+                        tc::fence_proxy_async_smem();
+                    }
+                    tc::fence_before_sync();
+                    dev::mbar_arrive(bar(kPbPFull + 2 * t + buf));
+                    ++u;
+                }
+                if (!ok) break;
+                if (loaded_next) publish_q();
+                if (r < it.nrows) a.part_ml[static_cast<int64_t>(it.slot_base) + r] = make_float2(m_use, l);
+                // the tile's O, once its last PV is done
+                if (!tc_warp_wait(bar(kPbOFull + t), jp & 1, limit, abort_flag, lane)) {
+                    ok = false;
+                    break;
+                }
+                tc::fence_after_sync();
+                float *dst = a.part_o + (static_cast<int64_t>(it.slot_base) + r) * D;
+#pragma unroll
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t ov[32];
+                    tc::ld32(tO + 32 * c, ov);
+                    tc::wait_ld();
+                    if (r < it.nrows) {
+#pragma unroll
+                        for (int q = 0; q < 32; q += 4)
+                            *reinterpret_cast<float4 *>(dst + 32 * c + q) =
+                                make_float4(__uint_as_float(ov[q]), __uint_as_float(ov[q + 1]),
+                                            __uint_as_float(ov[q + 2]), __uint_as_float(ov[q + 3]));
+                    }
+                }
+                tc::fence_before_sync();
+                __syncwarp();
+                if (lane == 0) dev::mbar_arrive(bar(kPbOEmpty + t));
+                ++jp;
+            } else {
+                // the tile has no rows in this pair; its Q buffer is free
+                more = has_pair(k + 1);
+                if (!ok) break;
+                if (more && on_in(k + 1)) {
+                    issue_q(k + 1);
+                    publish_q();
+                }
+            }
+            __syncwarp();
+            if (lane == 0) dev::mbar_arrive(bar(kPbMetaEmpty + k % kTcMeta));
+            have = more;
+        }
+        if (!ok && lane == 0) tc_fail(a, abort_flag, kSiteConsumerFull);
+    }
+}
+
 // One CTA per SM: 12 warps leave at most 168 registers per thread (three warps
 // on one sub-partition of 16K registers).
 template <int D, class KV>
@@ -1830,10 +2339,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool wide = static_cast<int>(blockIdx.x) < a.num_wide_ctas;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-    // the prefix pass at head_dim 128 (bf16 or e4m3 KV) runs on tcgen05
+    // the prefix pass at head_dim 128 (bf16 or e4m3 KV) runs on tcgen05; with
+    // bf16 KV the plan may hand it pairs of row tiles (pair mode)
     constexpr bool kTcPrefix = D == 128;
-    constexpr int kPrefixBars = kTcPrefix ? kTcBars : 2 * S::kWideStages + kIdSlots;
-    static_assert(!kTcPrefix || kTcBars <= S::kBars, "barrier area holds the tcgen05 barriers");
+    const bool tc_pairs = kTcPrefix && KV::kElemBytes == 2 && a.tc_pairs != 0;
+    const int prefix_bars =
+        kTcPrefix ? (tc_pairs ? static_cast<int>(kTcPairBars) : static_cast<int>(kTcBars))
+                  : 2 * S::kWideStages + kIdSlots;
+    static_assert(!kTcPrefix || (kTcBars <= S::kBars && kTcPairBars <= S::kBars),
+                  "barrier area holds the tcgen05 barriers");
     __shared__ TcMeta tc_meta[kTcPrefix ? kTcMeta : 1];
     auto init_suffix_barriers = [&]() {
         for (int s = 0; s < S::kNarrowBars; ++s) dev::mbar_init(bars + 8 * s, 1);
@@ -1841,7 +2355,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ uint32_t tmem_base;
     if (threadIdx.x == 0) {
         abort_flag = 0;
-        if (wide && kTcPrefix) {
+        if (wide && kTcPrefix && tc_pairs) {
+            for (int i = 0; i < kTcPairBars; ++i) dev::mbar_init(bars + 8 * i, tc_pair_bar_count(i));
+        } else if (wide && kTcPrefix) {
             for (int i = 0; i < kTcBars; ++i)
                 dev::mbar_init(bars + 8 * i, tc_bar_count(i, KV::kElemBytes == 1));
         } else if (wide) {
@@ -1868,8 +2384,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (wide) {
         if constexpr (kTcPrefix) {
             tc::fence_after_sync();
-            prefix_cta_tc<D, KV>(&maps, a, smem, bars, tmem_base, warp, lane, &abort_flag,
-                             tc_meta);
+            if constexpr (KV::kElemBytes == 2) {
+                if (tc_pairs)
+                    prefix_cta_tc_pair<D>(&maps, a, smem, bars, tmem_base, warp, lane, &abort_flag,
+                                          tc_meta);
+                else
+                    prefix_cta_tc<D, KV>(&maps, a, smem, bars, tmem_base, warp, lane, &abort_flag,
+                                         tc_meta);
+            } else {
+                prefix_cta_tc<D, KV>(&maps, a, smem, bars, tmem_base, warp, lane, &abort_flag,
+                                     tc_meta);
+            }
             tc::fence_before_sync();
             __syncthreads();
             tc::fence_after_sync();
@@ -1883,7 +2408,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncthreads();
         if (abort_flag) return;
         if (threadIdx.x == 0) {
-            for (int i = 0; i < kPrefixBars; ++i)
+            for (int i = 0; i < prefix_bars; ++i)
                 asm volatile("mbarrier.inval.shared::cta.b64 [%0];" ::"r"(bars + 8 * i) : "memory");
             init_suffix_barriers();
             dev::fence_mbar_init();

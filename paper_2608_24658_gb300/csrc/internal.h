@@ -91,6 +91,10 @@ struct AttnArgs {
     // first key when the item is causal, else -1; null for decode plans
     const int32_t *item_key0;
     int32_t suffix_warps;   // suffix-pass warps per CTA the plan was made for
+    // bf16 KV at head_dim 128: the prefix queue holds pairs of row tiles of
+    // one piece (position k: items 2k and 2k + 1, the second without rows
+    // when the piece has one tile), run by the tcgen05 tile in pair mode
+    int32_t tc_pairs;
 };
 
 struct MergeArgs {

@@ -56,7 +56,14 @@ constexpr int64_t kWidePiecesPerCta = 1;
 // 3: two-level step 79.7 -> 78.8 us, the Llama-3 shape level (its pieces
 // stay at the 8-page floor); 2 made the Llama-3-shape step 2 us slower.
 constexpr double kNarrowPiecesPerWarp = 2.5;
-constexpr double kWideProvision = 1.15; // prefix CTAs relative to the cost model
+constexpr double kWideProvision = 1.15;   // prefix CTAs relative to the cost model
+// pairs of tcgen05 row tiles when at least this share of the prefix
+// tile-pages sits in pieces of two or more tiles.  Same-box A/B, pairs
+// against single tiles: 32k prefix tile alone 207.4 -> 155.8 us, join
+// prefill 856.6 -> 721.8 us, fork prefill 84.5 -> 75.2 us, long prefix
+// 842.8 -> 839.4 us; the two-level tree (2/3 of its tile-pages in pieces of
+// two or more tiles) 77.6 -> 87.8 us, so it stays on single tiles.
+constexpr int64_t kPairShareNum = 3, kPairShareDen = 4;
 constexpr int kFp32ChunkPages = 32;
 // stream rows kept free after a branch's last item: half its pages, 4 to 64
 // (an item that grows further makes the launch's tail: build a new plan)
@@ -128,6 +135,10 @@ struct parason_plan_s {
     int32_t num_ctas = 0;
     int32_t num_wide_ctas = 0;
     int32_t suffix_warps = 8;          // suffix-pass warps per CTA (kernel instantiation)
+    // the prefix queue holds pairs of row tiles (bf16 KV, head_dim 128):
+    // position k is items 2k and 2k + 1, the second without rows when its
+    // piece has an odd number of tiles
+    bool tc_pairs = false;
     int64_t num_slots = 0;
     int64_t unique_tokens = 0;
     int64_t path_tokens = 0;
@@ -405,6 +416,38 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
             }
     }
 
+    // The row tiles of one (node, kv head) over the same pages: runs [i, j)
+    auto group_end = [&](size_t i) {
+        size_t j = i + 1;
+        while (j < runs.size() && runs[j].node == runs[i].node && runs[j].head == runs[i].head &&
+               runs[j].pages == runs[i].pages)
+            ++j;
+        return j;
+    };
+    // Pairs of tiles: with bf16 KV at head_dim 128, when most prefix
+    // tile-pages sit in pieces of two or more tiles, the tcgen05 tile runs
+    // two tiles of a piece against each staged block.  The cost model and
+    // the piece length still count tiles one by one (counting a pair as one
+    // unit made fewer prefix CTAs and longer pieces, and was slower: long
+    // prefix 841.8 -> 853.4 us, 32k prefix tile alone 156.1 -> 232.4 us).
+    p->tc_pairs = false;
+    if (mode == PARASON_BF16 && cfg->head_dim == 128) {
+        int64_t multi = 0, all = 0;
+        for (size_t i = 0; i < runs.size();) {
+            const size_t j = group_end(i);
+            if (runs[i].wide) {
+                const int64_t tp = static_cast<int64_t>(j - i) * runs[i].pages;
+                all += tp;
+                if (j - i >= 2) multi += tp;
+            }
+            i = j;
+        }
+        p->tc_pairs = all > 0 && multi * kPairShareDen >= all * kPairShareNum;
+    }
+    int64_t wide_units = 0;                 // tile-pages of the prefix pass
+    for (const Run &r : runs)
+        if (r.wide) wide_units += r.pages;
+
     // CTAs of the persistent kernel: the first n_wide start on the prefix
     // queue and join the suffix queue when it runs dry, the others run the
     // suffix queue only.  Prefix CTAs are over-provisioned on purpose: spare
@@ -442,7 +485,10 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     std::vector<std::pair<int64_t, int32_t>> wide_q, narrow_q;   // (pages, item)
     std::vector<std::pair<int32_t, int32_t>> tails;              // (branch, item)
     std::vector<int32_t> key0;                                   // per item (prefill)
-    auto emit = [&](const Run &run, int64_t pg0, int64_t np) -> bool {
+    // `queued`: the item starts a queue entry (the second tile of a pair
+    // does not); `blank`: a pair's second tile without rows
+    auto emit = [&](const Run &run, int64_t pg0, int64_t np, bool queued = true,
+                    bool blank = false) -> bool {
         WorkItem it;
         const int64_t P = run.node_pages;
         it.page_pos = node_page_ptr[run.node] + static_cast<int32_t>(pg0);
@@ -451,17 +497,17 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                             ? node_len[run.node] - static_cast<int32_t>(P - 1) * parason::kPageSize
                             : parason::kPageSize;
         it.leaf_lo = static_cast<int32_t>(run.leaf_lo);
-        it.row0 = run.row0;
-        it.nrows = run.nrows;
+        it.row0 = blank ? 0 : run.row0;
+        it.nrows = blank ? 0 : run.nrows;
         it.kv_head = run.head;
-        if (slots + run.nrows > INT32_MAX) return false;
+        if (slots + it.nrows > INT32_MAX) return false;
         it.slot_base = static_cast<int32_t>(slots);
-        slots += run.nrows;
+        slots += it.nrows;
         const int32_t id = static_cast<int32_t>(p->items.size());
         p->items.push_back(it);
-        (run.wide ? wide_q : narrow_q).emplace_back(np, id);
-        key0.push_back(run.causal ? static_cast<int32_t>(pg0 * parason::kPageSize) : -1);
-        if (!prefill && pg0 + np == P && leaf_of_node[run.node] >= 0)
+        if (queued) (run.wide ? wide_q : narrow_q).emplace_back(np, id);
+        key0.push_back(run.causal && !blank ? static_cast<int32_t>(pg0 * parason::kPageSize) : -1);
+        if (!prefill && !blank && pg0 + np == P && leaf_of_node[run.node] >= 0)
             tails.emplace_back(leaf_of_node[run.node], id);
         return true;
     };
@@ -486,33 +532,34 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                               static_cast<int64_t>(static_cast<double>(narrow_pages) /
                                                    (kNarrowPiecesPerWarp * std::max<int64_t>(1, total_warps)))));
         p->narrow_chunk = narrow_chunk;
-        int64_t wide_pages = 0;
-        for (const Run &r : runs)
-            if (r.wide) wide_pages += r.pages;
         const int64_t wide_chunk = std::min<int64_t>(
             kMaxTileItemPages,
             std::max<int64_t>(kWideBlockPages,
-                              wide_pages / std::max<int64_t>(1, static_cast<int64_t>(n_wide) *
+                              wide_units / std::max<int64_t>(1, static_cast<int64_t>(n_wide) *
                                                                     kWidePiecesPerCta)));
         // The row tiles of one (node, kv head) read the same pages: their
         // pieces are emitted piece by piece across the tiles, so that the
         // queue hands out the copies of one page range together and all but
         // the first read of each page come from L2.
         for (size_t i = 0; i < runs.size();) {
-            size_t j = i + 1;
-            while (j < runs.size() && runs[j].node == runs[i].node && runs[j].head == runs[i].head &&
-                   runs[j].pages == runs[i].pages)
-                ++j;
+            const size_t j = group_end(i);
             const Run &r = runs[i];
+            const bool pairs = r.wide && p->tc_pairs;
             const int64_t align = r.wide ? kWideBlockPages : 1;
             int64_t chunk = r.wide ? wide_chunk : narrow_chunk;
             chunk = std::max<int64_t>(align, chunk / align * align);
             const int64_t n = (r.pages + chunk - 1) / chunk;
             int64_t per = (r.pages + n - 1) / n;
             per = (per + align - 1) / align * align;
-            for (int64_t pg = 0; pg < r.pages; pg += per)
-                for (size_t t = i; t < j; ++t)
-                    if (!emit(runs[t], pg, std::min(per, r.pages - pg))) return PARASON_EUNSUPPORTED;
+            for (int64_t pg = 0; pg < r.pages; pg += per) {
+                const int64_t np = std::min(per, r.pages - pg);
+                for (size_t t = i; t < j; ++t) {
+                    const bool second = pairs && (t - i) % 2 == 1;
+                    if (!emit(runs[t], pg, np, !second)) return PARASON_EUNSUPPORTED;
+                    if (pairs && !second && t + 1 == j && !emit(runs[t], pg, np, false, true))
+                        return PARASON_EUNSUPPORTED;
+                }
+            }
             i = j;
         }
     }
@@ -528,6 +575,15 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     };
     order(wide_q, p->wide_queue);
     order(narrow_q, p->narrow_queue);
+    if (p->tc_pairs) {       // each queued first tile brings its second along
+        std::vector<int32_t> both;
+        both.reserve(2 * p->wide_queue.size());
+        for (int32_t id : p->wide_queue) {
+            both.push_back(id);
+            both.push_back(id + 1);
+        }
+        p->wide_queue.swap(both);
+    }
     if (mode == PARASON_FP32) {        // one CTA per item, no queues
         p->wide_queue.clear();
         p->narrow_queue.clear();
@@ -615,6 +671,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     std::vector<std::vector<int32_t>> ent(static_cast<size_t>(L_rows) * H_kv);
     for (size_t ii = 0; ii < p->items.size(); ++ii) {
         const WorkItem &it = p->items[ii];
+        if (it.nrows == 0) continue;                  // a pair's blank second tile
         const int32_t k0 = prefill ? key0[ii] : -1;
         const int32_t pos_lo = it.row0 / g, pos_hi = (it.row0 + it.nrows - 1) / g;
         for (int32_t pos = pos_lo; pos <= pos_hi; ++pos) {
@@ -1140,6 +1197,7 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
         a.kv_rows = static_cast<int32_t>(p->num_phys * p->cfg.num_kv_heads * parason::kPageSize);
         a.item_key0 = p->d_item_key0;
         a.suffix_warps = p->suffix_warps;
+        a.tc_pairs = p->tc_pairs ? 1 : 0;
         cudaError_t e;
         if (p->cfg.mode == PARASON_FP32) {
             e = parason::launch_attn_fp32(a, static_cast<const float *>(k_pages),
@@ -1271,6 +1329,7 @@ parason_status parason_plan_get_info(parason_plan p, parason_plan_info *info) {
     info->num_wide_items = static_cast<int32_t>(p->wide_queue.size());
     info->num_narrow_items = static_cast<int32_t>(p->narrow_queue.size());
     info->num_stream_rows = static_cast<int64_t>(p->stream_rows.size());
+    info->tile_pairs = p->tc_pairs ? 1 : 0;
     return PARASON_OK;
 }
 

@@ -330,6 +330,18 @@ def long_prefix_only(mode="bf16", device="cpu", branches=128, **kw) -> ForkTree:
                       head_dim=128, mode=mode, rng=rng, device=device, **kw)
 
 
+def pair_fixture(mode="bf16", device="cpu", **kw) -> ForkTree:
+    """A small tree whose prefix tiles come in pairs with bf16 KV (16 q / 2
+    kv heads, d 128, g 8): a 700-token root under 40 branches (320 rows: a
+    pair and an odd tile), inner nodes of 90 and 35 tokens under 17 and 23
+    branches (136 and 184 rows: pairs with 8- and 56-row second tiles), and
+    one-token to 40-token branch nodes."""
+    parent = [-1, 0, 0] + [1] * 17 + [2] * 23
+    lens = [700, 90, 35] + [1 + k for k in range(40)]
+    return build_tree("tile_pairs_odd", parent, lens, list(range(3, 43)), num_q_heads=16,
+                      num_kv_heads=2, head_dim=128, mode=mode, seed=12, device=device, **kw)
+
+
 CONFIGS = {1: tiny_fork, 2: llama3_trials, 3: subtask_trial_tree, 4: batched_serving,
            5: long_reasoning}
 

@@ -49,3 +49,30 @@ def definition(tree):
         for j in range(tree.num_kv_heads):
             out[(b, j)] = tuple(sorted(cov))
     return out
+
+
+def check_tile_pairs(plan):
+    """The prefix queue in pair mode: entries 2k and 2k + 1 are two row tiles
+    of one piece (the same pages and kv head, the second's rows right after
+    the first's) or a tile and a blank (no rows, never merged).  Returns the
+    blank items; outside pair mode there are none and every item has rows."""
+    info = plan.info()
+    items = plan.export(_lib.TABLE_ITEMS)
+    wq = plan.export(_lib.TABLE_WIDE_QUEUE)
+    blank = {i for i, it in enumerate(items) if int(it[5]) == 0}
+    if not info["tile_pairs"]:
+        assert not blank, "an item without rows outside pair mode"
+        return blank
+    assert len(wq) % 2 == 0
+    seconds = set()
+    for k in range(0, len(wq), 2):
+        a, b = items[wq[k]], items[wq[k + 1]]
+        assert int(a[5]) >= 1, "a pair's first tile has rows"
+        seconds.add(int(wq[k + 1]))
+        if int(b[5]) == 0:
+            continue
+        assert a[0] == b[0] and a[1] == b[1] and a[2] == b[2], "a pair reads one page range"
+        assert a[6] == b[6] and a[3] == b[3], "a pair is one kv head of one node"
+        assert b[4] == a[4] + a[5], "a pair's tiles are consecutive row tiles"
+    assert blank <= seconds, "a blank item outside a pair's second place"
+    return blank

@@ -8,7 +8,7 @@ import pytest
 from paper_2608_24658_gb300 import _lib, build
 from paper_2608_24658_gb300 import workloads as W
 from paper_2608_24658_gb300.api import Plan, ParasonError
-from tests.plan_cover import coverage, definition
+from tests.plan_cover import check_tile_pairs, coverage, definition
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -30,6 +30,7 @@ def check(tree, plan):
     nq = plan.export(_lib.TABLE_NARROW_QUEUE)
     wq = plan.export(_lib.TABLE_WIDE_QUEUE)
     assert sorted(wq.tolist() + nq.tolist()) == list(range(len(items)))
+    check_tile_pairs(plan)
 
 
 def base_tree(mode="bf16", **kw):

@@ -53,6 +53,10 @@ FIXTURES = {
         "ones", [-1, 0, 0, 0], [1, 1, 1, 1], [1, 2, 3], num_q_heads=8, num_kv_heads=1,
         head_dim=64, mode=m, seed=5, device="cuda"),
     "custom_scale": lambda m: W.figure3_tree(mode=m, sm_scale=0.21, device="cuda"),
+    # bf16 runs the prefix tile in pairs of row tiles here: 320 root rows (a
+    # pair and a tile without a partner), 136 and 184 rows under the two
+    # inner nodes (pairs whose second tile has 8 and 56 rows)
+    "tile_pairs_odd": lambda m: W.pair_fixture(mode=m, device="cuda", tail_value=float("nan")),
 }
 
 

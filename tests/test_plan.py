@@ -16,6 +16,7 @@ import numpy as np
 import pytest
 
 from paper_2608_24658_gb300 import _lib, build
+from tests.plan_cover import check_tile_pairs
 from paper_2608_24658_gb300.api import Plan
 from paper_2608_24658_gb300 import workloads as W
 
@@ -53,7 +54,10 @@ def verify_plan(tree, plan):
     coverage = collections.defaultdict(list)
     written = {}                                 # slot -> (node, kvh, branch, r)
     slots_of = collections.defaultdict(list)     # (branch, h) -> slots written for it
-    for it in items:
+    blank = check_tile_pairs(plan)
+    for i, it in enumerate(items):
+        if i in blank:
+            continue
         page_pos, npg, last_valid, leaf_lo, row0, nrows, kvh, slot_base = (int(x) for x in it)
         assert npg >= 1 and 1 <= nrows <= 128 and 0 <= kvh < H_kv
         assert row0 % g == 0, "tiles start at a multiple of g"
@@ -107,7 +111,8 @@ def verify_plan(tree, plan):
             pages = items[q, 1] if len(q) else np.zeros(0)
             assert np.all(np.diff(pages) <= 0), "queue not longest first"
         for i in wq:
-            assert len(under[int(owner[items[i][0]])]) * g > 16
+            if i not in blank:
+                assert len(under[int(owner[items[i][0]])]) * g > 16
         for i in nq:
             assert len(under[int(owner[items[i][0]])]) * g <= 16
         assert info["num_ctas"] <= max(info["num_sms"], 2)
@@ -148,6 +153,23 @@ def test_plan_covers_tree_exactly(name, mode):
         verify_plan(tree, plan)
 
 
+def test_tile_pairs_chosen_and_shaped():
+    """bf16 at head_dim 128 with most prefix tile-pages in multi-tile pieces:
+    pairs (blanks where a piece has an odd tile count); e4m3 and the
+    two-level workload (a third of its tile-pages in single-tile pieces):
+    single tiles."""
+    tree = W.pair_fixture(values=False)
+    with Plan.for_tree(tree, host_only=True) as plan:
+        assert plan.info()["tile_pairs"] == 1
+        assert len(check_tile_pairs(plan)) > 0
+        verify_plan(tree, plan)
+    for t in (W.pair_fixture(mode="fp8", values=False), W.make_config(3, values=False)):
+        with Plan.for_tree(t, host_only=True) as plan:
+            assert plan.info()["tile_pairs"] == 0
+    with Plan.for_tree(W.make_config(5, values=False), host_only=True) as plan:
+        assert plan.info()["tile_pairs"] == 1
+
+
 @pytest.mark.parametrize("idx", [4, 5])
 def test_plan_large_configs(idx):
     tree = W.make_config(idx, values=False)
@@ -160,7 +182,7 @@ def test_plan_large_configs(idx):
         assert part_bytes < 0.05 * kv_bytes, part_bytes / kv_bytes
         assert len(items) >= 152
         # pages of all items of one (kv head, first tile) sum to the unique pages
-        one = items[(items[:, 6] == 0) & (items[:, 4] == 0)]
+        one = items[(items[:, 6] == 0) & (items[:, 4] == 0) & (items[:, 5] > 0)]
         assert one[:, 1].sum() == sum(
             tree.node_page_ptr[n + 1] - tree.node_page_ptr[n]
             for n in range(tree.num_nodes) if tree.node_len[n] > 0)

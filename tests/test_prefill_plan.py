@@ -11,6 +11,7 @@ import pytest
 
 from paper_2608_24658_gb300 import _lib, build
 from paper_2608_24658_gb300 import workloads as W
+from tests.plan_cover import check_tile_pairs
 from paper_2608_24658_gb300.api import Plan, ParasonError
 
 
@@ -51,7 +52,11 @@ def verify_prefill_plan(tree, plan):
         owner[tree.node_page_ptr[n]:tree.node_page_ptr[n + 1]] = n
 
     seen = {}                                        # slot -> list of (node, token)
-    for it, k0 in zip(items, key0):
+    blank = check_tile_pairs(plan)
+    for i, (it, k0) in enumerate(zip(items, key0)):
+        if i in blank:
+            assert int(k0) == -1
+            continue
         page_pos, npg, last_valid, leaf_lo, row0, nrows, kvh, slot_base = (int(x) for x in it)
         assert 1 <= nrows <= 128 and row0 % g == 0 and 0 <= kvh < H_kv and npg >= 1
         n = int(owner[page_pos])
