@@ -1153,7 +1153,64 @@ struct TcMeta {
     int32_t rows[kTcMetaPages];      // TMA row of each page
     int32_t leaves[kTcRows];         // branch of rows [g i, g i + g)
     int32_t leavesB[kTcRows];        // pair mode: the same for the second tile
+    // per 64-token block, 4 bits a page: 16 - the valid tokens of a page
+    // that ends a node inside the item (a prefill piece over a whole path),
+    // 0 for a full page (the item's last page goes by last_valid)
+    uint16_t short_pages[kTcMetaPages / 4];
 };
+
+// causal mask: -1 when the item's rows see all of its keys
+constexpr int32_t kNoKey0 = -1;
+
+// An item's page rows into its metadata slot: the TMA row of every page, and
+// per block the code of its pages that end a node (the stream row's low 4
+// bits, which a TMA row (page * H_kv + kv head) * 16 leaves zero).
+__device__ __forceinline__ void stage_item_rows(TcMeta &m, const int32_t *src, int np, int lane) {
+    for (int p = lane; p < np; p += 32) m.rows[p] = src[p] & ~(kPageSize - 1);
+    for (int b = lane; b * 4 < np; b += 32) {
+        uint32_t code = 0;
+        for (int j = 0; j < 4 && b * 4 + j < np; ++j)
+            code |= static_cast<uint32_t>(src[b * 4 + j] & (kPageSize - 1)) << (4 * j);
+        m.short_pages[b] = static_cast<uint16_t>(code);
+    }
+}
+
+// Scores of keys in the unused part of a page that ends a node inside the
+// item become -inf (`code`: the block's short_pages entry).
+__device__ __forceinline__ void mask_short_pages(float (&x)[64], uint32_t code) {
+    int lim[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) lim[j] = kPageSize - static_cast<int>((code >> (4 * j)) & 15u);
+#pragma unroll
+    for (int q = 0; q < 64; ++q) x[q] = (q & 15) < lim[q >> 4] ? x[q] : -INFINITY;
+}
+
+// V rows of a staged block that no key stands for -- past the item's last
+// token (`valid`) or in the unused part of a page that ends a node -- may hold
+// anything (NaN included); P is 0 there but 0 * NaN is NaN, so they become
+// zeros.  `vst`: the stage's V; 128 threads, `r` this thread's index.
+__device__ __forceinline__ void zero_dead_v_rows(uint32_t vst, int valid, uint32_t code, int r) {
+    if (code == 0) {
+        const int n16 = (kTcBlockTokens - valid) * 2 * 8;     // 16-byte chunks
+        for (int q = r; q < n16; q += kTcRows) {
+            const int t = valid + q / 16, cb = (q / 8) & 1, c = q & 7;
+            asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
+                             vst + cb * kTcColBlockBytes + t * 128 + (c << 4)),
+                         "r"(0u)
+                         : "memory");
+        }
+    } else {
+        for (int q = r; q < kTcBlockTokens * 16; q += kTcRows) {
+            const int t = q / 16, cb = (q / 8) & 1, c = q & 7;
+            const int lim = kPageSize - static_cast<int>((code >> (4 * (t >> 4))) & 15u);
+            if (t >= valid || (t & 15) >= lim)
+                asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
+                                 vst + cb * kTcColBlockBytes + t * 128 + (c << 4)),
+                             "r"(0u)
+                             : "memory");
+        }
+    }
+}
 
 // barrier slots (8 bytes each) in the CTA's barrier area
 enum TcBar : int {
@@ -1285,10 +1342,9 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
                 } else {
                     if (lane == 0) {
                         m.it = it;
-                        m.key0 = a.item_key0 ? a.item_key0[id] : -1;
+                        m.key0 = a.item_key0 ? a.item_key0[id] : kNoKey0;
                     }
-                    const int32_t *src = a.stream_rows + a.item_rows[id];
-                    for (int p = lane; p < it.num_pages; p += 32) m.rows[p] = src[p];
+                    stage_item_rows(m, a.stream_rows + a.item_rows[id], it.num_pages, lane);
                     const int nbr = (it.nrows + a.group - 1) / a.group;
                     const int32_t *lv = a.dfs_leaf + it.leaf_lo + it.row0 / a.group;
                     for (int i = lane; i < nbr; i += 32) m.leaves[i] = lv[i];
@@ -1509,7 +1565,7 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
             // causal item (tree-masked prefill): the row's token, relative to
             // the item's first key, is the last key it sees
             const int key0 = meta[ms].key0;
-            const int t_rel = key0 < 0 ? (1 << 30) : (it.row0 + r) / a.group - key0;
+            const int t_rel = key0 == kNoKey0 ? (1 << 30) : (it.row0 + r) / a.group - key0;
             // e4m3 K: the kv head's scale goes into the logits
             const float sl = kF8 ? a.scale_log2 * a.k_scale[it.kv_head] : a.scale_log2;
             float m_use = -INFINITY, l = 0.f;
@@ -1537,6 +1593,8 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
 #pragma unroll
                     for (int j = 0; j < 64; ++j) x[j] = j < seen ? x[j] : -INFINITY;
                 }
+                const uint32_t code = meta[ms].short_pages[i];
+                if (code != 0) mask_short_pages(x, code);
                 // the block's max in the log2 domain (sl > 0)
                 float mr = x[0];
 #pragma unroll
@@ -1592,19 +1650,11 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
                 }
                 tc::st32(tS, pw);
                 tc::wait_st();
-                // V rows past the item's last token may hold anything (NaN
-                // included); P is 0 there but 0 * NaN is NaN, so zero them (the
-                // e4m3 converters write those rows as zeros)
-                if (!kF8 && valid < kTcBlockTokens) {
-                    const uint32_t vst = ring + (b % kTcStages) * kTcStageBytes + kTcKBytes;
-                    const int n16 = (kTcBlockTokens - valid) * 2 * 8;     // 16-byte chunks
-                    for (int q = r; q < n16; q += kTcRows) {
-                        const int t = valid + q / 16, cb = (q / 8) & 1, c = q & 7;
-                        asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
-                                         vst + cb * kTcColBlockBytes + t * 128 + (c << 4)),
-                                     "r"(0u)
-                                     : "memory");
-                    }
+                // V rows that no key stands for become zeros (the e4m3
+                // converters write rows past the last token as zeros; e4m3
+                // items never span nodes)
+                if (!kF8 && (valid < kTcBlockTokens || code != 0)) {
+                    zero_dead_v_rows(ring + (b % kTcStages) * kTcStageBytes + kTcKBytes, valid, code, r);
                     tc::fence_proxy_async_smem();
                 }
                 tc::fence_before_sync();
@@ -1925,11 +1975,10 @@ __device__ void prefix_cta_tc_pair(const KvMaps *maps, const AttnArgs &a, uint8_
                     if (lane == 0) {
                         m.it = it;
                         m.itB = itB;
-                        m.key0 = a.item_key0 ? a.item_key0[id] : -1;
-                        m.key0B = a.item_key0 ? a.item_key0[id + 1] : -1;
+                        m.key0 = a.item_key0 ? a.item_key0[id] : kNoKey0;
+                        m.key0B = a.item_key0 ? a.item_key0[id + 1] : kNoKey0;
                     }
-                    const int32_t *src = a.stream_rows + a.item_rows[id];
-                    for (int p = lane; p < it.num_pages; p += 32) m.rows[p] = src[p];
+                    stage_item_rows(m, a.stream_rows + a.item_rows[id], it.num_pages, lane);
                     const int nbr = (it.nrows + a.group - 1) / a.group;
                     const int32_t *lv = a.dfs_leaf + it.leaf_lo + it.row0 / a.group;
                     for (int i = lane; i < nbr; i += 32) m.leaves[i] = lv[i];
@@ -2174,7 +2223,7 @@ __device__ void prefix_cta_tc_pair(const KvMaps *maps, const AttnArgs &a, uint8_
                 const int nb = tc_blocks(it.num_pages);
                 const int tokens = (it.num_pages - 1) * kPageSize + it.last_valid;
                 const int key0 = t == 0 ? m.key0 : m.key0B;
-                const int t_rel = key0 < 0 ? (1 << 30) : (it.row0 + r) / a.group - key0;
+                const int t_rel = key0 == kNoKey0 ? (1 << 30) : (it.row0 + r) / a.group - key0;
                 float m_use = -INFINITY, l = 0.f;
                 for (int i = 0; i < nb; ++i) {
                     const int buf = u & 1;
@@ -2207,6 +2256,8 @@ __device__ void prefix_cta_tc_pair(const KvMaps *maps, const AttnArgs &a, uint8_
 #pragma unroll
                         for (int q = 0; q < 64; ++q) x[q] = q < seen ? x[q] : -INFINITY;
                     }
+                    const uint32_t code = m.short_pages[i];
+                    if (code != 0) mask_short_pages(x, code);
                     float mr = x[0];
 #pragma unroll
                     for (int q = 1; q + 1 < 64; q += 2) mr = dev::max3(mr, x[q], x[q + 1]);
@@ -2258,20 +2309,11 @@ __device__ void prefix_cta_tc_pair(const KvMaps *maps, const AttnArgs &a, uint8_
                     }
                     tc::st32(tS, pw);
                     tc::wait_st();
-                    // V rows past the item's last token may hold anything (NaN
-                    // included); P is 0 there but 0 * NaN is NaN, so tile A zeroes
-                    // them before its PV -- tile B's PV of the block is issued after
-                    if (t == 0 && valid < kTcBlockTokens) {
-                        const int stage = u % kTpStages;   // tile A has a block of every stage
-                        const uint32_t vst = ring + stage * kTcStageBytes + kTcKBytes;
-                        const int n16 = (kTcBlockTokens - valid) * 2 * 8;
-                        for (int q = r; q < n16; q += kTcRows) {
-                            const int tt = valid + q / 16, cb = (q / 8) & 1, c = q & 7;
-                            asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
-                                             vst + cb * kTcColBlockBytes + tt * 128 + (c << 4)),
-                                         "r"(0u)
-                                         : "memory");
-                        }
+                    // V rows that no key stands for become zeros: tile A does it
+                    // before its PV, and tile B's PV of the block is issued after
+                    // (tile A has a block of every stage)
+                    if (t == 0 && (valid < kTcBlockTokens || code != 0)) {
+                        zero_dead_v_rows(ring + (u % kTpStages) * kTcStageBytes + kTcKBytes, valid, code, r);
                         tc::fence_proxy_async_smem();
                     }
                     tc::fence_before_sync();

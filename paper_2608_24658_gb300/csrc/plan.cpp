@@ -51,6 +51,14 @@ constexpr int kWideBlockPages = 4;      // prefix pieces are whole 64-token bloc
 // 39.8 -> 39.2 us, long prefix 854.5 -> 843 us (e4m3 KV 655.4 -> 600.2
 // us), batched 2460 -> 2447 us.
 constexpr int64_t kWidePiecesPerCta = 1;
+// A prefill's queue is the whole launch, and nothing evens out the prefix
+// CTAs' ends: its piece length is the one, of a few candidates, under which
+// the queue, simulated, empties first.  An entry's start and its O cost
+// about kPieceStartPages pages; a lone tile of a pair kLoneTileShare of a
+// pair's time.
+constexpr double kPieceStartPages = 8.0;
+constexpr double kLoneTileShare = 0.6;
+constexpr int kPieceCountCandidates = 16;
 // suffix pieces: about this many per warp of the launch (at least
 // kMinPiecePages and at most kMaxPiecePages pages).  Same-box A/B against
 // 3: two-level step 79.7 -> 78.8 us, the Llama-3 shape level (its pieces
@@ -89,6 +97,56 @@ double wide_page_cost(int32_t rows, bool tensor_core_tile, bool e4m3) {
     if (tensor_core_tile) return e4m3 ? kTcPageCostE4m3 : kTcPageCost;
     const double groups = (rows + 15) / 16;
     return std::max(1.0, groups * kWideGroupPageCost);
+}
+
+// Pieces of a run of `pages` pages under the piece length `chunk`: equal
+// pieces, multiples of `align` pages except the last.  Sets the pages of
+// each piece but the last (`per`) and the piece count (`n`).
+void piece_split(int64_t pages, int64_t chunk, int64_t align, int64_t &per, int64_t &n) {
+    chunk = std::max<int64_t>(align, chunk / align * align);
+    n = (pages + chunk - 1) / chunk;
+    per = (pages + n - 1) / n;
+    per = (per + align - 1) / align * align;
+    n = (pages + per - 1) / per;
+}
+
+// Time, in pages, for `ctas` CTAs to empty a prefix queue whose (pages,
+// tiles) groups are cut into pieces of at most `chunk` pages.  The queue
+// hands its entries out longest first, the first `ctas` to the CTAs that own
+// them, each later one to the CTA that frees first.  An entry is a tile, or
+// with pairs two tiles (a lone tile at kLoneTileShare of a pair's time), and
+// costs its pages plus kPieceStartPages for its start and its O.
+double prefix_queue_time(const std::vector<std::pair<int64_t, int32_t>> &groups, int64_t chunk,
+                         int32_t ctas, bool pairs) {
+    std::vector<std::pair<int64_t, double>> entries;   // (pages, time)
+    for (const auto &g : groups) {
+        int64_t per = 0, n = 0;
+        piece_split(g.first, chunk, kWideBlockPages, per, n);
+        const int32_t full = pairs ? g.second / 2 : g.second;
+        const int32_t lone = pairs ? g.second % 2 : 0;
+        for (int64_t k = 0; k < n; ++k) {
+            const int64_t np = std::min(per, g.first - k * per);
+            for (int32_t t = 0; t < full; ++t)
+                entries.emplace_back(np, static_cast<double>(np) + kPieceStartPages);
+            for (int32_t t = 0; t < lone; ++t)
+                entries.emplace_back(np, kLoneTileShare * static_cast<double>(np) + kPieceStartPages);
+        }
+    }
+    std::stable_sort(entries.begin(), entries.end(),
+                     [](const auto &a, const auto &b) { return a.first > b.first; });
+    std::priority_queue<double, std::vector<double>, std::greater<double>> free_at;
+    double end = 0.0;
+    for (size_t e = 0; e < entries.size(); ++e) {
+        double t0 = 0.0;
+        if (e >= static_cast<size_t>(ctas)) {
+            t0 = free_at.top();
+            free_at.pop();
+        }
+        const double t1 = t0 + entries[e].second;
+        free_at.push(t1);
+        end = std::max(end, t1);
+    }
+    return end;
 }
 
 // Rows of one tile: a multiple of g (so a branch's rows never straddle two
@@ -332,7 +390,21 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         double cost_per_page;
         bool wide;
         bool causal = false;        // prefill: keys past the row's own token are masked
+        int32_t span = -1;          // bf16 prefill: its page list in `spans`
     };
+    // A bf16 prefill run reads its chunk's whole path in one list of pages:
+    // every page of every non-empty ancestor, root first, then the chunk's
+    // own pages up to the tile pair's last token.  Its pieces cross node
+    // boundaries, so that each query row has a partial per piece of its path
+    // rather than one per node.
+    struct Span {
+        std::vector<int32_t> pos;     // position in page_ids of each page
+        std::vector<int32_t> valid;   // valid tokens of each page
+        int64_t own = 0;              // pages before the chunk's own ones
+    };
+    std::vector<Span> spans;
+    std::vector<int32_t> item_span_rows;   // explicit page rows of span items, by item
+    std::vector<int64_t> item_span_off;    // their start in item_span_rows, -1: none
     std::vector<Run> runs;
     int64_t narrow_pages = 0;
     double wide_cost = 0.0;
@@ -350,6 +422,47 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
             std::vector<int32_t> path;
             for (int32_t m = n; m >= 0; m = parent[m]) path.push_back(m);
             std::reverse(path.begin(), path.end());
+            if (mode == PARASON_BF16 && cfg->head_dim == 128) {
+                // one list per tile pair, up to the pair's last token; a pair's
+                // first tile reads the few pages past its own last token masked
+                const int64_t pair_rows = 2 * static_cast<int64_t>(rt);
+                for (int64_t p0 = 0; p0 < R; p0 += pair_rows) {
+                    const int64_t tb = std::min<int64_t>(R, p0 + pair_rows) / g;   // tokens [.., tb)
+                    Span sp;
+                    for (int32_t m : path) {
+                        if (node_len[m] == 0) continue;
+                        const int64_t P = node_page_ptr[m + 1] - node_page_ptr[m];
+                        const int64_t use = m == n ? (tb + parason::kPageSize - 1) / parason::kPageSize : P;
+                        if (m == n) sp.own = static_cast<int64_t>(sp.pos.size());
+                        for (int64_t k = 0; k < use; ++k) {
+                            sp.pos.push_back(node_page_ptr[m] + static_cast<int32_t>(k));
+                            sp.valid.push_back(k == P - 1 ? node_len[m] - static_cast<int32_t>(P - 1) *
+                                                                              parason::kPageSize
+                                                          : parason::kPageSize);
+                        }
+                    }
+                    spans.push_back(std::move(sp));
+                    const int32_t si = static_cast<int32_t>(spans.size()) - 1;
+                    for (int32_t j = 0; j < H_kv; ++j)
+                        for (int64_t r0 = p0; r0 < std::min<int64_t>(R, p0 + pair_rows); r0 += rt) {
+                            Run run;
+                            run.node = n;
+                            run.head = j;
+                            run.row0 = static_cast<int32_t>(r0);
+                            run.nrows = static_cast<int32_t>(std::min<int64_t>(rt, R - r0));
+                            run.pages = static_cast<int64_t>(spans[si].pos.size());
+                            run.node_pages = run.pages;
+                            run.causal = true;
+                            run.span = si;
+                            run.leaf_lo = qbase[c];
+                            run.wide = true;
+                            run.cost_per_page = wide_page_cost(run.nrows, true, false);
+                            wide_cost += run.cost_per_page * static_cast<double>(run.pages);
+                            runs.push_back(run);
+                        }
+                }
+                continue;
+            }
             // (kv head, node, tile): the tiles of one ancestor read the same
             // pages and sit next to each other for the piece interleaving
             for (int32_t j = 0; j < H_kv; ++j)
@@ -491,11 +604,34 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                     bool blank = false) -> bool {
         WorkItem it;
         const int64_t P = run.node_pages;
-        it.page_pos = node_page_ptr[run.node] + static_cast<int32_t>(pg0);
         it.num_pages = static_cast<int32_t>(np);
-        it.last_valid = (pg0 + np == P)
-                            ? node_len[run.node] - static_cast<int32_t>(P - 1) * parason::kPageSize
-                            : parason::kPageSize;
+        int32_t k0 = run.causal && !blank ? static_cast<int32_t>(pg0 * parason::kPageSize) : -1;
+        if (run.span >= 0) {
+            // the item's page rows; a page that ends a node inside the item
+            // carries 16 - its valid tokens in the row's low bits
+            const Span &sp = spans[run.span];
+            it.page_pos = sp.pos[pg0];
+            it.last_valid = sp.valid[pg0 + np - 1];
+            item_span_off.push_back(static_cast<int64_t>(item_span_rows.size()));
+            for (int64_t k = pg0; k < pg0 + np; ++k) {
+                int32_t row = (page_ids[sp.pos[k]] * H_kv + run.head) * parason::kPageSize;
+                if (k < pg0 + np - 1) row |= parason::kPageSize - sp.valid[k];
+                item_span_rows.push_back(row);
+            }
+            // the chunk's own keys start at stream position 16 (own - pg0)
+            // when the item holds the first of them, at own token 16 (pg0 -
+            // own) when it starts among them; none when it holds none
+            k0 = blank || pg0 + np <= sp.own
+                     ? -1
+                     : (pg0 < sp.own ? -static_cast<int32_t>((sp.own - pg0) * parason::kPageSize)
+                                     : static_cast<int32_t>((pg0 - sp.own) * parason::kPageSize));
+        } else {
+            it.page_pos = node_page_ptr[run.node] + static_cast<int32_t>(pg0);
+            it.last_valid = (pg0 + np == P)
+                                ? node_len[run.node] - static_cast<int32_t>(P - 1) * parason::kPageSize
+                                : parason::kPageSize;
+            item_span_off.push_back(-1);
+        }
         it.leaf_lo = static_cast<int32_t>(run.leaf_lo);
         it.row0 = blank ? 0 : run.row0;
         it.nrows = blank ? 0 : run.nrows;
@@ -506,7 +642,7 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         const int32_t id = static_cast<int32_t>(p->items.size());
         p->items.push_back(it);
         if (queued) (run.wide ? wide_q : narrow_q).emplace_back(np, id);
-        key0.push_back(run.causal && !blank ? static_cast<int32_t>(pg0 * parason::kPageSize) : -1);
+        key0.push_back(k0);
         if (!prefill && !blank && pg0 + np == P && leaf_of_node[run.node] >= 0)
             tails.emplace_back(leaf_of_node[run.node], id);
         return true;
@@ -532,11 +668,35 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                               static_cast<int64_t>(static_cast<double>(narrow_pages) /
                                                    (kNarrowPiecesPerWarp * std::max<int64_t>(1, total_warps)))));
         p->narrow_chunk = narrow_chunk;
-        const int64_t wide_chunk = std::min<int64_t>(
+        int64_t wide_chunk = std::min<int64_t>(
             kMaxTileItemPages,
             std::max<int64_t>(kWideBlockPages,
                               wide_units / std::max<int64_t>(1, static_cast<int64_t>(n_wide) *
                                                                     kWidePiecesPerCta)));
+        if (prefill && n_wide > 0) {
+            // candidates: the longest run cut into n pieces, n from the
+            // fewest the tile allows up
+            std::vector<std::pair<int64_t, int32_t>> groups;   // (pages, tiles)
+            int64_t longest = 0;
+            for (size_t i = 0; i < runs.size();) {
+                const size_t j = group_end(i);
+                groups.emplace_back(runs[i].pages, static_cast<int32_t>(j - i));
+                longest = std::max(longest, runs[i].pages);
+                i = j;
+            }
+            double best = prefix_queue_time(groups, wide_chunk, n_wide, p->tc_pairs);
+            const int64_t n0 = (longest + kMaxTileItemPages - 1) / kMaxTileItemPages;
+            for (int64_t n = n0; n < n0 + kPieceCountCandidates; ++n) {
+                const int64_t c = std::min<int64_t>(
+                    kMaxTileItemPages,
+                    std::max<int64_t>(kWideBlockPages, (longest + n - 1) / n));
+                const double tq = prefix_queue_time(groups, c, n_wide, p->tc_pairs);
+                if (tq < best) {
+                    best = tq;
+                    wide_chunk = c;
+                }
+            }
+        }
         // The row tiles of one (node, kv head) read the same pages: their
         // pieces are emitted piece by piece across the tiles, so that the
         // queue hands out the copies of one page range together and all but
@@ -546,11 +706,8 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
             const Run &r = runs[i];
             const bool pairs = r.wide && p->tc_pairs;
             const int64_t align = r.wide ? kWideBlockPages : 1;
-            int64_t chunk = r.wide ? wide_chunk : narrow_chunk;
-            chunk = std::max<int64_t>(align, chunk / align * align);
-            const int64_t n = (r.pages + chunk - 1) / chunk;
-            int64_t per = (r.pages + n - 1) / n;
-            per = (per + align - 1) / align * align;
+            int64_t per = 0, n = 0;
+            piece_split(r.pages, r.wide ? wide_chunk : narrow_chunk, align, per, n);
             for (int64_t pg = 0; pg < r.pages; pg += per) {
                 const int64_t np = std::min(per, r.pages - pg);
                 for (size_t t = i; t < j; ++t) {
@@ -606,6 +763,9 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         std::vector<int32_t> key0_sorted(key0.size());
         for (size_t id = 0; id < key0.size(); ++id) key0_sorted[new_id[id]] = key0[id];
         key0.swap(key0_sorted);
+        std::vector<int64_t> span_sorted(item_span_off.size());
+        for (size_t id = 0; id < item_span_off.size(); ++id) span_sorted[new_id[id]] = item_span_off[id];
+        item_span_off.swap(span_sorted);
         for (size_t k = 0; k < p->wide_queue.size(); ++k) p->wide_queue[k] = static_cast<int32_t>(k);
         for (size_t k = 0; k < p->narrow_queue.size(); ++k)
             p->narrow_queue[k] = static_cast<int32_t>(p->wide_queue.size() + k);
@@ -639,9 +799,13 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     p->stream_rows.clear();
     for (size_t i = 0; i < p->items.size(); ++i) {
         const WorkItem &it = p->items[i];
-        for (int32_t pg = 0; pg < it.num_pages; ++pg)
-            p->stream_rows.push_back((page_ids[it.page_pos + pg] * H_kv + it.kv_head) *
-                                     parason::kPageSize);
+        if (item_span_off[i] >= 0)
+            p->stream_rows.insert(p->stream_rows.end(), item_span_rows.begin() + item_span_off[i],
+                                  item_span_rows.begin() + item_span_off[i] + it.num_pages);
+        else
+            for (int32_t pg = 0; pg < it.num_pages; ++pg)
+                p->stream_rows.push_back((page_ids[it.page_pos + pg] * H_kv + it.kv_head) *
+                                         parason::kPageSize);
         if (mode != PARASON_FP32 && is_tail[i])
             p->stream_rows.insert(p->stream_rows.end(),
                                   std::min(kAppendSlackMax, std::max(kAppendSlackMin, it.num_pages / 2)),

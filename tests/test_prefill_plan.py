@@ -29,6 +29,30 @@ def ancestors(tree, n):
     return out
 
 
+def item_keys(tree, it, rows):
+    """(node, token) of every stream position of an item (None where a page
+    ends a node or the item's last page ends), read from its page rows: row
+    (page * H_kv + kv head) * 16, plus 16 - valid tokens in the low bits of a
+    page that ends a node inside the item."""
+    H = tree.num_kv_heads
+    npg, last_valid, kvh = int(it[1]), int(it[2]), int(it[6])
+    where = {int(pg): i for i, pg in enumerate(tree.page_ids)}
+    keys = []
+    for k, row in enumerate(int(x) for x in rows):
+        short, base = row & 15, row >> 4
+        assert base % H == kvh
+        assert k < npg - 1 or short == 0, "the last page goes by last_valid"
+        valid = last_valid if k == npg - 1 else 16 - short
+        pos = where[base // H]
+        n = int(np.searchsorted(tree.node_page_ptr, pos, side="right")) - 1
+        idx = pos - int(tree.node_page_ptr[n])
+        P = int(tree.node_page_ptr[n + 1] - tree.node_page_ptr[n])
+        node_valid = int(tree.node_len[n]) - 16 * (P - 1) if idx == P - 1 else 16
+        assert valid == node_valid, "a page's valid tokens are the node's"
+        keys.extend((n, 16 * idx + x) if x < valid else None for x in range(16))
+    return keys
+
+
 def verify_prefill_plan(tree, plan):
     g, H_kv = tree.group, tree.num_kv_heads
     chunks = [int(c) for c in tree.leaf_node]
@@ -44,37 +68,32 @@ def verify_prefill_plan(tree, plan):
     ment = plan.export(_lib.TABLE_MERGE)
     wq = plan.export(_lib.TABLE_WIDE_QUEUE)
     nq = plan.export(_lib.TABLE_NARROW_QUEUE)
+    irows = plan.export(_lib.TABLE_ITEM_ROWS)
+    srows = plan.export(_lib.TABLE_STREAM_ROWS)
     assert dfs.tolist() == list(range(Q))
     assert len(key0) == len(items)
     assert len(nq) == 0 and wq.tolist() == list(range(len(items)))    # all on the tcgen05 tile
-    owner = np.full(int(tree.node_page_ptr[-1]), -1, dtype=np.int64)
-    for n in range(tree.num_nodes):
-        owner[tree.node_page_ptr[n]:tree.node_page_ptr[n + 1]] = n
 
-    seen = {}                                        # slot -> list of (node, token)
     blank = check_tile_pairs(plan)
+    seen = {}                                        # slot -> (query, q head, visible keys)
     for i, (it, k0) in enumerate(zip(items, key0)):
         if i in blank:
             assert int(k0) == -1
             continue
         page_pos, npg, last_valid, leaf_lo, row0, nrows, kvh, slot_base = (int(x) for x in it)
         assert 1 <= nrows <= 128 and row0 % g == 0 and 0 <= kvh < H_kv and npg >= 1
-        n = int(owner[page_pos])
-        assert owner[page_pos + npg - 1] == n
-        first = page_pos - int(tree.node_page_ptr[n])
-        P = int(tree.node_page_ptr[n + 1] - tree.node_page_ptr[n])
-        ends = first + npg == P
-        assert last_valid == (int(tree.node_len[n]) - 16 * (P - 1) if ends else 16)
         c = int(np.searchsorted(qbase, leaf_lo, side="right")) - 1
         assert qbase[c] == leaf_lo, "an item's rows start at its chunk's first query"
-        own = n == chunks[c]
-        assert n in ancestors(tree, chunks[c]) or own
-        assert int(k0) == (16 * first if own else -1)
-        tokens = list(range(16 * first, 16 * (first + npg - 1) + last_valid))
+        keys = item_keys(tree, it, srows[irows[i]:irows[i] + npg])
+        path = set(ancestors(tree, chunks[c])) | {chunks[c]}
+        assert all(k is None or k[0] in path for k in keys), "a key off the chunk's path"
         for row in range(row0, row0 + nrows):
             t = row // g
             assert t < lens[c]
-            vis = [(n, x) for x in tokens if not own or x <= t]
+            vis = [k for p, k in enumerate(keys)
+                   if k is not None and (int(k0) == -1 or p <= t - int(k0))]
+            # the causal rule: the chunk's own keys up to the row's token only
+            assert all(k[0] != chunks[c] or k[1] <= t for k in vis), (i, row)
             slot = slot_base + row - row0
             assert slot not in seen, "partial slot written twice"
             seen[slot] = (int(leaf_lo) + t, kvh * g + row % g, vis)
@@ -175,3 +194,24 @@ def test_prefill_plan_deterministic():
                                                   _lib.TABLE_MERGE_RANGES, _lib.TABLE_MERGE)])
     for a, b in zip(*tabs):
         assert np.array_equal(a, b)
+
+
+def test_bf16_pieces_span_the_path():
+    """With bf16 KV a piece reads across node boundaries along the chunk's
+    path, so a query row has fewer partials than its path has nodes (one each
+    on one SM, where every path fits one piece); e4m3 pieces stay within a
+    node."""
+    tree = CASES["join"]()
+    with Plan.for_prefill(tree, host_only=True, num_sms=1) as plan:
+        info = verify_prefill_plan(tree, plan)
+        mrng = plan.export(_lib.TABLE_MERGE_RANGES)
+        assert (mrng[:, 1] - mrng[:, 0] == 1).all()
+        srows = plan.export(_lib.TABLE_STREAM_ROWS)
+        assert (srows & 15).any(), "a page that ends a node inside a piece"
+    t8 = W.build_prefill("j8", tree.parent, tree.node_len, tree.leaf_node, num_q_heads=8,
+                         num_kv_heads=2, head_dim=128, mode="fp8", values=False)
+    with Plan.for_prefill(t8, host_only=True, num_sms=1) as plan:
+        verify_prefill_plan(t8, plan)
+        assert not (plan.export(_lib.TABLE_STREAM_ROWS) & 15).any()
+        mrng = plan.export(_lib.TABLE_MERGE_RANGES)
+        assert (mrng[:, 1] - mrng[:, 0] > 1).any()
