@@ -472,11 +472,20 @@ parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info)
  *                            rows in the stream (an item's rows are the first
  *                            page-count entries from there)
  *   PARASON_TABLE_STREAM_ROWS int32 [num_stream_rows]: the TMA row
- *                            (page * H_kv + kv head) * 16 of every item page
+ *                            (page * H_kv + kv head) * 16 of every item page;
+ *                            in a bf16 prefill piece over several nodes of a
+ *                            path, a page that ends a node before the item's
+ *                            last page adds 16 - its valid tokens (1..15)
  *   PARASON_TABLE_ITEM_KEY0  int32 [num_items] (prefill plans; empty for
- *                            decode plans): for an item over its chunk's own
- *                            node, the index in that node of its first key
- *                            (the causal mask's origin), else -1
+ *                            decode plans): the causal mask's origin.  Query
+ *                            token t of the chunk sees the key at position p
+ *                            of the item's page stream (16 per page) iff
+ *                            p <= t - key0: key0 is the own-node index of
+ *                            the item's first key when the item starts in
+ *                            the chunk's own node, minus the stream position
+ *                            of the own node's first key when the item
+ *                            reaches it from an ancestor, and -1 (no mask)
+ *                            for an item with no key of the chunk's node
  *   PARASON_TABLE_SHARD_BRANCHES int32 [num_leaves]: the global index of
  *                            each of the plan's branches (parason_attn_plan_
  *                            shard); b for a plan that is not a shard
