@@ -475,7 +475,10 @@ parason_status parason_plan_get_info(parason_plan plan, parason_plan_info *info)
  *                            (page * H_kv + kv head) * 16 of every item page;
  *                            in a bf16 prefill piece over several nodes of a
  *                            path, a page that ends a node before the item's
- *                            last page adds 16 - its valid tokens (1..15)
+ *                            last page adds 16 - its valid tokens (1..15),
+ *                            and is followed up to the next 4-page block by
+ *                            padding: the row num_physical_pages * H_kv * 16,
+ *                            past the pool, which reads as zeros
  *   PARASON_TABLE_ITEM_KEY0  int32 [num_items] (prefill plans; empty for
  *                            decode plans): the causal mask's origin.  Query
  *                            token t of the chunk sees the key at position p

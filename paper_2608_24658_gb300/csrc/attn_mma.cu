@@ -1153,62 +1153,38 @@ struct TcMeta {
     int32_t rows[kTcMetaPages];      // TMA row of each page
     int32_t leaves[kTcRows];         // branch of rows [g i, g i + g)
     int32_t leavesB[kTcRows];        // pair mode: the same for the second tile
-    // per 64-token block, 4 bits a page: 16 - the valid tokens of a page
-    // that ends a node inside the item (a prefill piece over a whole path),
-    // 0 for a full page (the item's last page goes by last_valid)
-    uint16_t short_pages[kTcMetaPages / 4];
+    // leading valid tokens of each 64-token block (64 but where a node ends
+    // inside the item: a prefill piece over a path pads each node that ends
+    // inside a page with zero-filled pages up to the next block); the item's
+    // last block also goes by last_valid
+    uint8_t block_valid[kTcMetaPages / 4];
 };
 
 // causal mask: -1 when the item's rows see all of its keys
 constexpr int32_t kNoKey0 = -1;
 
-// An item's page rows into its metadata slot: the TMA row of every page, and
-// per block the code of its pages that end a node (the stream row's low 4
-// bits, which a TMA row (page * H_kv + kv head) * 16 leaves zero).
-__device__ __forceinline__ void stage_item_rows(TcMeta &m, const int32_t *src, int np, int lane) {
-    for (int p = lane; p < np; p += 32) m.rows[p] = src[p] & ~(kPageSize - 1);
+// An item's page rows into its metadata slot: the TMA row of every page
+// (padding pages carry the first row past the pool, which TMA fills with
+// zeros), and the leading valid tokens of every block, from the low 4 bits
+// of the stream rows (16 - the valid tokens of a page that ends a node;
+// a TMA row (page * H_kv + kv head) * 16 leaves them zero).
+__device__ __forceinline__ void stage_item_rows(TcMeta &m, const int32_t *src, int np, int kv_rows,
+                                                int lane) {
+    // lane b takes block b: its 4 rows are loaded before any is looked at
     for (int b = lane; b * 4 < np; b += 32) {
-        uint32_t code = 0;
-        for (int j = 0; j < 4 && b * 4 + j < np; ++j)
-            code |= static_cast<uint32_t>(src[b * 4 + j] & (kPageSize - 1)) << (4 * j);
-        m.short_pages[b] = static_cast<uint16_t>(code);
-    }
-}
-
-// Scores of keys in the unused part of a page that ends a node inside the
-// item become -inf (`code`: the block's short_pages entry).
-__device__ __forceinline__ void mask_short_pages(float (&x)[64], uint32_t code) {
-    int lim[4];
+        int32_t row[4];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) lim[j] = kPageSize - static_cast<int>((code >> (4 * j)) & 15u);
+        for (int j = 0; j < 4; ++j) row[j] = b * 4 + j < np ? src[b * 4 + j] : kv_rows;
+        int v = 0;
+        bool open = true;                                  // no node has ended in the block yet
 #pragma unroll
-    for (int q = 0; q < 64; ++q) x[q] = (q & 15) < lim[q >> 4] ? x[q] : -INFINITY;
-}
-
-// V rows of a staged block that no key stands for -- past the item's last
-// token (`valid`) or in the unused part of a page that ends a node -- may hold
-// anything (NaN included); P is 0 there but 0 * NaN is NaN, so they become
-// zeros.  `vst`: the stage's V; 128 threads, `r` this thread's index.
-__device__ __forceinline__ void zero_dead_v_rows(uint32_t vst, int valid, uint32_t code, int r) {
-    if (code == 0) {
-        const int n16 = (kTcBlockTokens - valid) * 2 * 8;     // 16-byte chunks
-        for (int q = r; q < n16; q += kTcRows) {
-            const int t = valid + q / 16, cb = (q / 8) & 1, c = q & 7;
-            asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
-                             vst + cb * kTcColBlockBytes + t * 128 + (c << 4)),
-                         "r"(0u)
-                         : "memory");
+        for (int j = 0; j < 4; ++j) {
+            const int low = row[j] & (kPageSize - 1);
+            if (open && row[j] < kv_rows) v += kPageSize - low;
+            open = open && row[j] < kv_rows && low == 0;   // padding, or a node's last page
+            if (b * 4 + j < np) m.rows[b * 4 + j] = row[j] & ~(kPageSize - 1);
         }
-    } else {
-        for (int q = r; q < kTcBlockTokens * 16; q += kTcRows) {
-            const int t = q / 16, cb = (q / 8) & 1, c = q & 7;
-            const int lim = kPageSize - static_cast<int>((code >> (4 * (t >> 4))) & 15u);
-            if (t >= valid || (t & 15) >= lim)
-                asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
-                                 vst + cb * kTcColBlockBytes + t * 128 + (c << 4)),
-                             "r"(0u)
-                             : "memory");
-        }
+        m.block_valid[b] = static_cast<uint8_t>(v);
     }
 }
 
@@ -1344,7 +1320,7 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
                         m.it = it;
                         m.key0 = a.item_key0 ? a.item_key0[id] : kNoKey0;
                     }
-                    stage_item_rows(m, a.stream_rows + a.item_rows[id], it.num_pages, lane);
+                    stage_item_rows(m, a.stream_rows + a.item_rows[id], it.num_pages, a.kv_rows, lane);
                     const int nbr = (it.nrows + a.group - 1) / a.group;
                     const int32_t *lv = a.dfs_leaf + it.leaf_lo + it.row0 / a.group;
                     for (int i = lane; i < nbr; i += 32) m.leaves[i] = lv[i];
@@ -1572,7 +1548,7 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
             bool ok = true;
             for (int i = 0; i < nb; ++i) {
                 const int b = blk + i;
-                const int valid = min(kTcBlockTokens, tokens - i * kTcBlockTokens);
+                const int valid = min(static_cast<int>(meta[ms].block_valid[i]), tokens - i * kTcBlockTokens);
                 const int seen = min(valid, t_rel - i * kTcBlockTokens + 1);   // keys the row sees
                 const uint32_t tS = lane_base + kTmemS + 64u * (b & 1);
                 if (!tc_warp_wait(bar(kBarSFull + (b & 1)), (b >> 1) & 1, limit, abort_flag, lane)) {
@@ -1593,8 +1569,6 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
 #pragma unroll
                     for (int j = 0; j < 64; ++j) x[j] = j < seen ? x[j] : -INFINITY;
                 }
-                const uint32_t code = meta[ms].short_pages[i];
-                if (code != 0) mask_short_pages(x, code);
                 // the block's max in the log2 domain (sl > 0)
                 float mr = x[0];
 #pragma unroll
@@ -1650,11 +1624,19 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
                 }
                 tc::st32(tS, pw);
                 tc::wait_st();
-                // V rows that no key stands for become zeros (the e4m3
-                // converters write rows past the last token as zeros; e4m3
-                // items never span nodes)
-                if (!kF8 && (valid < kTcBlockTokens || code != 0)) {
-                    zero_dead_v_rows(ring + (b % kTcStages) * kTcStageBytes + kTcKBytes, valid, code, r);
+                // V rows past the block's valid tokens may hold anything (NaN
+                // included); P is 0 there but 0 * NaN is NaN, so zero them (the
+                // e4m3 converters write those rows as zeros)
+                if (!kF8 && valid < kTcBlockTokens) {
+                    const uint32_t vst = ring + (b % kTcStages) * kTcStageBytes + kTcKBytes;
+                    const int n16 = (kTcBlockTokens - valid) * 2 * 8;     // 16-byte chunks
+                    for (int q = r; q < n16; q += kTcRows) {
+                        const int t = valid + q / 16, cb = (q / 8) & 1, c = q & 7;
+                        asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
+                                         vst + cb * kTcColBlockBytes + t * 128 + (c << 4)),
+                                     "r"(0u)
+                                     : "memory");
+                    }
                     tc::fence_proxy_async_smem();
                 }
                 tc::fence_before_sync();
@@ -1978,7 +1960,7 @@ __device__ void prefix_cta_tc_pair(const KvMaps *maps, const AttnArgs &a, uint8_
                         m.key0 = a.item_key0 ? a.item_key0[id] : kNoKey0;
                         m.key0B = a.item_key0 ? a.item_key0[id + 1] : kNoKey0;
                     }
-                    stage_item_rows(m, a.stream_rows + a.item_rows[id], it.num_pages, lane);
+                    stage_item_rows(m, a.stream_rows + a.item_rows[id], it.num_pages, a.kv_rows, lane);
                     const int nbr = (it.nrows + a.group - 1) / a.group;
                     const int32_t *lv = a.dfs_leaf + it.leaf_lo + it.row0 / a.group;
                     for (int i = lane; i < nbr; i += 32) m.leaves[i] = lv[i];
@@ -2228,7 +2210,7 @@ __device__ void prefix_cta_tc_pair(const KvMaps *maps, const AttnArgs &a, uint8_
                 for (int i = 0; i < nb; ++i) {
                     const int buf = u & 1;
                     const uint32_t tS = lane_base + kTmemS + 128u * t + 64u * buf;
-                    const int valid = min(kTcBlockTokens, tokens - i * kTcBlockTokens);
+                    const int valid = min(static_cast<int>(m.block_valid[i]), tokens - i * kTcBlockTokens);
                     const int seen = min(valid, t_rel - i * kTcBlockTokens + 1);
                     if (!tc_warp_wait(bar(kPbSFull + 2 * t + buf), (u >> 1) & 1, limit, abort_flag, lane)) {
                         ok = false;
@@ -2256,8 +2238,6 @@ __device__ void prefix_cta_tc_pair(const KvMaps *maps, const AttnArgs &a, uint8_
 #pragma unroll
                         for (int q = 0; q < 64; ++q) x[q] = q < seen ? x[q] : -INFINITY;
                     }
-                    const uint32_t code = m.short_pages[i];
-                    if (code != 0) mask_short_pages(x, code);
                     float mr = x[0];
 #pragma unroll
                     for (int q = 1; q + 1 < 64; q += 2) mr = dev::max3(mr, x[q], x[q + 1]);
@@ -2309,11 +2289,20 @@ __device__ void prefix_cta_tc_pair(const KvMaps *maps, const AttnArgs &a, uint8_
                     }
                     tc::st32(tS, pw);
                     tc::wait_st();
-                    // V rows that no key stands for become zeros: tile A does it
-                    // before its PV, and tile B's PV of the block is issued after
-                    // (tile A has a block of every stage)
-                    if (t == 0 && (valid < kTcBlockTokens || code != 0)) {
-                        zero_dead_v_rows(ring + (u % kTpStages) * kTcStageBytes + kTcKBytes, valid, code, r);
+                    // V rows past the block's valid tokens may hold anything (NaN
+                    // included); P is 0 there but 0 * NaN is NaN, so tile A zeroes
+                    // them before its PV -- tile B's PV of the block is issued after
+                    if (t == 0 && valid < kTcBlockTokens) {
+                        const int stage = u % kTpStages;   // tile A has a block of every stage
+                        const uint32_t vst = ring + stage * kTcStageBytes + kTcKBytes;
+                        const int n16 = (kTcBlockTokens - valid) * 2 * 8;
+                        for (int q = r; q < n16; q += kTcRows) {
+                            const int tt = valid + q / 16, cb = (q / 8) & 1, c = q & 7;
+                            asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
+                                             vst + cb * kTcColBlockBytes + tt * 128 + (c << 4)),
+                                         "r"(0u)
+                                         : "memory");
+                        }
                         tc::fence_proxy_async_smem();
                     }
                     tc::fence_before_sync();

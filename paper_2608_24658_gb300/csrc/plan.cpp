@@ -54,9 +54,11 @@ constexpr int64_t kWidePiecesPerCta = 1;
 // A prefill's queue is the whole launch, and nothing evens out the prefix
 // CTAs' ends: its piece length is the one, of a few candidates, under which
 // the queue, simulated, empties first.  An entry's start and its O cost
-// about kPieceStartPages pages; a lone tile of a pair kLoneTileShare of a
-// pair's time.
-constexpr double kPieceStartPages = 8.0;
+// about kPieceStartPages pages (join prefill, 8 -> 16 pieces per path: the
+// kernel went from 606 to 672 us for 1024 more pairs on 152 CTAs, about 38
+// pages of a pair each); a lone tile of a pair kLoneTileShare of a pair's
+// time.
+constexpr double kPieceStartPages = 32.0;
 constexpr double kLoneTileShare = 0.6;
 constexpr int kPieceCountCandidates = 16;
 // suffix pieces: about this many per warp of the launch (at least
@@ -396,12 +398,15 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     // every page of every non-empty ancestor, root first, then the chunk's
     // own pages up to the tile pair's last token.  Its pieces cross node
     // boundaries, so that each query row has a partial per piece of its path
-    // rather than one per node.
+    // rather than one per node.  An ancestor that ends inside a page is
+    // followed by padding pages (zero-filled by TMA) up to the next 64-token
+    // block, so that the keys no token stands for always end a block.
     struct Span {
-        std::vector<int32_t> pos;     // position in page_ids of each page
+        std::vector<int32_t> pos;     // position in page_ids of each page, -1: padding
         std::vector<int32_t> valid;   // valid tokens of each page
         int64_t own = 0;              // pages before the chunk's own ones
     };
+    const int32_t pad_row = static_cast<int32_t>(num_phys * H_kv * parason::kPageSize);
     std::vector<Span> spans;
     std::vector<int32_t> item_span_rows;   // explicit page rows of span items, by item
     std::vector<int64_t> item_span_off;    // their start in item_span_rows, -1: none
@@ -439,6 +444,11 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                             sp.valid.push_back(k == P - 1 ? node_len[m] - static_cast<int32_t>(P - 1) *
                                                                               parason::kPageSize
                                                           : parason::kPageSize);
+                        }
+                        while (m != n && sp.valid.back() < parason::kPageSize &&
+                               sp.pos.size() % kWideBlockPages != 0) {
+                            sp.pos.push_back(-1);
+                            sp.valid.push_back(0);
                         }
                     }
                     spans.push_back(std::move(sp));
@@ -604,6 +614,9 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                     bool blank = false) -> bool {
         WorkItem it;
         const int64_t P = run.node_pages;
+        // a span piece ends at its last page with keys, not in padding
+        if (run.span >= 0)
+            while (np > 1 && spans[run.span].pos[pg0 + np - 1] < 0) --np;
         it.num_pages = static_cast<int32_t>(np);
         int32_t k0 = run.causal && !blank ? static_cast<int32_t>(pg0 * parason::kPageSize) : -1;
         if (run.span >= 0) {
@@ -614,8 +627,11 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
             it.last_valid = sp.valid[pg0 + np - 1];
             item_span_off.push_back(static_cast<int64_t>(item_span_rows.size()));
             for (int64_t k = pg0; k < pg0 + np; ++k) {
-                int32_t row = (page_ids[sp.pos[k]] * H_kv + run.head) * parason::kPageSize;
-                if (k < pg0 + np - 1) row |= parason::kPageSize - sp.valid[k];
+                int32_t row = pad_row;
+                if (sp.pos[k] >= 0) {
+                    row = (page_ids[sp.pos[k]] * H_kv + run.head) * parason::kPageSize;
+                    if (k < pg0 + np - 1) row |= parason::kPageSize - sp.valid[k];
+                }
                 item_span_rows.push_back(row);
             }
             // the chunk's own keys start at stream position 16 (own - pg0)

@@ -31,14 +31,22 @@ def ancestors(tree, n):
 
 def item_keys(tree, it, rows):
     """(node, token) of every stream position of an item (None where a page
-    ends a node or the item's last page ends), read from its page rows: row
-    (page * H_kv + kv head) * 16, plus 16 - valid tokens in the low bits of a
-    page that ends a node inside the item."""
+    ends a node or the item's last page ends, and in padding), read from its
+    page rows: row (page * H_kv + kv head) * 16, plus 16 - valid tokens in the
+    low bits of a page that ends a node inside the item; padding pages carry
+    the first row past the pool and only follow a page that ends a node, up to
+    the next 64-token block."""
     H = tree.num_kv_heads
     npg, last_valid, kvh = int(it[1]), int(it[2]), int(it[6])
     where = {int(pg): i for i, pg in enumerate(tree.page_ids)}
+    pad_row = tree.num_physical_pages * H * 16
     keys = []
     for k, row in enumerate(int(x) for x in rows):
+        if row == pad_row:
+            assert 0 < k < npg - 1 and k % 4 != 0, "padding ends a block, never an item"
+            assert keys[16 * k - 1] is None, "padding follows a page that ends a node"
+            keys.extend([None] * 16)
+            continue
         short, base = row & 15, row >> 4
         assert base % H == kvh
         assert k < npg - 1 or short == 0, "the last page goes by last_valid"
@@ -208,6 +216,7 @@ def test_bf16_pieces_span_the_path():
         assert (mrng[:, 1] - mrng[:, 0] == 1).all()
         srows = plan.export(_lib.TABLE_STREAM_ROWS)
         assert (srows & 15).any(), "a page that ends a node inside a piece"
+        assert (srows == tree.num_physical_pages * tree.num_kv_heads * 16).any(), "padding"
     t8 = W.build_prefill("j8", tree.parent, tree.node_len, tree.leaf_node, num_q_heads=8,
                          num_kv_heads=2, head_dim=128, mode="fp8", values=False)
     with Plan.for_prefill(t8, host_only=True, num_sms=1) as plan:
