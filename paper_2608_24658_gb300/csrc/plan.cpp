@@ -61,6 +61,7 @@ constexpr int64_t kWidePiecesPerCta = 1;
 constexpr double kPieceStartPages = 32.0;
 constexpr double kLoneTileShare = 0.6;
 constexpr int kPieceCountCandidates = 16;
+constexpr int64_t kPieceLengthSteps = 16;   // lengths tried per piece count, 4 pages apart
 // suffix pieces: about this many per warp of the launch (at least
 // kMinPiecePages and at most kMaxPiecePages pages).  Same-box A/B against
 // 3: two-level step 79.7 -> 78.8 us, the Llama-3 shape level (its pieces
@@ -691,25 +692,30 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                                                                     kWidePiecesPerCta)));
         if (prefill && n_wide > 0) {
             // candidates: the longest run cut into n pieces, n from the
-            // fewest the tile allows up
+            // fewest the tile allows up, and the lengths between that and
+            // the shortest run cut into n pieces (which give the longer runs
+            // n + 1 pieces and the shorter ones n)
             std::vector<std::pair<int64_t, int32_t>> groups;   // (pages, tiles)
-            int64_t longest = 0;
+            int64_t longest = 0, shortest = INT64_MAX;
             for (size_t i = 0; i < runs.size();) {
                 const size_t j = group_end(i);
                 groups.emplace_back(runs[i].pages, static_cast<int32_t>(j - i));
                 longest = std::max(longest, runs[i].pages);
+                shortest = std::min(shortest, runs[i].pages);
                 i = j;
             }
             double best = prefix_queue_time(groups, wide_chunk, n_wide, p->tc_pairs);
             const int64_t n0 = (longest + kMaxTileItemPages - 1) / kMaxTileItemPages;
             for (int64_t n = n0; n < n0 + kPieceCountCandidates; ++n) {
-                const int64_t c = std::min<int64_t>(
-                    kMaxTileItemPages,
-                    std::max<int64_t>(kWideBlockPages, (longest + n - 1) / n));
-                const double tq = prefix_queue_time(groups, c, n_wide, p->tc_pairs);
-                if (tq < best) {
-                    best = tq;
-                    wide_chunk = c;
+                const int64_t hi = (longest + n - 1) / n;
+                const int64_t lo = std::max<int64_t>((shortest + n - 1) / n, hi - kPieceLengthSteps * kWideBlockPages);
+                for (int64_t c0 = hi; c0 >= lo; c0 -= kWideBlockPages) {
+                    const int64_t c = std::min<int64_t>(kMaxTileItemPages, std::max<int64_t>(kWideBlockPages, c0));
+                    const double tq = prefix_queue_time(groups, c, n_wide, p->tc_pairs);
+                    if (tq < best) {
+                        best = tq;
+                        wide_chunk = c;
+                    }
                 }
             }
         }
