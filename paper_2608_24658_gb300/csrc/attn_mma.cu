@@ -1243,17 +1243,24 @@ __device__ __forceinline__ void convert_block_e4m3(uint32_t src, uint32_t dst, i
         const int r = (idx >> 3) & 63;
         const int c = idx & 7;
         if (r >= valid) w[q] = make_uint4(0u, 0u, 0u, 0u);
-        const uint32_t lo0 = e4m3x2_to_f16x2(w[q].x), lo1 = e4m3x2_to_f16x2(w[q].x >> 16);
-        const uint32_t lo2 = e4m3x2_to_f16x2(w[q].y), lo3 = e4m3x2_to_f16x2(w[q].y >> 16);
-        const uint32_t hi0 = e4m3x2_to_f16x2(w[q].z), hi1 = e4m3x2_to_f16x2(w[q].z >> 16);
-        const uint32_t hi2 = e4m3x2_to_f16x2(w[q].w), hi3 = e4m3x2_to_f16x2(w[q].w >> 16);
+        // chunks c and c + 4 of a row widen into the same 16-byte slots of
+        // the two column blocks; the 8 threads of a quarter warp (one row)
+        // would store two to a bank group, so the c >= 4 threads store their
+        // second half first
+        const bool second_first = (c & 4) != 0;
+        const uint4 v = second_first ? make_uint4(w[q].z, w[q].w, w[q].x, w[q].y) : w[q];
+        const uint32_t a0 = e4m3x2_to_f16x2(v.x), a1 = e4m3x2_to_f16x2(v.x >> 16);
+        const uint32_t a2 = e4m3x2_to_f16x2(v.y), a3 = e4m3x2_to_f16x2(v.y >> 16);
+        const uint32_t b0 = e4m3x2_to_f16x2(v.z), b1 = e4m3x2_to_f16x2(v.z >> 16);
+        const uint32_t b2 = e4m3x2_to_f16x2(v.w), b3 = e4m3x2_to_f16x2(v.w >> 16);
         const int c2 = 2 * (c & 3);              // f16 chunk in column block c / 4
+        const int first = second_first ? c2 + 1 : c2;
         const uint32_t row = dst + op * kTcKBytes + (c >> 2) * kTcColBlockBytes + r * 128;
-        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(row + ((c2 ^ (r & 7)) << 4)),
-                     "r"(lo0), "r"(lo1), "r"(lo2), "r"(lo3)
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(row + ((first ^ (r & 7)) << 4)),
+                     "r"(a0), "r"(a1), "r"(a2), "r"(a3)
                      : "memory");
-        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(row + (((c2 + 1) ^ (r & 7)) << 4)),
-                     "r"(hi0), "r"(hi1), "r"(hi2), "r"(hi3)
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(row + (((first ^ 1) ^ (r & 7)) << 4)),
+                     "r"(b0), "r"(b1), "r"(b2), "r"(b3)
                      : "memory");
     }
 }
