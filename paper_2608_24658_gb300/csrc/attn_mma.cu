@@ -1163,6 +1163,21 @@ struct TcMeta {
 // causal mask: -1 when the item's rows see all of its keys
 constexpr int32_t kNoKey0 = -1;
 
+// 32 consecutive fp32 values of one partial row (128 bytes, 32-byte
+// aligned), scaled, as four 32-byte stores: every store fills whole sectors
+// (16-byte stores from the 32 rows of a warp left each sector to be filled
+// by two instructions).
+__device__ __forceinline__ void store_row32(float *dst, const uint32_t (&v)[32], float scale) {
+#pragma unroll
+    for (int q = 0; q < 32; q += 8)
+        asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(dst + q),
+                     "f"(__uint_as_float(v[q]) * scale), "f"(__uint_as_float(v[q + 1]) * scale),
+                     "f"(__uint_as_float(v[q + 2]) * scale), "f"(__uint_as_float(v[q + 3]) * scale),
+                     "f"(__uint_as_float(v[q + 4]) * scale), "f"(__uint_as_float(v[q + 5]) * scale),
+                     "f"(__uint_as_float(v[q + 6]) * scale), "f"(__uint_as_float(v[q + 7]) * scale)
+                     : "memory");
+}
+
 // An item's page rows into its metadata slot: the TMA row of every page
 // (padding pages carry the first row past the pool, which TMA fills with
 // zeros), and the leading valid tokens of every block, from the low 4 bits
@@ -1723,13 +1738,7 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
                 uint32_t ov[32];
                 tc::ld32(tO + 32 * c, ov);
                 tc::wait_ld();
-                if (r < it.nrows) {
-#pragma unroll
-                    for (int q = 0; q < 32; q += 4)
-                        *reinterpret_cast<float4 *>(dst + 32 * c + q) =
-                            make_float4(__uint_as_float(ov[q]) * vs, __uint_as_float(ov[q + 1]) * vs,
-                                        __uint_as_float(ov[q + 2]) * vs, __uint_as_float(ov[q + 3]) * vs);
-                }
+                if (r < it.nrows) store_row32(dst + 32 * c, ov, vs);
             }
         };
             // The converters take every block of every item in order.  An
@@ -2331,13 +2340,7 @@ __device__ void prefix_cta_tc_pair(const KvMaps *maps, const AttnArgs &a, uint8_
                     uint32_t ov[32];
                     tc::ld32(tO + 32 * c, ov);
                     tc::wait_ld();
-                    if (r < it.nrows) {
-#pragma unroll
-                        for (int q = 0; q < 32; q += 4)
-                            *reinterpret_cast<float4 *>(dst + 32 * c + q) =
-                                make_float4(__uint_as_float(ov[q]), __uint_as_float(ov[q + 1]),
-                                            __uint_as_float(ov[q + 2]), __uint_as_float(ov[q + 3]));
-                    }
+                    if (r < it.nrows) store_row32(dst + 32 * c, ov, 1.f);
                 }
                 tc::fence_before_sync();
                 __syncwarp();
