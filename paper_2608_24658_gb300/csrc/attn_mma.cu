@@ -74,17 +74,23 @@ constexpr float kLazyRescaleLog2 = 8.f;   // mma.sync softmax: move the referenc
 // costs more issue per byte (widening to f16), so that pass runs more,
 // shallower warps; bf16 with few rows per tile (g <= 4) runs fewer, deeper
 // ones, whose extra pages in flight shorten the tail of the launch.
+// kStepPages: pages of a suffix item under one softmax update of the
+// transposed step (e4m3 pages are cheap to stream and costly to widen: two
+// pages per update give each warp two independent MMA chains)
 struct KvBf16 {
     static constexpr int kElemBytes = 2;
     static constexpr int kSuffixWarps = 8;
+    static constexpr int kStepPages = 1;
 };
 struct KvBf16Deep {
     static constexpr int kElemBytes = 2;
     static constexpr int kSuffixWarps = 6;
+    static constexpr int kStepPages = 1;
 };
 struct KvE4m3 {
     static constexpr int kElemBytes = 1;
     static constexpr int kSuffixWarps = 12;
+    static constexpr int kStepPages = 2;
 };
 
 template <int D, class KV>
@@ -186,6 +192,17 @@ __device__ __forceinline__ uint32_t e4m3x2_to_f16x2(uint32_t two_bytes) {
         : "=r"(out)
         : "r"(two_bytes));
     return out;
+}
+
+// Four e4m3 values (one word) widened exactly to two f16 pairs: bytes 0-1
+// to `lo`, bytes 2-3 to `hi`.
+__device__ __forceinline__ void e4m3x4_to_f16x2x2(uint32_t four_bytes, uint32_t &lo, uint32_t &hi) {
+    asm("{\n\t.reg .b16 l, h;\n\t"
+        "mov.b32 {l, h}, %2;\n\t"
+        "cvt.rn.f16x2.e4m3x2 %0, l;\n\t"
+        "cvt.rn.f16x2.e4m3x2 %1, h;\n\t}"
+        : "=r"(lo), "=r"(hi)
+        : "r"(four_bytes));
 }
 
 // A bf16 pair of q narrowed to an f16 pair for the e4m3 MMAs.  The f16
@@ -315,7 +332,9 @@ __device__ __forceinline__ void page_step(uint32_t kbase, uint32_t vbase, int va
 #pragma unroll
             for (int nt = 0; nt < 2; ++nt) {
                 const uint32_t w = lds32(kbase + dev::swz128(nt * 8 + gid, ks) + 4 * tig);
-                dev::mma_f16_16816(acc[nt], qa[ks], e4m3x2_to_f16x2(w), e4m3x2_to_f16x2(w >> 16));
+                uint32_t b0, b1;
+                e4m3x4_to_f16x2x2(w, b0, b1);
+                dev::mma_f16_16816(acc[nt], qa[ks], b0, b1);
             }
         }
     }
@@ -388,7 +407,7 @@ __device__ __forceinline__ void page_step(uint32_t kbase, uint32_t vbase, int va
 //   gid + 8.  O^T fragment of column tile dt: c0, c1 = column tcol(dt, gid),
 //   rows 2tig and 2tig + 1; c2, c3 = column tcol(dt, gid + 8).
 // The reduction index d of S^T may be permuted (the same way in K and Q); the
-// e4m3 path does so to read 4 bytes of K at a time, and picks its output
+// e4m3 path does so to read 16 bytes of K at a time, and picks its output
 // columns so that each lane's columns are one 16-byte chunk of V.
 // ---------------------------------------------------------------------------
 template <int D>
@@ -416,8 +435,9 @@ __device__ __forceinline__ int tcol(int dt, int r) {
 }
 
 // Q^T fragments (B operand, d x 8 rows): row gid of the tile, d pairs of
-// k-step ks -- (16 ks + 2 tig, 16 ks + 8 + 2 tig) for bf16, (16 ks + 4 tig,
-// 16 ks + 4 tig + 2) widened to f16 for e4m3
+// k-step ks -- (16 ks + 2 tig, 16 ks + 8 + 2 tig) for bf16; for e4m3, widened
+// to f16, (e, e + 2) with e = 32 tig + 16 (ks / 4) + 4 (ks % 4), the slice
+// that word ks % 4 of the lane's 16-byte K chunk 2 tig + ks / 4 holds
 template <int D, class KV>
 __device__ __forceinline__ void load_q_fragments_t(const AttnArgs &a, const WorkItem &it, int lane,
                                                    uint32_t (&qb)[D / 16][2]) {
@@ -437,7 +457,7 @@ __device__ __forceinline__ void load_q_fragments_t(const AttnArgs &a, const Work
             qb[ks][1] = qrow ? *reinterpret_cast<const uint32_t *>(qrow + ks * 16 + 8 + 2 * tig) : 0u;
         } else {
             uint2 u = make_uint2(0u, 0u);
-            if (qrow) u = *reinterpret_cast<const uint2 *>(qrow + ks * 16 + 4 * tig);
+            if (qrow) u = *reinterpret_cast<const uint2 *>(qrow + 32 * tig + 16 * (ks >> 2) + 4 * (ks & 3));
             qb[ks][0] = q_pair_to_f16(u.x, big);
             qb[ks][1] = q_pair_to_f16(u.y, big);
         }
@@ -445,80 +465,59 @@ __device__ __forceinline__ void load_q_fragments_t(const AttnArgs &a, const Work
     if constexpr (KV::kElemBytes == 1) report_q_range(a, big, lane);
 }
 
+// S^T of one page, unscaled: s[e] for token gid + 8 (e / 2), row 2 tig + e % 2
 template <int D, class KV>
-__device__ __forceinline__ void page_step_t(uint32_t kbase, uint32_t vbase, int valid,
-                                            const uint32_t (&qb)[D / 16][2], WarpStateT<D> &st,
-                                            float scale_log2, int lane) {
+__device__ __forceinline__ void scores_t(uint32_t kbase, const uint32_t (&qb)[D / 16][2], int lane,
+                                         float (&s)[4]) {
     using S = Shape<D, KV>;
     const int gid = lane >> 2, tig = lane & 3;
     const int mi = lane >> 3, r8 = lane & 7;
-
     // S^T = K Q^T, two accumulators (first and second half of d)
     float sc[4] = {0.f, 0.f, 0.f, 0.f}, sd[4] = {0.f, 0.f, 0.f, 0.f};
+    if constexpr (KV::kElemBytes == 2) {
 #pragma unroll
-    for (int ks = 0; ks < D / 16; ++ks) {
-        float(&acc)[4] = ks < D / 32 ? sc : sd;
-        uint32_t ka[4];
-        if constexpr (KV::kElemBytes == 2) {
+        for (int ks = 0; ks < D / 16; ++ks) {
+            float(&acc)[4] = ks < D / 32 ? sc : sd;
+            uint32_t ka[4];
             const int tok = r8 + ((mi & 1) << 3), dch = 2 * ks + (mi >> 1);
             dev::ldsm_x4(kbase + (dch >> 3) * S::kSegBytes + dev::swz128(tok, dch & 7), ka[0], ka[1],
                          ka[2], ka[3]);
             dev::mma_bf16_16816(acc, ka, qb[ks][0], qb[ks][1]);
-        } else {
-            const uint32_t w0 = lds32(kbase + dev::swz128(gid, ks) + 4 * tig);
-            const uint32_t w1 = lds32(kbase + dev::swz128(gid + 8, ks) + 4 * tig);
-            ka[0] = e4m3x2_to_f16x2(w0);
-            ka[1] = e4m3x2_to_f16x2(w1);
-            ka[2] = e4m3x2_to_f16x2(w0 >> 16);
-            ka[3] = e4m3x2_to_f16x2(w1 >> 16);
+        }
+    } else {
+        static_assert(D == 128, "e4m3 KV path is written for head_dim 128");
+        // 16-byte chunks 2 tig and 2 tig + 1 of tokens gid and gid + 8 (the
+        // eight lanes of a phase read eight distinct swizzled chunks)
+        uint4 kg[2], kh[2];
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+            kg[j] = lds128(kbase + dev::swz128(gid, 2 * tig + j));
+            kh[j] = lds128(kbase + dev::swz128(gid + 8, 2 * tig + j));
+        }
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+            float(&acc)[4] = ks < D / 32 ? sc : sd;
+            const uint4 &g = kg[ks >> 2], &h = kh[ks >> 2];
+            const int i = ks & 3;
+            const uint32_t w0 = i == 0 ? g.x : i == 1 ? g.y : i == 2 ? g.z : g.w;
+            const uint32_t w1 = i == 0 ? h.x : i == 1 ? h.y : i == 2 ? h.z : h.w;
+            uint32_t ka[4];
+            e4m3x4_to_f16x2x2(w0, ka[0], ka[2]);
+            e4m3x4_to_f16x2x2(w1, ka[1], ka[3]);
             dev::mma_f16_16816(acc, ka, qb[ks][0], qb[ks][1]);
         }
     }
-    float x[4];
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-        const int tok = gid + ((e >> 1) << 3);
-        x[e] = tok < valid ? (sc[e] + sd[e]) * scale_log2 : -INFINITY;
-    }
-    // row maxima over the 16 tokens: the 8 lanes of a tig
-    float mx0 = fmaxf(x[0], x[2]), mx1 = fmaxf(x[1], x[3]);
-#pragma unroll
-    for (int o = 4; o < 32; o <<= 1) {
-        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
-        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
-    }
-    // (token 0 of every page of an item is valid: the maxima are finite)
-    const bool grow = mx0 > st.m[0] + kLazyRescaleLog2 || mx1 > st.m[1] + kLazyRescaleLog2;
-    if (__any_sync(0xffffffffu, grow)) {
-        const float mn0 = fmaxf(st.m[0], mx0), mn1 = fmaxf(st.m[1], mx1);
-        const float al0 = dev::fast_exp2(st.m[0] - mn0), al1 = dev::fast_exp2(st.m[1] - mn1);
-        st.m[0] = mn0;
-        st.m[1] = mn1;
-        st.l[0] *= al0;
-        st.l[1] *= al1;
-#pragma unroll
-        for (int dt = 0; dt < D / 16; ++dt) {
-            st.o[dt][0] *= al0;
-            st.o[dt][1] *= al1;
-            st.o[dt][2] *= al0;
-            st.o[dt][3] *= al1;
-        }
-    }
-    const float p0 = dev::fast_exp2(x[0] - st.m[0]), p1 = dev::fast_exp2(x[1] - st.m[1]);
-    const float p2 = dev::fast_exp2(x[2] - st.m[0]), p3 = dev::fast_exp2(x[3] - st.m[1]);
-    st.l[0] += p0 + p2;
-    st.l[1] += p1 + p3;
-    // P^T as the B operand (tokens x rows): transpose the two 8 x 8 halves
-    uint32_t pb0, pb1;
-    if constexpr (KV::kElemBytes == 2) {
-        pb0 = dev::movmatrix_trans(dev::pack_bf16(p0, p1));
-        pb1 = dev::movmatrix_trans(dev::pack_bf16(p2, p3));
-    } else {
-        pb0 = dev::movmatrix_trans(dev::pack_f16(p0, p1));
-        pb1 = dev::movmatrix_trans(dev::pack_f16(p2, p3));
-    }
+    for (int e = 0; e < 4; ++e) s[e] = sc[e] + sd[e];
+}
 
-    // O^T += V^T P^T over the column tiles
+// O^T += V^T P^T of one page
+template <int D, class KV>
+__device__ __forceinline__ void pv_t(uint32_t vbase, int valid, uint32_t pb0, uint32_t pb1,
+                                     WarpStateT<D> &st, int lane) {
+    using S = Shape<D, KV>;
+    const int gid = lane >> 2, tig = lane & 3;
+    const int mi = lane >> 3, r8 = lane & 7;
     if constexpr (KV::kElemBytes == 2) {
         // slots past the node's length may hold anything (NaN included): V
         // of those tokens is zeroed (this lane's A columns are tokens 2tig,
@@ -543,7 +542,6 @@ __device__ __forceinline__ void page_step_t(uint32_t kbase, uint32_t vbase, int 
             dev::mma_bf16_16816(st.o[dt], va, pb0, pb1);
         }
     } else {
-        static_assert(D == 128, "e4m3 KV path is written for head_dim 128");
         // this lane's output columns are 16 gid .. 16 gid + 15: chunk gid of
         // its four tokens 2tig, 2tig + 1, 2tig + 8, 2tig + 9
         const int t0 = 2 * tig;
@@ -568,12 +566,78 @@ __device__ __forceinline__ void page_step_t(uint32_t kbase, uint32_t vbase, int 
             const uint32_t lo = __byte_perm(wa[dt >> 1], wb[dt >> 1], sel);   // tokens 2tig, 2tig+1
             const uint32_t hi = __byte_perm(wc[dt >> 1], wd[dt >> 1], sel);   // tokens 2tig+8, 2tig+9
             uint32_t a4[4];
-            a4[0] = e4m3x2_to_f16x2(lo);         // column 16 gid + 2 dt
-            a4[1] = e4m3x2_to_f16x2(lo >> 16);   // column 16 gid + 2 dt + 1
-            a4[2] = e4m3x2_to_f16x2(hi);
-            a4[3] = e4m3x2_to_f16x2(hi >> 16);
+            e4m3x4_to_f16x2x2(lo, a4[0], a4[1]);   // columns 16 gid + 2 dt, + 1
+            e4m3x4_to_f16x2x2(hi, a4[2], a4[3]);
             dev::mma_f16_16816(st.o[dt], a4, pb0, pb1);
         }
+    }
+}
+
+// NP consecutive pages of one item under one online-softmax update (their
+// scores share the row maxima, the rescale and the shuffles); all pages but
+// the last are full.
+template <int D, class KV, int NP>
+__device__ __forceinline__ void pages_step_t(const uint32_t *kbase, const uint32_t *vbase,
+                                             int valid_last, const uint32_t (&qb)[D / 16][2],
+                                             WarpStateT<D> &st, float scale_log2, int lane) {
+    const int gid = lane >> 2;
+    float x[NP][4];
+#pragma unroll
+    for (int p = 0; p < NP; ++p) {
+        float sp[4];
+        scores_t<D, KV>(kbase[p], qb, lane, sp);
+        const int valid = p == NP - 1 ? valid_last : kPageSize;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int tok = gid + ((e >> 1) << 3);
+            x[p][e] = tok < valid ? sp[e] * scale_log2 : -INFINITY;
+        }
+    }
+    // row maxima over the pages' tokens: the 8 lanes of a tig
+    float mx0 = fmaxf(x[0][0], x[0][2]), mx1 = fmaxf(x[0][1], x[0][3]);
+#pragma unroll
+    for (int p = 1; p < NP; ++p) {
+        mx0 = fmaxf(mx0, fmaxf(x[p][0], x[p][2]));
+        mx1 = fmaxf(mx1, fmaxf(x[p][1], x[p][3]));
+    }
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) {
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+    }
+    // (token 0 of every page of an item is valid: the maxima are finite)
+    const bool grow = mx0 > st.m[0] + kLazyRescaleLog2 || mx1 > st.m[1] + kLazyRescaleLog2;
+    if (__any_sync(0xffffffffu, grow)) {
+        const float mn0 = fmaxf(st.m[0], mx0), mn1 = fmaxf(st.m[1], mx1);
+        const float al0 = dev::fast_exp2(st.m[0] - mn0), al1 = dev::fast_exp2(st.m[1] - mn1);
+        st.m[0] = mn0;
+        st.m[1] = mn1;
+        st.l[0] *= al0;
+        st.l[1] *= al1;
+#pragma unroll
+        for (int dt = 0; dt < D / 16; ++dt) {
+            st.o[dt][0] *= al0;
+            st.o[dt][1] *= al1;
+            st.o[dt][2] *= al0;
+            st.o[dt][3] *= al1;
+        }
+    }
+#pragma unroll
+    for (int p = 0; p < NP; ++p) {
+        const float p0 = dev::fast_exp2(x[p][0] - st.m[0]), p1 = dev::fast_exp2(x[p][1] - st.m[1]);
+        const float p2 = dev::fast_exp2(x[p][2] - st.m[0]), p3 = dev::fast_exp2(x[p][3] - st.m[1]);
+        st.l[0] += p0 + p2;
+        st.l[1] += p1 + p3;
+        // P^T as the B operand (tokens x rows): transpose the two 8 x 8 halves
+        uint32_t pb0, pb1;
+        if constexpr (KV::kElemBytes == 2) {
+            pb0 = dev::movmatrix_trans(dev::pack_bf16(p0, p1));
+            pb1 = dev::movmatrix_trans(dev::pack_bf16(p2, p3));
+        } else {
+            pb0 = dev::movmatrix_trans(dev::pack_f16(p0, p1));
+            pb1 = dev::movmatrix_trans(dev::pack_f16(p2, p3));
+        }
+        pv_t<D, KV>(vbase[p], p == NP - 1 ? valid_last : kPageSize, pb0, pb1, st, lane);
     }
 }
 
@@ -825,19 +889,30 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
             load_q_fragments_t<D, KV>(a, it, lane, qb);
             WarpStateT<D> st;
             reset<D>(st);
-            for (int pg = 0; pg < it.num_pages; ++pg, ++consumed) {
-                const int s = consumed % NS;
-                if (!dev::mbar_wait_bounded(my_bar + s * 8, (consumed / NS) & 1, a.wait_limit_ns,
-                                            nullptr)) {
-                    ok = false;
-                    break;
+            for (int pg = 0; pg < it.num_pages;) {
+                // kStepPages pages per softmax update while the item has them
+                const int np = it.num_pages - pg >= KV::kStepPages ? KV::kStepPages : 1;
+                uint32_t kb[KV::kStepPages], vb[KV::kStepPages];
+#pragma unroll
+                for (int p = 0; p < KV::kStepPages; ++p) {
+                    const int c = consumed + (p < np ? p : 0);
+                    const int s = c % NS;
+                    kb[p] = my_ring + s * S::kStageBytes;
+                    vb[p] = kb[p] + S::kPageBytes;
+                    if (p < np && !dev::mbar_wait_bounded(my_bar + s * 8, (c / NS) & 1,
+                                                          a.wait_limit_ns, nullptr))
+                        ok = false;
                 }
-                const int valid = (pg == it.num_pages - 1) ? it.last_valid : kPageSize;
-                page_step_t<D, KV>(my_ring + s * S::kStageBytes,
-                                   my_ring + s * S::kStageBytes + S::kPageBytes, valid, qb, st, scl.x,
-                                   lane);
+                if (!ok) break;
+                const int valid = pg + np == it.num_pages ? it.last_valid : kPageSize;
+                if (KV::kStepPages > 1 && np == KV::kStepPages)
+                    pages_step_t<D, KV, KV::kStepPages>(kb, vb, valid, qb, st, scl.x, lane);
+                else
+                    pages_step_t<D, KV, 1>(kb, vb, valid, qb, st, scl.x, lane);
                 __syncwarp();
-                issue_next();
+                for (int p = 0; p < np; ++p) issue_next();
+                pg += np;
+                consumed += np;
             }
             if (!ok) break;
             store_warp_partials_t<D, KV>(a, it, st, lane, scl.y);
