@@ -1192,12 +1192,14 @@ constexpr int kTcKBytes = 2 * kTcColBlockBytes;               // d = 128: two co
 constexpr int kTcStageBytes = 2 * kTcKBytes;                  // K + V
 constexpr int kTcRingBytes = kTcStages * kTcStageBytes;       // 192 KB
 // e4m3 KV: TMA stages the raw bytes (K and V of a block, 64 rows of 128 B
-// each: 16 KB) in kTcStages stages; the epilogue warps convert each block
+// each: 16 KB) in kTcF8Stages stages; the epilogue warps convert each block
 // to f16 (exactly) into kTcCvStages stages laid out like a bf16 stage.
 constexpr int kTcF8Bytes = kTcBlockTokens * 128;              // 8 KB: K (or V) of a block
 constexpr int kTcF8StageBytes = 2 * kTcF8Bytes;
-constexpr int kTcCvStages = 3;
-constexpr int kTcCvOffset = kTcStages * kTcF8StageBytes;      // 96 KB
+constexpr int kTcF8Stages = 4;                                 // raw e4m3 stages
+constexpr int kTcCvStages = 4;
+constexpr int kTcCvOffset = kTcF8Stages * kTcF8StageBytes;    // 64 KB
+static_assert(kTcF8Stages <= kTcStages, "raw e4m3 stages use the ring's barriers");
 static_assert(kTcCvOffset + kTcCvStages * kTcStageBytes <= kTcRingBytes, "e4m3 rings fit");
 constexpr int kTcTmemCols = 512;
 constexpr uint32_t kTmemO = 0, kTmemS = 256, kTmemQ = 384;    // TMEM column bases
@@ -1339,10 +1341,11 @@ __device__ __forceinline__ void convert_block_e4m3(uint32_t src, uint32_t dst, i
         // second half first
         const bool second_first = (c & 4) != 0;
         const uint4 v = second_first ? make_uint4(w[q].z, w[q].w, w[q].x, w[q].y) : w[q];
-        const uint32_t a0 = e4m3x2_to_f16x2(v.x), a1 = e4m3x2_to_f16x2(v.x >> 16);
-        const uint32_t a2 = e4m3x2_to_f16x2(v.y), a3 = e4m3x2_to_f16x2(v.y >> 16);
-        const uint32_t b0 = e4m3x2_to_f16x2(v.z), b1 = e4m3x2_to_f16x2(v.z >> 16);
-        const uint32_t b2 = e4m3x2_to_f16x2(v.w), b3 = e4m3x2_to_f16x2(v.w >> 16);
+        uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
+        e4m3x4_to_f16x2x2(v.x, a0, a1);
+        e4m3x4_to_f16x2x2(v.y, a2, a3);
+        e4m3x4_to_f16x2x2(v.z, b0, b1);
+        e4m3x4_to_f16x2x2(v.w, b2, b3);
         const int c2 = 2 * (c & 3);              // f16 chunk in column block c / 4
         const int first = second_first ? c2 + 1 : c2;
         const uint32_t row = dst + op * kTcKBytes + (c >> 2) * kTcColBlockBytes + r * 128;
@@ -1438,8 +1441,9 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
         // e4m3 blocks keep the default L2 policy (the per-page boxes use no hint)
         const uint64_t f8_pol = dev::l2_evict_normal_policy();
         const int kv_page_rows = a.num_kv_heads * kPageSize;   // TMA rows between consecutive pages
-        int last_issue[kTcStages];
-        for (int s = 0; s < kTcStages; ++s) last_issue[s] = -1;
+        constexpr int NS = kF8 ? kTcF8Stages : kTcStages;
+        int last_issue[NS];
+        for (int s = 0; s < NS; ++s) last_issue[s] = -1;
         int blk = 0;
         bool ok = true;
         for (int k = 0; ok; ++k) {
@@ -1453,9 +1457,9 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
             const int np = m.it.num_pages;
             const int nb = tc_blocks(np);
             for (int bi = 0; bi < nb; ++bi, ++blk) {
-                const int s = blk % kTcStages;
-                if (blk >= kTcStages &&
-                    !tc_warp_wait(bar(kBarKvEmpty + s), ((blk / kTcStages) - 1) & 1, limit, abort_flag,
+                const int s = blk % NS;
+                if (blk >= NS &&
+                    !tc_warp_wait(bar(kBarKvEmpty + s), ((blk / NS) - 1) & 1, limit, abort_flag,
                                   lane)) {
                     if (lane == 0) tc_fail(a, abort_flag, kSiteProducerEmpty);
                     ok = false;
@@ -1521,9 +1525,9 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
         }
         // every copy this CTA issued must land before its shared memory is reused
         if (lane == 0)
-            for (int s = 0; s < kTcStages; ++s)
+            for (int s = 0; s < NS; ++s)
                 if (last_issue[s] >= 0)
-                    dev::mbar_wait_bounded(bar(kBarKvFull + s), (last_issue[s] / kTcStages) & 1,
+                    dev::mbar_wait_bounded(bar(kBarKvFull + s), (last_issue[s] / NS) & 1,
                                            kDrainLimitNs, nullptr);
     } else if (warp == kTcMmaWarp || warp == kTcPvWarp) {
         // ------------------------------------------------------------ MMA issuers
@@ -1824,8 +1828,8 @@ __device__ void prefix_cta_tc(const KvMaps *maps, const AttnArgs &a, uint8_t *sm
             // wait for the O is short (long-prefix step with e4m3 KV: 668 ->
             // 655 us).
             auto convert = [&](int gb, int valid) -> bool {
-                const int s = gb % kTcStages, c = gb % kTcCvStages;
-                if (!tc_warp_wait(bar(kBarKvFull + s), (gb / kTcStages) & 1, limit, abort_flag, lane))
+                const int s = gb % kTcF8Stages, c = gb % kTcCvStages;
+                if (!tc_warp_wait(bar(kBarKvFull + s), (gb / kTcF8Stages) & 1, limit, abort_flag, lane))
                     return false;
                 if (gb >= kTcCvStages &&
                     !tc_warp_wait(bar(kBarCvEmpty + c), ((gb / kTcCvStages) - 1) & 1, limit, abort_flag,

@@ -82,7 +82,7 @@ constexpr int32_t kAppendSlackMin = 4, kAppendSlackMax = 64;
 constexpr int kPatchesPerTail = 6;      // words one append may change per tail item
 constexpr double kWideGroupPageCost = 1.0;   // one 16-row group of one page, in suffix pages
 constexpr double kTcPageCost = 2.0;          // one page of a tcgen05 prefix tile (tuned)
-constexpr double kTcPageCostE4m3 = 4.0;      // the same with e4m3 KV, whose suffix pages
+constexpr double kTcPageCostE4m3 = 3.6;      // the same with e4m3 KV, whose suffix pages
                                              // take half the time (tuned)
 constexpr int64_t kDefaultWaitNs = 2000000000LL;
 constexpr size_t kAlign = 256;
