@@ -134,31 +134,40 @@ struct Shape {
 };
 
 // K then V of one (page, kv head) into a stage: one TMA box {128 bytes, 1
-// block, 16 tokens} per column block and tensor.  A suffix page is read by
-// one item only, so its lines go first when L2 needs room (the partials
-// written meanwhile stay for the merge); a prefix page may be read again by
-// another row tile of its node and keeps the normal policy.
-template <int D, class KV, bool kReadOnce>
+// block, 16 tokens} per column block and tensor (the prefix pass of the
+// mma.sync path; a prefix page may be read again by another row tile of its
+// node and keeps the normal L2 policy).
+template <int D, class KV>
 __device__ __forceinline__ void load_page(uint32_t dst, const CUtensorMap *tmap_k,
                                           const CUtensorMap *tmap_v, int row, uint32_t bar) {
     using S = Shape<D, KV>;
-    if constexpr (kReadOnce) {
-        const uint64_t pol = dev::l2_evict_first_policy();
 #pragma unroll
-        for (int sg = 0; sg < S::kSeg; ++sg) {
-            dev::tma_load_3d_hint(dst + sg * S::kSegBytes, tmap_k, 0, sg, row, bar, pol);
-            dev::tma_load_3d_hint(dst + S::kPageBytes + sg * S::kSegBytes, tmap_v, 0, sg, row, bar, pol);
-        }
-    } else {
-#pragma unroll
-        for (int sg = 0; sg < S::kSeg; ++sg) {
-            dev::tma_load_3d(dst + sg * S::kSegBytes, tmap_k, 0, sg, row, bar);
-            dev::tma_load_3d(dst + S::kPageBytes + sg * S::kSegBytes, tmap_v, 0, sg, row, bar);
-        }
+    for (int sg = 0; sg < S::kSeg; ++sg) {
+        dev::tma_load_3d(dst + sg * S::kSegBytes, tmap_k, 0, sg, row, bar);
+        dev::tma_load_3d(dst + S::kPageBytes + sg * S::kSegBytes, tmap_v, 0, sg, row, bar);
     }
 }
 
-// Online-softmax state of one warp: 16 rows, thread holds rows gid, gid+8.
+// The same for a suffix page, in one box per tensor (the page maps) where a
+// page has several column blocks: each TMA box costs the SM's copy engine a
+// fixed time, and with 2 KB boxes it held a suffix CTA to about 60 GB/s.  A
+// suffix page is read by one item only, so its lines go first when L2 needs
+// room (the partials written meanwhile stay for the merge).
+template <int D, class KV>
+__device__ __forceinline__ void load_suffix_page(uint32_t dst, const KvMaps &maps, int row,
+                                                 uint32_t bar) {
+    using S = Shape<D, KV>;
+    const uint64_t pol = dev::l2_evict_first_policy();
+    if constexpr (S::kSeg > 1) {
+        const int ph = row / kPageSize;
+        dev::tma_load_4d_hint(dst, &maps.k_page, 0, 0, 0, ph, bar, pol);
+        dev::tma_load_4d_hint(dst + S::kPageBytes, &maps.v_page, 0, 0, 0, ph, bar, pol);
+    } else {
+        dev::tma_load_3d_hint(dst, &maps.k, 0, 0, row, bar, pol);
+        dev::tma_load_3d_hint(dst + S::kPageBytes, &maps.v, 0, 0, row, bar, pol);
+    }
+}
+
 template <int D>
 struct WarpState {
     float o[D / 8][4];
@@ -790,9 +799,8 @@ struct ItemRows {
 // pages through its own ring
 // ---------------------------------------------------------------------------
 template <int D, class KV>
-__device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
-                            const AttnArgs &a, uint32_t ring, uint32_t bars, int warp, int lane,
-                            WorkItem *grab) {
+__device__ void suffix_warp(const KvMaps &maps, const AttnArgs &a, uint32_t ring, uint32_t bars,
+                            int warp, int lane, WorkItem *grab) {
     using S = Shape<D, KV>;
     constexpr int NS = S::kWarpStages;
     const uint32_t my_ring = ring + warp * S::kWarpRingBytes;
@@ -868,7 +876,7 @@ __device__ void suffix_warp(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v
             const int s = issued % NS;
             const uint32_t bar = my_bar + s * 8;
             dev::mbar_arrive_expect_tx(bar, S::kStageBytes);
-            load_page<D, KV, true>(my_ring + s * S::kStageBytes, tmap_k, tmap_v, row, bar);
+            load_suffix_page<D, KV>(my_ring + s * S::kStageBytes, maps, row, bar);
         }
         ++iss_pg;
         ++issued;
@@ -1025,7 +1033,7 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
                 const int row = rows.row(pg, lane);
                 if (lane == 0 && !(skip_first && stage == 0)) {
                     dev::mbar_arrive_expect_tx(bar_full + 8 * s, S::kStageBytes);
-                    load_page<D, KV, false>(k_page(s), tmap_k, tmap_v, row, bar_full + 8 * s);
+                    load_page<D, KV>(k_page(s), tmap_k, tmap_v, row, bar_full + 8 * s);
                     last_issue[s] = stage;
                 }
             }
@@ -2492,6 +2500,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         dev::fence_mbar_init();
         dev::prefetch_tensormap(&maps.k);
         dev::prefetch_tensormap(&maps.v);
+        if constexpr (S::kSeg > 1) {
+            dev::prefetch_tensormap(&maps.k_page);
+            dev::prefetch_tensormap(&maps.v_page);
+        }
     }
     if constexpr (kTcPrefix) {
         if (wide && warp == kTcMmaWarp) tc::alloc<kTcTmemCols>(dev::smem_addr(&tmem_base));
@@ -2536,7 +2548,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncthreads();
     }
     if (warp < S::kSuffixWarps)
-        suffix_warp<D, KV>(&maps.k, &maps.v, a, ring, bars, warp, lane, grab_items[warp]);
+        suffix_warp<D, KV>(maps, a, ring, bars, warp, lane, grab_items[warp]);
 }
 
 // Shared memory and carveout are set once per device (with that device

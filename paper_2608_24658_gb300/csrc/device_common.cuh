@@ -118,6 +118,18 @@ __device__ __forceinline__ void tma_load_3d_hint(uint32_t dst, const CUtensorMap
         : "memory");
 }
 
+// 4-D tensor copy with an L2 cache policy (a whole page of one kv head; see
+// the page maps of the KV pool).
+__device__ __forceinline__ void tma_load_4d_hint(uint32_t dst, const CUtensorMap *map, int32_t c0,
+                                                 int32_t c1, int32_t c2, int32_t c3, uint32_t bar,
+                                                 uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar), "l"(policy)
+        : "memory");
+}
+
 // 5-D tensor copy with an L2 cache policy (several pages of one kv head in
 // one box; see the run maps of the KV pool).
 __device__ __forceinline__ void tma_load_5d_hint(uint32_t dst, const CUtensorMap *map, int32_t c0,

@@ -122,10 +122,12 @@ cudaError_t attn_mma_ctas_per_sm(int head_dim, int mode, int *ctas_per_sm);
 // TMA views of the K and V pools.  k / v: one box is one 128-byte column
 // block of one page of one kv head (16 rows).  k_run / v_run: one box is the
 // same column block of kTcRunPages consecutive pages of one kv head, for
-// blocks whose pages are consecutive in the pool.
+// blocks whose pages are consecutive in the pool.  k_page / v_page: one box
+// is a whole page of one kv head, its column blocks one after another (the
+// layout the per-block boxes of k / v give).
 constexpr int kTcRunPages = 4;
 struct KvMaps {
-    CUtensorMap k, v, k_run, v_run;
+    CUtensorMap k, v, k_run, v_run, k_page, v_page;
 };
 
 // Kernel launchers; each returns the launch's cudaError_t.

@@ -1047,6 +1047,36 @@ parason_status encode_kv_run_map(CUtensorMap *map, const void *pages, int64_t nu
     return r == CUDA_SUCCESS ? PARASON_OK : PARASON_ECUDA;
 }
 
+// The same pool as a 4-D view whose dims are not in stride order: dim0 = 128
+// bytes of one segment, dim1 = slot in the page (16, stride one token row),
+// dim2 = segment (stride 128 bytes), dim3 = (page * H_kv + kv_head).  One box
+// {seg, 16, nseg, 1} is a whole page of one kv head with its column blocks
+// one after another, each 16 rows of 128 bytes (128-byte swizzle): what nseg
+// boxes of the 3-D view give, in one copy.
+parason_status encode_kv_page_map(CUtensorMap *map, const void *pages, int64_t num_phys,
+                                  int32_t H_kv, int32_t head_dim, int32_t mode) {
+    auto fn = encode_fn();
+    if (!fn) return PARASON_ECUDA;
+    const int esize = (mode == PARASON_FP8_E4M3_KV) ? 1 : 2;
+    const CUtensorMapDataType dt =
+        (mode == PARASON_FP8_E4M3_KV) ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    const int row_bytes = head_dim * esize;
+    if (row_bytes % 128 != 0) return PARASON_EUNSUPPORTED;
+    const int nseg = row_bytes / 128;
+    const int seg_elems = 128 / esize;
+    cuuint64_t dims[4] = {static_cast<cuuint64_t>(seg_elems), static_cast<cuuint64_t>(parason::kPageSize),
+                          static_cast<cuuint64_t>(nseg), static_cast<cuuint64_t>(num_phys) * H_kv};
+    cuuint64_t strides[3] = {static_cast<cuuint64_t>(row_bytes), 128,
+                             static_cast<cuuint64_t>(parason::kPageSize) * row_bytes};
+    cuuint32_t box[4] = {static_cast<cuuint32_t>(seg_elems), static_cast<cuuint32_t>(parason::kPageSize),
+                         static_cast<cuuint32_t>(nseg), 1u};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    CUresult r = fn(map, dt, 4, const_cast<void *>(pages), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? PARASON_OK : PARASON_ECUDA;
+}
+
 parason_status record_event(parason_plan_s *p, int which, cudaStream_t stream) {
     if (p->timing_cap <= 0 || p->timing_n >= p->timing_cap) return PARASON_OK;
     cudaEvent_t ev = p->events[3 * p->timing_n + which];
@@ -1398,6 +1428,8 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
                     st = encode_kv_map(&p->tm.k, k_pages, p->num_phys, H, d, mode);
                     if (st == PARASON_OK)
                         st = encode_kv_run_map(&p->tm.k_run, k_pages, p->num_phys, H, d, mode);
+                    if (st == PARASON_OK)
+                        st = encode_kv_page_map(&p->tm.k_page, k_pages, p->num_phys, H, d, mode);
                     if (st != PARASON_OK) return st;
                     p->tm_k_ptr = k_pages;
                 }
@@ -1406,6 +1438,8 @@ parason_status parason_attn_decode(parason_plan p, const void *q, const void *k_
                     st = encode_kv_map(&p->tm.v, v_pages, p->num_phys, H, d, mode);
                     if (st == PARASON_OK)
                         st = encode_kv_run_map(&p->tm.v_run, v_pages, p->num_phys, H, d, mode);
+                    if (st == PARASON_OK)
+                        st = encode_kv_page_map(&p->tm.v_page, v_pages, p->num_phys, H, d, mode);
                     if (st != PARASON_OK) return st;
                     p->tm_v_ptr = v_pages;
                 }
