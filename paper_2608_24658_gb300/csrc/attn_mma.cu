@@ -2477,9 +2477,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     static_assert(!kTcPrefix || (kTcBars <= S::kBars && kTcPairBars <= S::kBars),
                   "barrier area holds the tcgen05 barriers");
     __shared__ TcMeta tc_meta[kTcPrefix ? kTcMeta : 1];
-    auto init_suffix_barriers = [&]() {
-        for (int s = 0; s < S::kNarrowBars; ++s) dev::mbar_init(bars + 8 * s, 1);
-    };
     __shared__ uint32_t tmem_base;
     if (threadIdx.x == 0) {
         abort_flag = 0;
@@ -2495,7 +2492,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             for (int i = 0; i < kIdSlots; ++i) dev::mbar_init(bars + 8 * (2 * S::kWideStages + i), 1);
         } else {
-            init_suffix_barriers();
+            for (int s = 0; s < S::kNarrowBars; ++s) dev::mbar_init(bars + 8 * s, 1);
         }
         dev::fence_mbar_init();
         dev::prefetch_tensormap(&maps.k);
@@ -2536,15 +2533,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                               id_slots);
         }
         // the prefix queue is empty: this CTA joins the suffix queue with the
-        // same shared memory (every copy it issued has landed)
+        // same shared memory (every copy it issued has landed), unless every
+        // suffix position is already claimed (the counter only grows, so a
+        // stale read can only send the CTA to find the queue empty)
+        __shared__ int suffix_open;
+        if (threadIdx.x == 0)
+            suffix_open = *static_cast<volatile int *>(a.queue_next + 1) < a.num_narrow_items;
         __syncthreads();
-        if (abort_flag) return;
-        if (threadIdx.x == 0) {
-            for (int i = 0; i < prefix_bars; ++i)
+        if (abort_flag || !suffix_open) return;
+        // barrier i is invalidated and re-initialised by thread i
+        for (int i = threadIdx.x; i < prefix_bars || i < S::kNarrowBars; i += blockDim.x) {
+            if (i < prefix_bars)
                 asm volatile("mbarrier.inval.shared::cta.b64 [%0];" ::"r"(bars + 8 * i) : "memory");
-            init_suffix_barriers();
-            dev::fence_mbar_init();
+            if (i < S::kNarrowBars) dev::mbar_init(bars + 8 * i, 1);
         }
+        dev::fence_mbar_init();
         __syncthreads();
     }
     if (warp < S::kSuffixWarps)
