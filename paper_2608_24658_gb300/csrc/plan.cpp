@@ -68,6 +68,9 @@ constexpr int64_t kPieceLengthSteps = 16;   // lengths tried per piece count, 4 
 // stay at the 8-page floor); 2 made the Llama-3-shape step 2 us slower.
 constexpr double kNarrowPiecesPerWarp = 2.5;
 constexpr double kWideProvision = 1.15;   // prefix CTAs relative to the cost model
+// Decode: up to this many prefix queue entries per prefix CTA (num / den)
+// become one CTA each
+constexpr int64_t kSpareEntriesNum = 3, kSpareEntriesDen = 2;
 // pairs of tcgen05 row tiles when at least this share of the prefix
 // tile-pages sits in pieces of two or more tiles.  Same-box A/B, pairs
 // against single tiles: 32k prefix tile alone 207.4 -> 155.8 us, join
@@ -592,6 +595,34 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         }
         n_narrow_ctas = narrow_cost > 0 ? std::max(S - n_wide, 1) : 0;
     }
+    // Prefix pieces are about one prefix CTA's share each.  When the runs
+    // cut that way give a few more queue entries than prefix CTAs, the CTAs
+    // that take a second entry end a piece after the others, with nothing
+    // left for them to even out on the suffix queue: then every entry gets
+    // a CTA of its own, at the same piece length.
+    int64_t wide_chunk = std::min<int64_t>(
+        kMaxTileItemPages,
+        std::max<int64_t>(kWideBlockPages,
+                          wide_units / std::max<int64_t>(1, static_cast<int64_t>(n_wide) * kWidePiecesPerCta)));
+    if (!prefill && mode != PARASON_FP32 && n_wide > 0 && n_narrow_ctas > 0) {
+        int64_t entries = 0;
+        for (size_t i = 0; i < runs.size();) {
+            const size_t j = group_end(i);
+            if (runs[i].wide) {
+                int64_t per = 0, n = 0;
+                piece_split(runs[i].pages, wide_chunk, kWideBlockPages, per, n);
+                const int64_t tiles = static_cast<int64_t>(j - i);
+                entries += n * (p->tc_pairs ? (tiles + 1) / 2 : tiles);
+            }
+            i = j;
+        }
+        const int32_t S = p->num_sms;
+        if (entries > n_wide && entries * kSpareEntriesDen <= static_cast<int64_t>(n_wide) * kSpareEntriesNum &&
+            entries <= S - 1) {
+            n_wide = static_cast<int32_t>(entries);
+            n_narrow_ctas = S - n_wide;
+        }
+    }
     p->num_wide_ctas = n_wide;
     p->num_ctas = n_wide + n_narrow_ctas;
     // the kernel's CTAs own the first positions of each queue (one per
@@ -685,11 +716,6 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
                               static_cast<int64_t>(static_cast<double>(narrow_pages) /
                                                    (kNarrowPiecesPerWarp * std::max<int64_t>(1, total_warps)))));
         p->narrow_chunk = narrow_chunk;
-        int64_t wide_chunk = std::min<int64_t>(
-            kMaxTileItemPages,
-            std::max<int64_t>(kWideBlockPages,
-                              wide_units / std::max<int64_t>(1, static_cast<int64_t>(n_wide) *
-                                                                    kWidePiecesPerCta)));
         if (prefill && n_wide > 0) {
             // candidates: the longest run cut into n pieces, n from the
             // fewest the tile allows up, and the lengths between that and
