@@ -69,7 +69,7 @@ constexpr int64_t kPieceLengthSteps = 16;   // lengths tried per piece count, 4 
 constexpr double kNarrowPiecesPerWarp = 2.5;
 constexpr double kWideProvision = 1.15;   // prefix CTAs relative to the cost model
 // Decode: up to this many prefix queue entries per prefix CTA (num / den)
-// become one CTA each
+// become one CTA each; up to two, two entries each
 constexpr int64_t kSpareEntriesNum = 3, kSpareEntriesDen = 2;
 // pairs of tcgen05 row tiles when at least this share of the prefix
 // tile-pages sits in pieces of two or more tiles.  Same-box A/B, pairs
@@ -597,9 +597,14 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     }
     // Prefix pieces are about one prefix CTA's share each.  When the runs
     // cut that way give a few more queue entries than prefix CTAs, the CTAs
-    // that take a second entry end a piece after the others, with nothing
+    // that take a second entry end a piece after the others, with little
     // left for them to even out on the suffix queue: then every entry gets
-    // a CTA of its own, at the same piece length.
+    // a CTA of its own, at the same piece length (up to 3/2 entries per
+    // CTA), or every CTA two entries (up to 2; the CTAs spared run the
+    // suffix queue).  Same-box A/B: Llama-3 shape (24 entries, 18 -> 24
+    // CTAs) step 42.9 -> 39.4 us; two-level (128 entries, 68 -> 64 CTAs)
+    // 78.8 -> 77.2 us.  With 3 or more entries per CTA, evening them out
+    // was slower (long prefix bf16 835.9 -> 843.0 us).
     int64_t wide_chunk = std::min<int64_t>(
         kMaxTileItemPages,
         std::max<int64_t>(kWideBlockPages,
@@ -620,6 +625,9 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
         if (entries > n_wide && entries * kSpareEntriesDen <= static_cast<int64_t>(n_wide) * kSpareEntriesNum &&
             entries <= S - 1) {
             n_wide = static_cast<int32_t>(entries);
+            n_narrow_ctas = S - n_wide;
+        } else if (entries > n_wide && entries <= 2 * static_cast<int64_t>(n_wide)) {
+            n_wide = static_cast<int32_t>((entries + 1) / 2);
             n_narrow_ctas = S - n_wide;
         }
     }
