@@ -600,11 +600,13 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
     // that take a second entry end a piece after the others, with little
     // left for them to even out on the suffix queue: then every entry gets
     // a CTA of its own, at the same piece length (up to 3/2 entries per
-    // CTA), or every CTA two entries (up to 2; the CTAs spared run the
-    // suffix queue).  Same-box A/B: Llama-3 shape (24 entries, 18 -> 24
-    // CTAs) step 42.9 -> 39.4 us; two-level (128 entries, 68 -> 64 CTAs)
-    // 78.8 -> 77.2 us.  With 3 or more entries per CTA, evening them out
-    // was slower (long prefix bf16 835.9 -> 843.0 us).
+    // CTA, while that leaves half the SMs to the suffix queue), or every CTA
+    // two entries (up to 2; the CTAs spared run the suffix queue).  Same-box
+    // A/B: Llama-3 shape (24 entries, 18 -> 24 CTAs) step 42.9 -> 39.4 us;
+    // two-level (128 entries, 68 -> 64 CTAs) 78.8 -> 77.2 us.  Slower, and
+    // so left out: evening out 3 or more entries per CTA (long prefix bf16
+    // 835.9 -> 843.0 us), and 128 prefix CTAs of 152 for the two-level tree
+    // with e4m3 KV (71.8 -> 73.3 us).
     int64_t wide_chunk = std::min<int64_t>(
         kMaxTileItemPages,
         std::max<int64_t>(kWideBlockPages,
@@ -622,11 +624,12 @@ parason_status build_host(parason_plan_s *p, const parason_attn_config *cfg, int
             i = j;
         }
         const int32_t S = p->num_sms;
-        if (entries > n_wide && entries * kSpareEntriesDen <= static_cast<int64_t>(n_wide) * kSpareEntriesNum &&
-            entries <= S - 1) {
+        const bool one_each =
+            entries * kSpareEntriesDen <= static_cast<int64_t>(n_wide) * kSpareEntriesNum;
+        if (entries > n_wide && one_each && entries <= S / 2) {
             n_wide = static_cast<int32_t>(entries);
             n_narrow_ctas = S - n_wide;
-        } else if (entries > n_wide && entries <= 2 * static_cast<int64_t>(n_wide)) {
+        } else if (entries > n_wide && !one_each && entries <= 2 * static_cast<int64_t>(n_wide)) {
             n_wide = static_cast<int32_t>((entries + 1) / 2);
             n_narrow_ctas = S - n_wide;
         }
