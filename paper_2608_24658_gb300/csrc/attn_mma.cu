@@ -1187,8 +1187,8 @@ __device__ void prefix_cta(const CUtensorMap *tmap_k, const CUtensorMap *tmap_v,
 // TMEM, 512 columns: O[2] at 0 and 128, S/P[2] at 256 and 320, Q[2] at 384
 // and 448.  Shared memory: the ring [6][K: 2 col blocks x 64 tokens x 128 B |
 // V: same], 128-byte swizzled (K-major descriptors for K, MN-major for V),
-// and the metadata slots; with e4m3 KV the first half of the ring stages the
-// raw blocks (6 x 16 KB) and the second half holds 3 converted f16 blocks.
+// and the metadata slots; with e4m3 KV the first 64 KB stage the raw blocks
+// (4 x 16 KB) and the next 128 KB hold 4 converted f16 blocks.
 // ---------------------------------------------------------------------------
 constexpr int kTcRows = 128;
 constexpr int kTcBlockPages = 4;
