@@ -543,16 +543,41 @@ def algorithmic_bytes_of_plan(r):
     return {"kv": kv, "q": q, "out": q, "lse": lse, "step": kv + 2 * q + lse, "attn": kv + q}
 
 
+def _code_tokens(text: str) -> str:
+    """C/C++/CUDA source without comments, whitespace runs collapsed: edits
+    to comments or layout leave the hash alone."""
+    out, i, n = [], 0, len(text)
+    while i < n:
+        c = text[i]
+        if c in "\"'":                                   # string or char literal
+            j = i + 1
+            while j < n and text[j] != c:
+                j += 2 if text[j] == "\\" else 1
+            out.append(text[i:j + 1])
+            i = j + 1
+        elif text.startswith("//", i):
+            j = text.find("\n", i)
+            i = n if j < 0 else j
+        elif text.startswith("/*", i):
+            j = text.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+        else:
+            out.append(c)
+            i += 1
+    return " ".join("".join(out).split())
+
+
 def kernel_source_hash() -> str:
-    """Hash of the kernel sources, to tell whether stored ncu counters still apply."""
+    """Hash of the kernel sources' code (comments and whitespace aside), to
+    tell whether stored ncu counters still apply."""
     import hashlib
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_24658_gb300", "csrc")
     for name in sorted(os.listdir(csrc)):
         if name.endswith((".cu", ".cuh", ".h", ".cpp")):
-            with open(os.path.join(csrc, name), "rb") as f:
+            with open(os.path.join(csrc, name), encoding="utf-8") as f:
                 h.update(name.encode())
-                h.update(f.read())
+                h.update(_code_tokens(f.read()).encode())
     return h.hexdigest()[:16]
 
 
