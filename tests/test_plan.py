@@ -205,3 +205,35 @@ def test_plan_sm_count_changes_split_only():
         with Plan.for_tree(tree, host_only=True, num_sms=sms) as plan:
             assert plan.info()["num_sms"] == sms
             verify_plan(tree, plan)
+
+
+def test_prefix_ctas_even_out_queue_entries():
+    """Decode plans give every prefix CTA the same number of prefix queue
+    entries when the runs cut at one CTA's share give up to twice as many
+    entries as CTAs: one each up to 3/2 (while half the SMs stay on the
+    suffix queue), else two each; more entries keep the cost-model count."""
+    cases = {
+        (2, "bf16"): 1,      # Llama-3 shape: 24 entries, one per prefix CTA
+        (3, "bf16"): 2,      # two-level: 128 entries, two per prefix CTA
+    }
+    for (idx, mode), per_cta in cases.items():
+        tree = W.make_config(idx, mode, values=False)
+        with Plan.for_tree(tree, host_only=True, num_sms=152) as plan:
+            info = plan.info()
+            entries = info["num_wide_items"] // (2 if info["tile_pairs"] else 1)
+            assert entries == per_cta * info["num_wide_ctas"], (idx, mode, info)
+            assert info["num_ctas"] == 152
+            assert info["num_ctas"] - info["num_wide_ctas"] >= 152 // 2
+            verify_plan(tree, plan)
+    # the two-level tree with e4m3 KV: 128 entries would take 128 of 152
+    # SMs one each, so it keeps the cost model's count (more than 64)
+    tree = W.make_config(3, "fp8", values=False)
+    with Plan.for_tree(tree, host_only=True, num_sms=152) as plan:
+        info = plan.info()
+        assert 64 < info["num_wide_ctas"] < info["num_wide_items"]
+    # the long prefix (3 or more entries per CTA) is left to the cost model
+    tree = W.make_config(5, values=False)
+    with Plan.for_tree(tree, host_only=True, num_sms=152) as plan:
+        info = plan.info()
+        entries = info["num_wide_items"] // (2 if info["tile_pairs"] else 1)
+        assert entries > 2 * info["num_wide_ctas"]
