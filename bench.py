@@ -760,6 +760,11 @@ def run_prefill(args):
             plan.decode(tree.q, tree.k_pages, tree.v_pages, out=out, lse=lse, workspace=ws,
                         stream=stream)
 
+        # the clock sampler starts first, so that the warm-up runs right
+        # before the timed loop (the GPU does not idle in between)
+        sampler = ClockSampler(0)
+        sampler.start()
+        time.sleep(0.3)
         for _ in range(args.warmup):
             flush.fill_(1.0)
             step()
@@ -767,9 +772,6 @@ def run_prefill(args):
         K = min(args.steps, 200)
         ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
               for _ in range(K)]
-        sampler = ClockSampler(0)
-        sampler.start()
-        time.sleep(0.3)
         torch.cuda.synchronize(dev)
         for i in range(K):
             flush.fill_(float(i))
