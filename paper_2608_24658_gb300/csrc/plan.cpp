@@ -37,7 +37,10 @@ int32_t narrow_warps(int32_t mode, int32_t head_dim, int32_t g) {
     if (mode == PARASON_FP8_E4M3_KV) return 12;
     return (mode == PARASON_BF16 && head_dim == 128 && g <= 4) ? 6 : 8;
 }
-constexpr int kMinPiecePages = 8;       // suffix-pass pieces are at least this long
+// Suffix-pass pieces are at least kMinPiecePages long (4 against 8: tiny
+// fork 13.8 -> 11.7 us, the Llama-3 shape, whose pieces are 8 pages long by
+// the share below, level).
+constexpr int kMinPiecePages = 4;
 constexpr int kMaxPiecePages = 128;     // and at most this long
 // The tcgen05 tile holds an item of up to 512 pages (its metadata slot).
 constexpr int kMaxTileItemPages = 512;
@@ -65,7 +68,7 @@ constexpr int64_t kPieceLengthSteps = 16;   // lengths tried per piece count, 4 
 // suffix pieces: about this many per warp of the launch (at least
 // kMinPiecePages and at most kMaxPiecePages pages).  Same-box A/B against
 // 3: two-level step 79.7 -> 78.8 us, the Llama-3 shape level (its pieces
-// stay at the 8-page floor); 2 made the Llama-3-shape step 2 us slower.
+// were at an 8-page floor); 2 made the Llama-3-shape step 2 us slower.
 constexpr double kNarrowPiecesPerWarp = 2.5;
 constexpr double kWideProvision = 1.15;   // prefix CTAs relative to the cost model
 // Decode: up to this many prefix queue entries per prefix CTA (num / den)
