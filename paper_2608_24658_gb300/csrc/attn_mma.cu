@@ -149,10 +149,11 @@ __device__ __forceinline__ void load_page(uint32_t dst, const CUtensorMap *tmap_
 }
 
 // The same for a suffix page, in one box per tensor (the page maps) where a
-// page has several column blocks: each TMA box costs the SM's copy engine a
-// fixed time, and with 2 KB boxes it held a suffix CTA to about 60 GB/s.  A
-// suffix page is read by one item only, so its lines go first when L2 needs
-// room (the partials written meanwhile stay for the merge).
+// page has several column blocks: half the copies at head_dim 128 bf16, in
+// the same shared-memory layout (same-box A/B: two-level step 81.8 -> 79.6
+// us, long prefix 839.6 -> 834.2 us).  A suffix page is read by one item
+// only, so its lines go first when L2 needs room (the partials written
+// meanwhile stay for the merge).
 template <int D, class KV>
 __device__ __forceinline__ void load_suffix_page(uint32_t dst, const KvMaps &maps, int row,
                                                  uint32_t bar) {
