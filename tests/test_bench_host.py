@@ -63,3 +63,21 @@ def test_reference_arm_json_line():
     assert line["value"] > 0 and line["cpu_baseline"]["kind"] == "oracle"
     assert line["e2e"]["h2d_bytes_per_step"] == 0
     assert line["config"]["workload"] == "tiny_fork_h8_2_d64"
+
+
+def test_kernel_source_hash_ignores_comments_only():
+    """The hash that keys the stored DRAM counters sees code, not comments or
+    layout: a comment edit keeps it, a code edit (even inside a string
+    literal that looks like a comment) changes it."""
+    sys.path.insert(0, ROOT)
+    import bench
+    tok = bench._code_tokens
+    base = 'int a = 1; // note\n/* block\n comment */ const char *s = "// kept";\n'
+    assert tok(base) == tok(base.replace("note", "other note").replace("block", "x"))
+    assert tok(base) == tok(base.replace("int a = 1;", "int  a =\n 1;"))
+    assert tok(base) != tok(base.replace("int a = 1;", "int a = 2;"))
+    assert tok(base) != tok(base.replace('"// kept"', '"// changed"'))
+    assert "kept" in tok(base) and "note" not in tok(base) and "block" not in tok(base)
+    assert tok("char c = '\\'';  // q") == "char c = '\\'';"
+    h = bench.kernel_source_hash()
+    assert len(h) == 16 and int(h, 16) >= 0
