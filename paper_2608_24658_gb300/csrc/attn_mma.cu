@@ -13,12 +13,17 @@
 //        Warp roles: a scheduler warp stages each item's metadata; a
 //        producer warp moves 64-token blocks of K and V by TMA (one 5-D box
 //        per column block when the block's 4 pages are consecutive in the
-//        pool, else 3-D boxes per page) into a 6-stage ring; one thread
-//        issues S = Q K^T and another O += P V as tcgen05.mma with Q, S/P and
-//        O in TMEM and K, V from shared memory; 4 softmax warps own one row
-//        per thread (TMEM lane) and write P over S; 4 epilogue warps store an
-//        item's O and load Q two items ahead (with e4m3 KV they also convert
-//        each staged block to f16).
+//        pool, else 3-D boxes per page) into a 6-stage ring (with e4m3 KV,
+//        4 raw stages and 4 converted ones); one thread issues S = Q K^T and
+//        another O += P V as tcgen05.mma with Q, S/P and O in TMEM and K, V
+//        from shared memory; 4 softmax warps own one row per thread (TMEM
+//        lane) and write P over S; 4 epilogue warps store an item's O and
+//        load Q two items ahead (with e4m3 KV they also convert each staged
+//        block to f16).
+//      - bf16 at head_dim 128, when the planner pairs row tiles: two
+//        128-row tiles of a piece against each staged block
+//        (prefix_cta_tc_pair), Q in shared memory, each tile's S/P and O in
+//        TMEM, so that a block is staged once for 256 rows.
 //      - head_dim 64: mma.sync (prefix_cta): a producer warp streams pages
 //        into a ring, 8 consumer warps of 16 rows share the pages and combine
 //        through shared memory.
@@ -27,7 +32,9 @@
 //    an independent worker with its own TMA ring that pulls split-K pieces
 //    from a queue: no CTA barrier, no cross-warp combine.  QK^T and PV are
 //    mma.sync m16n8k16 with fp32 accumulation and a quad-shuffle online
-//    softmax; tiles of 5 to 8 rows run the transposed step (S^T = K Q^T).
+//    softmax; tiles of 5 to 8 rows run the transposed step (S^T = K Q^T),
+//    with e4m3 KV two pages per softmax update.  A bf16 page at head_dim 128
+//    comes in one TMA box per tensor (the 4-D page maps).
 //
 // Every item writes a partial (o, m, l) per row.  The merge kernel (merge.cu)
 // folds the partials of every branch's path; it is launched as a
@@ -42,8 +49,9 @@
 //    PARASON_ERANGE through the plan's error record).  The K scale joins the
 //    softmax scale, the V scale multiplies the partial o.  The suffix
 //    fragment layouts permute d so that each thread's bytes are contiguous:
-//    QK^T takes d = 16ks + 4t + {0..3} for thread t of a quad, PV gives
-//    thread column c of n-tile n the output d = 16c + n.
+//    the 16-row step's QK^T takes d = 16ks + 4t + {0..3} for thread t of a
+//    quad, the transposed step's two 16-byte runs per token row, and PV
+//    gives each thread one 16-byte chunk of V's columns.
 //
 // Scores are kept in the log2 domain: x = scale*log2(e)*<q,k>, so a partial
 // is m = max x, l = sum 2^(x-m), o = sum 2^(x-m) v (unnormalised).
